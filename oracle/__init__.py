@@ -1,0 +1,207 @@
+"""CPU oracle for the block-sparse INT8 linear layer (ctypes front end).
+
+TEST INFRASTRUCTURE ONLY: the test suite, the smoke check and the
+benchmark's CPU-baseline leg may import this package; the library and its
+Python binding never do.  The arithmetic lives in ``bsgemm_oracle.c``, a
+plain triple loop over the decompressed weights followed by the epilogue;
+every function there cites the passage of arXiv 2211.07715 it follows.
+
+ctypes releases the GIL during a foreign call, so ``linear(...,
+threads=n)`` runs row ranges on n host threads.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "bsgemm_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+I32, F32, F32_GELU, I8, I8_GELU = 0, 1, 2, 3, 4
+BLOCK = 4
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (IEEE fp32: no contraction, no fast-math)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math",
+                               "-fPIC", "-shared", _SRC, "-o", tmp, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            i8p = ctypes.POINTER(ctypes.c_int8)
+            i32p = ctypes.POINTER(ctypes.c_int32)
+            u8p = ctypes.POINTER(ctypes.c_uint8)
+            f32p = ctypes.POINTER(ctypes.c_float)
+            c_int, c_float, c_double = ctypes.c_int, ctypes.c_float, ctypes.c_double
+            lib.oracle_bsr_to_dense.argtypes = [c_int, c_int, i32p, i32p, i8p, i8p]
+            lib.oracle_bsr_to_dense.restype = c_int
+            lib.oracle_dense_to_bsr.argtypes = [c_int, c_int, i8p, u8p, i32p, i32p, i8p]
+            lib.oracle_dense_to_bsr.restype = c_int
+            lib.oracle_acc.argtypes = [c_int, c_int, c_int, i8p, i8p, i32p, c_int, c_int]
+            lib.oracle_acc.restype = c_int
+            lib.oracle_dequant_f32.argtypes = [ctypes.c_int32, c_float, c_float]
+            lib.oracle_dequant_f32.restype = c_float
+            lib.oracle_dequant_f64.argtypes = [ctypes.c_int32, c_float, c_float]
+            lib.oracle_dequant_f64.restype = c_double
+            lib.oracle_gelu_f64.argtypes = [c_double]
+            lib.oracle_gelu_f64.restype = c_double
+            lib.oracle_gelu_f32.argtypes = [c_float]
+            lib.oracle_gelu_f32.restype = c_float
+            lib.oracle_requant.argtypes = [c_float, c_float]
+            lib.oracle_requant.restype = ctypes.c_int8
+            lib.oracle_linear.argtypes = [c_int, c_int, c_int, i8p, i8p, f32p, f32p, c_int, c_float,
+                                          ctypes.c_void_p, c_int, c_int]
+            lib.oracle_linear.restype = c_int
+            lib.oracle_block_prune.argtypes = [c_int, c_int, f32p, c_double, u8p]
+            lib.oracle_block_prune.restype = ctypes.c_int64
+            _lib = lib
+    return _lib
+
+
+def _ptr(a: np.ndarray, ctype):
+    return a.ctypes.data_as(ctypes.POINTER(ctype))
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+# --- block-compressed format (App. A.1, App. A.3.4) ----------------------
+
+def bsr_to_dense(n_out: int, k_in: int, indptr, colidx, values) -> np.ndarray:
+    lib = _load()
+    indptr, colidx = _c(indptr, np.int32), _c(colidx, np.int32)
+    values = _c(values, np.int8).reshape(-1)
+    w = np.empty((n_out, k_in), dtype=np.int8)
+    rc = lib.oracle_bsr_to_dense(n_out, k_in, _ptr(indptr, ctypes.c_int32), _ptr(colidx, ctypes.c_int32),
+                                 _ptr(values, ctypes.c_int8), _ptr(w, ctypes.c_int8))
+    if rc:
+        raise ValueError("invalid block-compressed arrays")
+    return w
+
+
+def dense_to_bsr(w: np.ndarray, mask: np.ndarray):
+    lib = _load()
+    w = _c(w, np.int8)
+    n_out, k_in = w.shape
+    mask = _c(mask != 0, np.uint8)
+    indptr = np.empty(n_out // BLOCK + 1, dtype=np.int32)
+    nnzb = lib.oracle_dense_to_bsr(n_out, k_in, _ptr(w, ctypes.c_int8), _ptr(mask, ctypes.c_uint8),
+                                   _ptr(indptr, ctypes.c_int32), None, None)
+    colidx = np.empty(nnzb, dtype=np.int32)
+    values = np.empty((nnzb, BLOCK), dtype=np.int8)
+    lib.oracle_dense_to_bsr(n_out, k_in, _ptr(w, ctypes.c_int8), _ptr(mask, ctypes.c_uint8),
+                            _ptr(indptr, ctypes.c_int32), _ptr(colidx, ctypes.c_int32),
+                            _ptr(values, ctypes.c_int8))
+    return indptr, colidx, values
+
+
+def weight_dense(wt) -> np.ndarray:
+    """Decompress a synth.BsrWeight."""
+    return bsr_to_dense(wt.n_out, wt.k_in, wt.indptr, wt.colidx, wt.values)
+
+
+# --- accumulation and epilogue (Sec. 3, Algorithm 1, App. A.3.3) ---------
+
+def acc(x: np.ndarray, w: np.ndarray) -> np.ndarray:
+    lib = _load()
+    x, w = _c(x, np.int8), _c(w, np.int8)
+    m, k_in = x.shape
+    n_out = w.shape[0]
+    out = np.empty((m, n_out), dtype=np.int32)
+    rc = lib.oracle_acc(m, n_out, k_in, _ptr(x, ctypes.c_int8), _ptr(w, ctypes.c_int8),
+                        _ptr(out, ctypes.c_int32), 0, m)
+    if rc:
+        raise OverflowError("accumulator leaves the int32 range")
+    return out
+
+
+def dequant_f32(a: int, scale: float, bias: float) -> np.float32:
+    return np.float32(_load().oracle_dequant_f32(int(a), float(scale), float(bias)))
+
+
+def dequant_f64(a: int, scale: float, bias: float) -> float:
+    return _load().oracle_dequant_f64(int(a), float(scale), float(bias))
+
+
+def gelu_f32(y: float) -> np.float32:
+    return np.float32(_load().oracle_gelu_f32(float(np.float32(y))))
+
+
+def gelu_f64(y: float) -> float:
+    return _load().oracle_gelu_f64(float(y))
+
+
+def requant(v: float, inv_out_scale: float) -> int:
+    return int(_load().oracle_requant(float(np.float32(v)), float(np.float32(inv_out_scale))))
+
+
+def out_dtype(kind: int):
+    return {I32: np.int32, F32: np.float64, F32_GELU: np.float64, I8: np.int8, I8_GELU: np.int8}[kind]
+
+
+def linear(x: np.ndarray, w: np.ndarray, scales, bias, kind: int, out_scale: float = 1.0,
+           rows=None, threads: int = 1) -> np.ndarray:
+    """The whole layer on rows `rows` of x (all rows if None).
+
+    Output dtype by kind: I32 -> int32, F32/F32_GELU -> float64 (exact-valued
+    reference), I8/I8_GELU -> int8 decided in fp32.
+    """
+    lib = _load()
+    w = _c(w, np.int8)
+    n_out, k_in = w.shape
+    x = _c(x, np.int8)
+    if rows is not None:
+        x = np.ascontiguousarray(x[np.asarray(rows, dtype=np.int64)])
+    m = x.shape[0]
+    scales = _c(scales, np.float32)
+    bias_arr = None if bias is None else _c(bias, np.float32)
+    out = np.empty((m, n_out), dtype=out_dtype(kind))
+
+    def run(r0, r1):
+        return lib.oracle_linear(m, n_out, k_in, _ptr(x, ctypes.c_int8), _ptr(w, ctypes.c_int8),
+                                 _ptr(scales, ctypes.c_float),
+                                 None if bias_arr is None else _ptr(bias_arr, ctypes.c_float),
+                                 kind, float(out_scale), out.ctypes.data_as(ctypes.c_void_p), r0, r1)
+
+    threads = max(1, min(int(threads), m))
+    if threads == 1:
+        rcs = [run(0, m)]
+    else:
+        bounds = [m * i // threads for i in range(threads + 1)]
+        with ThreadPoolExecutor(threads) as ex:
+            rcs = list(ex.map(lambda i: run(bounds[i], bounds[i + 1]), range(threads)))
+    for rc in rcs:
+        if rc == -1:
+            raise ValueError("bad kind or out_scale")
+        if rc == -2:
+            raise OverflowError("accumulator leaves the int32 range")
+        if rc:
+            raise RuntimeError(f"oracle_linear failed ({rc})")
+    return out
+
+
+def block_prune(w: np.ndarray, sparsity: float) -> np.ndarray:
+    """Keep-mask [N/4][K] of the average-magnitude block pruning (App. A.1)."""
+    lib = _load()
+    w = _c(w, np.float32)
+    n_out, k_in = w.shape
+    keep = np.empty((n_out // BLOCK, k_in), dtype=np.uint8)
+    lib.oracle_block_prune(n_out, k_in, _ptr(w, ctypes.c_float), float(sparsity), _ptr(keep, ctypes.c_uint8))
+    return keep.astype(bool)

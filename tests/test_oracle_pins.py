@@ -1,0 +1,293 @@
+"""Pins for the CPU oracle: checks against values and identities that do not
+come from the oracle itself (hand-worked cases, closed forms, a library
+matmul, brute force, invariants).  CPU only.
+
+A mistake anywhere in the oracle (a dropped term, a wrong sign or index, a
+transposed operand, a wrong rounding mode or coefficient) fails one of them.
+"""
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _hand_cases():
+    with open(os.path.join(GOLDEN, "hand_small.json")) as f:
+        return json.load(f)["cases"]
+
+
+# ---------------------------------------------------------------- format --
+
+@pytest.mark.parametrize("case", _hand_cases(), ids=lambda c: c["name"])
+def test_hand_cases_acc(case):
+    """Hand-worked accumulators (App. A.1 block layout, Algorithm 1 dot)."""
+    w = oracle.bsr_to_dense(case["N"], case["K"], case["indptr"], case["colidx"], case["values"])
+    a = oracle.acc(np.array(case["X"], dtype=np.int8), w)
+    assert a.tolist() == case["acc"]
+
+
+def test_hand_case_epilogue():
+    """Hand-worked dequantisation and tie-heavy requantisation."""
+    case = [c for c in _hand_cases() if "q" in c][0]
+    w = oracle.bsr_to_dense(case["N"], case["K"], case["indptr"], case["colidx"], case["values"])
+    x = np.array(case["X"], dtype=np.int8)
+    s = np.full(case["N"], case["scale"], np.float32)
+    b = np.full(case["N"], case["bias"], np.float32)
+    y = oracle.linear(x, w, s, b, oracle.F32)
+    assert y.tolist() == case["y"]
+    q = oracle.linear(x, w, s, b, oracle.I8, out_scale=case["out_scale"])
+    assert q.tolist() == case["q"]
+
+
+def test_block_orientation_is_output_rows():
+    """A block covers 4 consecutive OUTPUT rows of one column (App. A.1)."""
+    w = oracle.bsr_to_dense(8, 5, [0, 0, 1], [3], [[1, 2, 3, 4]])
+    expect = np.zeros((8, 5), np.int8)
+    expect[4:8, 3] = [1, 2, 3, 4]
+    assert np.array_equal(w, expect)
+
+
+def test_bsr_rejects_bad_arrays():
+    with pytest.raises(ValueError):
+        oracle.bsr_to_dense(4, 3, [0, 2], [2, 1], [[1] * 4, [1] * 4])  # unsorted
+    with pytest.raises(ValueError):
+        oracle.bsr_to_dense(4, 3, [0, 1], [3], [[1] * 4])  # column out of range
+    with pytest.raises(ValueError):
+        oracle.bsr_to_dense(6, 3, [0, 0], [], np.zeros((0, 4)))  # N not a multiple of 4
+
+
+def test_dense_bsr_roundtrip_keeps_zero_valued_blocks():
+    rng = np.random.default_rng(1)
+    w = rng.integers(-127, 128, size=(12, 9)).astype(np.int8)
+    mask = rng.random((3, 9)) < 0.4
+    w[0:4, 2] = 0
+    mask[0, 2] = True  # a stored block whose values are all zero
+    indptr, colidx, values = oracle.dense_to_bsr(w, mask)
+    assert indptr[-1] == mask.sum()
+    back = oracle.bsr_to_dense(12, 9, indptr, colidx, values)
+    expect = np.where(np.repeat(mask, 4, axis=0), w, 0).astype(np.int8)
+    assert np.array_equal(back, expect)
+
+
+def test_generator_matches_requested_sparsity():
+    """Stored-block count = total - round(s * total); positions unique."""
+    for (n, k, s) in [(768, 768, 0.9), (3072, 768, 0.8), (768, 3072, 0.9), (20, 7, 0.5)]:
+        wt = synth.draw_weight(synth.rng_for(5), n, k, s)
+        total = n // 4 * k
+        assert wt.nnzb == total - int(math.floor(s * total + 0.5))
+        w = oracle.weight_dense(wt)  # validates sortedness and range
+        assert w.shape == (n, k)
+
+
+# ---------------------------------------------------------- accumulation --
+
+def test_fully_dense_equals_library_matmul():
+    """0% block sparsity: the oracle equals numpy's int64 matmul."""
+    rng = synth.rng_for(11)
+    wt = synth.draw_weight(rng, 16, 37, 0.0)
+    x = synth.draw_x(rng, 9, 37, "u127")
+    # independent construction of the dense weight from the block values
+    w_indep = wt.values.reshape(4, 37, 4).transpose(0, 2, 1).reshape(16, 37)
+    expect = x.astype(np.int64) @ w_indep.astype(np.int64).T
+    assert np.array_equal(oracle.acc(x, oracle.weight_dense(wt)), expect)
+
+
+def test_random_sparse_equals_library_matmul():
+    rng = synth.rng_for(12)
+    wt = synth.draw_weight(rng, 64, 200, 0.9)
+    x = synth.draw_x(rng, 33, 200, "n30")
+    w = np.zeros((64, 200), np.int64)
+    for r in range(16):
+        for j in range(wt.indptr[r], wt.indptr[r + 1]):
+            w[4 * r:4 * r + 4, wt.colidx[j]] = wt.values[j]
+    assert np.array_equal(oracle.acc(x, oracle.weight_dense(wt)), x.astype(np.int64) @ w.T)
+
+
+def test_all_blocks_zero_gives_bias():
+    rng = synth.rng_for(13)
+    wt = synth.draw_weight(rng, 32, 50, 1.0)
+    assert wt.nnzb == 0
+    x = synth.draw_x(rng, 7, 50, "u127")
+    w = oracle.weight_dense(wt)
+    assert not oracle.acc(x, w).any()
+    y = oracle.linear(x, w, wt.scales, wt.bias, oracle.F32)
+    assert np.array_equal(y, np.broadcast_to(wt.bias.astype(np.float64), y.shape))
+    y32 = oracle.linear(x, w, wt.scales, None, oracle.F32)
+    assert not y32.any()
+
+
+def test_one_hot_block():
+    rng = synth.rng_for(14)
+    x = synth.draw_x(rng, 5, 11, "u127")
+    v = [7, -128, 0, 127]
+    w = oracle.bsr_to_dense(12, 11, [0, 0, 1, 1], [6], [v])
+    a = oracle.acc(x, w)
+    expect = np.zeros((5, 12), np.int64)
+    for i in range(4):
+        expect[:, 4 + i] = x[:, 6].astype(np.int64) * v[i]
+    assert np.array_equal(a, expect)
+
+
+def test_k_permutation_invariance_and_linearity():
+    rng = synth.rng_for(15)
+    wt = synth.draw_weight(rng, 24, 40, 0.7)
+    w = oracle.weight_dense(wt)
+    x1 = rng.integers(-63, 64, size=(6, 40)).astype(np.int8)
+    x2 = rng.integers(-63, 64, size=(6, 40)).astype(np.int8)
+    a1 = oracle.acc(x1, w)
+    perm = rng.permutation(40)
+    assert np.array_equal(oracle.acc(x1[:, perm], w[:, perm]), a1)
+    assert np.array_equal(oracle.acc((x1 + x2).astype(np.int8), w), a1 + oracle.acc(x2, w))
+    # negating the input negates the accumulator
+    assert np.array_equal(oracle.acc((-x1).astype(np.int8), w), -a1)
+
+
+def test_int32_extreme_and_overflow():
+    """K = 131071 of (-128)*(-128) is the largest sum that fits int32."""
+    k = 131071
+    x = np.full((1, k), -128, np.int8)
+    w = np.full((4, k), -128, np.int8)
+    assert oracle.acc(x, w).tolist() == [[16384 * k] * 4]
+    assert 16384 * k <= 2**31 - 1 < 16384 * (k + 1)
+    with pytest.raises(OverflowError):
+        oracle.acc(np.full((1, k + 1), -128, np.int8), np.full((4, k + 1), -128, np.int8))
+
+
+# -------------------------------------------------------------- epilogue --
+
+def _nearest_f32(q: Fraction) -> np.float32:
+    """Round an exact rational to the nearest fp32, ties to even."""
+    f = np.float32(float(q))
+    best = None
+    for c in (np.nextafter(f, np.float32(-np.inf)), f, np.nextafter(f, np.float32(np.inf))):
+        d = abs(Fraction(float(c)) - q)
+        if best is None or d < best[0] or (d == best[0] and (c.view(np.int32) & 1) == 0):
+            best = (d, c)
+    return best[1]
+
+
+def test_dequant_f32_is_single_rounding_of_exact_value():
+    rng = np.random.default_rng(21)
+    for _ in range(2000):
+        a = int(rng.integers(-5_000_000, 5_000_000))
+        s = np.float32(rng.uniform(1e-3, 1e-2))
+        b = np.float32(rng.normal(0, 0.02))
+        exact = Fraction(a) * Fraction(float(s)) + Fraction(float(b))  # |a| < 2^24: (float)a exact
+        assert oracle.dequant_f32(a, s, b) == _nearest_f32(exact)
+        assert oracle.dequant_f64(a, s, b) == pytest.approx(float(exact), rel=1e-15, abs=1e-300)
+
+
+def test_requant_ties_and_saturation():
+    """Round half to even, saturate to [-128, 127]."""
+    cases = {2.5: 2, 3.5: 4, -2.5: -2, -3.5: -4, 0.5: 0, -0.5: 0, 1.4999999: 1,
+             126.5: 126, 127.4: 127, 127.5: 127, 1e6: 127, -127.5: -128, -128.5: -128,
+             -128.6: -128, -1e6: -128, 0.0: 0}
+    for t, q in cases.items():
+        assert oracle.requant(t, 1.0) == q, t
+    # the multiply happens in fp32: 0.05 -> inv = 1/0.05f
+    inv = np.float32(1.0) / np.float32(0.05)
+    assert oracle.requant(np.float32(1.275), inv) == int(np.rint(np.float32(1.275) * inv))
+
+
+def test_gelu_f64_closed_forms():
+    """GELU(y) = y * Phi(y); standard normal CDF values from tables."""
+    assert oracle.gelu_f64(0.0) == 0.0
+    assert oracle.gelu_f64(1.0) == pytest.approx(0.8413447460685429, abs=1e-15)
+    assert oracle.gelu_f64(-1.0) == pytest.approx(-0.15865525393145707, abs=1e-15)
+    assert oracle.gelu_f64(2.0) == pytest.approx(2 * 0.9772498680518208, abs=1e-14)
+    for y in (-3.0, -0.3, 0.7, 4.0):  # GELU(y) - GELU(-y) = y
+        assert oracle.gelu_f64(y) - oracle.gelu_f64(-y) == pytest.approx(y, abs=1e-14)
+
+
+def test_gelu_f32_within_derived_bound():
+    """A&S 7.1.28 error <= 3e-7 on erf; fp32 evaluation of p^16 adds at
+    most ~31 half-ulps relative; together |err| <= 1.2e-6 |y| + 1e-12."""
+    ys = np.concatenate([np.linspace(-12, 12, 4801), np.linspace(-0.05, 0.05, 401),
+                         np.linspace(-400, 400, 801)]).astype(np.float32)
+    for y in ys:
+        exact = 0.5 * float(y) * (1.0 + math.erf(float(y) / math.sqrt(2.0)))
+        assert abs(float(oracle.gelu_f32(y)) - exact) <= 1.2e-6 * abs(float(y)) + 1e-12, y
+
+
+def test_gelu_f32_special_values():
+    assert float(oracle.gelu_f32(0.0)) == 0.0
+    assert float(oracle.gelu_f32(1.0)) == pytest.approx(0.8413447460685429, abs=2e-7)
+    for y in (5.7, 6.0, 50.0, 1e30):
+        assert float(oracle.gelu_f32(y)) == np.float32(y)  # erf term rounds to exactly 1
+    for y in (-5.7, -6.0, -50.0, -1e30):
+        assert float(oracle.gelu_f32(y)) == 0.0
+
+
+def test_i8_gelu_path_uses_fp32_sequence():
+    """The int8 GELU output is requant(gelu_f32(fp32 dequant))."""
+    rng = synth.rng_for(31)
+    wt = synth.draw_weight(rng, 16, 64, 0.5)
+    x = synth.draw_x(rng, 8, 64, "n30")
+    w = oracle.weight_dense(wt)
+    a = oracle.acc(x, w)
+    q = oracle.linear(x, w, wt.scales, wt.bias, oracle.I8_GELU, out_scale=0.03)
+    inv = np.float32(1.0) / np.float32(0.03)
+    for m in range(8):
+        for n in range(16):
+            y = oracle.dequant_f32(a[m, n], wt.scales[n], wt.bias[n])
+            assert q[m, n] == oracle.requant(oracle.gelu_f32(y), inv)
+
+
+def test_row_sampling_and_threads_agree():
+    rng = synth.rng_for(41)
+    wt = synth.draw_weight(rng, 40, 96, 0.8)
+    x = synth.draw_x(rng, 50, 96, "u127")
+    w = oracle.weight_dense(wt)
+    full = oracle.linear(x, w, wt.scales, wt.bias, oracle.I8, out_scale=0.05)
+    par = oracle.linear(x, w, wt.scales, wt.bias, oracle.I8, out_scale=0.05, threads=4)
+    rows = [0, 7, 49, 23]
+    part = oracle.linear(x, w, wt.scales, wt.bias, oracle.I8, out_scale=0.05, rows=rows)
+    assert np.array_equal(full, par)
+    assert np.array_equal(full[rows], part)
+
+
+# --------------------------------------------------------------- pruning --
+
+def test_block_prune_hand_case():
+    """Average-magnitude block score (App. A.1); lowest scores pruned."""
+    w = np.array([[1, -8, 0.5],
+                  [1, 8, 0.5],
+                  [-1, 0, 0.5],
+                  [1, 0, 0.5]], np.float32)  # scores: col0 1.0, col1 4.0, col2 0.5
+    assert oracle.block_prune(w, 1 / 3).tolist() == [[True, True, False]]
+    assert oracle.block_prune(w, 2 / 3).tolist() == [[False, True, False]]
+    assert oracle.block_prune(w, 0.0).tolist() == [[True, True, True]]
+    assert oracle.block_prune(w, 1.0).tolist() == [[False, False, False]]
+    tie = np.ones((4, 3), np.float32)  # equal scores: lower index pruned first
+    assert oracle.block_prune(tie, 1 / 3).tolist() == [[False, True, True]]
+
+
+def test_block_prune_brute_force():
+    rng = np.random.default_rng(51)
+    for trial in range(20):
+        n, k = 4 * int(rng.integers(1, 5)), int(rng.integers(1, 9))
+        w = rng.normal(size=(n, k)).astype(np.float32)
+        if trial % 3 == 0:
+            w = np.round(w).astype(np.float32)  # many ties
+        s = float(rng.uniform())
+        keep = oracle.block_prune(w, s)
+        total = (n // 4) * k
+        npruned = int(math.floor(s * total + 0.5))
+        assert keep.sum() == total - npruned
+        # brute force: mean |w| of each block, stable order by (score, id)
+        scores = []
+        for r in range(n // 4):
+            for c in range(k):
+                scores.append((float(np.mean(np.abs(w[4 * r:4 * r + 4, c].astype(np.float64)))), r * k + c))
+        pruned = {i for (_, i) in sorted(scores)[:npruned]}
+        for r in range(n // 4):
+            for c in range(k):
+                assert keep[r, c] == ((r * k + c) not in pruned)
