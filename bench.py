@@ -1,0 +1,394 @@
+#!/usr/bin/env python
+"""Benchmark of the block-sparse INT8 linear layer on GB300.
+
+Default workload: the DistilBERT FFN2 linear, 3072 -> 768 at 90% block
+sparsity (4x1 blocks), M = 32 x 128 = 4096 tokens, int8 activations uniform
+in [0, 127], bias + requantise to int8 (scale 0.05).  One step = one pass of
+the layer over the whole batch (one kernel launch).
+
+Metric: effective INT8 TOPS = 2 * M * nnzb * 4 / t (every stored block's
+MACs, padding excluded) and achieved HBM GB/s = algorithmic bytes / t, where
+algorithmic bytes = stored values + column indices + indptr + scales + bias
++ activations + outputs.
+
+Timing: CUDA events on the launching stream around exactly --steps launches
+after --warmup launches (plus an untimed soak of about a second so that the
+clock sampler sees the GPU under this load), barrier + synchronize on both
+sides, max over ranks.  Input/output buffer sets rotate so that the working
+set of consecutive launches exceeds twice the L2 (no launch finds its
+activations in L2).
+
+--impl reference times the CPU oracle (plain C, the layer's definition) on
+the host cores on row samples of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "effective INT8 TOPS & HBM GB/s of block-sparse linear (% of roofline); stack tokens/s"
+UNIT = "TOPS"
+DP4A_LANES_PER_SM_CLK = 64   # int8 dot-4 lanes per SM per clock (half rate on sm_103)
+OPS_PER_DP4A = 8             # 4 multiply-adds
+KERNEL_SOURCES = ("paper_2211_07715_gb300/csrc/bsgemm_kernel.cu", "paper_2211_07715_gb300/csrc/bsgemm_internal.h",
+                  "paper_2211_07715_gb300/csrc/bsgemm_api.cpp")
+
+WORKLOADS = {"ffn2": synth.ffn2, "ffn1": synth.ffn1, "single": synth.single_768}
+
+
+def kernel_sha() -> str:
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def algorithmic_bytes(case) -> int:
+    wt = case.weight
+    out_elem = {synth.I32: 4, synth.F32: 4, synth.F32_GELU: 4, synth.I8: 1, synth.I8_GELU: 1}[case.kind]
+    return (wt.nnzb * 4 + wt.nnzb * 4 + (wt.n_out // 4 + 1) * 4 + wt.n_out * 8
+            + case.m * wt.k_in + case.m * wt.n_out * out_elem)
+
+
+def effective_ops(case, rows: int | None = None) -> float:
+    return 2.0 * (case.m if rows is None else rows) * case.weight.nnzb * 4
+
+
+def profile_traffic(workload: str):
+    """dram bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", f"{workload}_ncu.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    sha = re.search(r"kernel_source_sha256:\s*([0-9a-f]+)", text)
+    val = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
+    if not sha or not val or sha.group(1) != kernel_sha():
+        return None
+    return int(val.group(1))
+
+
+# ------------------------------------------------------------------ clocks --
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons for one GPU."""
+
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = (uuid or "").lower()
+        self.lines: list[str] = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def mark(self) -> int:
+        return len(self.lines)
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=5)
+
+    def summary(self, start: int, end: int) -> dict:
+        rows = []
+        for line in self.lines[start:end]:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            if self.uuid and self.uuid not in parts[0].lower():
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[4:8]))
+            except ValueError:
+                continue
+        if not rows and self.uuid:  # uuid formats differ: fall back to a single listed GPU
+            gpus = {ln.split(",")[0] for ln in self.lines[start:end] if "," in ln}
+            if len(gpus) == 1:
+                self.uuid = ""
+                return self.summary(start, end)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({names[i] for (_, _, flags) in rows for i, f in enumerate(flags) if f.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# -------------------------------------------------------------- our arm --
+
+def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
+    import torch
+    import paper_2211_07715_gb300 as bsg
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    props = torch.cuda.get_device_properties(dev)
+    case = WORKLOADS[args.workload]()
+    if world > 1:  # weak scaling: every rank runs its own batch of the same shape
+        case.x = synth.draw_x(synth.rng_for(case.meta["seed"] + 7919 * rank), case.m, case.weight.k_in,
+                              case.meta["x_dist"])
+    wt = case.weight
+    lin = bsg.SparseInt8Linear(wt.n_out, wt.k_in, wt.indptr, wt.colidx, wt.values, wt.scales, wt.bias)
+    out_dtype = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+                 synth.I8: torch.int8, synth.I8_GELU: torch.int8}[case.kind]
+    out_elem = torch.empty((), dtype=out_dtype).element_size()
+    set_bytes = case.m * wt.k_in + case.m * wt.n_out * out_elem
+    l2 = int(getattr(props, "L2_cache_size", 128 << 20))
+    nsets = max(2, math.ceil(2 * l2 / set_bytes) + 1)
+    x_host = torch.from_numpy(case.x)
+    xs = [x_host.to(dev) for _ in range(nsets)]
+    outs = [torch.empty((case.m, wt.n_out), dtype=out_dtype, device=dev) for _ in range(nsets)]
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i: int):
+        bsg.bsgemm_run(lin._h, xs[i % nsets].data_ptr(), case.m, outs[i % nsets].data_ptr(), case.kind,
+                       case.out_scale, stream.cuda_stream)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize(dev)
+    # probe one launch's duration to size the clock soak (~1 s)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(20):
+        step(i)
+    e1.record(stream)
+    e1.synchronize()
+    per_launch_ms = e0.elapsed_time(e1) / 20
+    soak = int(min(200000, max(0, 1000.0 / max(per_launch_ms, 1e-3))))
+
+    sampler = ClockSampler(str(getattr(props, "uuid", "")) if rank == 0 else None)
+    if rank == 0:
+        sampler.start()
+        time.sleep(0.3)
+    mark0 = sampler.mark()
+    for i in range(soak):
+        step(i)
+    barrier()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(args.steps):
+        step(i)
+    end.record(stream)
+    end.synchronize()
+    barrier()
+    mark1 = sampler.mark()
+    elapsed_ms = start.elapsed_time(end)
+    if rank == 0:
+        time.sleep(0.2)
+        sampler.stop()
+    clocks = sampler.summary(mark0, max(mark1, mark0 + 1)) if rank == 0 else {}
+
+    # end to end through the public call a user makes: a pinned host batch
+    # in, the result back in host memory (copies inside the timed region)
+    e2e_steps = max(3, min(args.steps, 200))
+    hx = [torch.from_numpy(case.x).pin_memory() for _ in range(2)]
+
+    def e2e_step(i: int):
+        lin(hx[i % 2], case.kind, case.out_scale)
+
+    for i in range(3):
+        e2e_step(i)
+    barrier()
+    s2, t2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s2.record(stream)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    t2.record(stream)
+    t2.synchronize()
+    barrier()
+    e2e_ms = s2.elapsed_time(t2)
+
+    # max over ranks
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([elapsed_ms, e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms, e2e_ms = float(t[0]), float(t[1])
+    lin.close()
+    if rank != 0:
+        return None
+
+    ms_per_step = elapsed_ms / args.steps
+    ops = effective_ops(case)
+    tops = world * ops / (ms_per_step * 1e-3) / 1e12
+    tops_rank = ops / (ms_per_step * 1e-3) / 1e12
+    hbm_gbs = algorithmic_bytes(case) / (ms_per_step * 1e-3) / 1e9
+    e2e_tops = world * ops / (e2e_ms / e2e_steps * 1e-3) / 1e12
+    max_mhz = clocks.get("sm_max_mhz") or 2070.0
+    peak = props.multi_processor_count * DP4A_LANES_PER_SM_CLK * OPS_PER_DP4A * max_mhz * 1e6 / 1e12
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except (OSError, ValueError):
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6683.8))
+    traffic = profile_traffic(args.workload)
+
+    result = {
+        "metric": METRIC,
+        "value": round(tops, 3),
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 6),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "s8",
+        "data": "synthetic",
+        "config": {"workload": case.name, "n_out": wt.n_out, "k_in": wt.k_in, "tokens": case.m,
+                   "block": "4x1", "sparsity": case.meta["sparsity"], "nnzb": wt.nnzb,
+                   "epilogue": synth.KIND_NAMES[case.kind], "out_scale": case.out_scale,
+                   "l2": f"rotating {nsets} activation/output sets ({nsets * set_bytes / 2**20:.0f} MiB > 2 x L2)",
+                   "parallelism": f"replicas x{world}", "soak_steps": soak},
+        "hbm_gbs": round(hbm_gbs, 1),
+        "hbm_frac": round(hbm_gbs / hbm_peak, 4),
+        "roofline": {"bound": "alu", "achieved": round(tops_rank, 3), "peak": round(peak, 2), "unit": "TOPS",
+                     "frac": round(tops_rank / peak, 4), "traffic": traffic,
+                     "peak_basis": f"{props.multi_processor_count} SMs x {DP4A_LANES_PER_SM_CLK} dp4a lanes/clk x "
+                                   f"{OPS_PER_DP4A} ops x {max_mhz:.0f} MHz (max SM clock)"},
+        "e2e": {"value": round(e2e_tops, 3), "unit": UNIT, "h2d_bytes_per_step": int(case.m * wt.k_in),
+                "d2h_bytes_per_step": int(case.m * wt.n_out * out_elem)},
+        "gpu_launches": args.steps,
+        "clocks": clocks,
+        "kernel_source_sha256": kernel_sha(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(case, rows=None)
+    return result
+
+
+def cpu_baseline(case, rows: int | None, threads: int | None = None, reps: int = 1) -> dict:
+    import oracle
+    threads = threads or os.cpu_count() or 1
+    w = oracle.weight_dense(case.weight)
+    wt = case.weight
+    sel = None if rows is None else np.arange(rows)
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        oracle.linear(case.x, w, wt.scales, wt.bias, case.kind, case.out_scale, rows=sel, threads=threads)
+    dt = (time.perf_counter() - t0) / reps
+    nrows = case.m if rows is None else rows
+    return {"value": round(effective_ops(case, nrows) / dt / 1e12, 6), "unit": UNIT, "cores": threads,
+            "kind": "oracle", "sample": f"{nrows} of {case.m} tokens, dense triple loop over the decompressed "
+                                        f"weight, {threads} host threads, {dt:.2f} s per pass"}
+
+
+# -------------------------------------------------------- reference arm --
+
+def run_reference(args, rank: int) -> dict | None:
+    if rank != 0:
+        return None
+    case = WORKLOADS[args.workload]()
+    threads = os.cpu_count() or 1
+    rows = min(case.m, args.ref_rows)
+    import oracle
+    w = oracle.weight_dense(case.weight)
+    wt = case.weight
+
+    def one(i: int):
+        start = (i * rows) % case.m
+        sel = (np.arange(rows) + start) % case.m
+        oracle.linear(case.x, w, wt.scales, wt.bias, case.kind, case.out_scale, rows=sel, threads=threads)
+
+    for i in range(args.warmup):
+        one(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        one(i)
+    dt = (time.perf_counter() - t0) / args.steps
+    value = effective_ops(case, rows) / dt / 1e12
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": UNIT, "n_gpus": 0,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "s8", "data": "synthetic",
+        "config": {"workload": case.name, "n_out": wt.n_out, "k_in": wt.k_in, "tokens": case.m,
+                   "block": "4x1", "sparsity": case.meta["sparsity"], "epilogue": synth.KIND_NAMES[case.kind]},
+        "cpu_baseline": {"value": round(value, 6), "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"{rows} of {case.m} tokens per step, {threads} host threads"},
+        "e2e": {"value": round(value, 6), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=2000)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    p.add_argument("--workload", choices=sorted(WORKLOADS), default="ffn2")
+    p.add_argument("--ref-rows", type=int, default=512, help="tokens per reference step")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    args = p.parse_args()
+    if args.warmup < 3:
+        p.error("--warmup must be >= 3")
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        res = run_reference(args, rank)
+    else:
+        if world > 1:
+            import torch
+            import torch.distributed as dist
+            torch.cuda.set_device(local_rank)
+            dist.init_process_group("nccl")
+        res = run_ours(args, rank, world, local_rank)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+    if res is not None:
+        print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

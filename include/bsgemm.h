@@ -1,0 +1,146 @@
+/*
+ * bsgemm.h -- C ABI of the block-sparse INT8 linear layer on one GB300
+ * (sm_103a): the hot path of the inference engine of "Fast DistilBERT on
+ * CPUs" (arXiv 2211.07715), re-designed for the GPU.
+ *
+ * The layer computes, for int8 activations X [M][K] and an int8 weight
+ * W [N][K] that is sparse in blocks of 4 consecutive output rows x 1 input
+ * column (App. A.1; "constant block size 4", App. A.3.4):
+ *
+ *   acc[m][n] = sum_k X[m][k] * W[n][k]                  exact int32
+ *                 (Sec. 3 "Sparse GEMM operators", Algorithm 1's dot-4)
+ *   y[m][n]   = fmaf((float)acc[m][n], scales[n], bias[n])
+ *   out       = acc | y | GELU(y) | q(y) | q(GELU(y))
+ *                 (the fused post-operators of App. A.3.3 / Algorithm 1's
+ *                  "downconvert and post-operator fusion")
+ *
+ * with q(v) = saturate_s8(round_half_even(v * (1.0f / out_scale))) and
+ * GELU the erf form 0.5 y (1 + erf(y / sqrt 2)) evaluated in fp32 by the
+ * Abramowitz & Stegun 7.1.28 rational approximation of erf (|error| <=
+ * 3e-7), by one fixed IEEE op sequence so that int8 results are
+ * reproducible bit for bit.
+ *
+ * Threading: every function may be called from any host thread.  A handle
+ * is immutable after bsgemm_create, so one handle (one copy of the weights
+ * in device memory) may serve concurrent bsgemm_run calls on several
+ * streams -- the GPU form of the paper's weight sharing across parallel
+ * instances (App. A.3.2).
+ *
+ * Errors: functions returning int give 0 on success or a negative
+ * BSGEMM_ERR_* code; bsgemm_create returns NULL on failure.  In both cases
+ * bsgemm_last_error() describes the last failure on the calling thread.
+ */
+#ifndef BSGEMM_H_
+#define BSGEMM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BSGEMM_BLOCK 4 /* output rows per block (App. A.1) */
+
+/* Return codes. */
+#define BSGEMM_OK 0
+#define BSGEMM_ERR_INVALID (-1)     /* a pointer, size or value is not allowed */
+#define BSGEMM_ERR_UNSUPPORTED (-2) /* valid, but outside what this build runs */
+#define BSGEMM_ERR_CUDA (-3)        /* a CUDA call failed (message has details) */
+
+/* Epilogue kinds: what bsgemm_run writes to `out` (App. A.3.3 post-ops). */
+typedef enum {
+    BSGEMM_OUT_I32 = 0,      /* int32 acc                               */
+    BSGEMM_OUT_F32 = 1,      /* float y = fmaf((float)acc, s[n], b[n])   */
+    BSGEMM_OUT_F32_GELU = 2, /* float GELU(y)                           */
+    BSGEMM_OUT_I8 = 3,       /* int8  q(y)                              */
+    BSGEMM_OUT_I8_GELU = 4   /* int8  q(GELU(y))                        */
+} bsgemm_out_kind;
+
+typedef struct {
+    int32_t kind;    /* a bsgemm_out_kind                                    */
+    float out_scale; /* int8 kinds only: finite and > 0; the library         */
+                     /* multiplies by 1.0f / out_scale (one fp32 division)   */
+} bsgemm_epilogue;
+
+typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
+
+/*
+ * bsgemm_create -- build the device form of a block-compressed weight.
+ *
+ * Block-compressed layout (App. A.1 blocks; App. A.3.4 "the sparse weight is
+ * compressed and the mask is used"), all HOST memory, read during the call
+ * only (the caller keeps ownership and may free them on return):
+ *   N        output features, a multiple of 4 (App. A.3.4: other N would
+ *            need padding, which the paper leaves out; so does this build:
+ *            N % 4 != 0 returns NULL with BSGEMM_ERR_UNSUPPORTED).
+ *   K        input features, 1 <= K <= bsgemm_max_k().
+ *   block    must be 4.
+ *   indices  int32: indptr[N/4 + 1] followed by colidx[nnzb], nnzb =
+ *            indptr[N/4].  Block j of block-row r (indptr[r] <= j <
+ *            indptr[r+1]) lies in column colidx[j]; columns strictly
+ *            increase within a block-row; indptr[0] = 0.
+ *   values   int8 [nnzb][4]: values[j][i] = W[4r + i][colidx[j]].  A stored
+ *            block may hold zeros; any int8 value is allowed.
+ *   scales   float [N]: per-output-channel dequantisation scale (the product
+ *            of the activation and weight scales); must be finite.
+ *   bias     float [N], or NULL for zeros; must be finite.
+ * The call allocates device memory on the CURRENT CUDA device, copies the
+ * repacked weights there and synchronises.  Returns NULL on failure.
+ */
+bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const int8_t* values,
+                       const float* scales, const float* bias);
+
+/*
+ * bsgemm_run -- out = epilogue(X * W^T) on `stream`.
+ *   act     DEVICE pointer, int8 [M][K] row-major (row stride K bytes).
+ *   M       tokens, M >= 0; M = 0 is a no-op returning BSGEMM_OK.
+ *   out     DEVICE pointer, [M][N] row-major of int32 / float / int8 by
+ *           epi.kind; 16-byte aligned; must not overlap act.
+ *   epi     epilogue kind and, for int8 kinds, the output scale.
+ *   stream  a cudaStream_t (NULL = the legacy default stream).
+ * Asynchronous: returns after enqueueing one kernel launch; allocates
+ * nothing, does not synchronise and keeps no reference to act or out.  The
+ * current device must be the one the handle was created on.
+ * Returns BSGEMM_OK, BSGEMM_ERR_INVALID (NULL handle or pointers, M < 0,
+ * bad kind, bad out_scale, misaligned out, wrong device) or
+ * BSGEMM_ERR_CUDA (launch failure).
+ */
+int bsgemm_run(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream);
+
+/*
+ * bsgemm_destroy -- free the handle and its device memory.  The caller must
+ * make sure no bsgemm_run on this handle is still executing (cudaFree
+ * itself waits for the device).  NULL is ignored.
+ */
+void bsgemm_destroy(bsgemm_t h);
+
+/* Message for the last failure on the calling thread ("" if none).  The
+ * string stays valid until the next bsgemm_* call on this thread. */
+const char* bsgemm_last_error(void);
+
+/* Code (BSGEMM_OK or BSGEMM_ERR_*) of the last bsgemm_* call on the calling
+ * thread; tells why bsgemm_create returned NULL. */
+int bsgemm_last_status(void);
+
+/* Largest K bsgemm_create accepts in this build (bounded by the shared
+ * memory that holds one token tile of activations for all of K). */
+int bsgemm_max_k(void);
+
+/*
+ * bsgemm_info -- describe a handle, for benchmarks and tests.  Fills up to
+ * `n` entries of `out` with: [0] N, [1] K, [2] nnzb (stored blocks),
+ * [3] padded quads (groups of 4 stored blocks of one block-row, the unit of
+ * the inner loop; the last quad of a block-row is padded with zero-weight
+ * entries), [4] token-tile height of the kernel, [5] CTAs of a launch once
+ * M is large enough to fill the GPU (SMs x resident CTAs per SM), [6] device
+ * bytes held by the handle.  Returns the number of entries
+ * available (7), or BSGEMM_ERR_INVALID.
+ */
+int bsgemm_info(bsgemm_t h, int64_t* out, int n);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BSGEMM_H_ */

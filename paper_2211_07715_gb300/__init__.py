@@ -1,0 +1,193 @@
+"""Block-sparse INT8 linear layer on GB300 -- Python binding of libbsgemm.so.
+
+The layer is the hot path of the inference engine of "Fast DistilBERT on
+CPUs" (arXiv 2211.07715): int8 activations times an int8 weight that is
+sparse in blocks of 4 output rows x 1 input column, exact int32
+accumulation, and a fused dequantise + bias (+ GELU) (+ requantise)
+epilogue.  All arithmetic runs in the CUDA kernels of libbsgemm.so; this
+module only marshals arguments (PyTorch provides device memory and
+streams).  There is no CPU fallback: importing fails loudly if the library
+has not been built (``python -m paper_2211_07715_gb300.build`` or
+``__graft_entry__.build()``).
+
+The functions below carry the C names (``bsgemm_create``, ``bsgemm_run``,
+...); :class:`SparseInt8Linear` wraps one handle.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libbsgemm.so")
+
+BLOCK = 4
+OUT_I32, OUT_F32, OUT_F32_GELU, OUT_I8, OUT_I8_GELU = 0, 1, 2, 3, 4
+ERR_INVALID, ERR_UNSUPPORTED, ERR_CUDA = -1, -2, -3
+
+
+class BsgemmError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"bsgemm error {code}: {msg}")
+        self.code = code
+
+
+class Epilogue(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("out_scale", ctypes.c_float)]
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2211_07715_gb300.build`")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp = ctypes.c_void_p
+    lib.bsgemm_create.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]
+    lib.bsgemm_create.restype = vp
+    lib.bsgemm_run.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp]
+    lib.bsgemm_run.restype = ctypes.c_int
+    lib.bsgemm_destroy.argtypes = [vp]
+    lib.bsgemm_destroy.restype = None
+    lib.bsgemm_last_error.argtypes = []
+    lib.bsgemm_last_error.restype = ctypes.c_char_p
+    lib.bsgemm_last_status.argtypes = []
+    lib.bsgemm_last_status.restype = ctypes.c_int
+    lib.bsgemm_max_k.argtypes = []
+    lib.bsgemm_max_k.restype = ctypes.c_int
+    lib.bsgemm_info.argtypes = [vp, ctypes.POINTER(ctypes.c_int64), ctypes.c_int]
+    lib.bsgemm_info.restype = ctypes.c_int
+    return lib
+
+
+_lib = _load()
+
+EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
+            "bsgemm_max_k", "bsgemm_info")
+
+
+def bsgemm_last_error() -> str:
+    return _lib.bsgemm_last_error().decode()
+
+
+def bsgemm_last_status() -> int:
+    return int(_lib.bsgemm_last_status())
+
+
+def bsgemm_max_k() -> int:
+    return int(_lib.bsgemm_max_k())
+
+
+def _host_array(a, dtype) -> np.ndarray:
+    if hasattr(a, "detach"):  # a torch tensor
+        a = a.detach().cpu().numpy()
+    return np.ascontiguousarray(np.asarray(a), dtype=dtype)
+
+
+def bsgemm_create(n_out: int, k_in: int, block: int, indices, values, scales, bias=None) -> int:
+    """Create a handle from host arrays (see include/bsgemm.h); raises on failure."""
+    indices = _host_array(indices, np.int32)
+    values = _host_array(values, np.int8)
+    scales = _host_array(scales, np.float32)
+    bias = None if bias is None else _host_array(bias, np.float32)
+    h = _lib.bsgemm_create(int(n_out), int(k_in), int(block), indices.ctypes.data, values.ctypes.data,
+                           scales.ctypes.data, None if bias is None else bias.ctypes.data)
+    if not h:
+        raise BsgemmError(bsgemm_last_status(), bsgemm_last_error())
+    return h
+
+
+def bsgemm_run(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float = 1.0,
+               stream: int = 0) -> None:
+    """Enqueue one run on `stream` (raw device pointers); raises on failure."""
+    rc = _lib.bsgemm_run(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_destroy(h: int) -> None:
+    _lib.bsgemm_destroy(h)
+
+
+def bsgemm_info(h: int) -> dict:
+    buf = (ctypes.c_int64 * 7)()
+    rc = _lib.bsgemm_info(h, buf, 7)
+    if rc < 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+    keys = ("n_out", "k_in", "nnzb", "quads", "tile_m", "ctas", "device_bytes")
+    return dict(zip(keys, (int(v) for v in buf)))
+
+
+_OUT_DTYPES = {OUT_I32: "int32", OUT_F32: "float32", OUT_F32_GELU: "float32", OUT_I8: "int8", OUT_I8_GELU: "int8"}
+
+
+def dense_to_blocks(w: np.ndarray):
+    """Block-compress a dense int8 weight [N][K], keeping every 4x1 block that
+    holds a nonzero value.  Returns (indptr, colidx, values)."""
+    w = _host_array(w, np.int8)
+    n_out, k_in = w.shape
+    if n_out % BLOCK:
+        raise ValueError("N must be a multiple of 4")
+    blocks = w.reshape(n_out // BLOCK, BLOCK, k_in)          # [r][i][k]
+    keep = (blocks != 0).any(axis=1)                          # [r][k]
+    r_idx, k_idx = np.nonzero(keep)                           # row-major: sorted by r, then k
+    indptr = np.zeros(n_out // BLOCK + 1, np.int32)
+    np.cumsum(keep.sum(axis=1), out=indptr[1:])
+    values = np.ascontiguousarray(blocks[r_idx, :, k_idx], dtype=np.int8)  # [nnzb][4]
+    return indptr, k_idx.astype(np.int32), values
+
+
+class SparseInt8Linear:
+    """One block-sparse int8 linear layer resident on the current CUDA device."""
+
+    def __init__(self, n_out: int, k_in: int, indptr, colidx, values, scales, bias=None):
+        indices = np.concatenate([_host_array(indptr, np.int32), _host_array(colidx, np.int32)])
+        self.n_out, self.k_in = int(n_out), int(k_in)
+        self._h = bsgemm_create(n_out, k_in, BLOCK, indices, values, scales, bias)
+        self.info = bsgemm_info(self._h)
+
+    @classmethod
+    def from_dense(cls, w, scales, bias=None) -> "SparseInt8Linear":
+        w = _host_array(w, np.int8)
+        indptr, colidx, values = dense_to_blocks(w)
+        return cls(w.shape[0], w.shape[1], indptr, colidx, values, scales, bias)
+
+    def run(self, x, out, kind: int, out_scale: float = 1.0, stream=None) -> None:
+        """out[M][N] = epilogue(x[M][K] W^T); both CUDA tensors, contiguous."""
+        import torch
+        if x.dtype != torch.int8 or not x.is_cuda or not x.is_contiguous() or x.dim() != 2 or x.shape[1] != self.k_in:
+            raise ValueError("x must be a contiguous CUDA int8 tensor [M][K]")
+        if (not out.is_cuda or not out.is_contiguous() or tuple(out.shape) != (x.shape[0], self.n_out)
+                or str(out.dtype).split(".")[-1] != _OUT_DTYPES[kind]):
+            raise ValueError(f"out must be a contiguous CUDA {_OUT_DTYPES[kind]} tensor [M][N]")
+        s = torch.cuda.current_stream() if stream is None else stream
+        bsgemm_run(self._h, x.data_ptr(), x.shape[0], out.data_ptr(), kind, out_scale, s.cuda_stream)
+
+    def __call__(self, x, kind: int, out_scale: float = 1.0, stream=None):
+        """Allocate the output and run.  A CPU `x` is copied in and the result
+        copied back (the end-to-end path); a CUDA `x` stays on the device."""
+        import torch
+        dtype = getattr(torch, _OUT_DTYPES[kind])
+        if x.is_cuda:
+            out = torch.empty((x.shape[0], self.n_out), dtype=dtype, device=x.device)
+            self.run(x, out, kind, out_scale, stream)
+            return out
+        pinned = x.is_pinned()
+        xd = x.to("cuda", non_blocking=pinned)
+        out = torch.empty((x.shape[0], self.n_out), dtype=dtype, device=xd.device)
+        self.run(xd, out, kind, out_scale, stream)
+        host = torch.empty(out.shape, dtype=dtype, pin_memory=pinned)
+        host.copy_(out, non_blocking=pinned)
+        (torch.cuda.current_stream() if stream is None else stream).synchronize()
+        return host
+
+    def close(self) -> None:
+        if getattr(self, "_h", None):
+            bsgemm_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,280 @@
+// Host side of the C ABI declared in include/bsgemm.h: argument checks, the
+// create-time repack of the block-compressed weight into quads (groups of 4
+// stored blocks of one block-row, the dot-4 unit of Algorithm 1), device
+// upload, and the launch of the kernel in bsgemm_kernel.cu.
+#include "bsgemm.h"
+
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "bsgemm_internal.h"
+
+struct bsgemm_ctx {
+    int device = -1;
+    int num_sms = 0;
+    int ctas_per_sm = 0;
+    int MT = 0;
+    int64_t nnzb = 0;
+    void* arena = nullptr;
+    size_t arena_bytes = 0;
+    bsg::DeviceWeights w{};
+};
+
+namespace {
+
+thread_local std::string g_error;
+thread_local int g_status = BSGEMM_OK;
+
+int fail(int code, const std::string& msg) {
+    g_error = msg;
+    g_status = code;
+    return code;
+}
+
+void clear_error() {
+    g_error.clear();
+    g_status = BSGEMM_OK;
+}
+
+std::string cuda_msg(const char* what, cudaError_t e) {
+    return std::string(what) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+}
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Check the block-compressed arrays; returns an empty string if valid.
+std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx) {
+    const int nbr = N / BSGEMM_BLOCK;
+    if (indptr[0] != 0) return "indptr[0] must be 0";
+    for (int r = 0; r < nbr; ++r) {
+        if (indptr[r + 1] < indptr[r]) return "indptr must be non-decreasing (block-row " + std::to_string(r) + ")";
+        for (int j = indptr[r]; j < indptr[r + 1]; ++j) {
+            const int k = colidx[j];
+            if (k < 0 || k >= K)
+                return "colidx[" + std::to_string(j) + "] = " + std::to_string(k) + " is outside [0, K)";
+            if (j > indptr[r] && colidx[j - 1] >= k)
+                return "columns must strictly increase within block-row " + std::to_string(r);
+        }
+    }
+    return "";
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* bsgemm_last_error(void) { return g_error.c_str(); }
+
+int bsgemm_last_status(void) { return g_status; }
+
+int bsgemm_max_k(void) { return bsg::max_k(); }
+
+bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const int8_t* values, const float* scales,
+                       const float* bias) {
+    clear_error();
+    if (block != BSGEMM_BLOCK) {
+        fail(BSGEMM_ERR_UNSUPPORTED, "block must be 4 (4 output rows x 1 input column)");
+        return nullptr;
+    }
+    if (N < BSGEMM_BLOCK || K < 1) {
+        fail(BSGEMM_ERR_INVALID, "need N >= 4 and K >= 1");
+        return nullptr;
+    }
+    if (N % BSGEMM_BLOCK != 0) {
+        fail(BSGEMM_ERR_UNSUPPORTED, "N must be a multiple of 4 (padding is not implemented)");
+        return nullptr;
+    }
+    if (K > bsg::max_k()) {
+        fail(BSGEMM_ERR_UNSUPPORTED, "K = " + std::to_string(K) + " exceeds bsgemm_max_k() = " +
+                                         std::to_string(bsg::max_k()));
+        return nullptr;
+    }
+    if (!indices || !scales) {
+        fail(BSGEMM_ERR_INVALID, "indices and scales must not be NULL");
+        return nullptr;
+    }
+    const int nbr = N / BSGEMM_BLOCK;
+    const int32_t* indptr = indices;
+    const int64_t nnzb = indptr[nbr];
+    if (indptr[0] != 0 || nnzb < 0 || nnzb > static_cast<int64_t>(nbr) * K) {
+        fail(BSGEMM_ERR_INVALID, "indptr[0] must be 0 and 0 <= indptr[N/4] <= (N/4) * K");
+        return nullptr;
+    }
+    if (nnzb > 0 && !values) {
+        fail(BSGEMM_ERR_INVALID, "values must not be NULL when blocks are stored");
+        return nullptr;
+    }
+    const int32_t* colidx = indices + nbr + 1;
+    std::string bad = check_bsr(N, K, indptr, colidx);
+    if (!bad.empty()) {
+        fail(BSGEMM_ERR_INVALID, bad);
+        return nullptr;
+    }
+    for (int n = 0; n < N; ++n) {
+        if (!std::isfinite(scales[n]) || (bias && !std::isfinite(bias[n]))) {
+            fail(BSGEMM_ERR_INVALID, "scales and bias must be finite (channel " + std::to_string(n) + ")");
+            return nullptr;
+        }
+    }
+
+    // Repack into quads: per block-row, stored blocks in groups of 4; the
+    // last group is padded by repeating the row's last column with zero
+    // weights.  Record q = {k0, k1, k2, k3} then 4 words, word c holding the
+    // bytes W[4r + c][k0..k3].
+    std::vector<int32_t> qptr(nbr + 1, 0), cost(nbr + 1, 0);
+    for (int r = 0; r < nbr; ++r) {
+        const int nz = indptr[r + 1] - indptr[r];
+        qptr[r + 1] = qptr[r] + (nz + 3) / 4;
+        cost[r + 1] = qptr[r + 1] + (r + 1);
+    }
+    const int Q = qptr[nbr];
+    std::vector<int32_t> quads(static_cast<size_t>(Q + 1) * 8, 0);  // + 1 padding record
+    for (int r = 0; r < nbr; ++r) {
+        const int j0 = indptr[r], j1 = indptr[r + 1];
+        for (int q = qptr[r]; q < qptr[r + 1]; ++q) {
+            int32_t* rec = &quads[static_cast<size_t>(q) * 8];
+            uint32_t wwords[4] = {0, 0, 0, 0};
+            for (int e = 0; e < 4; ++e) {
+                const int j = j0 + 4 * (q - qptr[r]) + e;
+                if (j < j1) {
+                    rec[e] = colidx[j];
+                    for (int c = 0; c < 4; ++c)
+                        wwords[c] |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(j) * 4 + c]))
+                                     << (8 * e);
+                } else {
+                    rec[e] = colidx[j1 - 1];  // padding: a valid column, zero weight
+                }
+            }
+            for (int c = 0; c < 4; ++c) rec[4 + c] = static_cast<int32_t>(wwords[c]);
+        }
+    }
+    std::vector<float> bias_v(N, 0.0f);
+    if (bias) std::memcpy(bias_v.data(), bias, sizeof(float) * N);
+
+    auto* h = new bsgemm_ctx();
+    cudaError_t e = cudaGetDevice(&h->device);
+    if (e != cudaSuccess) {
+        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
+        delete h;
+        return nullptr;
+    }
+    int optin = 0;
+    e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
+    if (e != cudaSuccess) {
+        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaDeviceGetAttribute", e));
+        delete h;
+        return nullptr;
+    }
+    h->MT = bsg::tile_for_k(K);
+    if (bsg::smem_bytes(h->MT, K) + 16 > static_cast<size_t>(optin)) {
+        fail(BSGEMM_ERR_UNSUPPORTED, "this device has too little shared memory per block for K = " + std::to_string(K));
+        delete h;
+        return nullptr;
+    }
+    e = bsg::prepare_kernels(h->MT, K, &h->ctas_per_sm);
+    if (e != cudaSuccess || h->ctas_per_sm < 1) {
+        fail(BSGEMM_ERR_CUDA, e != cudaSuccess ? cuda_msg("kernel setup", e) : "kernel cannot be resident on an SM");
+        delete h;
+        return nullptr;
+    }
+
+    const size_t off_qptr = 0;
+    const size_t off_cost = align_up(off_qptr + sizeof(int32_t) * (nbr + 1), 256);
+    const size_t off_quads = align_up(off_cost + sizeof(int32_t) * (nbr + 1), 256);
+    const size_t off_scale = align_up(off_quads + sizeof(int32_t) * quads.size(), 256);
+    const size_t off_bias = align_up(off_scale + sizeof(float) * N, 256);
+    h->arena_bytes = align_up(off_bias + sizeof(float) * N, 256);
+    e = cudaMalloc(&h->arena, h->arena_bytes);
+    if (e != cudaSuccess) {
+        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaMalloc", e));
+        delete h;
+        return nullptr;
+    }
+    char* base = static_cast<char*>(h->arena);
+    struct Piece { size_t off; const void* src; size_t bytes; } pieces[] = {
+        {off_qptr, qptr.data(), sizeof(int32_t) * qptr.size()},
+        {off_cost, cost.data(), sizeof(int32_t) * cost.size()},
+        {off_quads, quads.data(), sizeof(int32_t) * quads.size()},
+        {off_scale, scales, sizeof(float) * N},
+        {off_bias, bias_v.data(), sizeof(float) * N},
+    };
+    for (const Piece& p : pieces) {
+        e = cudaMemcpy(base + p.off, p.src, p.bytes, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) {
+            fail(BSGEMM_ERR_CUDA, cuda_msg("cudaMemcpy", e));
+            cudaFree(h->arena);
+            delete h;
+            return nullptr;
+        }
+    }
+    h->nnzb = nnzb;
+    h->w.qptr = reinterpret_cast<const int32_t*>(base + off_qptr);
+    h->w.cost = reinterpret_cast<const int32_t*>(base + off_cost);
+    h->w.quads = reinterpret_cast<const int4*>(base + off_quads);
+    h->w.scale = reinterpret_cast<const float*>(base + off_scale);
+    h->w.bias = reinterpret_cast<const float*>(base + off_bias);
+    h->w.N = N;
+    h->w.K = K;
+    h->w.nbr = nbr;
+    h->w.Q = Q;
+    return h;
+}
+
+int bsgemm_run(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream) {
+    clear_error();
+    if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
+    if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
+    if (epi.kind < BSGEMM_OUT_I32 || epi.kind > BSGEMM_OUT_I8_GELU)
+        return fail(BSGEMM_ERR_INVALID, "unknown epilogue kind " + std::to_string(epi.kind));
+    float inv = 0.0f;
+    if (epi.kind == BSGEMM_OUT_I8 || epi.kind == BSGEMM_OUT_I8_GELU) {
+        if (!(epi.out_scale > 0.0f) || !std::isfinite(epi.out_scale))
+            return fail(BSGEMM_ERR_INVALID, "out_scale must be finite and > 0 for int8 outputs");
+        inv = 1.0f / epi.out_scale;
+        if (!std::isfinite(inv)) return fail(BSGEMM_ERR_INVALID, "1 / out_scale overflows fp32");
+    }
+    if (M == 0) return BSGEMM_OK;
+    if (!act || !out) return fail(BSGEMM_ERR_INVALID, "act and out must not be NULL");
+    if (reinterpret_cast<uintptr_t>(out) % 16 != 0) return fail(BSGEMM_ERR_INVALID, "out must be 16-byte aligned");
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
+    if (dev != h->device)
+        return fail(BSGEMM_ERR_INVALID, "current device " + std::to_string(dev) + " is not the handle's device " +
+                                            std::to_string(h->device));
+
+    bsg::LaunchArgs a{};
+    a.x = act;
+    a.out = out;
+    a.M = M;
+    a.kind = epi.kind;
+    a.inv_out_scale = inv;
+    a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
+    const long long ntiles = (static_cast<long long>(M) + h->MT - 1) / h->MT;
+    const long long units = ntiles * h->w.nbr;
+    const long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
+    const int grid = static_cast<int>(units < cap ? units : cap);
+    e = bsg::launch(h->w, a, h->MT, grid, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("kernel launch", e));
+    return BSGEMM_OK;
+}
+
+void bsgemm_destroy(bsgemm_t h) {
+    if (!h) return;
+    if (h->arena) cudaFree(h->arena);
+    delete h;
+}
+
+int bsgemm_info(bsgemm_t h, int64_t* out, int n) {
+    clear_error();
+    if (!h || (!out && n > 0)) return fail(BSGEMM_ERR_INVALID, "NULL handle or output");
+    const int64_t v[7] = {h->w.N, h->w.K, h->nnzb, h->w.Q, h->MT,
+                          static_cast<int64_t>(h->num_sms) * h->ctas_per_sm, static_cast<int64_t>(h->arena_bytes)};
+    for (int i = 0; i < n && i < 7; ++i) out[i] = v[i];
+    return 7;
+}
+
+}  // extern "C"

@@ -1,0 +1,88 @@
+"""The C-ABI library builds, loads, exports every symbol include/bsgemm.h
+declares, and rejects bad arguments before touching a GPU.  CPU only."""
+import ctypes
+import os
+import re
+import shutil
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "bsgemm.h")
+
+
+@pytest.fixture(scope="module")
+def bsg():
+    if not shutil.which("nvcc") and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("nvcc not available")
+    from paper_2211_07715_gb300 import build
+    build.build()
+    import paper_2211_07715_gb300
+    return paper_2211_07715_gb300
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(bsgemm_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("bsgemm_create", "bsgemm_run", "bsgemm_destroy", "bsgemm_last_error"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(bsg):
+    lib = ctypes.CDLL(bsg.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(declared_functions()) == set(bsg.EXPORTED)
+
+
+def test_max_k(bsg):
+    k = bsg.bsgemm_max_k()
+    assert 3072 <= k < 131072  # covers the DistilBERT FFN2 (K = 3072)
+
+
+def _create(bsg, *args):
+    with pytest.raises(bsg.BsgemmError) as e:
+        bsg.bsgemm_create(*args)
+    return e.value.code
+
+
+def test_create_rejects_bad_arrays(bsg):
+    ones = [1.0] * 8
+    assert _create(bsg, 6, 8, 4, [0, 0], [], [1.0] * 6) == bsg.ERR_UNSUPPORTED       # N % 4
+    assert _create(bsg, 8, 8, 2, [0, 0, 0], [], ones) == bsg.ERR_UNSUPPORTED         # block != 4
+    assert _create(bsg, 8, 10**6, 4, [0, 0, 0], [], ones) == bsg.ERR_UNSUPPORTED     # K too large
+    assert _create(bsg, 8, 8, 4, [1, 1, 1], [], ones) == bsg.ERR_INVALID             # indptr[0] != 0
+    assert _create(bsg, 8, 8, 4, [0, 2, 1, 9, 3], [[1] * 4] * 2, ones) == bsg.ERR_INVALID  # decreasing
+    assert _create(bsg, 8, 8, 4, [0, 1, 1, 8], [[1] * 4], ones) == bsg.ERR_INVALID   # column = K
+    assert _create(bsg, 8, 8, 4, [0, 2, 2, 3, 3], [[1] * 4] * 2, ones) == bsg.ERR_INVALID  # repeated column
+    assert _create(bsg, 8, 8, 4, [0, 2, 2, 5, 3], [[1] * 4] * 2, ones) == bsg.ERR_INVALID  # unsorted
+    assert _create(bsg, 8, 8, 4, [0, 0, 0], [], [1.0] * 7 + [np.inf]) == bsg.ERR_INVALID  # scale inf
+    assert _create(bsg, 4, 8, 4, [0, 0], [], [1.0] * 4, [0, 0, np.nan, 0]) == bsg.ERR_INVALID  # bias nan
+    assert _create(bsg, 0, 8, 4, [0], [], []) == bsg.ERR_INVALID
+
+
+def test_run_rejects_bad_arguments_without_a_gpu(bsg):
+    # a NULL handle is rejected before any CUDA call
+    with pytest.raises(bsg.BsgemmError) as e:
+        bsg.bsgemm_run(None, 0, 1, 0, bsg.OUT_I32)
+    assert e.value.code == bsg.ERR_INVALID
+    assert "handle" in bsg.bsgemm_last_error()
+
+
+def test_dense_to_blocks(bsg):
+    rng = np.random.default_rng(3)
+    w = rng.integers(-3, 4, size=(12, 7)).astype(np.int8)
+    w[rng.random(w.shape) < 0.6] = 0
+    indptr, colidx, values = bsg.dense_to_blocks(w)
+    back = np.zeros_like(w)
+    for r in range(3):
+        for j in range(indptr[r], indptr[r + 1]):
+            back[4 * r:4 * r + 4, colidx[j]] = values[j]
+    assert np.array_equal(back, w)
+    assert all((values[j] != 0).any() for j in range(len(colidx)))

@@ -1,0 +1,295 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle.
+
+Integer outputs (int32 accumulators, requantised int8) must match bit for
+bit; fp32 outputs within |d| <= 1e-4 or |d| <= 1e-5 |oracle| per element,
+where the oracle gives the exact value in fp64.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+KINDS = (synth.I32, synth.F32, synth.F32_GELU, synth.I8, synth.I8_GELU)
+
+
+@pytest.fixture(scope="module")
+def bsg():
+    import paper_2211_07715_gb300
+    return paper_2211_07715_gb300
+
+
+def check(got: np.ndarray, want: np.ndarray, kind: int, what: str = ""):
+    assert got.shape == want.shape, what
+    if kind in (synth.F32, synth.F32_GELU):
+        err = np.abs(got.astype(np.float64) - want)
+        bad = ~((err <= 1e-4) | (err <= 1e-5 * np.abs(want)))
+        assert not bad.any(), (f"{what}: {bad.sum()} fp32 elements out of tolerance, max abs err "
+                               f"{err.max():.3g}, first at {np.argwhere(bad)[0].tolist()}")
+    else:
+        diff = got != want
+        assert not diff.any(), f"{what}: {diff.sum()} elements differ, first at {np.argwhere(diff)[0].tolist()}"
+
+
+def make_linear(bsg, wt):
+    return bsg.SparseInt8Linear(wt.n_out, wt.k_in, wt.indptr, wt.colidx, wt.values, wt.scales, wt.bias)
+
+
+def gpu_run(lin, x: np.ndarray, kind: int, out_scale: float) -> np.ndarray:
+    out = lin(torch.from_numpy(x).cuda(), kind, out_scale)
+    torch.cuda.synchronize()
+    return out.cpu().numpy()
+
+
+# -------------------------------------------------- small, every element --
+
+SMALL = [  # (n_out, k_in, m, sparsity, x_dist)
+    (768, 768, 300, 0.90, "u127"),    # 128-token tiles, 3 tiles + ragged tail
+    (256, 768, 129, 0.80, "n30"),
+    (64, 3072, 200, 0.90, "u0_127"),  # 64-token tiles (K > 1536)
+    (3072, 96, 70, 0.70, "u127"),
+]
+
+
+@pytest.mark.parametrize("shape", SMALL, ids=lambda s: "x".join(map(str, s[:3])))
+@pytest.mark.parametrize("kind", KINDS, ids=lambda k: synth.KIND_NAMES[k])
+def test_small_all_elements(bsg, shape, kind):
+    n, k, m, sp, dist = shape
+    rng = synth.rng_for(1000 + n + k + m)
+    wt = synth.draw_weight(rng, n, k, sp)
+    x = synth.draw_x(rng, m, k, dist)
+    lin = make_linear(bsg, wt)
+    got = gpu_run(lin, x, kind, 0.05)
+    want = oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
+    check(got, want, kind, f"{shape}")
+
+
+@pytest.mark.parametrize("m", [1, 3, 63, 64, 65, 127, 128, 129, 257])
+def test_token_counts_span_tiles(bsg, m):
+    for k in (768, 3072):
+        rng = synth.rng_for(2000 + m + k)
+        wt = synth.draw_weight(rng, 32, k, 0.85)
+        x = synth.draw_x(rng, m, k, "u127")
+        lin = make_linear(bsg, wt)
+        want = oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I32)
+        check(gpu_run(lin, x, synth.I32, 1.0), want, synth.I32, f"m={m} k={k}")
+
+
+@pytest.mark.parametrize("k", [1, 3, 5, 17, 37, 100, 1001, 1536, 1537, 2049])
+def test_ragged_k(bsg, k):
+    """K not a multiple of 4/16/32 takes the byte-wise staging path."""
+    rng = synth.rng_for(3000 + k)
+    wt = synth.draw_weight(rng, 48, k, 0.5)
+    x = synth.draw_x(rng, 77, k, "u127")
+    lin = make_linear(bsg, wt)
+    w = oracle.weight_dense(wt)
+    for kind in (synth.I32, synth.I8_GELU):
+        check(gpu_run(lin, x, kind, 0.07), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.07),
+              kind, f"k={k}")
+
+
+def test_max_k_and_int32_extremes(bsg):
+    """Largest supported K with the largest-magnitude values."""
+    k = bsg.bsgemm_max_k()
+    rng = synth.rng_for(4000)
+    wt = synth.draw_weight(rng, 16, k, 0.0, value_lo=-128, value_hi=127)
+    wt.values[:] = np.where(wt.values < 0, -128, 127).astype(np.int8)
+    x = synth.draw_x(rng, 40, k, "extreme")
+    x[0] = -128
+    wt.values[: k] = -128  # block-row 0 all -128: acc = 16384 * K on row 0
+    lin = make_linear(bsg, wt)
+    w = oracle.weight_dense(wt)
+    want = oracle.linear(x, w, wt.scales, wt.bias, synth.I32)
+    assert want[0, 0] == 16384 * k
+    check(gpu_run(lin, x, synth.I32, 1.0), want, synth.I32, "extremes i32")
+    for kind in (synth.I8, synth.F32):
+        check(gpu_run(lin, x, kind, 0.5), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.5), kind)
+
+
+def test_empty_and_dense_block_rows(bsg):
+    """Block-rows with no stored block, fully dense block-rows, and stored
+    blocks whose values are all zero."""
+    n, k = 40, 300
+    rng = synth.rng_for(5000)
+    dense = rng.integers(-127, 128, size=(n, k)).astype(np.int8)
+    mask = rng.random((n // 4, k)) < 0.2
+    mask[0] = False          # empty
+    mask[3] = False          # empty
+    mask[9] = False          # empty (last)
+    mask[1] = True           # fully dense
+    mask[5] = True
+    dense[8:12, :] = 0       # block-row 2: stored blocks of zeros
+    mask[2, ::3] = True
+    indptr, colidx, values = oracle.dense_to_bsr(dense, mask)
+    scales = rng.uniform(1e-3, 1e-2, n).astype(np.float32)
+    bias = rng.normal(0, 0.02, n).astype(np.float32)
+    lin = bsg.SparseInt8Linear(n, k, indptr, colidx, values, scales, bias)
+    w = oracle.bsr_to_dense(n, k, indptr, colidx, values)
+    x = synth.draw_x(rng, 150, k, "u127")
+    for kind in KINDS:
+        check(gpu_run(lin, x, kind, 0.05), oracle.linear(x, w, scales, bias, kind, out_scale=0.05), kind,
+              synth.KIND_NAMES[kind])
+
+
+def test_all_blocks_pruned_gives_bias(bsg):
+    rng = synth.rng_for(5100)
+    wt = synth.draw_weight(rng, 64, 768, 1.0)
+    assert wt.nnzb == 0
+    x = synth.draw_x(rng, 200, 768, "u127")
+    lin = make_linear(bsg, wt)
+    assert not gpu_run(lin, x, synth.I32, 1.0).any()
+    y = gpu_run(lin, x, synth.F32, 1.0)
+    assert np.array_equal(y, np.broadcast_to(wt.bias, y.shape))
+
+
+def test_null_bias_and_zero_m(bsg):
+    rng = synth.rng_for(5200)
+    wt = synth.draw_weight(rng, 16, 64, 0.5)
+    lin = bsg.SparseInt8Linear(16, 64, wt.indptr, wt.colidx, wt.values, wt.scales, None)
+    x = synth.draw_x(rng, 9, 64, "u127")
+    want = oracle.linear(x, oracle.weight_dense(wt), wt.scales, None, synth.F32)
+    check(gpu_run(lin, x, synth.F32, 1.0), want, synth.F32)
+    empty = torch.empty((0, 64), dtype=torch.int8, device="cuda")
+    assert lin(empty, synth.F32).shape == (0, 16)
+
+
+def test_run_argument_errors(bsg):
+    rng = synth.rng_for(5300)
+    wt = synth.draw_weight(rng, 16, 64, 0.5)
+    lin = make_linear(bsg, wt)
+    x = torch.zeros((4, 64), dtype=torch.int8, device="cuda")
+    out = torch.empty((4, 16), dtype=torch.int8, device="cuda")
+    for bad_scale in (0.0, -1.0, float("inf"), float("nan")):
+        with pytest.raises(bsg.BsgemmError) as e:
+            bsg.bsgemm_run(lin._h, x.data_ptr(), 4, out.data_ptr(), bsg.OUT_I8, bad_scale)
+        assert e.value.code == bsg.ERR_INVALID
+    with pytest.raises(bsg.BsgemmError):
+        bsg.bsgemm_run(lin._h, x.data_ptr(), 4, out.data_ptr(), 7, 1.0)
+    with pytest.raises(bsg.BsgemmError):
+        bsg.bsgemm_run(lin._h, x.data_ptr(), -1, out.data_ptr(), bsg.OUT_I32, 1.0)
+    raw = torch.empty(4 * 16 * 4 + 16, dtype=torch.uint8, device="cuda")
+    with pytest.raises(bsg.BsgemmError):  # misaligned output
+        bsg.bsgemm_run(lin._h, x.data_ptr(), 4, raw.data_ptr() + 4, bsg.OUT_I32, 1.0)
+
+
+def test_misaligned_activations(bsg):
+    """An activation pointer that is not 16-byte aligned is still exact."""
+    rng = synth.rng_for(5400)
+    wt = synth.draw_weight(rng, 32, 768, 0.9)
+    x = synth.draw_x(rng, 100, 768, "u127")
+    buf = torch.zeros(100 * 768 + 16, dtype=torch.int8, device="cuda")
+    buf[3:3 + 100 * 768] = torch.from_numpy(x.reshape(-1)).cuda()
+    lin = make_linear(bsg, wt)
+    out = torch.empty((100, 32), dtype=torch.int32, device="cuda")
+    bsg.bsgemm_run(lin._h, buf.data_ptr() + 3, 100, out.data_ptr(), bsg.OUT_I32, 1.0,
+                   torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    check(out.cpu().numpy(), oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I32), synth.I32)
+
+
+def test_guard_bands_and_determinism(bsg):
+    """Nothing is written outside out[M][N]; two runs are bit-identical."""
+    rng = synth.rng_for(5500)
+    wt = synth.draw_weight(rng, 96, 3072, 0.9)
+    m = 131
+    x = torch.from_numpy(synth.draw_x(rng, m, 3072, "u0_127")).cuda()
+    lin = make_linear(bsg, wt)
+    for kind, elem in ((synth.I8, 1), (synth.F32, 4)):
+        guard = 4096
+        raw = torch.full((guard * 2 + m * 96 * elem,), 0x5A, dtype=torch.uint8, device="cuda")
+        bsg.bsgemm_run(lin._h, x.data_ptr(), m, raw.data_ptr() + guard, kind, 0.05,
+                       torch.cuda.current_stream().cuda_stream)
+        first = raw.clone()
+        bsg.bsgemm_run(lin._h, x.data_ptr(), m, raw.data_ptr() + guard, kind, 0.05,
+                       torch.cuda.current_stream().cuda_stream)
+        torch.cuda.synchronize()
+        assert torch.equal(first, raw)
+        assert bool((raw[:guard] == 0x5A).all()) and bool((raw[-guard:] == 0x5A).all())
+
+
+def test_one_handle_many_streams(bsg):
+    """The handle is immutable: concurrent runs on several streams (weight
+    sharing across parallel instances) all give the oracle's result."""
+    rng = synth.rng_for(5600)
+    wt = synth.draw_weight(rng, 768, 768, 0.9)
+    lin = make_linear(bsg, wt)
+    w = oracle.weight_dense(wt)
+    xs = [synth.draw_x(rng, 64 * (i + 1), 768, "u127") for i in range(4)]
+    streams = [torch.cuda.Stream() for _ in xs]
+    outs = []
+    for x, s in zip(xs, streams):
+        with torch.cuda.stream(s):
+            xd = torch.from_numpy(x).cuda(non_blocking=False)
+            out = torch.empty((x.shape[0], 768), dtype=torch.int8, device="cuda")
+            lin.run(xd, out, synth.I8, 0.05, stream=s)
+            outs.append(out)
+    torch.cuda.synchronize()
+    for x, out in zip(xs, outs):
+        check(out.cpu().numpy(), oracle.linear(x, w, wt.scales, wt.bias, synth.I8, out_scale=0.05), synth.I8)
+
+
+def test_host_tensors_round_trip(bsg):
+    """The end-to-end call: CPU input in, CPU result out."""
+    rng = synth.rng_for(5700)
+    wt = synth.draw_weight(rng, 64, 768, 0.9)
+    x = synth.draw_x(rng, 50, 768, "u127")
+    lin = make_linear(bsg, wt)
+    got = lin(torch.from_numpy(x), synth.I8, 0.05)
+    assert not got.is_cuda
+    check(got.numpy(), oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I8, out_scale=0.05),
+          synth.I8)
+
+
+def test_from_dense(bsg):
+    rng = synth.rng_for(5800)
+    wt = synth.draw_weight(rng, 128, 768, 0.8)
+    w = oracle.weight_dense(wt)
+    lin = bsg.SparseInt8Linear.from_dense(w, wt.scales, wt.bias)
+    x = synth.draw_x(rng, 33, 768, "u127")
+    check(gpu_run(lin, x, synth.F32_GELU, 1.0), oracle.linear(x, w, wt.scales, wt.bias, synth.F32_GELU),
+          synth.F32_GELU)
+
+
+# ------------------------------------- full-size workloads, sampled rows --
+
+def sample_rows(m: int, tile: int, seed: int, n_random: int = 40) -> np.ndarray:
+    rng = np.random.default_rng(seed)
+    fixed = [0, 1, tile - 1, tile, m // 2, m - tile, m - 2, m - 1]
+    rows = set(r for r in fixed if 0 <= r < m) | set(rng.integers(0, m, n_random).tolist())
+    return np.array(sorted(rows))
+
+
+@pytest.mark.parametrize("case_fn", [synth.single_768, synth.ffn1, synth.ffn2], ids=lambda f: f.__name__)
+def test_full_size_workloads(bsg, case_fn):
+    case = case_fn()
+    wt = case.weight
+    lin = make_linear(bsg, wt)
+    got = gpu_run(lin, case.x, case.kind, case.out_scale)
+    rows = sample_rows(case.m, lin.info["tile_m"], 7)
+    want = oracle.linear(case.x, oracle.weight_dense(wt), wt.scales, wt.bias, case.kind,
+                         out_scale=case.out_scale, rows=rows, threads=8)
+    check(got[rows], want, case.kind, case.name)
+    if case.kind in (synth.I8, synth.I8_GELU):
+        # also the int32 accumulators, on the same rows
+        acc = gpu_run(lin, case.x, synth.I32, 1.0)
+        check(acc[rows], oracle.linear(case.x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I32,
+                                       rows=rows, threads=8), synth.I32, case.name + " acc")
+
+
+def test_encoder_layer_linears_full_size(bsg):
+    """The four linears of one encoder layer at M = 8 x 384, int8 between."""
+    ws, x0 = synth.encoder_layer()
+    x = x0
+    for (name, n, k, kind), wt in zip(synth.LAYER_LINEARS, ws):
+        if x.shape[1] != k:  # FFN2 consumes FFN1's width: use a seeded input
+            x = synth.draw_x(synth.rng_for(6000), x0.shape[0], k, "u0_127")
+        lin = make_linear(bsg, wt)
+        got = gpu_run(lin, x, kind, 0.05)
+        rows = sample_rows(x.shape[0], lin.info["tile_m"], 11, n_random=16)
+        want = oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, kind, out_scale=0.05, rows=rows,
+                             threads=8)
+        check(got[rows], want, kind, name)
