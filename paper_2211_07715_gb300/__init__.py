@@ -7,7 +7,7 @@ accumulation, and a fused dequantise + bias (+ GELU) (+ requantise)
 epilogue.  All arithmetic runs in the CUDA kernels of libbsgemm.so; this
 module only marshals arguments (PyTorch provides device memory and
 streams).  There is no CPU fallback: importing fails loudly if the library
-has not been built (``python -m paper_2211_07715_gb300.build`` or
+has not been built (``python paper_2211_07715_gb300/build.py`` or
 ``__graft_entry__.build()``).
 
 The functions below carry the C names (``bsgemm_create``, ``bsgemm_run``,
@@ -40,7 +40,7 @@ class Epilogue(ctypes.Structure):
 
 def _load() -> ctypes.CDLL:
     if not os.path.exists(LIB_PATH):
-        raise ImportError(f"{LIB_PATH} is missing: build it with `python -m paper_2211_07715_gb300.build`")
+        raise ImportError(f"{LIB_PATH} is missing: build it with `python paper_2211_07715_gb300/build.py`")
     lib = ctypes.CDLL(LIB_PATH)
     vp = ctypes.c_void_p
     lib.bsgemm_create.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]

@@ -16,8 +16,8 @@ HEADER = os.path.join(ROOT, "include", "bsgemm.h")
 def bsg():
     if not shutil.which("nvcc") and not os.path.exists("/usr/local/cuda/bin/nvcc"):
         pytest.skip("nvcc not available")
-    from paper_2211_07715_gb300 import build
-    build.build()
+    import __graft_entry__
+    __graft_entry__.build()
     import paper_2211_07715_gb300
     return paper_2211_07715_gb300
 
