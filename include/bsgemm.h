@@ -109,6 +109,54 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
 int bsgemm_run(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream);
 
 /*
+ * bsgemm_workspace_bytes -- device workspace bsgemm_run_ws needs for M
+ * tokens: a token-tiled, column-major copy of the activations
+ * (ceil(M / T) * round_up(K, 16) * T bytes, T = bsgemm_info()[4]).
+ * Returns 0 for M <= 0 or a NULL handle.
+ */
+size_t bsgemm_workspace_bytes(bsgemm_t h, int M);
+
+/*
+ * bsgemm_run_ws -- bsgemm_run with a caller-owned DEVICE workspace of at
+ * least bsgemm_workspace_bytes(h, M) bytes, 16-byte aligned.  Enqueues two
+ * kernels on `stream`: one rewrites act as token tiles into the workspace,
+ * the second streams each tile into shared memory with one bulk (TMA) copy
+ * and computes the layer.  This is the fast path; bsgemm_run (no
+ * workspace) gathers the activations with per-thread loads instead.  The
+ * workspace is scratch: its contents are undefined afterwards, and two runs
+ * in flight at the same time need two workspaces.  Same results, return
+ * codes and asynchrony as bsgemm_run; a workspace that is NULL, too small or
+ * misaligned returns BSGEMM_ERR_INVALID.
+ */
+int bsgemm_run_ws(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* workspace,
+                  size_t workspace_bytes, void* stream);
+
+/*
+ * The two steps of bsgemm_run_ws, for callers that keep activations in the
+ * token-tiled layout between layers or time the steps apart:
+ *   bsgemm_tile_activations -- act [M][K] (DEVICE) -> token tiles in
+ *     `tiles` (DEVICE, >= bsgemm_workspace_bytes(h, M) bytes, 16-byte
+ *     aligned): tile t = tokens tT..tT+T-1, stored column by column (all T
+ *     tokens' bytes of column k, then of column k+1, ...), columns padded to
+ *     round_up(K, 16) and tokens past M with zeros, T = bsgemm_info()[4].
+ *   bsgemm_run_tiled -- the layer from such tiles (one kernel).
+ * Both are asynchronous on `stream` and return BSGEMM_OK or BSGEMM_ERR_*.
+ */
+int bsgemm_tile_activations(bsgemm_t h, const int8_t* act, int M, void* tiles, size_t tiles_bytes, void* stream);
+int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, void* out, bsgemm_epilogue epi,
+                     void* stream);
+
+/*
+ * bsgemm_device_status -- read (and with clear != 0, reset) the handle's
+ * device status word.  0 means every wait in the kernels completed; bit 0
+ * (BSGEMM_STATUS_TIMEOUT) means a bounded wait on an asynchronous copy gave
+ * up and that run's output is incomplete.  Synchronises the device.  Returns
+ * the status, or a negative BSGEMM_ERR_* code.
+ */
+#define BSGEMM_STATUS_TIMEOUT 1
+int bsgemm_device_status(bsgemm_t h, int clear);
+
+/*
  * bsgemm_destroy -- free the handle and its device memory.  The caller must
  * make sure no bsgemm_run on this handle is still executing (cudaFree
  * itself waits for the device).  NULL is ignored.
@@ -134,8 +182,8 @@ int bsgemm_max_k(void);
  * the inner loop; the last quad of a block-row is padded with zero-weight
  * entries), [4] token-tile height of the kernel, [5] CTAs of a launch once
  * M is large enough to fill the GPU (SMs x resident CTAs per SM), [6] device
- * bytes held by the handle.  Returns the number of entries
- * available (7), or BSGEMM_ERR_INVALID.
+ * bytes held by the handle.  Returns the number of entries available (7),
+ * or BSGEMM_ERR_INVALID.
  */
 int bsgemm_info(bsgemm_t h, int64_t* out, int n);
 

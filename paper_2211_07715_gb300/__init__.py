@@ -57,12 +57,23 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_max_k.restype = ctypes.c_int
     lib.bsgemm_info.argtypes = [vp, ctypes.POINTER(ctypes.c_int64), ctypes.c_int]
     lib.bsgemm_info.restype = ctypes.c_int
+    lib.bsgemm_workspace_bytes.argtypes = [vp, ctypes.c_int]
+    lib.bsgemm_workspace_bytes.restype = ctypes.c_size_t
+    lib.bsgemm_run_ws.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp, ctypes.c_size_t, vp]
+    lib.bsgemm_run_ws.restype = ctypes.c_int
+    lib.bsgemm_tile_activations.argtypes = [vp, vp, ctypes.c_int, vp, ctypes.c_size_t, vp]
+    lib.bsgemm_tile_activations.restype = ctypes.c_int
+    lib.bsgemm_run_tiled.argtypes = [vp, vp, ctypes.c_size_t, ctypes.c_int, vp, Epilogue, vp]
+    lib.bsgemm_run_tiled.restype = ctypes.c_int
+    lib.bsgemm_device_status.argtypes = [vp, ctypes.c_int]
+    lib.bsgemm_device_status.restype = ctypes.c_int
     return lib
 
 
 _lib = _load()
 
-EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
+EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_workspace_bytes", "bsgemm_tile_activations",
+            "bsgemm_run_tiled", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status",
             "bsgemm_max_k", "bsgemm_info")
 
 
@@ -103,6 +114,40 @@ def bsgemm_run(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale:
     rc = _lib.bsgemm_run(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_run_ws(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float, ws_ptr: int,
+                  ws_bytes: int, stream: int = 0) -> None:
+    """Enqueue the two-kernel fast path with a device workspace; raises on failure."""
+    rc = _lib.bsgemm_run_ws(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), ws_ptr,
+                            int(ws_bytes), stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_tile_activations(h: int, act_ptr: int, m: int, tiles_ptr: int, tiles_bytes: int, stream: int = 0) -> None:
+    rc = _lib.bsgemm_tile_activations(h, act_ptr, int(m), tiles_ptr, int(tiles_bytes), stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_run_tiled(h: int, tiles_ptr: int, tiles_bytes: int, m: int, out_ptr: int, kind: int, out_scale: float,
+                     stream: int = 0) -> None:
+    rc = _lib.bsgemm_run_tiled(h, tiles_ptr, int(tiles_bytes), int(m), out_ptr, Epilogue(int(kind), float(out_scale)),
+                               stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_workspace_bytes(h: int, m: int) -> int:
+    return int(_lib.bsgemm_workspace_bytes(h, int(m)))
+
+
+def bsgemm_device_status(h: int, clear: bool = False) -> int:
+    rc = _lib.bsgemm_device_status(h, 1 if clear else 0)
+    if rc < 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+    return rc
 
 
 def bsgemm_destroy(h: int) -> None:
@@ -152,8 +197,16 @@ class SparseInt8Linear:
         indptr, colidx, values = dense_to_blocks(w)
         return cls(w.shape[0], w.shape[1], indptr, colidx, values, scales, bias)
 
-    def run(self, x, out, kind: int, out_scale: float = 1.0, stream=None) -> None:
-        """out[M][N] = epilogue(x[M][K] W^T); both CUDA tensors, contiguous."""
+    def workspace_bytes(self, m: int) -> int:
+        return bsgemm_workspace_bytes(self._h, m)
+
+    def run(self, x, out, kind: int, out_scale: float = 1.0, stream=None, workspace=None) -> None:
+        """out[M][N] = epilogue(x[M][K] W^T); both CUDA tensors, contiguous.
+
+        Takes the fast two-kernel path with a workspace: the given uint8 CUDA
+        tensor, or (workspace=None) one drawn from PyTorch's caching
+        allocator on the same stream.  workspace=False forces the
+        single-kernel path without scratch memory."""
         import torch
         if x.dtype != torch.int8 or not x.is_cuda or not x.is_contiguous() or x.dim() != 2 or x.shape[1] != self.k_in:
             raise ValueError("x must be a contiguous CUDA int8 tensor [M][K]")
@@ -161,7 +214,18 @@ class SparseInt8Linear:
                 or str(out.dtype).split(".")[-1] != _OUT_DTYPES[kind]):
             raise ValueError(f"out must be a contiguous CUDA {_OUT_DTYPES[kind]} tensor [M][N]")
         s = torch.cuda.current_stream() if stream is None else stream
-        bsgemm_run(self._h, x.data_ptr(), x.shape[0], out.data_ptr(), kind, out_scale, s.cuda_stream)
+        m = x.shape[0]
+        if workspace is False or m == 0:
+            bsgemm_run(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, s.cuda_stream)
+            return
+        need = self.workspace_bytes(m)
+        if workspace is None:
+            with torch.cuda.stream(s):
+                workspace = torch.empty(need, dtype=torch.uint8, device=x.device)
+        if workspace.numel() * workspace.element_size() < need:
+            raise ValueError(f"workspace must hold {need} bytes")
+        bsgemm_run_ws(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, workspace.data_ptr(),
+                      workspace.numel() * workspace.element_size(), s.cuda_stream)
 
     def __call__(self, x, kind: int, out_scale: float = 1.0, stream=None):
         """Allocate the output and run.  A CPU `x` is copied in and the result

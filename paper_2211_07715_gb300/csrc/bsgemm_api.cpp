@@ -4,6 +4,7 @@
 // upload, and the launch of the kernel in bsgemm_kernel.cu.
 #include "bsgemm.h"
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <string>
@@ -19,6 +20,7 @@ struct bsgemm_ctx {
     int64_t nnzb = 0;
     void* arena = nullptr;
     size_t arena_bytes = 0;
+    std::vector<int32_t> cost;  // host copy of the schedule's prefix cost [nbr + 1]
     bsg::DeviceWeights w{};
 };
 
@@ -43,6 +45,8 @@ std::string cuda_msg(const char* what, cudaError_t e) {
 }
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+const int kZeroStatus = 0;
 
 // Check the block-compressed arrays; returns an empty string if valid.
 std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx) {
@@ -119,18 +123,23 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         }
     }
 
-    // Repack into quads: per block-row, stored blocks in groups of 4; the
-    // last group is padded by repeating the row's last column with zero
-    // weights.  Record q = {k0, k1, k2, k3} then 4 words, word c holding the
-    // bytes W[4r + c][k0..k3].
+    // Repack into quads: per block-row, stored blocks in groups of 4, and
+    // the quad count rounded up to a multiple of the kernel's lane groups per
+    // warp; padding entries repeat the row's last column with zero weights.
+    // Record q = {k0, k1, k2, k3} then 4 words, word c holding the bytes
+    // W[4r + c][k0..k3].
+    const int MT = bsg::tile_for_k(K);
+    const int G = bsg::groups_for_tile(MT);
     std::vector<int32_t> qptr(nbr + 1, 0), cost(nbr + 1, 0);
     for (int r = 0; r < nbr; ++r) {
         const int nz = indptr[r + 1] - indptr[r];
-        qptr[r + 1] = qptr[r] + (nz + 3) / 4;
+        const int nq = (nz + 3) / 4;
+        qptr[r + 1] = qptr[r] + (nq + G - 1) / G * G;
         cost[r + 1] = qptr[r + 1] + (r + 1);
     }
     const int Q = qptr[nbr];
-    std::vector<int32_t> quads(static_cast<size_t>(Q + 1) * 8, 0);  // + 1 padding record
+    // + padding records: the kernel copies whole ring chunks of kQuadPad records
+    std::vector<int32_t> quads(static_cast<size_t>(Q + bsg::kQuadPad) * 8, 0);
     for (int r = 0; r < nbr; ++r) {
         const int j0 = indptr[r], j1 = indptr[r + 1];
         for (int q = qptr[r]; q < qptr[r + 1]; ++q) {
@@ -168,8 +177,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         delete h;
         return nullptr;
     }
-    h->MT = bsg::tile_for_k(K);
-    if (bsg::smem_bytes(h->MT, K) + 16 > static_cast<size_t>(optin)) {
+    h->MT = MT;
+    if (bsg::smem_bytes(h->MT, K) + bsg::kStaticSmem > static_cast<size_t>(optin)) {
         fail(BSGEMM_ERR_UNSUPPORTED, "this device has too little shared memory per block for K = " + std::to_string(K));
         delete h;
         return nullptr;
@@ -186,7 +195,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     const size_t off_quads = align_up(off_cost + sizeof(int32_t) * (nbr + 1), 256);
     const size_t off_scale = align_up(off_quads + sizeof(int32_t) * quads.size(), 256);
     const size_t off_bias = align_up(off_scale + sizeof(float) * N, 256);
-    h->arena_bytes = align_up(off_bias + sizeof(float) * N, 256);
+    const size_t off_status = align_up(off_bias + sizeof(float) * N, 256);
+    h->arena_bytes = align_up(off_status + sizeof(int), 256);
     e = cudaMalloc(&h->arena, h->arena_bytes);
     if (e != cudaSuccess) {
         fail(BSGEMM_ERR_CUDA, cuda_msg("cudaMalloc", e));
@@ -200,6 +210,7 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         {off_quads, quads.data(), sizeof(int32_t) * quads.size()},
         {off_scale, scales, sizeof(float) * N},
         {off_bias, bias_v.data(), sizeof(float) * N},
+        {off_status, &kZeroStatus, sizeof(int)},
     };
     for (const Piece& p : pieces) {
         e = cudaMemcpy(base + p.off, p.src, p.bytes, cudaMemcpyHostToDevice);
@@ -211,11 +222,13 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         }
     }
     h->nnzb = nnzb;
+    h->cost = cost;
     h->w.qptr = reinterpret_cast<const int32_t*>(base + off_qptr);
     h->w.cost = reinterpret_cast<const int32_t*>(base + off_cost);
     h->w.quads = reinterpret_cast<const int4*>(base + off_quads);
     h->w.scale = reinterpret_cast<const float*>(base + off_scale);
     h->w.bias = reinterpret_cast<const float*>(base + off_bias);
+    h->w.status = reinterpret_cast<int*>(base + off_status);
     h->w.N = N;
     h->w.K = K;
     h->w.nbr = nbr;
@@ -223,7 +236,11 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     return h;
 }
 
-int bsgemm_run(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream) {
+// mode: 0 = gather from act (no scratch), 1 = relayout act into workspace
+// then stage tiles, 2 = stage tiles already in workspace (act unused).
+static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* workspace,
+                      size_t workspace_bytes, int mode, void* stream) {
+    const bool use_ws = mode != 0;
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
     if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
@@ -237,29 +254,105 @@ int bsgemm_run(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue 
         if (!std::isfinite(inv)) return fail(BSGEMM_ERR_INVALID, "1 / out_scale overflows fp32");
     }
     if (M == 0) return BSGEMM_OK;
-    if (!act || !out) return fail(BSGEMM_ERR_INVALID, "act and out must not be NULL");
+    if ((mode != 2 && !act) || !out) return fail(BSGEMM_ERR_INVALID, "act and out must not be NULL");
     if (reinterpret_cast<uintptr_t>(out) % 16 != 0) return fail(BSGEMM_ERR_INVALID, "out must be 16-byte aligned");
+    if (use_ws) {
+        const size_t need = bsg::tiled_bytes(h->MT, h->w.K, M);
+        if (!workspace || workspace_bytes < need)
+            return fail(BSGEMM_ERR_INVALID, "workspace must hold bsgemm_workspace_bytes(h, M) = " +
+                                                std::to_string(need) + " bytes");
+        if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0)
+            return fail(BSGEMM_ERR_INVALID, "workspace must be 16-byte aligned");
+    }
     int dev = -1;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
     if (dev != h->device)
         return fail(BSGEMM_ERR_INVALID, "current device " + std::to_string(dev) + " is not the handle's device " +
                                             std::to_string(h->device));
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
 
     bsg::LaunchArgs a{};
     a.x = act;
+    a.xb = use_ws ? static_cast<const int8_t*>(workspace) : nullptr;
     a.out = out;
     a.M = M;
     a.kind = epi.kind;
     a.inv_out_scale = inv;
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
     const long long ntiles = (static_cast<long long>(M) + h->MT - 1) / h->MT;
-    const long long units = ntiles * h->w.nbr;
-    const long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
+    const long long nbr = h->w.nbr;
+    const long long units = ntiles * nbr;
+    long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
+    if (cap > bsg::kMaxGrid) cap = bsg::kMaxGrid;
     const int grid = static_cast<int>(units < cap ? units : cap);
-    e = bsg::launch(h->w, a, h->MT, grid, static_cast<cudaStream_t>(stream));
+    // Cost-balanced contiguous unit ranges: CTA c starts at the first unit
+    // whose start cost t * ctile + cost[r] reaches c * total / grid.
+    bsg::Schedule sched;
+    const long long ctile = h->cost[nbr];
+    const __int128 total = static_cast<__int128>(ntiles) * ctile;
+    for (int c = 0; c <= grid; ++c) {
+        const long long target = static_cast<long long>(total * c / grid);
+        const long long t = target / ctile, rem = target - t * ctile;
+        const long long r = std::lower_bound(h->cost.begin(), h->cost.begin() + nbr, rem) - h->cost.begin();
+        sched.u[c] = t * nbr + r;
+    }
+    if (mode == 1) {
+        e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(workspace), s);
+        if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("relayout launch", e));
+    }
+    e = bsg::launch(h->w, a, sched, h->MT, grid, s);
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("kernel launch", e));
     return BSGEMM_OK;
+}
+
+int bsgemm_run(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream) {
+    return run_common(h, act, M, out, epi, nullptr, 0, 0, stream);
+}
+
+int bsgemm_run_ws(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* workspace,
+                  size_t workspace_bytes, void* stream) {
+    return run_common(h, act, M, out, epi, workspace, workspace_bytes, 1, stream);
+}
+
+int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, void* out, bsgemm_epilogue epi,
+                     void* stream) {
+    return run_common(h, nullptr, M, out, epi, const_cast<void*>(tiles), tiles_bytes, 2, stream);
+}
+
+int bsgemm_tile_activations(bsgemm_t h, const int8_t* act, int M, void* tiles, size_t tiles_bytes, void* stream) {
+    clear_error();
+    if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
+    if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
+    if (M == 0) return BSGEMM_OK;
+    if (!act) return fail(BSGEMM_ERR_INVALID, "act must not be NULL");
+    const size_t need = bsg::tiled_bytes(h->MT, h->w.K, M);
+    if (!tiles || tiles_bytes < need)
+        return fail(BSGEMM_ERR_INVALID, "tiles must hold bsgemm_workspace_bytes(h, M) = " + std::to_string(need) +
+                                            " bytes");
+    if (reinterpret_cast<uintptr_t>(tiles) % 16 != 0) return fail(BSGEMM_ERR_INVALID, "tiles must be 16-byte aligned");
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
+    if (dev != h->device) return fail(BSGEMM_ERR_INVALID, "current device is not the handle's device");
+    e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(tiles), static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("relayout launch", e));
+    return BSGEMM_OK;
+}
+
+size_t bsgemm_workspace_bytes(bsgemm_t h, int M) {
+    if (!h || M <= 0) return 0;
+    return bsg::tiled_bytes(h->MT, h->w.K, M);
+}
+
+int bsgemm_device_status(bsgemm_t h, int clear) {
+    clear_error();
+    if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
+    int v = 0;
+    cudaError_t e = cudaMemcpy(&v, h->w.status, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && clear && v != 0) e = cudaMemcpy(h->w.status, &kZeroStatus, sizeof(int), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("reading the device status", e));
+    return v;
 }
 
 void bsgemm_destroy(bsgemm_t h) {

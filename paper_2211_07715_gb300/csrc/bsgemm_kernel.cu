@@ -27,9 +27,15 @@
 //   re-organised input block B and 4 vpdpbusd.  GB300 runs int8 dot products
 //   at the same rate on dp4a as on its int8 MMA paths, so no tensor-core path
 //   is faster here (the 4-channel block cannot fill an MMA tile).
-// * A CTA's quads are split evenly between its lane groups; a block-row that
-//   straddles a split point is summed in a shared-memory slot (int32 atomics)
-//   and finished after a barrier.  All sums are exact int32.
+// * A CTA's quads are split evenly between its 16 warps.  Each warp streams
+//   its contiguous range of 32-byte quad records through a two-chunk ring in
+//   shared memory (cp.async, 512 bytes per chunk, the next chunk in flight
+//   while the current one is consumed).  With 64-token tiles a lane covers
+//   only half the warp's width, so the two half-warps take alternate quads
+//   of a block-row and add their sums with one shuffle at the row's end.
+//   A block-row that straddles a split between warps is summed in a
+//   shared-memory slot (int32 atomics) and finished after a barrier.  All
+//   sums are exact int32.
 // * The epilogue runs in registers: int32 -> fp32 (RNE), one fma with scale
 //   and bias, optional GELU by a fixed fp32 op sequence (A&S 7.1.28 erf),
 //   optional requantise (fp32 multiply, round half to even, saturate).
@@ -42,9 +48,14 @@ namespace bsg {
 namespace {
 
 constexpr int kSmemOptin = 232448;  // sm_103 opt-in shared memory per block
+constexpr int kSlots = kWarps - 1;  // one per split point between warp ranges
+// Record ring per warp: kRingSlots chunks of ring_chunk(MT) quad records;
+// while one chunk is consumed the next kRingSlots - 1 are in flight.
+constexpr int kRingSlots = 4;
+__host__ __device__ constexpr int ring_chunk(int MT) { return MT == 64 ? 8 : 16; }
 
-__host__ __device__ constexpr int groups_per_cta(int MT) { return kThreads / (MT / 4); }
-__host__ __device__ constexpr int slot_words(int MT) { return 16 * (MT / 4); }
+__host__ __device__ constexpr int slot_words(int MT) { return 4 * MT; }  // MT tokens x 4 channels
+constexpr size_t ring_bytes(int MT) { return static_cast<size_t>(kWarps) * kRingSlots * ring_chunk(MT) * 32; }
 
 // 4x4 byte transpose.  In: a/b/c/d = bytes (x0..x3) of rows 0..3.  Out:
 // t_i = (a_i, b_i, c_i, d_i).
@@ -76,9 +87,30 @@ __device__ __forceinline__ float gelu_f32(float y) {
     const float p4 = __fmul_rn(p2, p2);
     const float p8 = __fmul_rn(p4, p4);
     const float p16 = __fmul_rn(p8, p8);
-    const float e = __fsub_rn(1.0f, __fdiv_rn(1.0f, p16));
+    const float e = __fsub_rn(1.0f, __frcp_rn(p16));  // IEEE 1/p16, round to nearest
     const float erf_x = (x < 0.0f) ? -e : e;
     return __fmul_rn(__fmul_rn(0.5f, y), __fadd_rn(1.0f, erf_x));
+}
+
+// The same erf-form GELU for fp32 outputs, with the hardware's approximate
+// reciprocal (relative error <= 2^-22) in place of the IEEE one: fp32
+// outputs are checked against a tolerance, not bit for bit, and the extra
+// error stays below 2e-7 |y|.  int8 outputs use gelu_f32, which an int8
+// decision must reproduce exactly.
+__device__ __forceinline__ float gelu_f32_fast(float y) {
+    const float x = y * 0.70710678f;
+    const float ax = fabsf(x);
+    float h = fmaf(ax, 0.0000430638f, 0.0002765672f);
+    h = fmaf(ax, h, 0.0001520143f);
+    h = fmaf(ax, h, 0.0092705272f);
+    h = fmaf(ax, h, 0.0422820123f);
+    h = fmaf(ax, h, 0.0705230784f);
+    const float p = fmaf(ax, h, 1.0f);
+    const float p2 = p * p, p4 = p2 * p2, p8 = p4 * p4, p16 = p8 * p8;
+    float rcp;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rcp) : "f"(p16));
+    const float e = 1.0f - rcp;
+    return 0.5f * y * (1.0f + ((x < 0.0f) ? -e : e));
 }
 
 // fp32 -> int8: one fp32 multiply, round half to even, saturate.
@@ -88,31 +120,32 @@ __device__ __forceinline__ uint32_t requant_s8(float v, float inv) {
     return static_cast<uint32_t>(q) & 0xffu;
 }
 
-// Epilogue for one lane: tokens m_first..m_first+3 (rows < M only) x the 4
-// channels of block-row r.  acc[i * 4 + c] = token i, channel c.
-template <int KIND>
-__device__ __forceinline__ void store_tile(const DeviceWeights& w, const LaunchArgs& a, long long m_first,
-                                           int r, const int (&acc)[16]) {
+// Epilogue for one lane: tokens m_first + i, i < T (rows < M only), x the
+// 4 channels of block-row r (scales s, bias b).  v[i * 4 + c] = token i,
+// channel c.
+template <int KIND, int T>
+__device__ __forceinline__ void store_rows(const DeviceWeights& w, const LaunchArgs& a, long long m_first, int r,
+                                           const int (&v)[T * 4], float4 s, float4 b) {
     const int N = w.N;
-    float4 s = make_float4(0.f, 0.f, 0.f, 0.f), b = s;
-    if (KIND != 0) {
-        s = __ldg(reinterpret_cast<const float4*>(w.scale) + r);
-        b = __ldg(reinterpret_cast<const float4*>(w.bias) + r);
-    }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < T; ++i) {
         const long long m = m_first + i;
         if (m >= a.M) break;
         const size_t o = static_cast<size_t>(m) * N + 4 * r;
-        const int* v = acc + 4 * i;
+        const int* vi = v + 4 * i;
         if (KIND == 0) {
-            *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(v[0], v[1], v[2], v[3]);
+            *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(vi[0], vi[1], vi[2], vi[3]);
         } else {
-            float y0 = __fmaf_rn(__int2float_rn(v[0]), s.x, b.x);
-            float y1 = __fmaf_rn(__int2float_rn(v[1]), s.y, b.y);
-            float y2 = __fmaf_rn(__int2float_rn(v[2]), s.z, b.z);
-            float y3 = __fmaf_rn(__int2float_rn(v[3]), s.w, b.w);
-            if (KIND == 2 || KIND == 4) {
+            float y0 = __fmaf_rn(__int2float_rn(vi[0]), s.x, b.x);
+            float y1 = __fmaf_rn(__int2float_rn(vi[1]), s.y, b.y);
+            float y2 = __fmaf_rn(__int2float_rn(vi[2]), s.z, b.z);
+            float y3 = __fmaf_rn(__int2float_rn(vi[3]), s.w, b.w);
+            if (KIND == 2) {
+                y0 = gelu_f32_fast(y0);
+                y1 = gelu_f32_fast(y1);
+                y2 = gelu_f32_fast(y2);
+                y3 = gelu_f32_fast(y3);
+            } else if (KIND == 4) {
                 y0 = gelu_f32(y0);
                 y1 = gelu_f32(y1);
                 y2 = gelu_f32(y2);
@@ -130,227 +163,484 @@ __device__ __forceinline__ void store_tile(const DeviceWeights& w, const LaunchA
     }
 }
 
-// Last block-row r in [lo, hi) with qptr[r] <= q, given qptr[lo] <= q < qptr[hi].
-__device__ __forceinline__ int row_of(const int32_t* qptr, int lo, int hi, int q) {
+__device__ __forceinline__ float4 load_s4(const float* p, int r) { return __ldg(reinterpret_cast<const float4*>(p) + r); }
+
+// Last index r in [lo, hi) with qp[r] <= q, given qp[lo] <= q < qp[hi]
+// (qp: the shared-memory window of quad offsets).
+__device__ __forceinline__ int row_of(const int* qp, int lo, int hi, int q) {
     while (hi - lo > 1) {
         const int mid = (lo + hi) >> 1;
-        if (__ldg(qptr + mid) <= q) lo = mid; else hi = mid;
+        if (qp[mid] <= q) lo = mid; else hi = mid;
     }
     return lo;
 }
 
-// Stage activations rows m0..m0+MT-1, all K columns, into xt as k-major rows
-// of MT bytes (word g of row k = tokens 4g..4g+3 at column k).  Rows >= M and
-// columns >= K read as zero.
-template <int MT>
-__device__ __forceinline__ void stage_tile(uint32_t* xt, const LaunchArgs& a, int K, int kpad, long long m0) {
-    constexpr int G = MT / 4;
-    const int nkc = kpad >> 4;
-    for (int id = threadIdx.x; id < G * nkc; id += kThreads) {
-        const int g = id % G, kc = id / G;
-        uint32_t rw[4][4];
+// One staging unit: tokens 4g..4g+3 of the tile x columns 16kc..16kc+15.
+// rw[i][j] = bytes of token 4g+i at columns 16kc+4j..16kc+4j+3 (zero past M
+// or K).
+__device__ __forceinline__ void load_unit(const LaunchArgs& a, int K, long long m0, int g, int kc,
+                                          uint32_t (&rw)[4][4]) {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const long long m = m0 + 4 * g + i;
-            if (m < a.M) {
-                const int8_t* src = a.x + static_cast<size_t>(m) * K + 16 * kc;
-                if (a.x_vec16) {
-                    const int4 v = __ldg(reinterpret_cast<const int4*>(src));
-                    rw[i][0] = v.x; rw[i][1] = v.y; rw[i][2] = v.z; rw[i][3] = v.w;
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        uint32_t word = 0;
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const int k = 16 * kc + 4 * j + e;
-                            const uint32_t byte = (k < K) ? static_cast<uint8_t>(src[4 * j + e]) : 0u;
-                            word |= byte << (8 * e);
-                        }
-                        rw[i][j] = word;
-                    }
-                }
+    for (int i = 0; i < 4; ++i) {
+        const long long m = m0 + 4 * g + i;
+        if (m < a.M) {
+            const int8_t* src = a.x + static_cast<size_t>(m) * K + 16 * kc;
+            if (a.x_vec16) {
+                const int4 v = __ldg(reinterpret_cast<const int4*>(src));
+                rw[i][0] = v.x; rw[i][1] = v.y; rw[i][2] = v.z; rw[i][3] = v.w;
             } else {
-                rw[i][0] = rw[i][1] = rw[i][2] = rw[i][3] = 0u;
-            }
-        }
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            uint32_t t0, t1, t2, t3;
-            transpose4(rw[0][j], rw[1][j], rw[2][j], rw[3][j], t0, t1, t2, t3);
-            uint32_t* dst = xt + static_cast<size_t>(16 * kc + 4 * j) * G + g;
-            dst[0] = t0;
-            dst[G] = t1;
-            dst[2 * G] = t2;
-            dst[3 * G] = t3;
+                for (int j = 0; j < 4; ++j) {
+                    uint32_t word = 0;
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int k = 16 * kc + 4 * j + e;
+                        const uint32_t byte = (k < K) ? static_cast<uint8_t>(src[4 * j + e]) : 0u;
+                        word |= byte << (8 * e);
+                    }
+                    rw[i][j] = word;
+                }
+            }
+        } else {
+            rw[i][0] = rw[i][1] = rw[i][2] = rw[i][3] = 0u;
         }
     }
 }
 
-template <int MT, int KIND>
+// Write one unit k-major: word g of rows 16kc..16kc+15 (tokens 4g..4g+3).
+template <int MT>
+__device__ __forceinline__ void store_unit(uint32_t* xt, int g, int kc, const uint32_t (&rw)[4][4]) {
+    constexpr int RW = MT / 4;  // words per k-row
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        uint32_t t0, t1, t2, t3;
+        transpose4(rw[0][j], rw[1][j], rw[2][j], rw[3][j], t0, t1, t2, t3);
+        uint32_t* dst = xt + static_cast<size_t>(16 * kc + 4 * j) * RW + g;
+        dst[0] = t0;
+        dst[RW] = t1;
+        dst[2 * RW] = t2;
+        dst[3 * RW] = t3;
+    }
+}
+
+// Stage activation rows m0..m0+MT-1, all K columns, into xt as k-major rows
+// of MT bytes (word g of row k = tokens 4g..4g+3 at column k).  Each thread
+// keeps kStageBatch units' loads in flight before transposing them.
+template <int MT>
+__device__ __forceinline__ void stage_tile(uint32_t* xt, const LaunchArgs& a, int K, int kpad, long long m0) {
+    constexpr int G = MT / 4;
+    constexpr int kStageBatch = 2;
+    const int total = G * (kpad >> 4);
+    for (int base = threadIdx.x; base < total; base += kStageBatch * kThreads) {
+        uint32_t rw[kStageBatch][4][4];
+#pragma unroll
+        for (int b = 0; b < kStageBatch; ++b) {
+            const int id = base + b * kThreads;
+            if (id < total) load_unit(a, K, m0, id % G, id / G, rw[b]);
+        }
+#pragma unroll
+        for (int b = 0; b < kStageBatch; ++b) {
+            const int id = base + b * kThreads;
+            if (id < total) store_unit<MT>(xt, id % G, id / G, rw[b]);
+        }
+    }
+}
+
+// cp.async (16 bytes, L2 only) into shared memory, and its group fences.
+__device__ __forceinline__ void cp_async16(uint32_t smem_dst, const void* gmem_src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(smem_dst), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+// Shared-memory loads with 32-bit shared-window addresses.
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ int4 lds128(uint32_t addr) {
+    int4 v;
+    asm volatile("ld.shared.v4.s32 {%0, %1, %2, %3}, [%4];\n"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ uint2 lds64(uint32_t addr) {
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];\n" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+// mbarrier + bulk-copy (TMA) helpers.  Waits are bounded: a wait that
+// gives up reports false and the caller records kStatusTimeout.
+constexpr unsigned kWaitLimit = 1u << 20;
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, unsigned count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, unsigned bytes) {
+    asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}\n"
+                 ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, unsigned parity) {
+    for (unsigned i = 0; i < kWaitLimit; ++i) {
+        unsigned done;
+        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+                     " selp.u32 %0, 1, 0, p;\n}\n"
+                     : "=r"(done) : "r"(bar), "r"(parity) : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+// Global -> shared bulk copy completing on an mbarrier (16-byte aligned, size % 16 == 0).
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, unsigned bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
+                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+// Order this thread's earlier generic-proxy shared-memory accesses before
+// later asynchronous-proxy (bulk copy) writes.
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
+
+// One quad for one lane's 8 tokens: 4 x 8 bytes from the k-major tile at the
+// quad's columns, two 4x4 byte transposes, 32 dp4a (8 tokens x 4 channels).
+template <int MT>
+__device__ __forceinline__ void quad8(uint32_t xlane, const int4& kk, const int4& ww, int (&acc)[32]) {
+    const uint2 x0 = lds64(xlane + kk.x * MT), x1 = lds64(xlane + kk.y * MT);
+    const uint2 x2 = lds64(xlane + kk.z * MT), x3 = lds64(xlane + kk.w * MT);
+    uint32_t t[8];
+    transpose4(x0.x, x1.x, x2.x, x3.x, t[0], t[1], t[2], t[3]);
+    transpose4(x0.y, x1.y, x2.y, x3.y, t[4], t[5], t[6], t[7]);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        acc[4 * i + 0] = __dp4a(static_cast<int>(t[i]), ww.x, acc[4 * i + 0]);
+        acc[4 * i + 1] = __dp4a(static_cast<int>(t[i]), ww.y, acc[4 * i + 1]);
+        acc[4 * i + 2] = __dp4a(static_cast<int>(t[i]), ww.z, acc[4 * i + 2]);
+        acc[4 * i + 3] = __dp4a(static_cast<int>(t[i]), ww.w, acc[4 * i + 3]);
+    }
+}
+
+// Sum the G lane groups' partial accumulators of one block-row and scatter
+// the result: afterwards group g holds tokens [g*8/G, (g+1)*8/G) of its
+// lanes' 8 (red[j*4 + c] = token g*8/G + j, channel c).
+template <int G>
+__device__ __forceinline__ void reduce_groups(int lane, const int (&acc)[32], int (&red)[32 / G]) {
+    constexpr unsigned kFull = 0xffffffffu;
+    const bool up = (lane & 16) != 0;
+    if (G == 1) {
+#pragma unroll
+        for (int j = 0; j < 32 / G; ++j) red[j] = acc[j];
+    } else if (G == 2) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int send = up ? acc[j] : acc[16 + j];
+            const int keep = up ? acc[16 + j] : acc[j];
+            red[j % (32 / G)] = keep + __shfl_xor_sync(kFull, send, 16);
+        }
+    } else {
+        int k1[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+            const int send = up ? acc[j] : acc[16 + j];
+            const int keep = up ? acc[16 + j] : acc[j];
+            k1[j] = keep + __shfl_xor_sync(kFull, send, 16);
+        }
+        const bool up2 = (lane & 8) != 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int send = up2 ? k1[j] : k1[8 + j];
+            const int keep = up2 ? k1[8 + j] : k1[j];
+            red[j % (32 / G)] = keep + __shfl_xor_sync(kFull, send, 8);
+        }
+    }
+}
+
+template <int MT, int KIND, bool TMA>
 __global__ void __launch_bounds__(kThreads, 1)
-bsgemm_kernel(DeviceWeights w, LaunchArgs a, long long ntiles, long long ctile, int grid) {
-    constexpr int GL = MT / 4;               // lanes per block-row group
-    constexpr int H = groups_per_cta(MT);    // lane groups per CTA
-    constexpr int SW = slot_words(MT);       // int32 words per slot
+bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sched) {
+    constexpr int LW = MT / 8;          // lanes spanning the token tile (8 tokens per lane)
+    constexpr int G = 32 / LW;          // lane groups per warp; they interleave a block-row's quads
+    constexpr int TPG = 8 / G;          // tokens per lane after the groups' sums are combined
+    constexpr int SW = slot_words(MT);  // MT tokens x 4 channels
+    constexpr int RC = ring_chunk(MT);  // records per ring chunk
+    constexpr int S = RC / G;           // steps (G quads each) per ring chunk
+    constexpr int kRec = 32;            // bytes per quad record
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ long long s_range[2];
+    __shared__ int s_qp[kRowWin + 1];          // quad offsets of the current block-row window
+    __shared__ __align__(8) unsigned long long s_bar;  // completion of the token tile's bulk copy
+    __shared__ int s_cnt[kSlots];                      // warps that have added into each slot
 
     const int K = w.K;
     const int kpad = (K + 15) & ~15;
     uint32_t* xt = reinterpret_cast<uint32_t*>(smem);
     int* slots = reinterpret_cast<int*>(smem + static_cast<size_t>(kpad) * MT);
+    unsigned char* ring = reinterpret_cast<unsigned char*>(slots + kSlots * SW);
     const int tid = threadIdx.x;
-    const int h = tid / GL, li = tid % GL;
+    const int warp = tid >> 5, lane = tid & 31;
+    const int g = lane / LW, li = lane % LW;
     const long long nbr = w.nbr;
 
-    // This CTA's units: [U(c), U(c+1)), U(c) = first unit whose start cost
-    // reaches c * total / grid (unit (t, r) starts at t * ctile + cost[r]).
-    if (tid < 2) {
-        const long long c = static_cast<long long>(blockIdx.x) + tid;
-        const long long target = c * ctile * ntiles / grid;
-        const long long t = target / ctile, rem = target - t * ctile;
-        int lo = 0, hi = static_cast<int>(nbr);
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (__ldg(w.cost + mid) >= rem) hi = mid; else lo = mid + 1;
-        }
-        s_range[tid] = t * nbr + lo;
-    }
+    const uint32_t bar = smem_addr(&s_bar);
+    if (TMA && tid == 0) mbar_init(bar, 1);
+    // slots and their counters start at zero; whoever finishes a slot resets it
+    for (int i = tid; i < kSlots * SW; i += kThreads) slots[i] = 0;
+    if (tid < kSlots) s_cnt[tid] = 0;
     __syncthreads();
-    long long u = s_range[0];
-    const long long u_end = s_range[1];
+    unsigned phase = 0;
+    long long u = sched.u[blockIdx.x];
+    const long long u_end = sched.u[blockIdx.x + 1];
+    unsigned char* ringw = ring + warp * (kRingSlots * RC * kRec);
+    const uint32_t ring_s = smem_addr(ringw);
+    const uint32_t xlane = smem_addr(xt) + 8 * li;  // this lane's 8 tokens in every k-row
+    const int i0 = g * TPG;
 
+    long long staged = -1;  // token tile currently in xt
     while (u < u_end) {
+        // next window: one token tile, at most kRowWin consecutive block-rows
         const long long t = u / nbr;
         const int r_lo = static_cast<int>(u - t * nbr);
-        const int r_hi = static_cast<int>(min(nbr, r_lo + (u_end - u)));
+        const int r_hi = static_cast<int>(min(min(nbr, r_lo + (u_end - u)), static_cast<long long>(r_lo + kRowWin)));
         u += r_hi - r_lo;
         const long long m0 = t * MT;
+        const long long m_lane = m0 + 8 * li + i0;  // first token this lane finishes
+        // quad offset of block-row r (r_lo <= r <= r_hi), from the window
+        auto qp = [&](int r) { return s_qp[r - r_lo]; };
+        auto row_of_q = [&](int q) { return r_lo + row_of(s_qp, 0, r_hi - r_lo, q); };
 
-        stage_tile<MT>(xt, a, K, kpad, m0);
-        for (int i = tid; i < (H - 1) * SW; i += kThreads) slots[i] = 0;
-        __syncthreads();
+        for (int i = tid; i <= r_hi - r_lo; i += kThreads) s_qp[i] = __ldg(w.qptr + r_lo + i);
+        const bool stage = (t != staged);
+        if (TMA && stage && tid == 0) {
+            // one bulk copy of the token tile (already k-major in a.xb)
+            const unsigned bytes = static_cast<unsigned>(kpad) * MT;
+            const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * MT;
+            fence_proxy_async();
+            mbar_arrive_expect_tx(bar, bytes);
+            for (unsigned off = 0; off < bytes; off += 65536u)
+                bulk_g2s(smem_addr(xt) + off, src + off, min(65536u, bytes - off), bar);
+        }
+        __syncthreads();  // the block-row window is visible
+        if (!TMA && stage) {  // gather the tile with per-thread loads
+            stage_tile<MT>(xt, a, K, kpad, m0);
+            __syncthreads();
+            staged = t;
+        }
 
-        const int qa = __ldg(w.qptr + r_lo), qb = __ldg(w.qptr + r_hi);
-        const int qn = qb - qa;
-        const int q_begin = qa + static_cast<int>(static_cast<long long>(h) * qn / H);
-        const int q_end = qa + static_cast<int>(static_cast<long long>(h + 1) * qn / H);
-        const long long m_first = m0 + 4 * li;
+        const int qa = qp(r_lo), qb = qp(r_hi);
+        // Every block-row holds a multiple of G quads, so the tile's quads form
+        // nst steps of G; warps take an even split of the steps.
+        const int nst = (qb - qa) / G;
+        auto wstep = [&](int wi) { return static_cast<int>(static_cast<long long>(wi) * nst / kWarps); };
+        const int ws0 = wstep(warp), ws1 = wstep(warp + 1);
+        const int wq0 = qa + ws0 * G, wq1 = qa + ws1 * G;
 
-        if (q_begin < q_end) {
-            const uint32_t* xl = xt + li;
-            int r = row_of(w.qptr, r_lo, r_hi, q_begin);
-            int q = q_begin;
-            while (q < q_end) {
-                const int rs = __ldg(w.qptr + r), re = __ldg(w.qptr + r + 1);
-                const int seg_end = min(re, q_end);
-                int acc[16];
+        // Stream the warp's records [wq0, wq1) through the ring: chunk c =
+        // records wq0 + RC*c ..; one 16-byte copy per lane (RC*2 lanes).  The
+        // first chunks load while the token tile does.
+        const unsigned char* gsrc = reinterpret_cast<const unsigned char*>(w.quads) + static_cast<size_t>(wq0) * kRec;
+        const int nchunks = (wq1 - wq0 + RC - 1) / RC;
+        auto issue = [&](int c) {
+            if (c < nchunks && lane < RC * 2)
+                cp_async16(ring_s + (c % kRingSlots) * (RC * kRec) + 16 * lane,
+                           gsrc + static_cast<size_t>(c) * (RC * kRec) + 16 * lane);
+            cp_async_commit();
+        };
 #pragma unroll
-                for (int i = 0; i < 16; ++i) acc[i] = 0;
-                int4 kk = __ldg(w.quads + 2 * q);
-                int4 ww = __ldg(w.quads + 2 * q + 1);
-                for (; q < seg_end; ++q) {
-                    // the quad array carries one padding record, so q + 1 is in bounds
-                    const int4 kn = __ldg(w.quads + 2 * q + 2);
-                    const int4 wn = __ldg(w.quads + 2 * q + 3);
-                    const uint32_t x0 = xl[kk.x * GL], x1 = xl[kk.y * GL];
-                    const uint32_t x2 = xl[kk.z * GL], x3 = xl[kk.w * GL];
-                    uint32_t t0, t1, t2, t3;
-                    transpose4(x0, x1, x2, x3, t0, t1, t2, t3);
-                    acc[0] = __dp4a(static_cast<int>(t0), ww.x, acc[0]);
-                    acc[1] = __dp4a(static_cast<int>(t0), ww.y, acc[1]);
-                    acc[2] = __dp4a(static_cast<int>(t0), ww.z, acc[2]);
-                    acc[3] = __dp4a(static_cast<int>(t0), ww.w, acc[3]);
-                    acc[4] = __dp4a(static_cast<int>(t1), ww.x, acc[4]);
-                    acc[5] = __dp4a(static_cast<int>(t1), ww.y, acc[5]);
-                    acc[6] = __dp4a(static_cast<int>(t1), ww.z, acc[6]);
-                    acc[7] = __dp4a(static_cast<int>(t1), ww.w, acc[7]);
-                    acc[8] = __dp4a(static_cast<int>(t2), ww.x, acc[8]);
-                    acc[9] = __dp4a(static_cast<int>(t2), ww.y, acc[9]);
-                    acc[10] = __dp4a(static_cast<int>(t2), ww.z, acc[10]);
-                    acc[11] = __dp4a(static_cast<int>(t2), ww.w, acc[11]);
-                    acc[12] = __dp4a(static_cast<int>(t3), ww.x, acc[12]);
-                    acc[13] = __dp4a(static_cast<int>(t3), ww.y, acc[13]);
-                    acc[14] = __dp4a(static_cast<int>(t3), ww.z, acc[14]);
-                    acc[15] = __dp4a(static_cast<int>(t3), ww.w, acc[15]);
-                    kk = kn;
-                    ww = wn;
-                }
-                if (rs >= q_begin && re <= q_end) {
-                    store_tile<KIND>(w, a, m_first, r, acc);
-                } else {
-                    // Block-row shared with other groups: its slot is the first
-                    // split point inside it, b = ceil((rs - qa + 1) * H / qn).
-                    const long long d = rs - qa;
-                    const int b = static_cast<int>(((d + 1) * H + qn - 1) / qn);
-                    int* sl = slots + (b - 1) * SW + li;
+        for (int c = 0; c < kRingSlots; ++c) issue(c);
+
+        // Block-rows with no stored block: acc = 0.
+        for (int r = r_lo + warp; r < r_hi; r += kWarps) {
+            if (qp(r) == qp(r + 1)) {
+                int red[TPG * 4];
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) atomicAdd(sl + i * GL, acc[i]);
-                }
-                while (r < r_hi && __ldg(w.qptr + r + 1) <= q) ++r;
+                for (int j = 0; j < TPG * 4; ++j) red[j] = 0;
+                store_rows<KIND, TPG>(w, a, m_lane, r, red, load_s4(w.scale, r), load_s4(w.bias, r));
             }
         }
-        __syncthreads();
 
-        // Finish the shared block-rows: group h owns split point b = h + 1.
-        if (h < H - 1 && qn > 0) {
-            const int b = h + 1;
-            const int pb = qa + static_cast<int>(static_cast<long long>(b) * qn / H);
-            if (pb < qb) {
-                const int r = row_of(w.qptr, r_lo, r_hi, pb);
-                const int rs = __ldg(w.qptr + r);
-                if (rs < pb) {
-                    const long long d = rs - qa;
-                    const int bf = static_cast<int>(((d + 1) * H + qn - 1) / qn);
-                    if (bf == b) {
-                        int acc[16];
-                        const int* sl = slots + (b - 1) * SW + li;
+        if (TMA && stage) {
+            const bool ok = mbar_wait(bar, phase & 1u);
+            ++phase;
+            if (__syncthreads_or(!ok)) {
+                if (tid == 0) {
+                    atomicOr(w.status, kStatusTimeout);
+                    mbar_wait(bar, (phase - 1) & 1u);  // give the copy one more bounded chance to land
+                }
+                cp_async_wait<0>();
+                __syncthreads();
+                return;
+            }
+            staged = t;
+        }
+
+        if (wq0 < wq1) {
+            cp_async_wait<kRingSlots - 1>();  // chunk 0 has landed
+            __syncwarp();
+            int cur = 0;
+            int r = row_of_q(wq0);
+            int p = 0;  // step index relative to ws0
+            const int p_all = ws1 - ws0;
+            while (p < p_all) {
+                const int rs = qp(r), re_row = qp(r + 1);
+                const int p_end = min(p_all, (re_row - wq0) / G);
+                float4 sc = make_float4(0.f, 0.f, 0.f, 0.f), bi = sc;
+                if (KIND != 0) {  // needed at the row's end; load it now
+                    sc = load_s4(w.scale, r);
+                    bi = load_s4(w.bias, r);
+                }
+                int acc[32];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) acc[i] = sl[i * GL];
-                        store_tile<KIND>(w, a, m_first, r, acc);
+                for (int i = 0; i < 32; ++i) acc[i] = 0;
+                while (p < p_end) {
+                    const int cq = p / S;
+                    if (cq != cur) {  // entering the next chunk (cq == cur + 1)
+                        cur = cq;
+                        __syncwarp();  // everyone is done with chunk cur - 1, whose slot is refilled
+                        issue(cur + kRingSlots - 1);
+                        cp_async_wait<kRingSlots - 1>();  // chunk cur has landed
+                        __syncwarp();
+                    }
+                    const int seg_end = min(p_end, (cur + 1) * S);
+                    uint32_t rec = ring_s + (cur % kRingSlots) * (RC * kRec) + ((p - cur * S) * G + g) * kRec;
+                    for (; p + 1 < seg_end; p += 2, rec += 2 * G * kRec) {
+                        const int4 k0 = lds128(rec), w0 = lds128(rec + 16);
+                        const int4 k1 = lds128(rec + G * kRec), w1 = lds128(rec + G * kRec + 16);
+                        quad8<MT>(xlane, k0, w0, acc);
+                        quad8<MT>(xlane, k1, w1, acc);
+                    }
+                    if (p < seg_end) {
+                        const int4 k0 = lds128(rec), w0 = lds128(rec + 16);
+                        quad8<MT>(xlane, k0, w0, acc);
+                        ++p;
                     }
                 }
-            }
-        }
-        // Block-rows with no stored block: acc = 0.
-        for (int r = r_lo + h; r < r_hi; r += H) {
-            if (__ldg(w.qptr + r) == __ldg(w.qptr + r + 1)) {
-                int acc[16];
+                int red[TPG * 4];
+                reduce_groups<G>(lane, acc, red);
+                if (rs >= wq0 && re_row <= wq1) {
+                    store_rows<KIND, TPG>(w, a, m_lane, r, red, sc, bi);
+                } else {
+                    // Shared with other warps: sum into the slot of the first warp
+                    // split inside the block-row; the last warp to add finishes it.
+                    const int s0 = (rs - qa) / G, s1 = (re_row - qa) / G;  // the row's steps
+                    const int b = static_cast<int>((static_cast<long long>(s0 + 1) * kWarps + nst - 1) / nst);
+                    int* sl = slots + (b - 1) * SW + li;
 #pragma unroll
-                for (int i = 0; i < 16; ++i) acc[i] = 0;
-                store_tile<KIND>(w, a, m_first, r, acc);
+                    for (int j = 0; j < TPG * 4; ++j) atomicAdd(sl + (4 * i0 + j) * LW, red[j]);
+                    __syncwarp();
+                    int arrived = 0;
+                    if (lane == 0) {
+                        __threadfence_block();
+                        arrived = atomicAdd(&s_cnt[b - 1], 1) + 1;
+                    }
+                    arrived = __shfl_sync(0xffffffffu, arrived, 0);
+                    int parts = 0;  // warps whose step range meets the row's
+                    for (int wi = 0; wi < kWarps; ++wi) {
+                        const int a0 = wstep(wi), a1 = wstep(wi + 1);
+                        parts += (a0 < a1 && a0 < s1 && a1 > s0) ? 1 : 0;
+                    }
+                    if (arrived == parts) {
+                        __threadfence_block();
+#pragma unroll
+                        for (int j = 0; j < TPG * 4; ++j) red[j] = atomicExch(sl + (4 * i0 + j) * LW, 0);
+                        store_rows<KIND, TPG>(w, a, m_lane, r, red, sc, bi);
+                        if (lane == 0) s_cnt[b - 1] = 0;
+                    }
+                }
+                ++r;
+                while (r < r_hi && qp(r + 1) == qp(r)) ++r;  // skip block-rows without quads
             }
         }
-        __syncthreads();
+        cp_async_wait<0>();
+        __syncthreads();  // the tile, window, ring and slots may be reused
     }
 }
 
+// Token-tile relayout: xb[t][k][j] = x[t*MT + j][k] for k < kpad (zero when
+// t*MT + j >= M or k >= K).  One CTA moves MT tokens x KC columns (16 KB)
+// through shared memory: 16-byte row loads (4 in flight per thread), a 4x4
+// byte transpose per thread, 16-byte stores of the k-major block, which is
+// contiguous in xb.
 template <int MT>
+__global__ void __launch_bounds__(256)
+pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __restrict__ xb) {
+    constexpr int KC = 16384 / MT;     // columns per CTA (256 or 128)
+    constexpr int C16 = KC / 16;       // 16-byte chunks per raw row
+    constexpr int RW = KC / 4 + 4;     // raw row stride in words (rows shift by 4 banks)
+    constexpr int OS = MT / 4 + 1;     // transposed row stride in words
+    __shared__ __align__(16) uint32_t raw[MT * RW];
+    __shared__ uint32_t tr[KC * OS];
+    const long long t = blockIdx.x;
+    const int k0 = blockIdx.y * KC;
+    const long long m0 = t * MT;
+    const int kc = min(KC, kpad - k0);  // a multiple of 16
+    const bool vec16 = ((K & 15) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
+#pragma unroll
+    for (int i = 0; i < (MT * C16) / 256; ++i) {
+        const int c = i * 256 + threadIdx.x;
+        const int rho = c / C16, c16 = c % C16;
+        const long long m = m0 + rho;
+        const int k = k0 + 16 * c16;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (m < M && k < K) {
+            const int8_t* src = x + static_cast<size_t>(m) * K + k;
+            if (vec16) {
+                v = __ldg(reinterpret_cast<const uint4*>(src));
+            } else {
+                uint32_t wv[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                    if (k + e < K) wv[e >> 2] |= static_cast<uint32_t>(static_cast<uint8_t>(src[e])) << (8 * (e & 3));
+                v = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+            }
+        }
+        *reinterpret_cast<uint4*>(raw + rho * RW + 4 * c16) = v;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < (MT / 4) * (KC / 4); i += 256) {
+        const int j = i % (KC / 4), g = i / (KC / 4);
+        uint32_t t0, t1, t2, t3;
+        transpose4(raw[(4 * g + 0) * RW + j], raw[(4 * g + 1) * RW + j], raw[(4 * g + 2) * RW + j],
+                   raw[(4 * g + 3) * RW + j], t0, t1, t2, t3);
+        tr[(4 * j + 0) * OS + g] = t0;
+        tr[(4 * j + 1) * OS + g] = t1;
+        tr[(4 * j + 2) * OS + g] = t2;
+        tr[(4 * j + 3) * OS + g] = t3;
+    }
+    __syncthreads();
+    int8_t* dst = xb + (static_cast<size_t>(t) * kpad + k0) * MT;
+    for (int i = threadIdx.x; i < kc * (MT / 16); i += 256) {
+        const int row = i / (MT / 16), c = i % (MT / 16);
+        const uint32_t* srow = tr + row * OS + 4 * c;
+        *reinterpret_cast<uint4*>(dst + static_cast<size_t>(row) * MT + 16 * c) =
+            make_uint4(srow[0], srow[1], srow[2], srow[3]);
+    }
+}
+
+template <int MT, bool TMA>
 const void* kernel_for(int kind) {
     switch (kind) {
-    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 0>);
-    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 1>);
-    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 2>);
-    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 3>);
-    default: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 4>);
+    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 0, TMA>);
+    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 1, TMA>);
+    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 2, TMA>);
+    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 3, TMA>);
+    default: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 4, TMA>);
     }
 }
 
-const void* kernel_ptr(int MT, int kind) { return MT == 128 ? kernel_for<128>(kind) : kernel_for<64>(kind); }
+const void* kernel_ptr(int MT, int kind, bool tma) {
+    if (MT == 128) return tma ? kernel_for<128, true>(kind) : kernel_for<128, false>(kind);
+    return tma ? kernel_for<64, true>(kind) : kernel_for<64, false>(kind);
+}
 
 }  // namespace
 
 size_t smem_bytes(int MT, int K) {
     const size_t kpad = (static_cast<size_t>(K) + 15) & ~static_cast<size_t>(15);
-    return kpad * MT + static_cast<size_t>(groups_per_cta(MT) - 1) * slot_words(MT) * 4;
+    return kpad * MT + static_cast<size_t>(kSlots) * slot_words(MT) * 4 + ring_bytes(MT);
 }
 
 int tile_for_k(int K) {
     if (K < 1) return 0;
-    // static shared memory (the CTA's unit range) takes 16 bytes
-    if (smem_bytes(128, K) + 16 <= static_cast<size_t>(kSmemOptin)) return 128;
-    if (smem_bytes(64, K) + 16 <= static_cast<size_t>(kSmemOptin)) return 64;
+    if (smem_bytes(128, K) + kStaticSmem <= static_cast<size_t>(kSmemOptin)) return 128;
+    if (smem_bytes(64, K) + kStaticSmem <= static_cast<size_t>(kSmemOptin)) return 64;
     return 0;
 }
 
@@ -363,19 +653,23 @@ int max_k() {
 cudaError_t prepare_kernels(int MT, int K, int* ctas_per_sm) {
     const int smem = static_cast<int>(smem_bytes(MT, K));
     for (int kind = 0; kind < 5; ++kind) {
-        cudaError_t e = cudaFuncSetAttribute(kernel_ptr(MT, kind), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kSmemOptin - 16);
-        if (e != cudaSuccess) return e;
+        for (int tma = 0; tma < 2; ++tma) {
+            cudaError_t e = cudaFuncSetAttribute(kernel_ptr(MT, kind, tma != 0),
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemOptin - kStaticSmem);
+            if (e != cudaSuccess) return e;
+        }
     }
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_ptr(MT, 0), kThreads, smem);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_ptr(MT, 0, true), kThreads, smem);
 }
 
-cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, int MT, int grid, cudaStream_t s) {
-    const long long ntiles = (static_cast<long long>(a.M) + MT - 1) / MT;
-    const long long ctile = static_cast<long long>(w.Q) + w.nbr;  // cost[nbr]
+cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int MT, int grid,
+                   cudaStream_t s) {
     const size_t smem = smem_bytes(MT, w.K);
-#define BSG_LAUNCH(MTV, KV) \
-    bsgemm_kernel<MTV, KV><<<grid, kThreads, smem, s>>>(w, a, ntiles, ctile, grid)
+#define BSG_LAUNCH(MTV, KV)                                                                   \
+    do {                                                                                      \
+        if (a.xb) bsgemm_kernel<MTV, KV, true><<<grid, kThreads, smem, s>>>(w, a, sched);     \
+        else bsgemm_kernel<MTV, KV, false><<<grid, kThreads, smem, s>>>(w, a, sched);         \
+    } while (0)
     if (MT == 128) {
         switch (a.kind) {
         case 0: BSG_LAUNCH(128, 0); break;
@@ -394,6 +688,20 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, int MT, int grid
         }
     }
 #undef BSG_LAUNCH
+    return cudaGetLastError();
+}
+
+size_t tiled_bytes(int MT, int K, long long M) {
+    const size_t kpad = (static_cast<size_t>(K) + 15) & ~static_cast<size_t>(15);
+    return static_cast<size_t>((M + MT - 1) / MT) * kpad * MT;
+}
+
+cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, cudaStream_t s) {
+    const int kpad = (K + 15) & ~15;
+    const dim3 grid(static_cast<unsigned>((static_cast<long long>(M) + MT - 1) / MT),
+                    static_cast<unsigned>((kpad + 16384 / MT - 1) / (16384 / MT)));
+    if (MT == 128) pretile_kernel<128><<<grid, 256, 0, s>>>(x, M, K, kpad, xb);
+    else pretile_kernel<64><<<grid, 256, 0, s>>>(x, M, K, kpad, xb);
     return cudaGetLastError();
 }
 

@@ -39,10 +39,19 @@ def make_linear(bsg, wt):
     return bsg.SparseInt8Linear(wt.n_out, wt.k_in, wt.indptr, wt.colidx, wt.values, wt.scales, wt.bias)
 
 
-def gpu_run(lin, x: np.ndarray, kind: int, out_scale: float) -> np.ndarray:
-    out = lin(torch.from_numpy(x).cuda(), kind, out_scale)
+def gpu_run(lin, x: np.ndarray, kind: int, out_scale: float, workspace=None) -> np.ndarray:
+    """workspace=None: the two-kernel path (token-tile relayout + bulk-copy
+    staging); workspace=False: the single kernel without scratch memory."""
+    xd = torch.from_numpy(x).cuda()
+    dtype = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+             synth.I8: torch.int8, synth.I8_GELU: torch.int8}[kind]
+    out = torch.empty((x.shape[0], lin.n_out), dtype=dtype, device="cuda")
+    lin.run(xd, out, kind, out_scale, workspace=workspace)
     torch.cuda.synchronize()
     return out.cpu().numpy()
+
+
+PATHS = {"ws": None, "nows": False}
 
 
 # -------------------------------------------------- small, every element --
@@ -55,40 +64,43 @@ SMALL = [  # (n_out, k_in, m, sparsity, x_dist)
 ]
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("shape", SMALL, ids=lambda s: "x".join(map(str, s[:3])))
 @pytest.mark.parametrize("kind", KINDS, ids=lambda k: synth.KIND_NAMES[k])
-def test_small_all_elements(bsg, shape, kind):
+def test_small_all_elements(bsg, shape, kind, path):
     n, k, m, sp, dist = shape
     rng = synth.rng_for(1000 + n + k + m)
     wt = synth.draw_weight(rng, n, k, sp)
     x = synth.draw_x(rng, m, k, dist)
     lin = make_linear(bsg, wt)
-    got = gpu_run(lin, x, kind, 0.05)
+    got = gpu_run(lin, x, kind, 0.05, PATHS[path])
     want = oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
     check(got, want, kind, f"{shape}")
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("m", [1, 3, 63, 64, 65, 127, 128, 129, 257])
-def test_token_counts_span_tiles(bsg, m):
+def test_token_counts_span_tiles(bsg, m, path):
     for k in (768, 3072):
         rng = synth.rng_for(2000 + m + k)
         wt = synth.draw_weight(rng, 32, k, 0.85)
         x = synth.draw_x(rng, m, k, "u127")
         lin = make_linear(bsg, wt)
         want = oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I32)
-        check(gpu_run(lin, x, synth.I32, 1.0), want, synth.I32, f"m={m} k={k}")
+        check(gpu_run(lin, x, synth.I32, 1.0, PATHS[path]), want, synth.I32, f"m={m} k={k}")
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("k", [1, 3, 5, 17, 37, 100, 1001, 1536, 1537, 2049])
-def test_ragged_k(bsg, k):
-    """K not a multiple of 4/16/32 takes the byte-wise staging path."""
+def test_ragged_k(bsg, k, path):
+    """K not a multiple of 4/16/32 takes the byte-wise load paths."""
     rng = synth.rng_for(3000 + k)
     wt = synth.draw_weight(rng, 48, k, 0.5)
     x = synth.draw_x(rng, 77, k, "u127")
     lin = make_linear(bsg, wt)
     w = oracle.weight_dense(wt)
     for kind in (synth.I32, synth.I8_GELU):
-        check(gpu_run(lin, x, kind, 0.07), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.07),
+        check(gpu_run(lin, x, kind, 0.07, PATHS[path]), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.07),
               kind, f"k={k}")
 
 
@@ -176,39 +188,82 @@ def test_run_argument_errors(bsg):
         bsg.bsgemm_run(lin._h, x.data_ptr(), 4, raw.data_ptr() + 4, bsg.OUT_I32, 1.0)
 
 
-def test_misaligned_activations(bsg):
-    """An activation pointer that is not 16-byte aligned is still exact."""
-    rng = synth.rng_for(5400)
+@pytest.mark.parametrize("offset", [1, 3, 4, 8])
+def test_misaligned_activations(bsg, offset):
+    """An activation pointer that is not 16-byte aligned is still exact, on
+    both paths."""
+    rng = synth.rng_for(5400 + offset)
     wt = synth.draw_weight(rng, 32, 768, 0.9)
     x = synth.draw_x(rng, 100, 768, "u127")
     buf = torch.zeros(100 * 768 + 16, dtype=torch.int8, device="cuda")
-    buf[3:3 + 100 * 768] = torch.from_numpy(x.reshape(-1)).cuda()
+    buf[offset:offset + 100 * 768] = torch.from_numpy(x.reshape(-1)).cuda()
     lin = make_linear(bsg, wt)
+    want = oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I32)
+    stream = torch.cuda.current_stream().cuda_stream
     out = torch.empty((100, 32), dtype=torch.int32, device="cuda")
-    bsg.bsgemm_run(lin._h, buf.data_ptr() + 3, 100, out.data_ptr(), bsg.OUT_I32, 1.0,
-                   torch.cuda.current_stream().cuda_stream)
+    bsg.bsgemm_run(lin._h, buf.data_ptr() + offset, 100, out.data_ptr(), bsg.OUT_I32, 1.0, stream)
     torch.cuda.synchronize()
-    check(out.cpu().numpy(), oracle.linear(x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I32), synth.I32)
+    check(out.cpu().numpy(), want, synth.I32, "no workspace")
+    ws = torch.empty(lin.workspace_bytes(100), dtype=torch.uint8, device="cuda")
+    out.zero_()
+    bsg.bsgemm_run_ws(lin._h, buf.data_ptr() + offset, 100, out.data_ptr(), bsg.OUT_I32, 1.0, ws.data_ptr(),
+                      ws.numel(), stream)
+    torch.cuda.synchronize()
+    check(out.cpu().numpy(), want, synth.I32, "workspace")
 
 
-def test_guard_bands_and_determinism(bsg):
-    """Nothing is written outside out[M][N]; two runs are bit-identical."""
+def test_workspace_validation_and_status(bsg):
+    rng = synth.rng_for(5450)
+    wt = synth.draw_weight(rng, 64, 3072, 0.9)
+    lin = make_linear(bsg, wt)
+    m = 70
+    need = lin.workspace_bytes(m)
+    assert need == -(-m // lin.info["tile_m"]) * 3072 * lin.info["tile_m"]
+    x = torch.zeros((m, 3072), dtype=torch.int8, device="cuda")
+    out = torch.empty((m, 64), dtype=torch.int8, device="cuda")
+    ws = torch.empty(need + 16, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    with pytest.raises(bsg.BsgemmError):  # too small
+        bsg.bsgemm_run_ws(lin._h, x.data_ptr(), m, out.data_ptr(), bsg.OUT_I8, 0.05, ws.data_ptr(), need - 16, stream)
+    with pytest.raises(bsg.BsgemmError):  # misaligned
+        bsg.bsgemm_run_ws(lin._h, x.data_ptr(), m, out.data_ptr(), bsg.OUT_I8, 0.05, ws.data_ptr() + 8, need, stream)
+    with pytest.raises(bsg.BsgemmError):  # NULL
+        bsg.bsgemm_run_ws(lin._h, x.data_ptr(), m, out.data_ptr(), bsg.OUT_I8, 0.05, None, need, stream)
+    bsg.bsgemm_run_ws(lin._h, x.data_ptr(), m, out.data_ptr(), bsg.OUT_I8, 0.05, ws.data_ptr(), need, stream)
+    torch.cuda.synchronize()
+    assert bsg.bsgemm_device_status(lin._h) == 0
+
+
+@pytest.mark.parametrize("path", sorted(PATHS))
+def test_guard_bands_and_determinism(bsg, path):
+    """Nothing is written outside out[M][N] (nor outside the workspace); two
+    runs are bit-identical."""
     rng = synth.rng_for(5500)
     wt = synth.draw_weight(rng, 96, 3072, 0.9)
     m = 131
     x = torch.from_numpy(synth.draw_x(rng, m, 3072, "u0_127")).cuda()
     lin = make_linear(bsg, wt)
+    stream = torch.cuda.current_stream().cuda_stream
+    guard = 4096
+    need = lin.workspace_bytes(m)
+    wsraw = torch.full((guard * 2 + need,), 0x3C, dtype=torch.uint8, device="cuda")
+
+    def run(kind, ptr):
+        if path == "ws":
+            bsg.bsgemm_run_ws(lin._h, x.data_ptr(), m, ptr, kind, 0.05, wsraw.data_ptr() + guard, need, stream)
+        else:
+            bsg.bsgemm_run(lin._h, x.data_ptr(), m, ptr, kind, 0.05, stream)
+
     for kind, elem in ((synth.I8, 1), (synth.F32, 4)):
-        guard = 4096
         raw = torch.full((guard * 2 + m * 96 * elem,), 0x5A, dtype=torch.uint8, device="cuda")
-        bsg.bsgemm_run(lin._h, x.data_ptr(), m, raw.data_ptr() + guard, kind, 0.05,
-                       torch.cuda.current_stream().cuda_stream)
+        run(kind, raw.data_ptr() + guard)
         first = raw.clone()
-        bsg.bsgemm_run(lin._h, x.data_ptr(), m, raw.data_ptr() + guard, kind, 0.05,
-                       torch.cuda.current_stream().cuda_stream)
+        run(kind, raw.data_ptr() + guard)
         torch.cuda.synchronize()
         assert torch.equal(first, raw)
         assert bool((raw[:guard] == 0x5A).all()) and bool((raw[-guard:] == 0x5A).all())
+        assert bool((wsraw[:guard] == 0x3C).all()) and bool((wsraw[-guard:] == 0x3C).all())
+    assert bsg.bsgemm_device_status(lin._h) == 0
 
 
 def test_one_handle_many_streams(bsg):
@@ -263,19 +318,20 @@ def sample_rows(m: int, tile: int, seed: int, n_random: int = 40) -> np.ndarray:
     return np.array(sorted(rows))
 
 
+@pytest.mark.parametrize("path", sorted(PATHS))
 @pytest.mark.parametrize("case_fn", [synth.single_768, synth.ffn1, synth.ffn2], ids=lambda f: f.__name__)
-def test_full_size_workloads(bsg, case_fn):
+def test_full_size_workloads(bsg, case_fn, path):
     case = case_fn()
     wt = case.weight
     lin = make_linear(bsg, wt)
-    got = gpu_run(lin, case.x, case.kind, case.out_scale)
+    got = gpu_run(lin, case.x, case.kind, case.out_scale, PATHS[path])
     rows = sample_rows(case.m, lin.info["tile_m"], 7)
     want = oracle.linear(case.x, oracle.weight_dense(wt), wt.scales, wt.bias, case.kind,
                          out_scale=case.out_scale, rows=rows, threads=8)
     check(got[rows], want, case.kind, case.name)
     if case.kind in (synth.I8, synth.I8_GELU):
         # also the int32 accumulators, on the same rows
-        acc = gpu_run(lin, case.x, synth.I32, 1.0)
+        acc = gpu_run(lin, case.x, synth.I32, 1.0, PATHS[path])
         check(acc[rows], oracle.linear(case.x, oracle.weight_dense(wt), wt.scales, wt.bias, synth.I32,
                                        rows=rows, threads=8), synth.I32, case.name + " acc")
 
