@@ -132,6 +132,30 @@ int bsgemm_run_ws(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilog
                   size_t workspace_bytes, void* stream);
 
 /*
+ * bsgemm_run_static -- bsgemm_run_ws without a caller workspace and without
+ * any allocation: the token tiles go to a fixed scratch array of
+ * BSGEMM_STATIC_SCRATCH_BYTES (16 MiB) that the library holds in device
+ * memory, one per device.  The paper has no counterpart; this entry point
+ * serves callers that must not allocate at run time.
+ *   Limit: bsgemm_workspace_bytes(h, M) <= BSGEMM_STATIC_SCRATCH_BYTES,
+ *   i.e. M <= floor(16 MiB / (round_up(K, 16) * T)) * T tokens
+ *   (T = bsgemm_info()[4]; M <= 5440 at K = 3072, M <= 21760 at K = 768).
+ *   A larger M returns BSGEMM_ERR_INVALID (use bsgemm_run_ws).
+ *   Set-up: the first call on each device looks up the scratch array's
+ *   address (cudaGetSymbolAddress) with that device current and caches it;
+ *   make that first call before any stream capture.
+ *   Races: every call on a device uses the same scratch, whatever the
+ *   handle, stream or thread.  Two calls whose kernels overlap in time race
+ *   and give undefined output; serialise them (one stream, or events).
+ *   Nothing has to start at zero: each run writes every scratch byte it
+ *   reads.
+ * Results, return codes, asynchrony and the other arguments are those of
+ * bsgemm_run_ws.
+ */
+#define BSGEMM_STATIC_SCRATCH_BYTES (16u << 20)
+int bsgemm_run_static(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream);
+
+/*
  * The two steps of bsgemm_run_ws, for callers that keep activations in the
  * token-tiled layout between layers or time the steps apart:
  *   bsgemm_tile_activations -- act [M][K] (DEVICE) -> token tiles in

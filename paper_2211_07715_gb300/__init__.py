@@ -26,6 +26,7 @@ LIB_PATH = os.path.join(_PKG, "libbsgemm.so")
 BLOCK = 4
 OUT_I32, OUT_F32, OUT_F32_GELU, OUT_I8, OUT_I8_GELU = 0, 1, 2, 3, 4
 ERR_INVALID, ERR_UNSUPPORTED, ERR_CUDA = -1, -2, -3
+STATIC_SCRATCH_BYTES = 16 << 20  # BSGEMM_STATIC_SCRATCH_BYTES: the token-tile scratch of bsgemm_run_static
 
 
 class BsgemmError(RuntimeError):
@@ -61,6 +62,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_workspace_bytes.restype = ctypes.c_size_t
     lib.bsgemm_run_ws.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp, ctypes.c_size_t, vp]
     lib.bsgemm_run_ws.restype = ctypes.c_int
+    lib.bsgemm_run_static.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp]
+    lib.bsgemm_run_static.restype = ctypes.c_int
     lib.bsgemm_tile_activations.argtypes = [vp, vp, ctypes.c_int, vp, ctypes.c_size_t, vp]
     lib.bsgemm_tile_activations.restype = ctypes.c_int
     lib.bsgemm_run_tiled.argtypes = [vp, vp, ctypes.c_size_t, ctypes.c_int, vp, Epilogue, vp]
@@ -72,9 +75,9 @@ def _load() -> ctypes.CDLL:
 
 _lib = _load()
 
-EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_workspace_bytes", "bsgemm_tile_activations",
-            "bsgemm_run_tiled", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status",
-            "bsgemm_max_k", "bsgemm_info")
+EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
+            "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
+            "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
 
 
 def bsgemm_last_error() -> str:
@@ -121,6 +124,15 @@ def bsgemm_run_ws(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_sca
     """Enqueue the two-kernel fast path with a device workspace; raises on failure."""
     rc = _lib.bsgemm_run_ws(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), ws_ptr,
                             int(ws_bytes), stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_run_static(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float = 1.0,
+                      stream: int = 0) -> None:
+    """The fast path with the library's fixed device scratch: allocates
+    nothing; calls overlapping in time on one device race (see the header)."""
+    rc = _lib.bsgemm_run_static(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 

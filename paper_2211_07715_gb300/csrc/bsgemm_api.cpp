@@ -320,6 +320,33 @@ int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, v
     return run_common(h, nullptr, M, out, epi, const_cast<void*>(tiles), tiles_bytes, 2, stream);
 }
 
+int bsgemm_run_static(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream) {
+    clear_error();
+    if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
+    if (M > 0) {
+        const size_t need = bsg::tiled_bytes(h->MT, h->w.K, M);
+        if (need > BSGEMM_STATIC_SCRATCH_BYTES) {
+            const size_t per_tile = bsg::tiled_bytes(h->MT, h->w.K, h->MT);
+            const long long m_max = static_cast<long long>(BSGEMM_STATIC_SCRATCH_BYTES / per_tile) * h->MT;
+            return fail(BSGEMM_ERR_INVALID, "M = " + std::to_string(M) + " needs " + std::to_string(need) +
+                                                " bytes of token tiles; the static scratch holds " +
+                                                std::to_string(static_cast<size_t>(BSGEMM_STATIC_SCRATCH_BYTES)) +
+                                                " (M <= " + std::to_string(m_max) + " at K = " +
+                                                std::to_string(h->w.K) + "): use bsgemm_run_ws");
+        }
+    }
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
+    if (dev != h->device)
+        return fail(BSGEMM_ERR_INVALID, "current device " + std::to_string(dev) + " is not the handle's device " +
+                                            std::to_string(h->device));
+    int8_t* scratch = nullptr;
+    e = bsg::static_scratch(dev, &scratch);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetSymbolAddress (static scratch)", e));
+    return run_common(h, act, M, out, epi, scratch, BSGEMM_STATIC_SCRATCH_BYTES, 1, stream);
+}
+
 int bsgemm_tile_activations(bsgemm_t h, const int8_t* act, int M, void* tiles, size_t tiles_bytes, void* stream) {
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");

@@ -69,5 +69,9 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
                    cudaStream_t s);
 // x [M][K] -> token tiles [ntiles][kpad][MT] in xb (the layout the kernel stages by TMA).
 cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, cudaStream_t s);
+// Address of the fixed token-tile scratch (BSGEMM_STATIC_SCRATCH_BYTES) on
+// `device`, which must be the current device; looked up on the first call
+// per device, then cached.
+cudaError_t static_scratch(int device, int8_t** ptr);
 
 }  // namespace bsg

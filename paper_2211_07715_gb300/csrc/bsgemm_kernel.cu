@@ -40,8 +40,10 @@
 //   and bias, optional GELU by a fixed fp32 op sequence (A&S 7.1.28 erf),
 //   optional requantise (fp32 multiply, round half to even, saturate).
 #include <cstdint>
+#include <mutex>
 #include <cuda_runtime.h>
 
+#include "bsgemm.h"
 #include "bsgemm_internal.h"
 
 namespace bsg {
@@ -703,6 +705,34 @@ cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, cu
     if (MT == 128) pretile_kernel<128><<<grid, 256, 0, s>>>(x, M, K, kpad, xb);
     else pretile_kernel<64><<<grid, 256, 0, s>>>(x, M, K, kpad, xb);
     return cudaGetLastError();
+}
+
+}  // namespace bsg
+
+// Token-tile scratch of bsgemm_run_static: one fixed array per device, so
+// that entry point allocates nothing.  Every byte a run reads from it is
+// written by the relayout kernel of the same run (tokens past M and columns
+// past K as zeros), so nothing in it has to start at zero.
+static __device__ __align__(256) int8_t g_static_tiles[BSGEMM_STATIC_SCRATCH_BYTES];
+
+namespace bsg {
+
+cudaError_t static_scratch(int device, int8_t** ptr) {
+    constexpr int kMaxDevices = 64;
+    static std::mutex mu;
+    static int8_t* addr[kMaxDevices] = {};
+    if (device < 0 || device >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[device]) {
+        // Resolved once per device, with that device current (the caller
+        // checks): the address of this module's copy in its context.
+        void* p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_static_tiles);
+        if (e != cudaSuccess) return e;
+        addr[device] = static_cast<int8_t*>(p);
+    }
+    *ptr = addr[device];
+    return cudaSuccess;
 }
 
 }  // namespace bsg
