@@ -7,6 +7,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -22,6 +23,10 @@ struct bsgemm_ctx {
     size_t arena_bytes = 0;
     std::vector<int32_t> cost;  // host copy of the schedule's prefix cost [nbr + 1]
     bsg::DeviceWeights w{};
+    std::mutex sched_mu;        // guards the cached schedule of the last token count
+    long long sched_m = -1;
+    int sched_grid = 0;
+    bsg::Schedule sched{};
 };
 
 namespace {
@@ -63,6 +68,65 @@ std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx
         }
     }
     return "";
+}
+
+// Schedule cost of one token tile in a CTA's range, in quads: a CTA holds
+// one tile in shared memory, so every further tile in its range costs a
+// copy-in and the start-up around it.  1000 quads (a few microseconds of a
+// CTA's work) gave the shortest layer kernels on GB300 in a sweep over
+// 0-4000 at K = 3072 and K = 768.
+constexpr long long kTileCost = 1000;
+
+// End of the greedy range that starts at unit u under the cost bound C: it
+// takes whole units while the cost (units' cost + tc per token tile
+// touched) stays within C, and at least one unit.
+long long fill_range(const std::vector<int32_t>& cost, long long nbr, long long ntiles, long long tc, long long C,
+                     long long u) {
+    long long t = u / nbr, r = u - t * nbr, left = C;
+    bool first = true;
+    while (t < ntiles) {
+        left -= tc;
+        const long long rest = cost[nbr] - cost[r];
+        if (left >= rest) {  // the rest of this tile fits
+            left -= rest;
+            ++t;
+            r = 0;
+            first = false;
+            continue;
+        }
+        // the largest e with cost[e] - cost[r] <= left
+        long long e = std::upper_bound(cost.begin() + r, cost.begin() + nbr + 1, cost[r] + (left > 0 ? left : 0)) -
+                      cost.begin() - 1;
+        if (e <= r && first) e = r + 1;  // at least one unit
+        return t * nbr + (e > r ? e : r);
+    }
+    return ntiles * nbr;
+}
+
+// Contiguous unit ranges (tile-major units t * nbr + r), one per CTA, with
+// the largest range cost as small as bisection on the bound finds it;
+// returns the number of ranges (<= cap, each non-empty).
+int make_schedule(const std::vector<int32_t>& cost, long long nbr, long long ntiles, int cap, long long tc,
+                  bsg::Schedule& sched) {
+    const long long end = ntiles * nbr;
+    auto ranges = [&](long long C) {
+        int n = 0;
+        for (long long u = 0; u < end; u = fill_range(cost, nbr, ntiles, tc, C, u))
+            if (++n > cap) break;
+        return n;
+    };
+    long long hi = ntiles * (cost[nbr] + tc), lo = 0;
+    while (hi - lo > 1) {
+        const long long mid = lo + (hi - lo) / 2;
+        if (ranges(mid) <= cap) hi = mid; else lo = mid;
+    }
+    int n = 0;
+    sched.u[0] = 0;
+    for (long long u = 0; u < end;) {
+        u = fill_range(cost, nbr, ntiles, tc, hi, u);
+        sched.u[++n] = u;
+    }
+    return n;
 }
 
 }  // namespace
@@ -282,20 +346,18 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
     const long long ntiles = (static_cast<long long>(M) + h->MT - 1) / h->MT;
     const long long nbr = h->w.nbr;
-    const long long units = ntiles * nbr;
     long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
     if (cap > bsg::kMaxGrid) cap = bsg::kMaxGrid;
-    const int grid = static_cast<int>(units < cap ? units : cap);
-    // Cost-balanced contiguous unit ranges: CTA c starts at the first unit
-    // whose start cost t * ctile + cost[r] reaches c * total / grid.
     bsg::Schedule sched;
-    const long long ctile = h->cost[nbr];
-    const __int128 total = static_cast<__int128>(ntiles) * ctile;
-    for (int c = 0; c <= grid; ++c) {
-        const long long target = static_cast<long long>(total * c / grid);
-        const long long t = target / ctile, rem = target - t * ctile;
-        const long long r = std::lower_bound(h->cost.begin(), h->cost.begin() + nbr, rem) - h->cost.begin();
-        sched.u[c] = t * nbr + r;
+    int grid = 0;
+    {
+        std::lock_guard<std::mutex> lock(h->sched_mu);
+        if (h->sched_m != M) {
+            h->sched_grid = make_schedule(h->cost, nbr, ntiles, static_cast<int>(cap), kTileCost, h->sched);
+            h->sched_m = M;
+        }
+        grid = h->sched_grid;
+        std::memcpy(sched.u, h->sched.u, sizeof(long long) * (grid + 1));
     }
     if (mode == 1) {
         e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(workspace), s);
