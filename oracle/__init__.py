@@ -205,3 +205,94 @@ def block_prune(w: np.ndarray, sparsity: float) -> np.ndarray:
     keep = np.empty((n_out // BLOCK, k_in), dtype=np.uint8)
     lib.oracle_block_prune(n_out, k_in, _ptr(w, ctypes.c_float), float(sparsity), _ptr(keep, ctypes.c_uint8))
     return keep.astype(bool)
+
+
+# ------------------------------------------------------------------ encoder layer chain --
+# The layer chain of the DistilBERT encoder: QKV, attention, output
+# projection, FFN1 (+GELU), FFN2, int8 between the linears (Sec. 3; the
+# paper's engine quantises every linear, Sec. 2).  Attention itself is not
+# part of the sparse linear; it is the plain reference step below, run on
+# the host between the QKV and output linears of both chains.  Residual
+# connections and LayerNorm are omitted.
+
+HEADS = 12
+
+
+def requant_f32(y: np.ndarray, out_scale) -> np.ndarray:
+    """fp32 -> int8: multiply by the fp32 reciprocal of the scale, round half
+    to even, saturate -- the same requantisation as the linears' epilogue."""
+    inv = np.float32(1.0) / np.float32(out_scale)
+    t = (np.asarray(y, dtype=np.float32) * inv).astype(np.float32)
+    return np.clip(np.rint(t), -128, 127).astype(np.int8)
+
+
+def attention_f32(qkv: np.ndarray, qkv_scale, batch: int, seq: int, heads: int = HEADS) -> np.ndarray:
+    """Multi-head self-attention in fp32 on an int8 QKV output [M][3d],
+    M = batch x seq: q, k, v are its dequantised thirds (int8 x qkv_scale);
+    per sequence and head (d / heads wide) P = softmax(q k^T / sqrt(d /
+    heads)) with the row maximum subtracted, context = P v.  Returns the
+    context [M][d] in fp32."""
+    m, d3 = qkv.shape
+    assert m == batch * seq and d3 % 3 == 0
+    d = d3 // 3
+    hd = d // heads
+    x = qkv.astype(np.float32) * np.float32(qkv_scale)
+
+    def split(part):  # [M][d] -> [batch][heads][seq][hd]
+        return np.ascontiguousarray(part.reshape(batch, seq, heads, hd).transpose(0, 2, 1, 3))
+
+    q, k, v = split(x[:, :d]), split(x[:, d:2 * d]), split(x[:, 2 * d:])
+    s = np.matmul(q, k.transpose(0, 1, 3, 2)) * np.float32(1.0 / np.sqrt(hd))
+    s = s - s.max(axis=-1, keepdims=True)
+    p = np.exp(s, dtype=np.float32)
+    p = p / p.sum(axis=-1, keepdims=True, dtype=np.float32)
+    ctx = np.matmul(p, v)  # [batch][heads][seq][hd]
+    return np.ascontiguousarray(ctx.transpose(0, 2, 1, 3).reshape(m, d)).astype(np.float32)
+
+
+def attention(qkv: np.ndarray, qkv_scale, batch: int, seq: int, ctx_scale, heads: int = HEADS) -> np.ndarray:
+    """attention_f32, requantised to int8 with ctx_scale."""
+    return requant_f32(attention_f32(qkv, qkv_scale, batch, seq, heads), ctx_scale)
+
+
+CHAIN_STAGES = ("qkv", "ctx", "attn_out", "ffn1", "ffn2")
+
+
+def layer_chain(x0: np.ndarray, weights, out_scales: dict, batch: int, seq: int, threads: int = 8) -> dict:
+    """The int8 outputs of every stage of one encoder layer for input x0
+    [M][768]; weights = the four linears' BsrWeight (QKV, attention output,
+    FFN1, FFN2), out_scales = the frozen output scales per stage."""
+    wq, wo, w1, w2 = weights
+    dense = [weight_dense(w) for w in weights]
+    out = {}
+    out["qkv"] = linear(x0, dense[0], wq.scales, wq.bias, I8, out_scales["qkv"], threads=threads)
+    out["ctx"] = attention(out["qkv"], out_scales["qkv"], batch, seq, out_scales["ctx"])
+    out["attn_out"] = linear(out["ctx"], dense[1], wo.scales, wo.bias, I8, out_scales["attn_out"], threads=threads)
+    out["ffn1"] = linear(out["attn_out"], dense[2], w1.scales, w1.bias, I8_GELU, out_scales["ffn1"], threads=threads)
+    out["ffn2"] = linear(out["ffn1"], dense[3], w2.scales, w2.bias, I8, out_scales["ffn2"], threads=threads)
+    return out
+
+
+def calibrate_chain(x0: np.ndarray, weights, batch: int, seq: int, threads: int = 8) -> dict:
+    """Post-training calibration of the chain's output scales: each stage's
+    scale is max |y| / 127 (in fp32) of its unquantised output y on these
+    inputs, stage by stage, so that every stage sees the int8 input the
+    chain will give it."""
+    wq, wo, w1, w2 = weights
+    dense = [weight_dense(w) for w in weights]
+
+    def scale_of(y) -> float:
+        return float(np.float32(np.max(np.abs(y))) / np.float32(127.0))
+
+    s = {}
+    s["qkv"] = scale_of(linear(x0, dense[0], wq.scales, wq.bias, F32, threads=threads))
+    qkv = linear(x0, dense[0], wq.scales, wq.bias, I8, s["qkv"], threads=threads)
+    ctx_f = attention_f32(qkv, s["qkv"], batch, seq)
+    s["ctx"] = scale_of(ctx_f)
+    ctx = requant_f32(ctx_f, s["ctx"])
+    s["attn_out"] = scale_of(linear(ctx, dense[1], wo.scales, wo.bias, F32, threads=threads))
+    o = linear(ctx, dense[1], wo.scales, wo.bias, I8, s["attn_out"], threads=threads)
+    s["ffn1"] = scale_of(linear(o, dense[2], w1.scales, w1.bias, F32_GELU, threads=threads))
+    f1 = linear(o, dense[2], w1.scales, w1.bias, I8_GELU, s["ffn1"], threads=threads)
+    s["ffn2"] = scale_of(linear(f1, dense[3], w2.scales, w2.bias, F32, threads=threads))
+    return s
