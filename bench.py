@@ -380,13 +380,241 @@ def run_reference(args, rank: int) -> dict | None:
     }
 
 
+# ---------------------------------------------- encoder-layer chain and stack --
+
+LAYER_SCALES = os.path.join(ROOT, "tests", "golden", "layer_scales.json")
+
+
+def _layer_linears(bsg, weights):
+    return [bsg.SparseInt8Linear(w.n_out, w.k_in, w.indptr, w.colidx, w.values, w.scales, w.bias) for w in weights]
+
+
+def _peak_tops(props, max_mhz) -> float:
+    return props.multi_processor_count * DP4A_LANES_PER_SM_CLK * OPS_PER_DP4A * max_mhz * 1e6 / 1e12
+
+
+class _Chain:
+    """One encoder layer's four linears on the device, back to back on one
+    stream through the C ABI (relayout + layer kernel each): QKV on the
+    layer input, the attention output on a context buffer (the attention
+    step itself is outside the timed path), FFN1 + GELU on its result, FFN2
+    on FFN1's.  int8 everywhere, frozen calibrated output scales."""
+
+    def __init__(self, bsg, torch, dev, weights, m: int, scales: dict):
+        self.bsg, self.torch, self.m = bsg, torch, m
+        self.lins = _layer_linears(bsg, weights)
+        self.weights = weights
+        self.scales = [scales["qkv"], scales["attn_out"], scales["ffn1"], scales["ffn2"]]
+        self.kinds = [synth.I8, synth.I8, synth.I8_GELU, synth.I8]
+        ws = max(l.workspace_bytes(m) for l in self.lins)
+        self.ws = torch.empty(ws, dtype=torch.uint8, device=dev)
+        self.ws_bytes = ws
+
+    def buffers(self, dev):
+        t = self.torch
+        return {"qkv": t.empty((self.m, 2304), dtype=t.int8, device=dev),
+                "o": t.empty((self.m, 768), dtype=t.int8, device=dev),
+                "f1": t.empty((self.m, 3072), dtype=t.int8, device=dev),
+                "f2": t.empty((self.m, 768), dtype=t.int8, device=dev)}
+
+    def linear(self, i, x, out, stream, ev=None):
+        bsg = self.bsg
+        lin = self.lins[i]
+        bsg.bsgemm_tile_activations(lin._h, x.data_ptr(), self.m, self.ws.data_ptr(), self.ws_bytes, stream)
+        if ev is not None:
+            ev[0].record()
+        bsg.bsgemm_run_tiled(lin._h, self.ws.data_ptr(), self.ws_bytes, self.m, out.data_ptr(), self.kinds[i],
+                             self.scales[i], stream)
+        if ev is not None:
+            ev[1].record()
+
+    def run(self, x, ctx, b, stream, evs=None):
+        self.linear(0, x, b["qkv"], stream, None if evs is None else evs[0])
+        self.linear(1, ctx, b["o"], stream, None if evs is None else evs[1])
+        self.linear(2, b["o"], b["f1"], stream, None if evs is None else evs[2])
+        self.linear(3, b["f1"], b["f2"], stream, None if evs is None else evs[3])
+        return b["f2"]
+
+    def ops(self):
+        return [2.0 * self.m * w.nnzb * 4 for w in self.weights]
+
+    def close(self):
+        for lin in self.lins:
+            lin.close()
+
+
+def run_layer(args) -> dict:
+    """cfg 4: one encoder layer's four linears chained on the device,
+    M = 8 x 384 tokens, 80% block sparsity."""
+    import torch
+    import paper_2211_07715_gb300 as bsg
+
+    dev = torch.device("cuda", 0)
+    props = torch.cuda.get_device_properties(dev)
+    with open(LAYER_SCALES) as f:
+        scales = json.load(f)["scales"]
+    weights, x0 = synth.encoder_layer()
+    m = x0.shape[0]
+    ctx_host = synth.draw_x(synth.rng_for(synth.SEED_BASE + 3 + 7), m, 768, "u127")
+    chain = _Chain(bsg, torch, dev, weights, m, scales)
+    set_bytes = m * (768 + 768 + 2304 + 768 + 3072 + 768)
+    nsets = max(2, math.ceil(2 * int(getattr(props, "L2_cache_size", 128 << 20)) / set_bytes) + 1)
+    xs = [torch.from_numpy(x0).to(dev) for _ in range(nsets)]
+    ctxs = [torch.from_numpy(ctx_host).to(dev) for _ in range(nsets)]
+    bufs = [chain.buffers(dev) for _ in range(nsets)]
+    stream = torch.cuda.current_stream(dev)
+    sh = stream.cuda_stream
+    for i in range(args.warmup):
+        chain.run(xs[i % nsets], ctxs[i % nsets], bufs[i % nsets], sh)
+    torch.cuda.synchronize(dev)
+    sampler = ClockSampler(str(getattr(props, "uuid", "")))
+    sampler.start()
+    time.sleep(0.3)
+    mark0 = sampler.mark()
+    steps = args.steps
+    evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(4)] for _ in range(steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(steps):
+        chain.run(xs[i % nsets], ctxs[i % nsets], bufs[i % nsets], sh, evs[i])
+    end.record(stream)
+    end.synchronize()
+    mark1 = sampler.mark()
+    time.sleep(0.2)
+    sampler.stop()
+    clocks = sampler.summary(mark0, max(mark1, mark0 + 1))
+    ms = start.elapsed_time(end) / steps
+    ops = chain.ops()
+    kern_ms = [statistics.fmean(evs[i][j][0].elapsed_time(evs[i][j][1]) for i in range(steps)) for j in range(4)]
+    peak = _peak_tops(props, clocks.get("sm_max_mhz") or 2070.0)
+    names = ["qkv", "attn_out", "ffn1", "ffn2"]
+    per = {n: {"kernel_ms": round(k, 6), "tops": round(o / (k * 1e-3) / 1e12, 3),
+               "frac": round(o / (k * 1e-3) / 1e12 / peak, 4)} for n, k, o in zip(names, kern_ms, ops)}
+    kernel_tops = sum(ops) / (sum(kern_ms) * 1e-3) / 1e12
+    chain.close()
+    return {
+        "metric": METRIC, "value": round(sum(ops) / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "n_gpus": 1,
+        "steps": steps, "warmup": args.warmup, "ms_per_step": round(ms, 6), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "s8", "data": "synthetic",
+        "config": {"workload": "encoder layer chain: QKV 768->2304, attention output 768->768, FFN1 768->3072 + GELU, "
+                               "FFN2 3072->768; int8 between (frozen calibrated scales); attention replaced in the "
+                               "timed path by a seeded int8 context buffer",
+                   "tokens": m, "batch": 8, "seq": 384, "sparsity": 0.8,
+                   "l2": f"rotating {nsets} input/output sets ({nsets * set_bytes / 2**20:.0f} MiB > 2 x L2)"},
+        "tokens_per_s": round(m / (ms * 1e-3), 1),
+        "roofline": {"bound": "alu", "achieved": round(kernel_tops, 3), "peak": round(peak, 2), "unit": "TOPS",
+                     "frac": round(kernel_tops / peak, 4), "traffic": None, "kernel": "bsgemm_kernel (4 linears)"},
+        "per_linear": per, "gpu_launches": 8 * steps, "clocks": clocks, "kernel_source_sha256": kernel_sha(),
+    }
+
+
+def run_stack(args) -> dict:
+    """cfg 5: the six-layer stack of 24 sparse linears swept over batch
+    {1, 8, 32, 128} x seq {128, 384} x sparsity {70, 80, 90}%.  One pass =
+    24 linears (48 launches) back to back on one stream, the attention step
+    replaced by a seeded int8 context buffer; also replayed as one CUDA
+    graph.  Tokens/s = M / pass time."""
+    import torch
+    import paper_2211_07715_gb300 as bsg
+
+    dev = torch.device("cuda", 0)
+    props = torch.cuda.get_device_properties(dev)
+    with open(LAYER_SCALES) as f:
+        scales = json.load(f)["scales"]
+    peak = _peak_tops(props, 2070.0)
+    reps = max(3, min(args.steps, 20))
+    points = []
+    sampler = ClockSampler(str(getattr(props, "uuid", "")))
+    sampler.start()
+    time.sleep(0.3)
+    mark0 = sampler.mark()
+    for pi, (batch, seq, sp) in enumerate(synth.STACK_POINTS):
+        layers, x0, ctx0 = synth.stack_point(batch, seq, sp, pi)
+        m = batch * seq
+        chains = [_Chain(bsg, torch, dev, w, m, scales) for w in layers]
+        x = torch.from_numpy(x0).to(dev)
+        ctx = torch.from_numpy(ctx0).to(dev)
+        b = chains[0].buffers(dev)
+        stream = torch.cuda.current_stream(dev)
+
+        def stack_pass(sh, evs=None):
+            h = x
+            for li, c in enumerate(chains):
+                # the next layer's QKV reads this layer's FFN2 output (b["f2"]) before its own FFN2
+                # overwrites it: one stream, so one buffer set serves all six layers
+                h = c.run(h, ctx, b, sh, None if evs is None else evs[li])
+            return h
+
+        for _ in range(3):
+            stack_pass(stream.cuda_stream)
+        torch.cuda.synchronize(dev)
+        # per-linear kernel times on one instrumented pass
+        evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(4)] for _ in chains]
+        stack_pass(stream.cuda_stream, evs)
+        torch.cuda.synchronize(dev)
+        kern = [[evs[l][j][0].elapsed_time(evs[l][j][1]) for l in range(len(chains))] for j in range(4)]
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            stack_pass(stream.cuda_stream)
+        e1.record(stream)
+        e1.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        # the same pass captured once as a CUDA graph
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(stream)
+        with torch.cuda.graph(g, stream=side):
+            stack_pass(side.cuda_stream)
+        torch.cuda.synchronize(dev)
+        for _ in range(2):
+            g.replay()
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+        e1.synchronize()
+        ms_graph = e0.elapsed_time(e1) / reps
+        ops = chains[0].ops()
+        names = ["qkv", "attn_out", "ffn1", "ffn2"]
+        per = {n: round(sum(ops[j] for _ in range(len(chains))) / (sum(kern[j]) * 1e-3) / 1e12 / peak, 4)
+               for j, n in enumerate(names)}
+        total_ops = sum(sum(c.ops()) for c in chains)
+        points.append({"batch": batch, "seq": seq, "sparsity": sp, "tokens": m, "ms": round(ms, 4),
+                       "tokens_per_s": round(m / (ms * 1e-3), 1), "ms_graph": round(ms_graph, 4),
+                       "tokens_per_s_graph": round(m / (ms_graph * 1e-3), 1),
+                       "tops": round(total_ops / (ms * 1e-3) / 1e12, 3), "roofline_frac_per_linear": per})
+        del g
+        for c in chains:
+            c.close()
+        torch.cuda.synchronize(dev)
+    mark1 = sampler.mark()
+    time.sleep(0.2)
+    sampler.stop()
+    clocks = sampler.summary(mark0, max(mark1, mark0 + 1))
+    ref = next(pt for pt in points if (pt["batch"], pt["seq"], pt["sparsity"]) == (8, 384, 0.8))
+    return {
+        "metric": METRIC, "value": ref["tokens_per_s"], "unit": "tokens/s", "n_gpus": 1, "steps": reps,
+        "warmup": 3, "ms_per_step": ref["ms"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "s8", "data": "synthetic",
+        "config": {"workload": "six-layer stack of 24 sparse INT8 linears (QKV, attention output, FFN1 + GELU, FFN2 "
+                               "per layer); value = the batch 8 x seq 384, 80% point; attention replaced in the "
+                               "timed path by a seeded int8 context buffer", "points": len(points)},
+        "points": points, "gpu_launches": 48 * reps * len(points) * 2, "clocks": clocks,
+        "kernel_source_sha256": kernel_sha(),
+    }
+
+
 def main():
     p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=2000)
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    p.add_argument("--workload", choices=sorted(WORKLOADS), default="ffn2")
+    p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "stack"], default="ffn2",
+                   help="ffn2/ffn1/single: one linear; layer: the encoder layer's four linears; stack: the "
+                        "six-layer stack sweep")
     p.add_argument("--ref-rows", type=int, default=512, help="tokens per reference step")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--soak-seconds", type=float, default=1.0, help="untimed load before the timed region")
@@ -406,7 +634,12 @@ def main():
             import torch.distributed as dist
             torch.cuda.set_device(local_rank)
             dist.init_process_group("nccl")
-        res = run_ours(args, rank, world, local_rank)
+        if args.workload == "layer":
+            res = run_layer(args) if rank == 0 else None
+        elif args.workload == "stack":
+            res = run_stack(args) if rank == 0 else None
+        else:
+            res = run_ours(args, rank, world, local_rank)
         if world > 1:
             import torch.distributed as dist
             dist.destroy_process_group()
