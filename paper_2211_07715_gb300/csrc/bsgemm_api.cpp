@@ -360,7 +360,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
         std::memcpy(sched.u, h->sched.u, sizeof(long long) * (grid + 1));
     }
     if (mode == 1) {
-        e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(workspace), s);
+        e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(workspace), h->num_sms, s);
         if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("relayout launch", e));
     }
     e = bsg::launch(h->w, a, sched, h->MT, grid, s);
@@ -424,7 +424,8 @@ int bsgemm_tile_activations(bsgemm_t h, const int8_t* act, int M, void* tiles, s
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
     if (dev != h->device) return fail(BSGEMM_ERR_INVALID, "current device is not the handle's device");
-    e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(tiles), static_cast<cudaStream_t>(stream));
+    e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(tiles), h->num_sms,
+                            static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("relayout launch", e));
     return BSGEMM_OK;
 }

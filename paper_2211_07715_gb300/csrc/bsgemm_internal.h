@@ -68,7 +68,7 @@ cudaError_t prepare_kernels(int MT, int K, int* ctas_per_sm);  // set attributes
 cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int MT, int grid,
                    cudaStream_t s);
 // x [M][K] -> token tiles [ntiles][kpad][MT] in xb (the layout the kernel stages by TMA).
-cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, cudaStream_t s);
+cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, int sms, cudaStream_t s);
 // Address of the fixed token-tile scratch (BSGEMM_STATIC_SCRATCH_BYTES) on
 // `device`, which must be the current device; looked up on the first call
 // per device, then cached.

@@ -556,63 +556,79 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
 }
 
 // Token-tile relayout: xb[t][k][j] = x[t*MT + j][k] for k < kpad (zero when
-// t*MT + j >= M or k >= K).  One CTA moves MT tokens x KC columns (16 KB)
-// through shared memory: 16-byte row loads (4 in flight per thread), a 4x4
-// byte transpose per thread, 16-byte stores of the k-major block, which is
-// contiguous in xb.
+// t*MT + j >= M or k >= K).  A persistent CTA walks items (tile t, block of
+// KC columns): MT tokens x KC columns (16 KB) through shared memory --
+// 16-byte row loads, a 4x4 byte transpose per thread, 16-byte stores of the
+// k-major block, which is contiguous in xb.  The next item's loads are in
+// flight (in registers) while the current item is transposed and stored.
 template <int MT>
 __global__ void __launch_bounds__(256)
-pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __restrict__ xb) {
-    constexpr int KC = 16384 / MT;     // columns per CTA (256 or 128)
+pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __restrict__ xb, long long items,
+               int ncb) {
+    constexpr int KC = 16384 / MT;     // columns per item (256 or 128)
     constexpr int C16 = KC / 16;       // 16-byte chunks per raw row
     constexpr int RW = KC / 4 + 4;     // raw row stride in words (rows shift by 4 banks)
     constexpr int OS = MT / 4 + 1;     // transposed row stride in words
+    constexpr int NL = (MT * C16) / 256;  // row loads per thread and item
     __shared__ __align__(16) uint32_t raw[MT * RW];
     __shared__ uint32_t tr[KC * OS];
-    const long long t = blockIdx.x;
-    const int k0 = blockIdx.y * KC;
-    const long long m0 = t * MT;
-    const int kc = min(KC, kpad - k0);  // a multiple of 16
     const bool vec16 = ((K & 15) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
+    auto load_item = [&](long long it, uint4 (&v)[NL]) {
+        const long long m0 = (it / ncb) * MT;
+        const int k0 = static_cast<int>(it % ncb) * KC;
 #pragma unroll
-    for (int i = 0; i < (MT * C16) / 256; ++i) {
-        const int c = i * 256 + threadIdx.x;
-        const int rho = c / C16, c16 = c % C16;
-        const long long m = m0 + rho;
-        const int k = k0 + 16 * c16;
-        uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if (m < M && k < K) {
-            const int8_t* src = x + static_cast<size_t>(m) * K + k;
-            if (vec16) {
-                v = __ldg(reinterpret_cast<const uint4*>(src));
-            } else {
-                uint32_t wv[4] = {0u, 0u, 0u, 0u};
+        for (int i = 0; i < NL; ++i) {
+            const int c = i * 256 + threadIdx.x;
+            const int rho = c / C16, c16 = c % C16;
+            const long long m = m0 + rho;
+            const int k = k0 + 16 * c16;
+            v[i] = make_uint4(0u, 0u, 0u, 0u);
+            if (m < M && k < K) {
+                const int8_t* src = x + static_cast<size_t>(m) * K + k;
+                if (vec16) {
+                    v[i] = __ldg(reinterpret_cast<const uint4*>(src));
+                } else {
+                    uint32_t wv[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-                for (int e = 0; e < 16; ++e)
-                    if (k + e < K) wv[e >> 2] |= static_cast<uint32_t>(static_cast<uint8_t>(src[e])) << (8 * (e & 3));
-                v = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                    for (int e = 0; e < 16; ++e)
+                        if (k + e < K) wv[e >> 2] |= static_cast<uint32_t>(static_cast<uint8_t>(src[e])) << (8 * (e & 3));
+                    v[i] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                }
             }
         }
-        *reinterpret_cast<uint4*>(raw + rho * RW + 4 * c16) = v;
-    }
-    __syncthreads();
-    for (int i = threadIdx.x; i < (MT / 4) * (KC / 4); i += 256) {
-        const int j = i % (KC / 4), g = i / (KC / 4);
-        uint32_t t0, t1, t2, t3;
-        transpose4(raw[(4 * g + 0) * RW + j], raw[(4 * g + 1) * RW + j], raw[(4 * g + 2) * RW + j],
-                   raw[(4 * g + 3) * RW + j], t0, t1, t2, t3);
-        tr[(4 * j + 0) * OS + g] = t0;
-        tr[(4 * j + 1) * OS + g] = t1;
-        tr[(4 * j + 2) * OS + g] = t2;
-        tr[(4 * j + 3) * OS + g] = t3;
-    }
-    __syncthreads();
-    int8_t* dst = xb + (static_cast<size_t>(t) * kpad + k0) * MT;
-    for (int i = threadIdx.x; i < kc * (MT / 16); i += 256) {
-        const int row = i / (MT / 16), c = i % (MT / 16);
-        const uint32_t* srow = tr + row * OS + 4 * c;
-        *reinterpret_cast<uint4*>(dst + static_cast<size_t>(row) * MT + 16 * c) =
-            make_uint4(srow[0], srow[1], srow[2], srow[3]);
+    };
+    uint4 v[NL];
+    long long it = blockIdx.x;
+    if (it < items) load_item(it, v);
+    for (; it < items; it += gridDim.x) {
+        const long long t = it / ncb;
+        const int k0 = static_cast<int>(it % ncb) * KC;
+        const int kc = min(KC, kpad - k0);  // a multiple of 16
+#pragma unroll
+        for (int i = 0; i < NL; ++i) {
+            const int c = i * 256 + threadIdx.x;
+            *reinterpret_cast<uint4*>(raw + (c / C16) * RW + 4 * (c % C16)) = v[i];
+        }
+        __syncthreads();  // raw is complete; every thread is past the previous item's stores
+        if (it + gridDim.x < items) load_item(it + gridDim.x, v);
+        for (int i = threadIdx.x; i < (MT / 4) * (KC / 4); i += 256) {
+            const int j = i % (KC / 4), g = i / (KC / 4);
+            uint32_t t0, t1, t2, t3;
+            transpose4(raw[(4 * g + 0) * RW + j], raw[(4 * g + 1) * RW + j], raw[(4 * g + 2) * RW + j],
+                       raw[(4 * g + 3) * RW + j], t0, t1, t2, t3);
+            tr[(4 * j + 0) * OS + g] = t0;
+            tr[(4 * j + 1) * OS + g] = t1;
+            tr[(4 * j + 2) * OS + g] = t2;
+            tr[(4 * j + 3) * OS + g] = t3;
+        }
+        __syncthreads();  // tr is complete; raw may be refilled
+        int8_t* dst = xb + (static_cast<size_t>(t) * kpad + k0) * MT;
+        for (int i = threadIdx.x; i < kc * (MT / 16); i += 256) {
+            const int row = i / (MT / 16), c = i % (MT / 16);
+            const uint32_t* srow = tr + row * OS + 4 * c;
+            *reinterpret_cast<uint4*>(dst + static_cast<size_t>(row) * MT + 16 * c) =
+                make_uint4(srow[0], srow[1], srow[2], srow[3]);
+        }
     }
 }
 
@@ -698,12 +714,14 @@ size_t tiled_bytes(int MT, int K, long long M) {
     return static_cast<size_t>((M + MT - 1) / MT) * kpad * MT;
 }
 
-cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, cudaStream_t s) {
+cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, int sms, cudaStream_t s) {
     const int kpad = (K + 15) & ~15;
-    const dim3 grid(static_cast<unsigned>((static_cast<long long>(M) + MT - 1) / MT),
-                    static_cast<unsigned>((kpad + 16384 / MT - 1) / (16384 / MT)));
-    if (MT == 128) pretile_kernel<128><<<grid, 256, 0, s>>>(x, M, K, kpad, xb);
-    else pretile_kernel<64><<<grid, 256, 0, s>>>(x, M, K, kpad, xb);
+    const int ncb = (kpad + 16384 / MT - 1) / (16384 / MT);
+    const long long items = (static_cast<long long>(M) + MT - 1) / MT * ncb;
+    const long long cap = 4LL * (sms > 0 ? sms : 1);  // 4 resident CTAs per SM (35 KB of shared memory each)
+    const unsigned grid = static_cast<unsigned>(items < cap ? items : cap);
+    if (MT == 128) pretile_kernel<128><<<grid, 256, 0, s>>>(x, M, K, kpad, xb, items, ncb);
+    else pretile_kernel<64><<<grid, 256, 0, s>>>(x, M, K, kpad, xb, items, ncb);
     return cudaGetLastError();
 }
 
