@@ -12,10 +12,12 @@ MACs, padding excluded) and achieved HBM GB/s = algorithmic bytes / t, where
 algorithmic bytes = stored values + column indices + indptr + scales + bias
 + activations + outputs.
 
-Timing: CUDA events on the launching stream around exactly --steps launches
-after --warmup launches (plus an untimed soak of about a second so that the
-clock sampler sees the GPU under this load), barrier + synchronize on both
-sides, max over ranks.  Input/output buffer sets rotate so that the working
+Timing: the --steps timed steps are captured once as one CUDA graph and
+replayed between CUDA events on the launching stream, after --warmup
+stream-launched steps and an untimed soak of about a second (so that the
+clock sampler sees the GPU under this load); barrier + synchronize on both
+sides, max over ranks.  A second, stream-launched loop with events around
+each kernel gives the per-kernel times.  Input/output buffer sets rotate so that the working
 set of consecutive launches exceeds twice the L2 (no launch finds its
 activations in L2).
 
