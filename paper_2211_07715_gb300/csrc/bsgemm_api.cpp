@@ -1,6 +1,6 @@
 // Host side of the C ABI declared in include/bsgemm.h: argument checks, the
-// create-time repack of the block-compressed weight into quads (groups of 4
-// stored blocks of one block-row, the dot-4 unit of Algorithm 1), device
+// create-time repack of the block-compressed weight into steps (16 stored
+// blocks of one block-row = 4 quads, the dot-4 unit of Algorithm 1), device
 // upload, and the launch of the kernel in bsgemm_kernel.cu.
 #include "bsgemm.h"
 
@@ -17,7 +17,6 @@ struct bsgemm_ctx {
     int device = -1;
     int num_sms = 0;
     int ctas_per_sm = 0;
-    int MT = 0;
     int64_t nnzb = 0;
     void* arena = nullptr;
     size_t arena_bytes = 0;
@@ -70,12 +69,12 @@ std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx
     return "";
 }
 
-// Schedule cost of one token tile in a CTA's range, in quads: a CTA holds
-// one tile in shared memory, so every further tile in its range costs a
-// copy-in and the start-up around it.  1000 quads (a few microseconds of a
-// CTA's work) gave the shortest layer kernels on GB300 in a sweep over
-// 0-4000 at K = 3072 and K = 768.
-constexpr long long kTileCost = 1000;
+// Schedule costs, in steps (16 stored blocks of one block-row for 64
+// tokens: 32 dp4a per lane): every block-row adds kRowCost for its
+// cross-lane sum and epilogue, every token tile in a CTA's range adds
+// kTileCost for its copy into shared memory and the start-up around it.
+constexpr long long kRowCost = 2;
+constexpr long long kTileCost = 250;
 
 // End of the greedy range that starts at unit u under the cost bound C: it
 // takes whole units while the cost (units' cost + tc per token tile
@@ -187,40 +186,84 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         }
     }
 
-    // Repack into quads: per block-row, stored blocks in groups of 4, and
-    // the quad count rounded up to a multiple of the kernel's lane groups per
-    // warp; padding entries repeat the row's last column with zero weights.
-    // Record q = {k0, k1, k2, k3} then 4 words, word c holding the bytes
-    // W[4r + c][k0..k3].
-    const int MT = bsg::tile_for_k(K);
-    const int G = bsg::groups_for_tile(MT);
-    std::vector<int32_t> qptr(nbr + 1, 0), cost(nbr + 1, 0);
+    // Repack into steps.  Per block-row the stored columns are ordered so
+    // that each half-step (8 consecutive columns, one pass of the kernel's
+    // shared-memory gather) takes its columns from distinct bank groups of
+    // the swizzled token tile where it can: every half-step draws one
+    // column from each of the 8 bank-key buckets with the most columns left,
+    // then (if fewer than 8 buckets are left) again from the fullest; the
+    // last step is padded with zero-weight entries on unused keys (columns
+    // 0..7 cover all 8 keys and are rows of every tile, which has
+    // round_up(K, 16) >= 16 rows).
+    std::vector<int32_t> sptr(nbr + 1, 0);
+    std::vector<int32_t> cost(nbr + 1, 0);
     for (int r = 0; r < nbr; ++r) {
         const int nz = indptr[r + 1] - indptr[r];
-        const int nq = (nz + 3) / 4;
-        qptr[r + 1] = qptr[r] + (nq + G - 1) / G * G;
-        cost[r + 1] = qptr[r + 1] + (r + 1);
+        sptr[r + 1] = sptr[r] + (nz + 15) / 16;
+        cost[r + 1] = static_cast<int32_t>(cost[r] + (nz + 15) / 16 + (nz > 0 ? kRowCost : 0));
     }
-    const int Q = qptr[nbr];
-    // + padding records: the kernel copies whole ring chunks of kQuadPad records
-    std::vector<int32_t> quads(static_cast<size_t>(Q + bsg::kQuadPad) * 8, 0);
-    for (int r = 0; r < nbr; ++r) {
-        const int j0 = indptr[r], j1 = indptr[r + 1];
-        for (int q = qptr[r]; q < qptr[r + 1]; ++q) {
-            int32_t* rec = &quads[static_cast<size_t>(q) * 8];
-            uint32_t wwords[4] = {0, 0, 0, 0};
-            for (int e = 0; e < 4; ++e) {
-                const int j = j0 + 4 * (q - qptr[r]) + e;
-                if (j < j1) {
-                    rec[e] = colidx[j];
-                    for (int c = 0; c < 4; ++c)
-                        wwords[c] |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(j) * 4 + c]))
-                                     << (8 * e);
-                } else {
-                    rec[e] = colidx[j1 - 1];  // padding: a valid column, zero weight
+    const int S = sptr[nbr];
+    std::vector<int32_t> recs(static_cast<size_t>(S + bsg::kStepPad) * 32, 0);
+    int pad_col[8];
+    for (int k = 0; k < 8; ++k) pad_col[bsg::bank_key(k)] = k;
+    {
+        std::vector<int> bucket[8];
+        std::vector<int> order;  // stored-block index j, or -1 - key for a padding entry
+        for (int r = 0; r < nbr; ++r) {
+            const int j0 = indptr[r], j1 = indptr[r + 1];
+            if (j1 == j0) continue;
+            for (auto& b : bucket) b.clear();
+            for (int j = j1 - 1; j >= j0; --j) bucket[bsg::bank_key(colidx[j])].push_back(j);  // popped in column order
+            const int entries = (sptr[r + 1] - sptr[r]) * 16;
+            order.clear();
+            int left = j1 - j0;
+            while (static_cast<int>(order.size()) < entries) {
+                int keys[8] = {0, 1, 2, 3, 4, 5, 6, 7};
+                std::stable_sort(keys, keys + 8, [&](int x, int y) { return bucket[x].size() > bucket[y].size(); });
+                bool used[8] = {false, false, false, false, false, false, false, false};
+                int taken = 0;
+                for (int i = 0; i < 8 && taken < 8; ++i) {
+                    if (bucket[keys[i]].empty()) continue;
+                    order.push_back(bucket[keys[i]].back());
+                    bucket[keys[i]].pop_back();
+                    used[keys[i]] = true;
+                    ++taken;
+                    --left;
+                }
+                while (taken < 8 && left > 0) {  // fewer than 8 keys left: repeat the fullest
+                    int best = 0;
+                    for (int x = 1; x < 8; ++x)
+                        if (bucket[x].size() > bucket[best].size()) best = x;
+                    order.push_back(bucket[best].back());
+                    bucket[best].pop_back();
+                    used[best] = true;
+                    ++taken;
+                    --left;
+                }
+                for (int x = 0; x < 8 && taken < 8; ++x) {  // padding on keys this half-step does not use
+                    if (used[x]) continue;
+                    order.push_back(-1 - x);
+                    used[x] = true;
+                    ++taken;
                 }
             }
-            for (int c = 0; c < 4; ++c) rec[4 + c] = static_cast<int32_t>(wwords[c]);
+            for (int s = 0; s < sptr[r + 1] - sptr[r]; ++s) {
+                int32_t* rec = &recs[static_cast<size_t>(sptr[r] + s) * 32];
+                uint32_t wwords[4][4] = {};
+                for (int e = 0; e < 16; ++e) {
+                    const int o = order[16 * s + e];
+                    if (o >= 0) {
+                        rec[e] = static_cast<int32_t>(bsg::tile_row_offset(colidx[o]));
+                        for (int c = 0; c < 4; ++c)
+                            wwords[e / 4][c] |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(o) * 4 + c]))
+                                                << (8 * (e % 4));
+                    } else {
+                        rec[e] = static_cast<int32_t>(bsg::tile_row_offset(pad_col[-1 - o]));
+                    }
+                }
+                for (int qd = 0; qd < 4; ++qd)
+                    for (int c = 0; c < 4; ++c) rec[16 + 4 * qd + c] = static_cast<int32_t>(wwords[qd][c]);
+            }
         }
     }
     std::vector<float> bias_v(N, 0.0f);
@@ -241,23 +284,21 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         delete h;
         return nullptr;
     }
-    h->MT = MT;
-    if (bsg::smem_bytes(h->MT, K) + bsg::kStaticSmem > static_cast<size_t>(optin)) {
+    if (bsg::smem_bytes(K) + bsg::kStaticSmem > static_cast<size_t>(optin)) {
         fail(BSGEMM_ERR_UNSUPPORTED, "this device has too little shared memory per block for K = " + std::to_string(K));
         delete h;
         return nullptr;
     }
-    e = bsg::prepare_kernels(h->MT, K, &h->ctas_per_sm);
+    e = bsg::prepare_kernels(K, &h->ctas_per_sm);
     if (e != cudaSuccess || h->ctas_per_sm < 1) {
         fail(BSGEMM_ERR_CUDA, e != cudaSuccess ? cuda_msg("kernel setup", e) : "kernel cannot be resident on an SM");
         delete h;
         return nullptr;
     }
 
-    const size_t off_qptr = 0;
-    const size_t off_cost = align_up(off_qptr + sizeof(int32_t) * (nbr + 1), 256);
-    const size_t off_quads = align_up(off_cost + sizeof(int32_t) * (nbr + 1), 256);
-    const size_t off_scale = align_up(off_quads + sizeof(int32_t) * quads.size(), 256);
+    const size_t off_sptr = 0;
+    const size_t off_recs = align_up(off_sptr + sizeof(int32_t) * (nbr + 1), 256);
+    const size_t off_scale = align_up(off_recs + sizeof(int32_t) * recs.size(), 256);
     const size_t off_bias = align_up(off_scale + sizeof(float) * N, 256);
     const size_t off_status = align_up(off_bias + sizeof(float) * N, 256);
     h->arena_bytes = align_up(off_status + sizeof(int), 256);
@@ -269,9 +310,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     }
     char* base = static_cast<char*>(h->arena);
     struct Piece { size_t off; const void* src; size_t bytes; } pieces[] = {
-        {off_qptr, qptr.data(), sizeof(int32_t) * qptr.size()},
-        {off_cost, cost.data(), sizeof(int32_t) * cost.size()},
-        {off_quads, quads.data(), sizeof(int32_t) * quads.size()},
+        {off_sptr, sptr.data(), sizeof(int32_t) * sptr.size()},
+        {off_recs, recs.data(), sizeof(int32_t) * recs.size()},
         {off_scale, scales, sizeof(float) * N},
         {off_bias, bias_v.data(), sizeof(float) * N},
         {off_status, &kZeroStatus, sizeof(int)},
@@ -287,16 +327,15 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     }
     h->nnzb = nnzb;
     h->cost = cost;
-    h->w.qptr = reinterpret_cast<const int32_t*>(base + off_qptr);
-    h->w.cost = reinterpret_cast<const int32_t*>(base + off_cost);
-    h->w.quads = reinterpret_cast<const int4*>(base + off_quads);
+    h->w.sptr = reinterpret_cast<const int32_t*>(base + off_sptr);
+    h->w.recs = reinterpret_cast<const int4*>(base + off_recs);
     h->w.scale = reinterpret_cast<const float*>(base + off_scale);
     h->w.bias = reinterpret_cast<const float*>(base + off_bias);
     h->w.status = reinterpret_cast<int*>(base + off_status);
     h->w.N = N;
     h->w.K = K;
     h->w.nbr = nbr;
-    h->w.Q = Q;
+    h->w.S = S;
     return h;
 }
 
@@ -321,7 +360,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     if ((mode != 2 && !act) || !out) return fail(BSGEMM_ERR_INVALID, "act and out must not be NULL");
     if (reinterpret_cast<uintptr_t>(out) % 16 != 0) return fail(BSGEMM_ERR_INVALID, "out must be 16-byte aligned");
     if (use_ws) {
-        const size_t need = bsg::tiled_bytes(h->MT, h->w.K, M);
+        const size_t need = bsg::tiled_bytes(h->w.K, M);
         if (!workspace || workspace_bytes < need)
             return fail(BSGEMM_ERR_INVALID, "workspace must hold bsgemm_workspace_bytes(h, M) = " +
                                                 std::to_string(need) + " bytes");
@@ -344,7 +383,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.kind = epi.kind;
     a.inv_out_scale = inv;
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
-    const long long ntiles = (static_cast<long long>(M) + h->MT - 1) / h->MT;
+    const long long ntiles = (static_cast<long long>(M) + bsg::kTile - 1) / bsg::kTile;
     const long long nbr = h->w.nbr;
     long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
     if (cap > bsg::kMaxGrid) cap = bsg::kMaxGrid;
@@ -360,10 +399,10 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
         std::memcpy(sched.u, h->sched.u, sizeof(long long) * (grid + 1));
     }
     if (mode == 1) {
-        e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(workspace), h->num_sms, s);
+        e = bsg::launch_pretile(act, M, h->w.K, static_cast<int8_t*>(workspace), h->num_sms, s);
         if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("relayout launch", e));
     }
-    e = bsg::launch(h->w, a, sched, h->MT, grid, s);
+    e = bsg::launch(h->w, a, sched, grid, s);
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("kernel launch", e));
     return BSGEMM_OK;
 }
@@ -386,10 +425,10 @@ int bsgemm_run_static(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
     if (M > 0) {
-        const size_t need = bsg::tiled_bytes(h->MT, h->w.K, M);
+        const size_t need = bsg::tiled_bytes(h->w.K, M);
         if (need > BSGEMM_STATIC_SCRATCH_BYTES) {
-            const size_t per_tile = bsg::tiled_bytes(h->MT, h->w.K, h->MT);
-            const long long m_max = static_cast<long long>(BSGEMM_STATIC_SCRATCH_BYTES / per_tile) * h->MT;
+            const size_t per_tile = bsg::tiled_bytes(h->w.K, bsg::kTile);
+            const long long m_max = static_cast<long long>(BSGEMM_STATIC_SCRATCH_BYTES / per_tile) * bsg::kTile;
             return fail(BSGEMM_ERR_INVALID, "M = " + std::to_string(M) + " needs " + std::to_string(need) +
                                                 " bytes of token tiles; the static scratch holds " +
                                                 std::to_string(static_cast<size_t>(BSGEMM_STATIC_SCRATCH_BYTES)) +
@@ -415,7 +454,7 @@ int bsgemm_tile_activations(bsgemm_t h, const int8_t* act, int M, void* tiles, s
     if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
     if (M == 0) return BSGEMM_OK;
     if (!act) return fail(BSGEMM_ERR_INVALID, "act must not be NULL");
-    const size_t need = bsg::tiled_bytes(h->MT, h->w.K, M);
+    const size_t need = bsg::tiled_bytes(h->w.K, M);
     if (!tiles || tiles_bytes < need)
         return fail(BSGEMM_ERR_INVALID, "tiles must hold bsgemm_workspace_bytes(h, M) = " + std::to_string(need) +
                                             " bytes");
@@ -424,15 +463,14 @@ int bsgemm_tile_activations(bsgemm_t h, const int8_t* act, int M, void* tiles, s
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
     if (dev != h->device) return fail(BSGEMM_ERR_INVALID, "current device is not the handle's device");
-    e = bsg::launch_pretile(act, M, h->w.K, h->MT, static_cast<int8_t*>(tiles), h->num_sms,
-                            static_cast<cudaStream_t>(stream));
+    e = bsg::launch_pretile(act, M, h->w.K, static_cast<int8_t*>(tiles), h->num_sms, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("relayout launch", e));
     return BSGEMM_OK;
 }
 
 size_t bsgemm_workspace_bytes(bsgemm_t h, int M) {
     if (!h || M <= 0) return 0;
-    return bsg::tiled_bytes(h->MT, h->w.K, M);
+    return bsg::tiled_bytes(h->w.K, M);
 }
 
 int bsgemm_device_status(bsgemm_t h, int clear) {
@@ -454,7 +492,7 @@ void bsgemm_destroy(bsgemm_t h) {
 int bsgemm_info(bsgemm_t h, int64_t* out, int n) {
     clear_error();
     if (!h || (!out && n > 0)) return fail(BSGEMM_ERR_INVALID, "NULL handle or output");
-    const int64_t v[7] = {h->w.N, h->w.K, h->nnzb, h->w.Q, h->MT,
+    const int64_t v[7] = {h->w.N, h->w.K, h->nnzb, 4 * static_cast<int64_t>(h->w.S), bsg::kTile,
                           static_cast<int64_t>(h->num_sms) * h->ctas_per_sm, static_cast<int64_t>(h->arena_bytes)};
     for (int i = 0; i < n && i < 7; ++i) out[i] = v[i];
     return 7;

@@ -8,34 +8,34 @@
 //
 // GB300 design (not a translation of the paper's AVX-512 loop nest):
 //
-// * Unit of work: (token tile t, block-row r) -- MT tokens x 4 output
+// * Unit of work: (token tile t, block-row r) -- 64 tokens x 4 output
 //   channels, reduced over the block-row's stored columns.  Units are
 //   ordered tile-major and split into one contiguous, cost-balanced range per
-//   CTA of a persistent grid (CTAs = SMs x resident CTAs), so every SM gets
-//   the same number of quads regardless of M.
+//   CTA of a persistent grid (CTAs = SMs x resident CTAs).
 // * The CTA stages its token tile of the activations for ALL of K in shared
-//   memory, transposed to "k-major" rows (row k holds the MT tokens' bytes at
-//   column k), once per tile; every block-row of the tile then gathers from
-//   it.  This is the re-organisation of the input by the mask that
-//   Algorithm 1 does with vpermt2d/vpshufb, done once per tile instead of
-//   once per block.
-// * Lanes own 4 consecutive tokens.  For one quad (4 stored columns k0..k3 of
-//   one block-row) a lane reads 4 words (one per column, 4 tokens each),
-//   transposes the 4x4 bytes with 8 byte-permutes into one dot-4 operand per
-//   token, and issues 16 dp4a (4 tokens x 4 channels) against the quad's 4
-//   weight words -- the analogue of Algorithm 1's broadcast weight block A,
-//   re-organised input block B and 4 vpdpbusd.  GB300 runs int8 dot products
-//   at the same rate on dp4a as on its int8 MMA paths, so no tensor-core path
-//   is faster here (the 4-channel block cannot fill an MMA tile).
-// * A CTA's quads are split evenly between its 16 warps.  Each warp streams
-//   its contiguous range of 32-byte quad records through a two-chunk ring in
-//   shared memory (cp.async, 512 bytes per chunk, the next chunk in flight
-//   while the current one is consumed).  With 64-token tiles a lane covers
-//   only half the warp's width, so the two half-warps take alternate quads
-//   of a block-row and add their sums with one shuffle at the row's end.
-//   A block-row that straddles a split between warps is summed in a
-//   shared-memory slot (int32 atomics) and finished after a barrier.  All
-//   sums are exact int32.
+//   memory once (one bulk TMA copy of a tile the relayout kernel has already
+//   swizzled); every block-row of the tile then gathers from it.  This is the
+//   re-organisation of the input by the mask that Algorithm 1 does with
+//   vpermt2d/vpshufb, done once per tile instead of once per block.
+// * A block-row's stored columns come in steps of 16 (4 quads).  One step of
+//   one warp is two transposed shared-memory gathers (ldmatrix .m16n16 .b8):
+//   each lane receives 8 dot-4 operands -- 8 tokens x 4 consecutive columns
+//   of its quad -- with no byte permutes, and issues 32 dp4a against the
+//   quad's 4 channel words: Algorithm 1's broadcast weight block A,
+//   re-organised input block B and vpdpbusd, 8 tokens at a time.  The
+//   columns of each half-step are chosen at create time to fall in distinct
+//   shared-memory bank groups of the swizzled tile, so a gather reads in one
+//   pass per 8 rows.
+// * The 4 lanes that hold the same tokens took different quads; at the end
+//   of a block-row their sums are added with 24 shuffles (exact int32).
+// * A CTA's steps are split evenly between its 16 warps.  Each warp reads its
+//   contiguous range of 128-byte step records straight from global memory
+//   (L1/L2) into a 4-deep register ring, three steps ahead of their use.  A block-row that straddles a
+//   split between warps is summed in a shared-memory slot (int32 atomics);
+//   the last warp to add finishes it.
+// * GB300 runs int8 dot products on dp4a at the rate of its int8 MMA paths
+//   (tcgen05 has no int8 kind on sm_103a), and a 4-channel block cannot fill
+//   an MMA tile, so the contraction stays on dp4a.
 // * The epilogue runs in registers: int32 -> fp32 (RNE), one fma with scale
 //   and bias, optional GELU by a fixed fp32 op sequence (A&S 7.1.28 erf),
 //   optional requantise (fp32 multiply, round half to even, saturate).
@@ -51,13 +51,6 @@ namespace {
 
 constexpr int kSmemOptin = 232448;  // sm_103 opt-in shared memory per block
 constexpr int kSlots = kWarps - 1;  // one per split point between warp ranges
-// Record ring per warp: kRingSlots chunks of ring_chunk(MT) quad records;
-// while one chunk is consumed the next kRingSlots - 1 are in flight.
-constexpr int kRingSlots = 4;
-__host__ __device__ constexpr int ring_chunk(int MT) { return MT == 64 ? 8 : 16; }
-
-__host__ __device__ constexpr int slot_words(int MT) { return 4 * MT; }  // MT tokens x 4 channels
-constexpr size_t ring_bytes(int MT) { return static_cast<size_t>(kWarps) * kRingSlots * ring_chunk(MT) * 32; }
 
 // 4x4 byte transpose.  In: a/b/c/d = bytes (x0..x3) of rows 0..3.  Out:
 // t_i = (a_i, b_i, c_i, d_i).
@@ -122,59 +115,60 @@ __device__ __forceinline__ uint32_t requant_s8(float v, float inv) {
     return static_cast<uint32_t>(q) & 0xffu;
 }
 
-// Epilogue for one lane: tokens m_first + i, i < T (rows < M only), x the
-// 4 channels of block-row r (scales s, bias b).  v[i * 4 + c] = token i,
-// channel c.
-template <int KIND, int T>
-__device__ __forceinline__ void store_rows(const DeviceWeights& w, const LaunchArgs& a, long long m_first, int r,
-                                           const int (&v)[T * 4], float4 s, float4 b) {
-    const int N = w.N;
-#pragma unroll
-    for (int i = 0; i < T; ++i) {
-        const long long m = m_first + i;
-        if (m >= a.M) break;
-        const size_t o = static_cast<size_t>(m) * N + 4 * r;
-        const int* vi = v + 4 * i;
-        if (KIND == 0) {
-            *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(vi[0], vi[1], vi[2], vi[3]);
-        } else {
-            float y0 = __fmaf_rn(__int2float_rn(vi[0]), s.x, b.x);
-            float y1 = __fmaf_rn(__int2float_rn(vi[1]), s.y, b.y);
-            float y2 = __fmaf_rn(__int2float_rn(vi[2]), s.z, b.z);
-            float y3 = __fmaf_rn(__int2float_rn(vi[3]), s.w, b.w);
-            if (KIND == 2) {
-                y0 = gelu_f32_fast(y0);
-                y1 = gelu_f32_fast(y1);
-                y2 = gelu_f32_fast(y2);
-                y3 = gelu_f32_fast(y3);
-            } else if (KIND == 4) {
-                y0 = gelu_f32(y0);
-                y1 = gelu_f32(y1);
-                y2 = gelu_f32(y2);
-                y3 = gelu_f32(y3);
-            }
-            if (KIND == 1 || KIND == 2) {
-                *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y0, y1, y2, y3);
-            } else {
-                const float inv = a.inv_out_scale;
-                const uint32_t packed = requant_s8(y0, inv) | (requant_s8(y1, inv) << 8) |
-                                        (requant_s8(y2, inv) << 16) | (requant_s8(y3, inv) << 24);
-                *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = packed;
-            }
-        }
+// Epilogue for one token m (nothing past M): v = acc of the 4 channels of
+// block-row r (scales s, bias b), written as out[m][4r .. 4r+3].
+template <int KIND>
+__device__ __forceinline__ void store_token(const LaunchArgs& a, int N, long long m, int r, const int* v, float4 s,
+                                            float4 b) {
+    if (m >= a.M) return;
+    const size_t o = static_cast<size_t>(m) * N + 4 * r;
+    if (KIND == 0) {
+        *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(v[0], v[1], v[2], v[3]);
+        return;
+    }
+    float y0 = __fmaf_rn(__int2float_rn(v[0]), s.x, b.x);
+    float y1 = __fmaf_rn(__int2float_rn(v[1]), s.y, b.y);
+    float y2 = __fmaf_rn(__int2float_rn(v[2]), s.z, b.z);
+    float y3 = __fmaf_rn(__int2float_rn(v[3]), s.w, b.w);
+    if (KIND == 2) {
+        y0 = gelu_f32_fast(y0);
+        y1 = gelu_f32_fast(y1);
+        y2 = gelu_f32_fast(y2);
+        y3 = gelu_f32_fast(y3);
+    } else if (KIND == 4) {
+        y0 = gelu_f32(y0);
+        y1 = gelu_f32(y1);
+        y2 = gelu_f32(y2);
+        y3 = gelu_f32(y3);
+    }
+    if (KIND == 1 || KIND == 2) {
+        *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y0, y1, y2, y3);
+    } else {
+        const float inv = a.inv_out_scale;
+        const uint32_t packed = requant_s8(y0, inv) | (requant_s8(y1, inv) << 8) | (requant_s8(y2, inv) << 16) |
+                                (requant_s8(y3, inv) << 24);
+        *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = packed;
     }
 }
 
 __device__ __forceinline__ float4 load_s4(const float* p, int r) { return __ldg(reinterpret_cast<const float4*>(p) + r); }
 
-// Last index r in [lo, hi) with qp[r] <= q, given qp[lo] <= q < qp[hi]
-// (qp: the shared-memory window of quad offsets).
-__device__ __forceinline__ int row_of(const int* qp, int lo, int hi, int q) {
+// Last index r in [lo, hi) with sp[r] <= q, given sp[lo] <= q < sp[hi]
+// (sp: the shared-memory window of step offsets).
+__device__ __forceinline__ int row_of(const int* sp, int lo, int hi, int q) {
     while (hi - lo > 1) {
         const int mid = (lo + hi) >> 1;
-        if (qp[mid] <= q) lo = mid; else hi = mid;
+        if (sp[mid] <= q) lo = mid; else hi = mid;
     }
     return lo;
+}
+
+// Byte offset of chunk 0 of activation column k in a swizzled token tile
+// (rows 2i, 2i+1 share 128-byte line i; chunk c of row k in 16-byte slot
+// (4 (k & 1) + c) XOR (i & 7)); chunk c is at row_off(k) XOR 16 c.
+__device__ __forceinline__ uint32_t row_off(int k) {
+    const uint32_t line = static_cast<uint32_t>(k) >> 1;
+    return (line << 7) | ((((static_cast<uint32_t>(k) & 1u) << 2) ^ (line & 7u)) << 4);
 }
 
 // One staging unit: tokens 4g..4g+3 of the tile x columns 16kc..16kc+15.
@@ -209,28 +203,25 @@ __device__ __forceinline__ void load_unit(const LaunchArgs& a, int K, long long 
     }
 }
 
-// Write one unit k-major: word g of rows 16kc..16kc+15 (tokens 4g..4g+3).
-template <int MT>
-__device__ __forceinline__ void store_unit(uint32_t* xt, int g, int kc, const uint32_t (&rw)[4][4]) {
-    constexpr int RW = MT / 4;  // words per k-row
+// Write one unit into the swizzled tile: word (tokens 4g..4g+3) of rows
+// 16kc..16kc+15; the word lies in chunk g / 4 at byte 4 (g % 4).
+__device__ __forceinline__ void store_unit(unsigned char* xt, int g, int kc, const uint32_t (&rw)[4][4]) {
+    const uint32_t cx = static_cast<uint32_t>(g >> 2) << 4, wb = 4u * static_cast<uint32_t>(g & 3);
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-        uint32_t t0, t1, t2, t3;
-        transpose4(rw[0][j], rw[1][j], rw[2][j], rw[3][j], t0, t1, t2, t3);
-        uint32_t* dst = xt + static_cast<size_t>(16 * kc + 4 * j) * RW + g;
-        dst[0] = t0;
-        dst[RW] = t1;
-        dst[2 * RW] = t2;
-        dst[3 * RW] = t3;
+        uint32_t t[4];
+        transpose4(rw[0][j], rw[1][j], rw[2][j], rw[3][j], t[0], t[1], t[2], t[3]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            *reinterpret_cast<uint32_t*>(xt + ((row_off(16 * kc + 4 * j + e) ^ cx) + wb)) = t[e];
     }
 }
 
-// Stage activation rows m0..m0+MT-1, all K columns, into xt as k-major rows
-// of MT bytes (word g of row k = tokens 4g..4g+3 at column k).  Each thread
-// keeps kStageBatch units' loads in flight before transposing them.
-template <int MT>
-__device__ __forceinline__ void stage_tile(uint32_t* xt, const LaunchArgs& a, int K, int kpad, long long m0) {
-    constexpr int G = MT / 4;
+// Stage activation rows m0..m0+63, all kpad columns, into the swizzled tile
+// with per-thread loads.  Each thread keeps kStageBatch units' loads in
+// flight before transposing them.
+__device__ __forceinline__ void stage_tile(unsigned char* xt, const LaunchArgs& a, int K, int kpad, long long m0) {
+    constexpr int G = kTile / 4;
     constexpr int kStageBatch = 2;
     const int total = G * (kpad >> 4);
     for (int base = threadIdx.x; base < total; base += kStageBatch * kThreads) {
@@ -243,33 +234,25 @@ __device__ __forceinline__ void stage_tile(uint32_t* xt, const LaunchArgs& a, in
 #pragma unroll
         for (int b = 0; b < kStageBatch; ++b) {
             const int id = base + b * kThreads;
-            if (id < total) store_unit<MT>(xt, id % G, id / G, rw[b]);
+            if (id < total) store_unit(xt, id % G, id / G, rw[b]);
         }
     }
 }
 
-// cp.async (16 bytes, L2 only) into shared memory, and its group fences.
-__device__ __forceinline__ void cp_async16(uint32_t smem_dst, const void* gmem_src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(smem_dst), "l"(gmem_src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
-
-// Shared-memory loads with 32-bit shared-window addresses.
+// 32-bit shared-window address of a shared-memory pointer.
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
-__device__ __forceinline__ int4 lds128(uint32_t addr) {
-    int4 v;
-    asm volatile("ld.shared.v4.s32 {%0, %1, %2, %3}, [%4];\n"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
-    return v;
-}
-__device__ __forceinline__ uint2 lds64(uint32_t addr) {
-    uint2 v;
-    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];\n" : "=r"(v.x), "=r"(v.y) : "r"(addr));
-    return v;
+
+// Gather two 16 x 16 byte matrices from shared memory, transposed: lane i
+// gives the address of row (i % 16) of matrix i / 16 (16 bytes, 16-byte
+// aligned); lane l receives, for matrix 0 (r0, r1) and matrix 1 (r2, r3),
+// the bytes of rows 4 (l % 4) .. 4 (l % 4) + 3 at column l / 4 (r0, r2) and
+// column l / 4 + 8 (r1, r3), row 4 (l % 4) in the lowest byte.
+__device__ __forceinline__ void ldsm_x2_trans_b8(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                                 uint32_t& r3) {
+    asm volatile("ldmatrix.sync.aligned.m16n16.x2.trans.shared.b8 {%0, %1, %2, %3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
 }
 
 // mbarrier + bulk-copy (TMA) helpers.  Waits are bounded: a wait that
@@ -303,82 +286,90 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, unsigned
 // later asynchronous-proxy (bulk copy) writes.
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
 
-// One quad for one lane's 8 tokens: 4 x 8 bytes from the k-major tile at the
-// quad's columns, two 4x4 byte transposes, 32 dp4a (8 tokens x 4 channels).
-template <int MT>
-__device__ __forceinline__ void quad8(uint32_t xlane, const int4& kk, const int4& ww, int (&acc)[32]) {
-    const uint2 x0 = lds64(xlane + kk.x * MT), x1 = lds64(xlane + kk.y * MT);
-    const uint2 x2 = lds64(xlane + kk.z * MT), x3 = lds64(xlane + kk.w * MT);
+// One step for one lane: the step's 16 columns x the tile's 64 tokens come
+// in by two transposed gathers (tokens 0-31, then 32-63); lane l (g = l / 4,
+// q = l % 4) receives x[g + 8 i][k_{4q} .. k_{4q+3}] as word t[i], i < 8, and
+// issues 32 dp4a against quad q's 4 channel words.  `off` is the step's
+// column offset for row l % 16, lb = 16 (l / 16) selects the chunk (16
+// tokens) of matrix l / 16.  tb is 128-byte aligned, so XOR with 16 c moves
+// to chunk c of the same row.
+__device__ __forceinline__ void step16(uint32_t tb, uint32_t lb, int off, const int4& w, int (&acc)[32]) {
+    const uint32_t a0 = tb + (static_cast<uint32_t>(off) ^ lb);
     uint32_t t[8];
-    transpose4(x0.x, x1.x, x2.x, x3.x, t[0], t[1], t[2], t[3]);
-    transpose4(x0.y, x1.y, x2.y, x3.y, t[4], t[5], t[6], t[7]);
+    ldsm_x2_trans_b8(a0, t[0], t[1], t[2], t[3]);
+    ldsm_x2_trans_b8(a0 ^ 32u, t[4], t[5], t[6], t[7]);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-        acc[4 * i + 0] = __dp4a(static_cast<int>(t[i]), ww.x, acc[4 * i + 0]);
-        acc[4 * i + 1] = __dp4a(static_cast<int>(t[i]), ww.y, acc[4 * i + 1]);
-        acc[4 * i + 2] = __dp4a(static_cast<int>(t[i]), ww.z, acc[4 * i + 2]);
-        acc[4 * i + 3] = __dp4a(static_cast<int>(t[i]), ww.w, acc[4 * i + 3]);
+        acc[4 * i + 0] = __dp4a(static_cast<int>(t[i]), w.x, acc[4 * i + 0]);
+        acc[4 * i + 1] = __dp4a(static_cast<int>(t[i]), w.y, acc[4 * i + 1]);
+        acc[4 * i + 2] = __dp4a(static_cast<int>(t[i]), w.z, acc[4 * i + 2]);
+        acc[4 * i + 3] = __dp4a(static_cast<int>(t[i]), w.w, acc[4 * i + 3]);
     }
 }
 
-// Sum the G lane groups' partial accumulators of one block-row and scatter
-// the result: afterwards group g holds tokens [g*8/G, (g+1)*8/G) of its
-// lanes' 8 (red[j*4 + c] = token g*8/G + j, channel c).
-template <int G>
-__device__ __forceinline__ void reduce_groups(int lane, const int (&acc)[32], int (&red)[32 / G]) {
+// Sum the partial accumulators of the 4 lanes that share g (they took
+// different quads of each step) and scatter: afterwards lane l holds red[j]
+// = token g + 16 (l % 4) + 8 (j / 4), channel j % 4.  Exact int32 adds.
+__device__ __forceinline__ void reduce_quads(int lane, const int (&acc)[32], int (&red)[8]) {
     constexpr unsigned kFull = 0xffffffffu;
-    const bool up = (lane & 16) != 0;
-    if (G == 1) {
+    const bool b1 = (lane & 2) != 0;
+    int k1[16];
 #pragma unroll
-        for (int j = 0; j < 32 / G; ++j) red[j] = acc[j];
-    } else if (G == 2) {
+    for (int j = 0; j < 16; ++j) {
+        const int send = b1 ? acc[j] : acc[16 + j];
+        const int keep = b1 ? acc[16 + j] : acc[j];
+        k1[j] = keep + __shfl_xor_sync(kFull, send, 2);
+    }
+    const bool b0 = (lane & 1) != 0;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int send = up ? acc[j] : acc[16 + j];
-            const int keep = up ? acc[16 + j] : acc[j];
-            red[j % (32 / G)] = keep + __shfl_xor_sync(kFull, send, 16);
-        }
-    } else {
-        int k1[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            const int send = up ? acc[j] : acc[16 + j];
-            const int keep = up ? acc[16 + j] : acc[j];
-            k1[j] = keep + __shfl_xor_sync(kFull, send, 16);
-        }
-        const bool up2 = (lane & 8) != 0;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int send = up2 ? k1[j] : k1[8 + j];
-            const int keep = up2 ? k1[8 + j] : k1[j];
-            red[j % (32 / G)] = keep + __shfl_xor_sync(kFull, send, 8);
-        }
+    for (int j = 0; j < 8; ++j) {
+        const int send = b0 ? k1[j] : k1[8 + j];
+        const int keep = b0 ? k1[8 + j] : k1[j];
+        red[j] = keep + __shfl_xor_sync(kFull, send, 1);
     }
 }
 
-template <int MT, int KIND, bool TMA>
+// This lane's view of the step records: ro points at the column offset of
+// row (lane % 16) of a step, rw at quad q's 4 channel words of the same
+// step; step s + i is at ro + 32 i, rw + 8 i.
+struct RecPtr {
+    const int* ro;
+    const int4* rw;
+    __device__ __forceinline__ RecPtr(const int4* recs, long long s, int lane, int q)
+        : ro(reinterpret_cast<const int*>(recs + s * 8) + (lane & 15)), rw(recs + s * 8 + 4 + q) {}
+    __device__ __forceinline__ void load(int i, int& off, int4& w) const {
+        off = __ldg(ro + 32 * i);
+        w = __ldg(rw + 8 * i);
+    }
+    __device__ __forceinline__ void advance(int steps) {
+        ro += 32 * steps;
+        rw += 8 * steps;
+    }
+};
+
+template <int KIND, bool TMA>
 __global__ void __launch_bounds__(kThreads, 1)
 bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sched) {
-    constexpr int LW = MT / 8;          // lanes spanning the token tile (8 tokens per lane)
-    constexpr int G = 32 / LW;          // lane groups per warp; they interleave a block-row's quads
-    constexpr int TPG = 8 / G;          // tokens per lane after the groups' sums are combined
-    constexpr int SW = slot_words(MT);  // MT tokens x 4 channels
-    constexpr int RC = ring_chunk(MT);  // records per ring chunk
-    constexpr int S = RC / G;           // steps (G quads each) per ring chunk
-    constexpr int kRec = 32;            // bytes per quad record
+    constexpr int SW = kTile * 4;  // slot words: 64 tokens x 4 channels
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ int s_qp[kRowWin + 1];          // quad offsets of the current block-row window
+    __shared__ int s_sp[kRowWin + 1];                  // step offsets of the current block-row window
     __shared__ __align__(8) unsigned long long s_bar;  // completion of the token tile's bulk copy
     __shared__ int s_cnt[kSlots];                      // warps that have added into each slot
+    __shared__ int s_wst[kWarps + 1];                  // first step of each warp in the window (relative)
 
-    const int K = w.K;
+    const int K = w.K, N = w.N;
     const int kpad = (K + 15) & ~15;
-    uint32_t* xt = reinterpret_cast<uint32_t*>(smem);
-    int* slots = reinterpret_cast<int*>(smem + static_cast<size_t>(kpad) * MT);
-    unsigned char* ring = reinterpret_cast<unsigned char*>(slots + kSlots * SW);
+    const uint32_t sbase = smem_addr(smem);
+    const uint32_t tb = (sbase + 127u) & ~127u;  // the token tile, 128-byte aligned
+    unsigned char* tile = smem + (tb - sbase);
+    int* slots = reinterpret_cast<int*>(tile + static_cast<size_t>(kpad) * kTile);
+    float4* s_scale = reinterpret_cast<float4*>(slots + kSlots * SW);  // [kRowWin]: block-row r - r_lo
+    float4* s_bias = s_scale + kRowWin;
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
-    const int g = lane / LW, li = lane % LW;
+    const int q = lane & 3, g = lane >> 2;
+    const uint32_t lb = 16u * static_cast<uint32_t>(lane >> 4);
+    const int ta = g + 16 * q;  // tokens this lane finishes: ta and ta + 8 of the tile
     const long long nbr = w.nbr;
 
     const uint32_t bar = smem_addr(&s_bar);
@@ -390,71 +381,70 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     unsigned phase = 0;
     long long u = sched.u[blockIdx.x];
     const long long u_end = sched.u[blockIdx.x + 1];
-    unsigned char* ringw = ring + warp * (kRingSlots * RC * kRec);
-    const uint32_t ring_s = smem_addr(ringw);
-    const uint32_t xlane = smem_addr(xt) + 8 * li;  // this lane's 8 tokens in every k-row
-    const int i0 = g * TPG;
 
-    long long staged = -1;  // token tile currently in xt
+    long long staged = -1;  // token tile currently in shared memory
     while (u < u_end) {
         // next window: one token tile, at most kRowWin consecutive block-rows
         const long long t = u / nbr;
         const int r_lo = static_cast<int>(u - t * nbr);
         const int r_hi = static_cast<int>(min(min(nbr, r_lo + (u_end - u)), static_cast<long long>(r_lo + kRowWin)));
         u += r_hi - r_lo;
-        const long long m0 = t * MT;
-        const long long m_lane = m0 + 8 * li + i0;  // first token this lane finishes
-        // quad offset of block-row r (r_lo <= r <= r_hi), from the window
-        auto qp = [&](int r) { return s_qp[r - r_lo]; };
-        auto row_of_q = [&](int q) { return r_lo + row_of(s_qp, 0, r_hi - r_lo, q); };
+        const long long m0 = t * kTile;
+        auto sp = [&](int r) { return s_sp[r - r_lo]; };
 
-        for (int i = tid; i <= r_hi - r_lo; i += kThreads) s_qp[i] = __ldg(w.qptr + r_lo + i);
+        for (int i = tid; i <= r_hi - r_lo; i += kThreads) s_sp[i] = __ldg(w.sptr + r_lo + i);
+        if (tid <= kWarps) {
+            // warps take an even split of the window's steps
+            const long long nst_w = __ldg(w.sptr + r_hi) - __ldg(w.sptr + r_lo);
+            s_wst[tid] = static_cast<int>(nst_w * tid / kWarps);
+        }
+        if (KIND != 0) {
+            for (int i = tid; i < 2 * (r_hi - r_lo); i += kThreads) {
+                const int rr = i >> 1;
+                if (i & 1) s_bias[rr] = load_s4(w.bias, r_lo + rr);
+                else s_scale[rr] = load_s4(w.scale, r_lo + rr);
+            }
+        }
         const bool stage = (t != staged);
         if (TMA && stage && tid == 0) {
-            // one bulk copy of the token tile (already k-major in a.xb)
-            const unsigned bytes = static_cast<unsigned>(kpad) * MT;
-            const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * MT;
+            // one bulk copy of the token tile (already swizzled in a.xb)
+            const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
+            const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * kTile;
             fence_proxy_async();
             mbar_arrive_expect_tx(bar, bytes);
             for (unsigned off = 0; off < bytes; off += 65536u)
-                bulk_g2s(smem_addr(xt) + off, src + off, min(65536u, bytes - off), bar);
+                bulk_g2s(tb + off, src + off, min(65536u, bytes - off), bar);
         }
         __syncthreads();  // the block-row window is visible
         if (!TMA && stage) {  // gather the tile with per-thread loads
-            stage_tile<MT>(xt, a, K, kpad, m0);
+            stage_tile(tile, a, K, kpad, m0);
             __syncthreads();
             staged = t;
         }
 
-        const int qa = qp(r_lo), qb = qp(r_hi);
-        // Every block-row holds a multiple of G quads, so the tile's quads form
-        // nst steps of G; warps take an even split of the steps.
-        const int nst = (qb - qa) / G;
-        auto wstep = [&](int wi) { return static_cast<int>(static_cast<long long>(wi) * nst / kWarps); };
-        const int ws0 = wstep(warp), ws1 = wstep(warp + 1);
-        const int wq0 = qa + ws0 * G, wq1 = qa + ws1 * G;
+        const int sa = sp(r_lo);
+        const int ws0 = s_wst[warp], ws1 = s_wst[warp + 1];
 
-        // Stream the warp's records [wq0, wq1) through the ring: chunk c =
-        // records wq0 + RC*c ..; one 16-byte copy per lane (RC*2 lanes).  The
-        // first chunks load while the token tile does.
-        const unsigned char* gsrc = reinterpret_cast<const unsigned char*>(w.quads) + static_cast<size_t>(wq0) * kRec;
-        const int nchunks = (wq1 - wq0 + RC - 1) / RC;
-        auto issue = [&](int c) {
-            if (c < nchunks && lane < RC * 2)
-                cp_async16(ring_s + (c % kRingSlots) * (RC * kRec) + 16 * lane,
-                           gsrc + static_cast<size_t>(c) * (RC * kRec) + 16 * lane);
-            cp_async_commit();
-        };
+        // The warp's first four step records load while the tile does; a
+        // record is loaded three steps before its use (the record array has
+        // kStepPad spare steps for the loads past the last one).
+        RecPtr rec(w.recs, sa + ws0, lane, q);  // at step p of the loop below
+        int off[4];
+        int4 wq[4];
 #pragma unroll
-        for (int c = 0; c < kRingSlots; ++c) issue(c);
+        for (int i = 0; i < 4; ++i) {
+            off[i] = 0;
+            wq[i] = make_int4(0, 0, 0, 0);
+            if (ws0 < ws1) rec.load(i, off[i], wq[i]);
+        }
 
         // Block-rows with no stored block: acc = 0.
         for (int r = r_lo + warp; r < r_hi; r += kWarps) {
-            if (qp(r) == qp(r + 1)) {
-                int red[TPG * 4];
-#pragma unroll
-                for (int j = 0; j < TPG * 4; ++j) red[j] = 0;
-                store_rows<KIND, TPG>(w, a, m_lane, r, red, load_s4(w.scale, r), load_s4(w.bias, r));
+            if (sp(r) == sp(r + 1)) {
+                const int zero[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                const float4 sc = s_scale[r - r_lo], bi = s_bias[r - r_lo];
+                store_token<KIND>(a, N, m0 + ta, r, zero, sc, bi);
+                store_token<KIND>(a, N, m0 + ta + 8, r, zero + 4, sc, bi);
             }
         }
 
@@ -466,66 +456,60 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                     atomicOr(w.status, kStatusTimeout);
                     mbar_wait(bar, (phase - 1) & 1u);  // give the copy one more bounded chance to land
                 }
-                cp_async_wait<0>();
                 __syncthreads();
                 return;
             }
             staged = t;
         }
 
-        if (wq0 < wq1) {
-            cp_async_wait<kRingSlots - 1>();  // chunk 0 has landed
-            __syncwarp();
-            int cur = 0;
-            int r = row_of_q(wq0);
-            int p = 0;  // step index relative to ws0
-            const int p_all = ws1 - ws0;
-            while (p < p_all) {
-                const int rs = qp(r), re_row = qp(r + 1);
-                const int p_end = min(p_all, (re_row - wq0) / G);
-                float4 sc = make_float4(0.f, 0.f, 0.f, 0.f), bi = sc;
-                if (KIND != 0) {  // needed at the row's end; load it now
-                    sc = load_s4(w.scale, r);
-                    bi = load_s4(w.bias, r);
-                }
+        if (ws0 < ws1) {
+            int r = r_lo + row_of(s_sp, 0, r_hi - r_lo, sa + ws0);
+            int p = ws0;  // step index relative to sa
+            while (p < ws1) {
+                const int rs = sp(r), re = sp(r + 1);
+                const int p_end = min(ws1, re - sa);
                 int acc[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) acc[i] = 0;
-                while (p < p_end) {
-                    const int cq = p / S;
-                    if (cq != cur) {  // entering the next chunk (cq == cur + 1)
-                        cur = cq;
-                        __syncwarp();  // everyone is done with chunk cur - 1, whose slot is refilled
-                        issue(cur + kRingSlots - 1);
-                        cp_async_wait<kRingSlots - 1>();  // chunk cur has landed
-                        __syncwarp();
+                // invariant: off/wq[i] hold step p + i
+                for (; p + 3 < p_end; p += 4) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        step16(tb, lb, off[i], wq[i], acc);
+                        rec.load(4 + i, off[i], wq[i]);
                     }
-                    const int seg_end = min(p_end, (cur + 1) * S);
-                    uint32_t rec = ring_s + (cur % kRingSlots) * (RC * kRec) + ((p - cur * S) * G + g) * kRec;
-                    for (; p + 1 < seg_end; p += 2, rec += 2 * G * kRec) {
-                        const int4 k0 = lds128(rec), w0 = lds128(rec + 16);
-                        const int4 k1 = lds128(rec + G * kRec), w1 = lds128(rec + G * kRec + 16);
-                        quad8<MT>(xlane, k0, w0, acc);
-                        quad8<MT>(xlane, k1, w1, acc);
-                    }
-                    if (p < seg_end) {
-                        const int4 k0 = lds128(rec), w0 = lds128(rec + 16);
-                        quad8<MT>(xlane, k0, w0, acc);
-                        ++p;
-                    }
+                    rec.advance(4);
                 }
-                int red[TPG * 4];
-                reduce_groups<G>(lane, acc, red);
-                if (rs >= wq0 && re_row <= wq1) {
-                    store_rows<KIND, TPG>(w, a, m_lane, r, red, sc, bi);
+                for (; p < p_end; ++p) {  // the row's last 0-3 steps: shift the ring by one
+                    step16(tb, lb, off[0], wq[0], acc);
+#pragma unroll
+                    for (int i = 0; i < 3; ++i) {
+                        off[i] = off[i + 1];
+                        wq[i] = wq[i + 1];
+                    }
+                    rec.load(4, off[3], wq[3]);
+                    rec.advance(1);
+                }
+                float4 sc = make_float4(0.f, 0.f, 0.f, 0.f), bi = sc;
+                if (KIND != 0) {
+                    sc = s_scale[r - r_lo];
+                    bi = s_bias[r - r_lo];
+                }
+                int red[8];
+                reduce_quads(lane, acc, red);
+                if (rs >= sa + ws0 && re <= sa + ws1) {
+                    store_token<KIND>(a, N, m0 + ta, r, red, sc, bi);
+                    store_token<KIND>(a, N, m0 + ta + 8, r, red + 4, sc, bi);
                 } else {
                     // Shared with other warps: sum into the slot of the first warp
-                    // split inside the block-row; the last warp to add finishes it.
-                    const int s0 = (rs - qa) / G, s1 = (re_row - qa) / G;  // the row's steps
-                    const int b = static_cast<int>((static_cast<long long>(s0 + 1) * kWarps + nst - 1) / nst);
-                    int* sl = slots + (b - 1) * SW + li;
+                    // boundary inside the block-row (the first b with s_wst[b] > s0);
+                    // the last warp to add finishes it.
+                    const int s0 = rs - sa, s1 = re - sa;  // the row's steps
+                    int b = 1;
+                    while (s_wst[b] <= s0) ++b;
+                    int* sl = slots + (b - 1) * SW;
 #pragma unroll
-                    for (int j = 0; j < TPG * 4; ++j) atomicAdd(sl + (4 * i0 + j) * LW, red[j]);
+                    for (int j = 0; j < 8; ++j) atomicAdd(sl + (ta + 8 * (j >> 2)) * 4 + (j & 3), red[j]);
                     __syncwarp();
                     int arrived = 0;
                     if (lane == 0) {
@@ -534,47 +518,46 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                     }
                     arrived = __shfl_sync(0xffffffffu, arrived, 0);
                     int parts = 0;  // warps whose step range meets the row's
-                    for (int wi = 0; wi < kWarps; ++wi) {
-                        const int a0 = wstep(wi), a1 = wstep(wi + 1);
-                        parts += (a0 < a1 && a0 < s1 && a1 > s0) ? 1 : 0;
-                    }
+                    for (int wi = b - 1; wi < kWarps && s_wst[wi] < s1; ++wi)
+                        parts += (s_wst[wi] < s_wst[wi + 1]) ? 1 : 0;
                     if (arrived == parts) {
                         __threadfence_block();
 #pragma unroll
-                        for (int j = 0; j < TPG * 4; ++j) red[j] = atomicExch(sl + (4 * i0 + j) * LW, 0);
-                        store_rows<KIND, TPG>(w, a, m_lane, r, red, sc, bi);
+                        for (int j = 0; j < 8; ++j) red[j] = atomicExch(sl + (ta + 8 * (j >> 2)) * 4 + (j & 3), 0);
+                        store_token<KIND>(a, N, m0 + ta, r, red, sc, bi);
+                        store_token<KIND>(a, N, m0 + ta + 8, r, red + 4, sc, bi);
                         if (lane == 0) s_cnt[b - 1] = 0;
                     }
                 }
                 ++r;
-                while (r < r_hi && qp(r + 1) == qp(r)) ++r;  // skip block-rows without quads
+                while (r < r_hi && sp(r + 1) == sp(r)) ++r;  // skip block-rows without steps
             }
         }
-        cp_async_wait<0>();
-        __syncthreads();  // the tile, window, ring and slots may be reused
+        __syncthreads();  // the tile, window and slots may be reused
     }
 }
 
-// Token-tile relayout: xb[t][k][j] = x[t*MT + j][k] for k < kpad (zero when
-// t*MT + j >= M or k >= K).  A persistent CTA walks items (tile t, block of
-// KC columns): MT tokens x KC columns (16 KB) through shared memory --
-// 16-byte row loads, a 4x4 byte transpose per thread, 16-byte stores of the
-// k-major block, which is contiguous in xb.  The next item's loads are in
-// flight (in registers) while the current item is transposed and stored.
-template <int MT>
+// Token-tile relayout: x [M][K] -> swizzled tiles (tile t = tokens
+// 64t..64t+63, all kpad columns; zero past M or K).  A persistent CTA walks
+// items (tile t, block of 256 columns): 64 tokens x 256 columns (16 KB)
+// through shared memory -- 16-byte row loads, a 4x4 byte transpose per
+// thread, then each 16-token chunk of a column is one 16-byte store into its
+// slot of the swizzled tile (a block of 256 columns is 128 whole lines,
+// written contiguously).  The next item's loads are in flight (in
+// registers) while the current item is transposed and stored.
 __global__ void __launch_bounds__(256)
 pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __restrict__ xb, long long items,
                int ncb) {
-    constexpr int KC = 16384 / MT;     // columns per item (256 or 128)
-    constexpr int C16 = KC / 16;       // 16-byte chunks per raw row
-    constexpr int RW = KC / 4 + 4;     // raw row stride in words (rows shift by 4 banks)
-    constexpr int OS = MT / 4 + 1;     // transposed row stride in words
-    constexpr int NL = (MT * C16) / 256;  // row loads per thread and item
-    __shared__ __align__(16) uint32_t raw[MT * RW];
+    constexpr int KC = 256;               // columns per item
+    constexpr int C16 = KC / 16;          // 16-byte chunks per raw row
+    constexpr int RW = KC / 4 + 4;        // raw row stride in words (rows shift by 4 banks)
+    constexpr int OS = kTile / 4 + 1;     // transposed row stride in words
+    constexpr int NL = (kTile * C16) / 256;  // row loads per thread and item
+    __shared__ __align__(16) uint32_t raw[kTile * RW];
     __shared__ uint32_t tr[KC * OS];
     const bool vec16 = ((K & 15) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
     auto load_item = [&](long long it, uint4 (&v)[NL]) {
-        const long long m0 = (it / ncb) * MT;
+        const long long m0 = (it / ncb) * kTile;
         const int k0 = static_cast<int>(it % ncb) * KC;
 #pragma unroll
         for (int i = 0; i < NL; ++i) {
@@ -611,7 +594,7 @@ pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __r
         }
         __syncthreads();  // raw is complete; every thread is past the previous item's stores
         if (it + gridDim.x < items) load_item(it + gridDim.x, v);
-        for (int i = threadIdx.x; i < (MT / 4) * (KC / 4); i += 256) {
+        for (int i = threadIdx.x; i < (kTile / 4) * (KC / 4); i += 256) {
             const int j = i % (KC / 4), g = i / (KC / 4);
             uint32_t t0, t1, t2, t3;
             transpose4(raw[(4 * g + 0) * RW + j], raw[(4 * g + 1) * RW + j], raw[(4 * g + 2) * RW + j],
@@ -622,106 +605,85 @@ pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __r
             tr[(4 * j + 3) * OS + g] = t3;
         }
         __syncthreads();  // tr is complete; raw may be refilled
-        int8_t* dst = xb + (static_cast<size_t>(t) * kpad + k0) * MT;
-        for (int i = threadIdx.x; i < kc * (MT / 16); i += 256) {
-            const int row = i / (MT / 16), c = i % (MT / 16);
+        int8_t* dst = xb + static_cast<size_t>(t) * kpad * kTile;
+        for (int i = threadIdx.x; i < kc * 4; i += 256) {
+            const int row = i >> 2, c = i & 3;
             const uint32_t* srow = tr + row * OS + 4 * c;
-            *reinterpret_cast<uint4*>(dst + static_cast<size_t>(row) * MT + 16 * c) =
+            *reinterpret_cast<uint4*>(dst + (row_off(k0 + row) ^ (static_cast<uint32_t>(c) << 4))) =
                 make_uint4(srow[0], srow[1], srow[2], srow[3]);
         }
     }
 }
 
-template <int MT, bool TMA>
+template <bool TMA>
 const void* kernel_for(int kind) {
     switch (kind) {
-    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 0, TMA>);
-    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 1, TMA>);
-    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 2, TMA>);
-    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 3, TMA>);
-    default: return reinterpret_cast<const void*>(&bsgemm_kernel<MT, 4, TMA>);
+    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<0, TMA>);
+    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<1, TMA>);
+    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<2, TMA>);
+    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<3, TMA>);
+    default: return reinterpret_cast<const void*>(&bsgemm_kernel<4, TMA>);
     }
-}
-
-const void* kernel_ptr(int MT, int kind, bool tma) {
-    if (MT == 128) return tma ? kernel_for<128, true>(kind) : kernel_for<128, false>(kind);
-    return tma ? kernel_for<64, true>(kind) : kernel_for<64, false>(kind);
 }
 
 }  // namespace
 
-size_t smem_bytes(int MT, int K) {
+size_t smem_bytes(int K) {
     const size_t kpad = (static_cast<size_t>(K) + 15) & ~static_cast<size_t>(15);
-    return kpad * MT + static_cast<size_t>(kSlots) * slot_words(MT) * 4 + ring_bytes(MT);
-}
-
-int tile_for_k(int K) {
-    if (K < 1) return 0;
-    if (smem_bytes(128, K) + kStaticSmem <= static_cast<size_t>(kSmemOptin)) return 128;
-    if (smem_bytes(64, K) + kStaticSmem <= static_cast<size_t>(kSmemOptin)) return 64;
-    return 0;
+    // 128 bytes of slack to align the tile, the tile, the split-row slots,
+    // the window's scales and biases
+    return 128 + kpad * kTile + static_cast<size_t>(kSlots) * kTile * 4 * sizeof(int) +
+           2 * static_cast<size_t>(kRowWin) * sizeof(float4);
 }
 
 int max_k() {
     int k = 16;
-    while (tile_for_k(k + 16)) k += 16;
+    while (smem_bytes(k + 16) + kStaticSmem <= static_cast<size_t>(kSmemOptin)) k += 16;
     return k;
 }
 
-cudaError_t prepare_kernels(int MT, int K, int* ctas_per_sm) {
-    const int smem = static_cast<int>(smem_bytes(MT, K));
+cudaError_t prepare_kernels(int K, int* ctas_per_sm) {
+    const int smem = static_cast<int>(smem_bytes(K));
     for (int kind = 0; kind < 5; ++kind) {
         for (int tma = 0; tma < 2; ++tma) {
-            cudaError_t e = cudaFuncSetAttribute(kernel_ptr(MT, kind, tma != 0),
+            cudaError_t e = cudaFuncSetAttribute(tma ? kernel_for<true>(kind) : kernel_for<false>(kind),
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemOptin - kStaticSmem);
             if (e != cudaSuccess) return e;
         }
     }
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_ptr(MT, 0, true), kThreads, smem);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_for<true>(0), kThreads, smem);
 }
 
-cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int MT, int grid,
-                   cudaStream_t s) {
-    const size_t smem = smem_bytes(MT, w.K);
-#define BSG_LAUNCH(MTV, KV)                                                                   \
-    do {                                                                                      \
-        if (a.xb) bsgemm_kernel<MTV, KV, true><<<grid, kThreads, smem, s>>>(w, a, sched);     \
-        else bsgemm_kernel<MTV, KV, false><<<grid, kThreads, smem, s>>>(w, a, sched);         \
+cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int grid, cudaStream_t s) {
+    const size_t smem = smem_bytes(w.K);
+#define BSG_LAUNCH(KV)                                                                  \
+    do {                                                                                \
+        if (a.xb) bsgemm_kernel<KV, true><<<grid, kThreads, smem, s>>>(w, a, sched);    \
+        else bsgemm_kernel<KV, false><<<grid, kThreads, smem, s>>>(w, a, sched);        \
     } while (0)
-    if (MT == 128) {
-        switch (a.kind) {
-        case 0: BSG_LAUNCH(128, 0); break;
-        case 1: BSG_LAUNCH(128, 1); break;
-        case 2: BSG_LAUNCH(128, 2); break;
-        case 3: BSG_LAUNCH(128, 3); break;
-        default: BSG_LAUNCH(128, 4); break;
-        }
-    } else {
-        switch (a.kind) {
-        case 0: BSG_LAUNCH(64, 0); break;
-        case 1: BSG_LAUNCH(64, 1); break;
-        case 2: BSG_LAUNCH(64, 2); break;
-        case 3: BSG_LAUNCH(64, 3); break;
-        default: BSG_LAUNCH(64, 4); break;
-        }
+    switch (a.kind) {
+    case 0: BSG_LAUNCH(0); break;
+    case 1: BSG_LAUNCH(1); break;
+    case 2: BSG_LAUNCH(2); break;
+    case 3: BSG_LAUNCH(3); break;
+    default: BSG_LAUNCH(4); break;
     }
 #undef BSG_LAUNCH
     return cudaGetLastError();
 }
 
-size_t tiled_bytes(int MT, int K, long long M) {
+size_t tiled_bytes(int K, long long M) {
     const size_t kpad = (static_cast<size_t>(K) + 15) & ~static_cast<size_t>(15);
-    return static_cast<size_t>((M + MT - 1) / MT) * kpad * MT;
+    return static_cast<size_t>((M + kTile - 1) / kTile) * kpad * kTile;
 }
 
-cudaError_t launch_pretile(const int8_t* x, int M, int K, int MT, int8_t* xb, int sms, cudaStream_t s) {
+cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, cudaStream_t s) {
     const int kpad = (K + 15) & ~15;
-    const int ncb = (kpad + 16384 / MT - 1) / (16384 / MT);
-    const long long items = (static_cast<long long>(M) + MT - 1) / MT * ncb;
+    const int ncb = (kpad + 255) / 256;
+    const long long items = (static_cast<long long>(M) + kTile - 1) / kTile * ncb;
     const long long cap = 4LL * (sms > 0 ? sms : 1);  // 4 resident CTAs per SM (35 KB of shared memory each)
     const unsigned grid = static_cast<unsigned>(items < cap ? items : cap);
-    if (MT == 128) pretile_kernel<128><<<grid, 256, 0, s>>>(x, M, K, kpad, xb, items, ncb);
-    else pretile_kernel<64><<<grid, 256, 0, s>>>(x, M, K, kpad, xb, items, ncb);
+    pretile_kernel<<<grid, 256, 0, s>>>(x, M, K, kpad, xb, items, ncb);
     return cudaGetLastError();
 }
 
