@@ -20,7 +20,7 @@ struct bsgemm_ctx {
     int64_t nnzb = 0;
     void* arena = nullptr;
     size_t arena_bytes = 0;
-    std::vector<int32_t> cost;  // host copy of the schedule's prefix cost [nbr + 1]
+    std::vector<int32_t> cost;  // schedule prefix cost of the row groups [ngroups + 1]
     bsg::DeviceWeights w{};
     std::mutex sched_mu;        // guards the cached schedule of the last token count
     long long sched_m = -1;
@@ -69,23 +69,23 @@ std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx
     return "";
 }
 
-// Schedule costs, in steps (16 stored blocks of one block-row for 64
-// tokens: 32 dp4a per lane): every block-row adds kRowCost for its
-// cross-lane sum and epilogue, every token tile in a CTA's range adds
-// kTileCost for its copy into shared memory and the start-up around it.
-constexpr long long kRowCost = 2;
+// Schedule costs, in steps (one quad of each of a row group's 4 block-rows
+// for 64 tokens: 32 dp4a per lane): every row group adds kGroupCost for its
+// epilogue, every token tile in a CTA's range adds kTileCost for its copy
+// into shared memory and the start-up around it.
+constexpr long long kGroupCost = 4;
 constexpr long long kTileCost = 250;
 
 // End of the greedy range that starts at unit u under the cost bound C: it
 // takes whole units while the cost (units' cost + tc per token tile
 // touched) stays within C, and at least one unit.
-long long fill_range(const std::vector<int32_t>& cost, long long nbr, long long ntiles, long long tc, long long C,
+long long fill_range(const std::vector<int32_t>& cost, long long upt, long long ntiles, long long tc, long long C,
                      long long u) {
-    long long t = u / nbr, r = u - t * nbr, left = C;
+    long long t = u / upt, r = u - t * upt, left = C;
     bool first = true;
     while (t < ntiles) {
         left -= tc;
-        const long long rest = cost[nbr] - cost[r];
+        const long long rest = cost[upt] - cost[r];
         if (left >= rest) {  // the rest of this tile fits
             left -= rest;
             ++t;
@@ -94,27 +94,28 @@ long long fill_range(const std::vector<int32_t>& cost, long long nbr, long long 
             continue;
         }
         // the largest e with cost[e] - cost[r] <= left
-        long long e = std::upper_bound(cost.begin() + r, cost.begin() + nbr + 1, cost[r] + (left > 0 ? left : 0)) -
+        long long e = std::upper_bound(cost.begin() + r, cost.begin() + upt + 1, cost[r] + (left > 0 ? left : 0)) -
                       cost.begin() - 1;
         if (e <= r && first) e = r + 1;  // at least one unit
-        return t * nbr + (e > r ? e : r);
+        return t * upt + (e > r ? e : r);
     }
-    return ntiles * nbr;
+    return ntiles * upt;
 }
 
-// Contiguous unit ranges (tile-major units t * nbr + r), one per CTA, with
-// the largest range cost as small as bisection on the bound finds it;
-// returns the number of ranges (<= cap, each non-empty).
-int make_schedule(const std::vector<int32_t>& cost, long long nbr, long long ntiles, int cap, long long tc,
+// Contiguous unit ranges (tile-major units t * upt + r, upt = row groups
+// per token tile), one per CTA, with the largest range cost as small as
+// bisection on the bound finds it; returns the number of ranges (<= cap,
+// each non-empty).
+int make_schedule(const std::vector<int32_t>& cost, long long upt, long long ntiles, int cap, long long tc,
                   bsg::Schedule& sched) {
-    const long long end = ntiles * nbr;
+    const long long end = ntiles * upt;
     auto ranges = [&](long long C) {
         int n = 0;
-        for (long long u = 0; u < end; u = fill_range(cost, nbr, ntiles, tc, C, u))
+        for (long long u = 0; u < end; u = fill_range(cost, upt, ntiles, tc, C, u))
             if (++n > cap) break;
         return n;
     };
-    long long hi = ntiles * (cost[nbr] + tc), lo = 0;
+    long long hi = ntiles * (cost[upt] + tc), lo = 0;
     while (hi - lo > 1) {
         const long long mid = lo + (hi - lo) / 2;
         if (ranges(mid) <= cap) hi = mid; else lo = mid;
@@ -122,7 +123,7 @@ int make_schedule(const std::vector<int32_t>& cost, long long nbr, long long nti
     int n = 0;
     sched.u[0] = 0;
     for (long long u = 0; u < end;) {
-        u = fill_range(cost, nbr, ntiles, tc, hi, u);
+        u = fill_range(cost, upt, ntiles, tc, hi, u);
         sched.u[++n] = u;
     }
     return n;
@@ -186,83 +187,108 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         }
     }
 
-    // Repack into steps.  Per block-row the stored columns are ordered so
-    // that each half-step (8 consecutive columns, one pass of the kernel's
-    // shared-memory gather) takes its columns from distinct bank groups of
-    // the swizzled token tile where it can: every half-step draws one
-    // column from each of the 8 bank-key buckets with the most columns left,
-    // then (if fewer than 8 buckets are left) again from the fullest; the
-    // last step is padded with zero-weight entries on unused keys (columns
-    // 0..7 cover all 8 keys and are rows of every tile, which has
-    // round_up(K, 16) >= 16 rows).
-    std::vector<int32_t> sptr(nbr + 1, 0);
-    std::vector<int32_t> cost(nbr + 1, 0);
-    for (int r = 0; r < nbr; ++r) {
-        const int nz = indptr[r + 1] - indptr[r];
-        sptr[r + 1] = sptr[r] + (nz + 15) / 16;
-        cost[r + 1] = static_cast<int32_t>(cost[r] + (nz + 15) / 16 + (nz > 0 ? kRowCost : 0));
+    // Repack into row groups and steps.  Block-rows sorted by stored-block
+    // count (longest first, ties by index) are taken 4 at a time, so a
+    // group's block-rows need about the same number of quads.  Each half of
+    // a step (8 columns: one quad of block-row 2h, one of block-row 2h + 1,
+    // one pass of the kernel's shared-memory gather) takes its columns from
+    // distinct bank groups of the swizzled token tile where it can: pick by
+    // pick, the block-row whose fullest bucket of an unused bank key is
+    // largest takes a column from it; a block-row whose remaining columns
+    // all sit on used keys takes one anyway (a conflict, never an extra
+    // step); a block-row with no columns left is padded with a zero-weight
+    // entry on an unused key (columns 0..7 cover all 8 keys and are rows of
+    // every tile, which has round_up(K, 16) >= 16 rows).
+    const int ngroups = (nbr + 3) / 4;
+    std::vector<int> rows_sorted(nbr);
+    for (int r = 0; r < nbr; ++r) rows_sorted[r] = r;
+    std::stable_sort(rows_sorted.begin(), rows_sorted.end(),
+                     [&](int x, int y) { return indptr[x + 1] - indptr[x] > indptr[y + 1] - indptr[y]; });
+    std::vector<int32_t> grow(static_cast<size_t>(ngroups) * 4, -1);
+    std::vector<int32_t> gptr(ngroups + 1, 0);
+    std::vector<int32_t> cost(ngroups + 1, 0);
+    for (int gi = 0; gi < ngroups; ++gi) {
+        int quads = 0;
+        for (int q = 0; q < 4 && 4 * gi + q < nbr; ++q) {
+            const int r = rows_sorted[4 * gi + q];
+            grow[4 * gi + q] = r;
+            quads = std::max(quads, (indptr[r + 1] - indptr[r] + 3) / 4);
+        }
+        gptr[gi + 1] = gptr[gi] + quads;
+        cost[gi + 1] = static_cast<int32_t>(cost[gi] + quads + (quads > 0 ? kGroupCost : 0));
     }
-    const int S = sptr[nbr];
+    const int S = gptr[ngroups];
     std::vector<int32_t> recs(static_cast<size_t>(S + bsg::kStepPad) * 32, 0);
     int pad_col[8];
     for (int k = 0; k < 8; ++k) pad_col[bsg::bank_key(k)] = k;
     {
-        std::vector<int> bucket[8];
-        std::vector<int> order;  // stored-block index j, or -1 - key for a padding entry
-        for (int r = 0; r < nbr; ++r) {
-            const int j0 = indptr[r], j1 = indptr[r + 1];
-            if (j1 == j0) continue;
-            for (auto& b : bucket) b.clear();
-            for (int j = j1 - 1; j >= j0; --j) bucket[bsg::bank_key(colidx[j])].push_back(j);  // popped in column order
-            const int entries = (sptr[r + 1] - sptr[r]) * 16;
-            order.clear();
-            int left = j1 - j0;
-            while (static_cast<int>(order.size()) < entries) {
-                int keys[8] = {0, 1, 2, 3, 4, 5, 6, 7};
-                std::stable_sort(keys, keys + 8, [&](int x, int y) { return bucket[x].size() > bucket[y].size(); });
-                bool used[8] = {false, false, false, false, false, false, false, false};
-                int taken = 0;
-                for (int i = 0; i < 8 && taken < 8; ++i) {
-                    if (bucket[keys[i]].empty()) continue;
-                    order.push_back(bucket[keys[i]].back());
-                    bucket[keys[i]].pop_back();
-                    used[keys[i]] = true;
-                    ++taken;
-                    --left;
-                }
-                while (taken < 8 && left > 0) {  // fewer than 8 keys left: repeat the fullest
-                    int best = 0;
-                    for (int x = 1; x < 8; ++x)
-                        if (bucket[x].size() > bucket[best].size()) best = x;
-                    order.push_back(bucket[best].back());
-                    bucket[best].pop_back();
-                    used[best] = true;
-                    ++taken;
-                    --left;
-                }
-                for (int x = 0; x < 8 && taken < 8; ++x) {  // padding on keys this half-step does not use
-                    if (used[x]) continue;
-                    order.push_back(-1 - x);
-                    used[x] = true;
-                    ++taken;
-                }
+        std::vector<int> bucket[4][8];  // stored-block indices j of each block-row, by bank key
+        int left[4];
+        for (int gi = 0; gi < ngroups; ++gi) {
+            for (int q = 0; q < 4; ++q) {
+                for (auto& bk : bucket[q]) bk.clear();
+                left[q] = 0;
+                const int r = grow[4 * gi + q];
+                if (r < 0) continue;
+                for (int j = indptr[r + 1] - 1; j >= indptr[r]; --j) bucket[q][bsg::bank_key(colidx[j])].push_back(j);
+                left[q] = indptr[r + 1] - indptr[r];
             }
-            for (int s = 0; s < sptr[r + 1] - sptr[r]; ++s) {
-                int32_t* rec = &recs[static_cast<size_t>(sptr[r] + s) * 32];
+            for (int s = gptr[gi]; s < gptr[gi + 1]; ++s) {
+                int32_t* rec = &recs[static_cast<size_t>(s) * 32];
                 uint32_t wwords[4][4] = {};
-                for (int e = 0; e < 16; ++e) {
-                    const int o = order[16 * s + e];
-                    if (o >= 0) {
-                        rec[e] = static_cast<int32_t>(bsg::tile_row_offset(colidx[o]));
-                        for (int c = 0; c < 4; ++c)
-                            wwords[e / 4][c] |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(o) * 4 + c]))
+                for (int h = 0; h < 2; ++h) {
+                    bool used[8] = {false, false, false, false, false, false, false, false};
+                    int placed[2] = {0, 0};
+                    for (int n = 0; n < 8; ++n) {
+                        // candidate of each of the two block-rows still short of 4 entries:
+                        // the size of its fullest bucket on an unused key (-1: none)
+                        int best_x = -1, best_key = -1, best_size = -2;
+                        for (int x = 0; x < 2; ++x) {
+                            const int q = 2 * h + x;
+                            if (placed[x] == 4) continue;
+                            int key = -1, size = -1;
+                            for (int kk = 0; kk < 8; ++kk)
+                                if (!used[kk] && static_cast<int>(bucket[q][kk].size()) > size &&
+                                    !bucket[q][kk].empty()) {
+                                    key = kk;
+                                    size = static_cast<int>(bucket[q][kk].size());
+                                }
+                            if (size > best_size || (size == best_size && left[q] > left[2 * h + best_x])) {
+                                best_x = x;
+                                best_key = key;
+                                best_size = size;
+                            }
+                        }
+                        const int q = 2 * h + best_x;
+                        const int e = 4 * q + placed[best_x];
+                        int j = -1, key = best_key;
+                        if (key < 0 && left[q] > 0) {  // its columns sit on used keys only: take a conflict
+                            for (int kk = 0; kk < 8; ++kk)
+                                if (key < 0 || bucket[q][kk].size() > bucket[q][key].size()) key = kk;
+                        }
+                        if (key >= 0 && left[q] > 0) {
+                            j = bucket[q][key].back();
+                            bucket[q][key].pop_back();
+                            --left[q];
+                        } else {  // padding on an unused key (any key if all are used)
+                            key = 0;
+                            for (int kk = 7; kk >= 0; --kk)
+                                if (!used[kk]) key = kk;
+                        }
+                        used[key] = true;
+                        ++placed[best_x];
+                        if (j >= 0) {
+                            rec[e] = static_cast<int32_t>(bsg::tile_row_offset(colidx[j]));
+                            for (int c = 0; c < 4; ++c)
+                                wwords[q][c] |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(j) * 4 + c]))
                                                 << (8 * (e % 4));
-                    } else {
-                        rec[e] = static_cast<int32_t>(bsg::tile_row_offset(pad_col[-1 - o]));
+                        } else {
+                            rec[e] = static_cast<int32_t>(bsg::tile_row_offset(pad_col[key]));
+                        }
                     }
                 }
-                for (int qd = 0; qd < 4; ++qd)
-                    for (int c = 0; c < 4; ++c) rec[16 + 4 * qd + c] = static_cast<int32_t>(wwords[qd][c]);
+                for (int q = 0; q < 4; ++q)
+                    for (int c = 0; c < 4; ++c) rec[16 + 4 * q + c] = static_cast<int32_t>(wwords[q][c]);
             }
         }
     }
@@ -296,8 +322,9 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         return nullptr;
     }
 
-    const size_t off_sptr = 0;
-    const size_t off_recs = align_up(off_sptr + sizeof(int32_t) * (nbr + 1), 256);
+    const size_t off_gptr = 0;
+    const size_t off_grow = align_up(off_gptr + sizeof(int32_t) * (ngroups + 1), 256);
+    const size_t off_recs = align_up(off_grow + sizeof(int32_t) * grow.size(), 256);
     const size_t off_scale = align_up(off_recs + sizeof(int32_t) * recs.size(), 256);
     const size_t off_bias = align_up(off_scale + sizeof(float) * N, 256);
     const size_t off_status = align_up(off_bias + sizeof(float) * N, 256);
@@ -310,7 +337,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     }
     char* base = static_cast<char*>(h->arena);
     struct Piece { size_t off; const void* src; size_t bytes; } pieces[] = {
-        {off_sptr, sptr.data(), sizeof(int32_t) * sptr.size()},
+        {off_gptr, gptr.data(), sizeof(int32_t) * gptr.size()},
+        {off_grow, grow.data(), sizeof(int32_t) * grow.size()},
         {off_recs, recs.data(), sizeof(int32_t) * recs.size()},
         {off_scale, scales, sizeof(float) * N},
         {off_bias, bias_v.data(), sizeof(float) * N},
@@ -327,14 +355,15 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     }
     h->nnzb = nnzb;
     h->cost = cost;
-    h->w.sptr = reinterpret_cast<const int32_t*>(base + off_sptr);
+    h->w.gptr = reinterpret_cast<const int32_t*>(base + off_gptr);
+    h->w.grow = reinterpret_cast<const int4*>(base + off_grow);
     h->w.recs = reinterpret_cast<const int4*>(base + off_recs);
     h->w.scale = reinterpret_cast<const float*>(base + off_scale);
     h->w.bias = reinterpret_cast<const float*>(base + off_bias);
     h->w.status = reinterpret_cast<int*>(base + off_status);
     h->w.N = N;
     h->w.K = K;
-    h->w.nbr = nbr;
+    h->w.ngroups = ngroups;
     h->w.S = S;
     return h;
 }
@@ -384,7 +413,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.inv_out_scale = inv;
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
     const long long ntiles = (static_cast<long long>(M) + bsg::kTile - 1) / bsg::kTile;
-    const long long nbr = h->w.nbr;
+    const long long upt = h->w.ngroups;  // units per token tile
     long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
     if (cap > bsg::kMaxGrid) cap = bsg::kMaxGrid;
     bsg::Schedule sched;
@@ -392,7 +421,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     {
         std::lock_guard<std::mutex> lock(h->sched_mu);
         if (h->sched_m != M) {
-            h->sched_grid = make_schedule(h->cost, nbr, ntiles, static_cast<int>(cap), kTileCost, h->sched);
+            h->sched_grid = make_schedule(h->cost, upt, ntiles, static_cast<int>(cap), kTileCost, h->sched);
             h->sched_m = M;
         }
         grid = h->sched_grid;

@@ -28,23 +28,29 @@ inline int bank_key(int k) { return static_cast<int>((tile_row_offset(k) >> 4) &
 
 // Device form of one block-compressed weight (built once by bsgemm_create).
 //
-// A block-row r holds output rows 4r..4r+3.  Its stored blocks (columns)
-// are ordered and grouped in "steps" of 16; steps of block-row r are
-// [sptr[r], sptr[r+1]).  A step is a 128-byte record (8 int4):
-//   int32 off[16]  : tile_row_offset(k_j) of its columns k_0..k_15
-//   uint32 w[4][4] : w[q][c] = bytes W[4r+c][k_{4q}] .. W[4r+c][k_{4q+3}],
-//                    one dot-4 operand per output channel c and quad q
-// (quad q = columns 4q..4q+3, the analogue of Algorithm 1's k_block = 4).
-// The last step of a block-row is padded with zero-weight entries whose
-// columns are valid tile rows.  Within each half of a step (columns 0-7,
-// 8-15) the columns' bank keys differ wherever the row's columns allow it.
+// A block-row r holds output rows 4r..4r+3.  Block-rows are sorted by their
+// number of stored blocks and taken 4 at a time into "row groups"
+// (grow[gi] = the group's block-rows, -1 where the last group has fewer
+// than 4).  A group is processed in steps; step s of group gi (gptr[gi] <=
+// s < gptr[gi+1]) holds one quad -- 4 stored columns, the analogue of
+// Algorithm 1's k_block = 4 -- of each of the group's 4 block-rows, as a
+// 128-byte record (8 int4):
+//   int32 off[16]  : tile_row_offset(k_e) of its 16 columns; columns 4q..4q+3
+//                    belong to the group's block-row q
+//   uint32 w[4][4] : w[q][c] = bytes W[4 r_q + c][k_{4q}] .. W[4 r_q + c][k_{4q+3}],
+//                    one dot-4 operand per output channel c of block-row q
+// A group has as many steps as its longest block-row has quads; shorter
+// block-rows are padded with zero-weight entries whose columns are valid
+// tile rows.  Within each half of a step (columns 0-7, 8-15) the columns'
+// bank keys differ wherever the two block-rows' columns allow it.
 struct DeviceWeights {
-    const int32_t* sptr;   // [nbr + 1]
+    const int32_t* gptr;   // [ngroups + 1]
+    const int4* grow;      // [ngroups]
     const int4* recs;      // [8 * (S + kStepPad)]
     const float* scale;    // [N]
     const float* bias;     // [N]
     int* status;           // device status word (bounded-wait timeouts), 0 = fine
-    int N, K, nbr, S;
+    int N, K, ngroups, S;
 };
 
 // Device status bits written by the kernels.
@@ -60,17 +66,19 @@ struct LaunchArgs {
     bool x_vec16;          // x 16-byte aligned and K % 16 == 0
 };
 
-// Kernel configuration: 16 warps per CTA.
-constexpr int kWarps = 16;
+// Kernel configuration: 8 warps per CTA (2 per SM sub-partition, up to 255
+// registers a thread).
+constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
-constexpr int kStepPad = 4;         // zero step records after the last one (record prefetch runs ahead)
-constexpr int kRowWin = 256;        // block-rows whose step offsets, scales and biases a CTA keeps in shared memory
+constexpr int kRing = 8;            // step records a warp keeps in flight (registers)
+constexpr int kStepPad = kRing;     // zero step records after the last one (the record prefetch runs ahead)
+constexpr int kGroupWin = 512;      // row groups whose step offsets a CTA keeps in shared memory
 constexpr int kStaticSmem = 2304;   // bytes of static shared memory the kernel may use
 constexpr int kMaxGrid = 512;       // CTAs per launch at most
 
 // Unit ranges of a launch: CTA c processes units [u[c], u[c+1]) of the
-// tile-major list (token tile t, block-row r) -> t * nbr + r.  Computed on
-// the host so that the kernel starts without a search.
+// tile-major list (token tile t, row group gi) -> t * ngroups + gi.
+// Computed on the host so that the kernel starts without a search.
 struct Schedule {
     long long u[kMaxGrid + 1];
 };

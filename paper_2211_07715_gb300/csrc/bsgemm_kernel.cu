@@ -8,31 +8,31 @@
 //
 // GB300 design (not a translation of the paper's AVX-512 loop nest):
 //
-// * Unit of work: (token tile t, block-row r) -- 64 tokens x 4 output
-//   channels, reduced over the block-row's stored columns.  Units are
-//   ordered tile-major and split into one contiguous, cost-balanced range per
-//   CTA of a persistent grid (CTAs = SMs x resident CTAs).
+// * Block-rows are sorted by length and taken 4 at a time into row groups
+//   (16 output channels).  Unit of work: (token tile t, row group) -- 64
+//   tokens x 16 channels.  Units are ordered tile-major and split into one
+//   contiguous, cost-balanced range per CTA of a persistent grid (CTAs =
+//   SMs x resident CTAs).
 // * The CTA stages its token tile of the activations for ALL of K in shared
 //   memory once (one bulk TMA copy of a tile the relayout kernel has already
-//   swizzled); every block-row of the tile then gathers from it.  This is the
-//   re-organisation of the input by the mask that Algorithm 1 does with
+//   swizzled); every row group of the tile then gathers from it.  This is
+//   the re-organisation of the input by the mask that Algorithm 1 does with
 //   vpermt2d/vpshufb, done once per tile instead of once per block.
-// * A block-row's stored columns come in steps of 16 (4 quads).  One step of
-//   one warp is two transposed shared-memory gathers (ldmatrix .m16n16 .b8):
-//   each lane receives 8 dot-4 operands -- 8 tokens x 4 consecutive columns
-//   of its quad -- with no byte permutes, and issues 32 dp4a against the
-//   quad's 4 channel words: Algorithm 1's broadcast weight block A,
-//   re-organised input block B and vpdpbusd, 8 tokens at a time.  The
-//   columns of each half-step are chosen at create time to fall in distinct
-//   shared-memory bank groups of the swizzled tile, so a gather reads in one
-//   pass per 8 rows.
-// * The 4 lanes that hold the same tokens took different quads; at the end
-//   of a block-row their sums are added with 24 shuffles (exact int32).
-// * A CTA's steps are split evenly between its 16 warps.  Each warp reads its
-//   contiguous range of 128-byte step records straight from global memory
-//   (L1/L2) into a 4-deep register ring, three steps ahead of their use.  A block-row that straddles a
-//   split between warps is summed in a shared-memory slot (int32 atomics);
-//   the last warp to add finishes it.
+// * One step of a warp takes one quad (4 stored columns) of each of the
+//   group's 4 block-rows: two transposed shared-memory gathers (ldmatrix
+//   .m16n16 .b8) give lane l (q = l % 4, g = l / 4) 8 dot-4 operands -- tokens
+//   g + 8 i x the 4 columns of block-row q's quad -- with no byte permutes,
+//   and the lane issues 32 dp4a against the quad's 4 channel words:
+//   Algorithm 1's broadcast weight block A, re-organised input block B and
+//   vpdpbusd, 8 tokens at a time.  Each lane thus owns whole outputs of its
+//   block-row: no cross-lane sum.  The columns of each half-step are chosen
+//   at create time to fall in distinct shared-memory bank groups of the
+//   swizzled tile, so a gather reads in one pass per 8 rows.
+// * A CTA's steps are split evenly between its 8 warps.  Each warp reads
+//   its contiguous range of 128-byte step records straight from global
+//   memory (L1/L2) into an 8-deep register ring.  A row group that
+//   straddles a split between warps is summed in a shared-memory slot
+//   (int32 atomics); the last warp to add finishes it.
 // * GB300 runs int8 dot products on dp4a at the rate of its int8 MMA paths
 //   (tcgen05 has no int8 kind on sm_103a), and a 4-channel block cannot fill
 //   an MMA tile, so the contraction stays on dp4a.
@@ -154,7 +154,7 @@ __device__ __forceinline__ void store_token(const LaunchArgs& a, int N, long lon
 __device__ __forceinline__ float4 load_s4(const float* p, int r) { return __ldg(reinterpret_cast<const float4*>(p) + r); }
 
 // Last index r in [lo, hi) with sp[r] <= q, given sp[lo] <= q < sp[hi]
-// (sp: the shared-memory window of step offsets).
+// (sp: the shared-memory window of row-group step offsets).
 __device__ __forceinline__ int row_of(const int* sp, int lo, int hi, int q) {
     while (hi - lo > 1) {
         const int mid = (lo + hi) >> 1;
@@ -307,28 +307,6 @@ __device__ __forceinline__ void step16(uint32_t tb, uint32_t lb, int off, const 
     }
 }
 
-// Sum the partial accumulators of the 4 lanes that share g (they took
-// different quads of each step) and scatter: afterwards lane l holds red[j]
-// = token g + 16 (l % 4) + 8 (j / 4), channel j % 4.  Exact int32 adds.
-__device__ __forceinline__ void reduce_quads(int lane, const int (&acc)[32], int (&red)[8]) {
-    constexpr unsigned kFull = 0xffffffffu;
-    const bool b1 = (lane & 2) != 0;
-    int k1[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-        const int send = b1 ? acc[j] : acc[16 + j];
-        const int keep = b1 ? acc[16 + j] : acc[j];
-        k1[j] = keep + __shfl_xor_sync(kFull, send, 2);
-    }
-    const bool b0 = (lane & 1) != 0;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const int send = b0 ? k1[j] : k1[8 + j];
-        const int keep = b0 ? k1[8 + j] : k1[j];
-        red[j] = keep + __shfl_xor_sync(kFull, send, 1);
-    }
-}
-
 // This lane's view of the step records: ro points at the column offset of
 // row (lane % 16) of a step, rw at quad q's 4 channel words of the same
 // step; step s + i is at ro + 32 i, rw + 8 i.
@@ -347,12 +325,22 @@ struct RecPtr {
     }
 };
 
+// Epilogue of one lane for one row group: its block-row r (channels
+// 4r..4r+3; r < 0 for none) at tokens m_g + 8 i, i < 8, from acc[4 i + c].
+template <int KIND>
+__device__ __forceinline__ void store_lane(const LaunchArgs& a, int N, long long m_g, int r, const int (&acc)[32],
+                                           float4 sc, float4 bi) {
+    if (r < 0) return;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) store_token<KIND>(a, N, m_g + 8 * i, r, acc + 4 * i, sc, bi);
+}
+
 template <int KIND, bool TMA>
 __global__ void __launch_bounds__(kThreads, 1)
 bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sched) {
-    constexpr int SW = kTile * 4;  // slot words: 64 tokens x 4 channels
+    constexpr int SW = kTile * 16;  // slot words: 64 tokens x 4 block-rows x 4 channels
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ int s_sp[kRowWin + 1];                  // step offsets of the current block-row window
+    __shared__ int s_gp[kGroupWin + 1];                // step offsets of the current group window
     __shared__ __align__(8) unsigned long long s_bar;  // completion of the token tile's bulk copy
     __shared__ int s_cnt[kSlots];                      // warps that have added into each slot
     __shared__ int s_wst[kWarps + 1];                  // first step of each warp in the window (relative)
@@ -363,14 +351,11 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     const uint32_t tb = (sbase + 127u) & ~127u;  // the token tile, 128-byte aligned
     unsigned char* tile = smem + (tb - sbase);
     int* slots = reinterpret_cast<int*>(tile + static_cast<size_t>(kpad) * kTile);
-    float4* s_scale = reinterpret_cast<float4*>(slots + kSlots * SW);  // [kRowWin]: block-row r - r_lo
-    float4* s_bias = s_scale + kRowWin;
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
-    const int q = lane & 3, g = lane >> 2;
+    const int q = lane & 3, g = lane >> 2;  // block-row q of each group; tokens g + 8 i
     const uint32_t lb = 16u * static_cast<uint32_t>(lane >> 4);
-    const int ta = g + 16 * q;  // tokens this lane finishes: ta and ta + 8 of the tile
-    const long long nbr = w.nbr;
+    const long long ng = w.ngroups;
 
     const uint32_t bar = smem_addr(&s_bar);
     if (TMA && tid == 0) mbar_init(bar, 1);
@@ -384,26 +369,19 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
 
     long long staged = -1;  // token tile currently in shared memory
     while (u < u_end) {
-        // next window: one token tile, at most kRowWin consecutive block-rows
-        const long long t = u / nbr;
-        const int r_lo = static_cast<int>(u - t * nbr);
-        const int r_hi = static_cast<int>(min(min(nbr, r_lo + (u_end - u)), static_cast<long long>(r_lo + kRowWin)));
-        u += r_hi - r_lo;
+        // next window: one token tile, at most kGroupWin consecutive row groups
+        const long long t = u / ng;
+        const int g_lo = static_cast<int>(u - t * ng);
+        const int g_hi = static_cast<int>(min(min(ng, g_lo + (u_end - u)), static_cast<long long>(g_lo + kGroupWin)));
+        u += g_hi - g_lo;
         const long long m0 = t * kTile;
-        auto sp = [&](int r) { return s_sp[r - r_lo]; };
+        auto gp = [&](int gi) { return s_gp[gi - g_lo]; };
 
-        for (int i = tid; i <= r_hi - r_lo; i += kThreads) s_sp[i] = __ldg(w.sptr + r_lo + i);
+        for (int i = tid; i <= g_hi - g_lo; i += kThreads) s_gp[i] = __ldg(w.gptr + g_lo + i);
         if (tid <= kWarps) {
             // warps take an even split of the window's steps
-            const long long nst_w = __ldg(w.sptr + r_hi) - __ldg(w.sptr + r_lo);
-            s_wst[tid] = static_cast<int>(nst_w * tid / kWarps);
-        }
-        if (KIND != 0) {
-            for (int i = tid; i < 2 * (r_hi - r_lo); i += kThreads) {
-                const int rr = i >> 1;
-                if (i & 1) s_bias[rr] = load_s4(w.bias, r_lo + rr);
-                else s_scale[rr] = load_s4(w.scale, r_lo + rr);
-            }
+            const long long nst = __ldg(w.gptr + g_hi) - __ldg(w.gptr + g_lo);
+            s_wst[tid] = static_cast<int>(nst * tid / kWarps);
         }
         const bool stage = (t != staged);
         if (TMA && stage && tid == 0) {
@@ -415,36 +393,38 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             for (unsigned off = 0; off < bytes; off += 65536u)
                 bulk_g2s(tb + off, src + off, min(65536u, bytes - off), bar);
         }
-        __syncthreads();  // the block-row window is visible
+        __syncthreads();  // the group window is visible
         if (!TMA && stage) {  // gather the tile with per-thread loads
             stage_tile(tile, a, K, kpad, m0);
             __syncthreads();
             staged = t;
         }
 
-        const int sa = sp(r_lo);
+        const int sa = gp(g_lo);
         const int ws0 = s_wst[warp], ws1 = s_wst[warp + 1];
 
-        // The warp's first four step records load while the tile does; a
-        // record is loaded three steps before its use (the record array has
-        // kStepPad spare steps for the loads past the last one).
-        RecPtr rec(w.recs, sa + ws0, lane, q);  // at step p of the loop below
-        int off[4];
-        int4 wq[4];
+        // The warp's first kRing step records load while the tile does; the
+        // record of a step is loaded kRing steps before its use (the record
+        // array has kStepPad spare steps for the loads past the last one).
+        RecPtr rec(w.recs, sa + ws0, lane, q);  // step of ring slot 0
+        int off[kRing];
+        int4 wq[kRing];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < kRing; ++i) {
             off[i] = 0;
             wq[i] = make_int4(0, 0, 0, 0);
             if (ws0 < ws1) rec.load(i, off[i], wq[i]);
         }
 
-        // Block-rows with no stored block: acc = 0.
-        for (int r = r_lo + warp; r < r_hi; r += kWarps) {
-            if (sp(r) == sp(r + 1)) {
-                const int zero[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-                const float4 sc = s_scale[r - r_lo], bi = s_bias[r - r_lo];
-                store_token<KIND>(a, N, m0 + ta, r, zero, sc, bi);
-                store_token<KIND>(a, N, m0 + ta + 8, r, zero + 4, sc, bi);
+        // Row groups without any stored block: acc = 0.
+        for (int gi = g_lo + warp; gi < g_hi; gi += kWarps) {
+            if (gp(gi) == gp(gi + 1)) {
+                const int4 gr = __ldg(w.grow + gi);
+                const int r = q == 0 ? gr.x : q == 1 ? gr.y : q == 2 ? gr.z : gr.w;
+                int zero[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) zero[i] = 0;
+                if (r >= 0) store_lane<KIND>(a, N, m0 + g, r, zero, load_s4(w.scale, r), load_s4(w.bias, r));
             }
         }
 
@@ -463,53 +443,76 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         }
 
         if (ws0 < ws1) {
-            int r = r_lo + row_of(s_sp, 0, r_hi - r_lo, sa + ws0);
+            int gi = g_lo + row_of(s_gp, 0, g_hi - g_lo, sa + ws0);
             int p = ws0;  // step index relative to sa
+            int ph = 0;   // ring slot holding step p
             while (p < ws1) {
-                const int rs = sp(r), re = sp(r + 1);
-                const int p_end = min(ws1, re - sa);
+                const int gs = gp(gi), ge = gp(gi + 1);
+                const int p_end = min(ws1, ge - sa);
+                const int4 gr = __ldg(w.grow + gi);
+                const int r = q == 0 ? gr.x : q == 1 ? gr.y : q == 2 ? gr.z : gr.w;
+                float4 sc = make_float4(0.f, 0.f, 0.f, 0.f), bi = sc;
+                if (KIND != 0 && r >= 0) {  // needed at the group's end; load it now
+                    sc = load_s4(w.scale, r);
+                    bi = load_s4(w.bias, r);
+                }
                 int acc[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) acc[i] = 0;
-                // invariant: off/wq[i] hold step p + i
-                for (; p + 3 < p_end; p += 4) {
+                // Steps p .. p_end - 1.  Ring slot i holds step (ring base + i);
+                // after its step it loads step (base + kRing + i), and after
+                // slot kRing - 1 the base moves on by kRing.  Whole rounds of
+                // the ring run as one straight block (the compiler overlaps
+                // one step's gathers with the previous step's dp4a); the
+                // switch enters at the slot of step p, so a group may start
+                // or end at any slot.
+                while (p < p_end) {
+                    if (ph == 0 && p + kRing <= p_end) {
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        step16(tb, lb, off[i], wq[i], acc);
-                        rec.load(4 + i, off[i], wq[i]);
+                        for (int i = 0; i < kRing; ++i) {
+                            step16(tb, lb, off[i], wq[i], acc);
+                            rec.load(kRing + i, off[i], wq[i]);
+                        }
+                        rec.advance(kRing);
+                        p += kRing;
+                        continue;
                     }
-                    rec.advance(4);
-                }
-                for (; p < p_end; ++p) {  // the row's last 0-3 steps: shift the ring by one
-                    step16(tb, lb, off[0], wq[0], acc);
-#pragma unroll
-                    for (int i = 0; i < 3; ++i) {
-                        off[i] = off[i + 1];
-                        wq[i] = wq[i + 1];
+                    switch (ph) {
+#define BSG_RING_SLOT(i)                                 \
+    case i:                                              \
+        step16(tb, lb, off[i], wq[i], acc);              \
+        rec.load(kRing + (i), off[i], wq[i]);            \
+        ++p;                                             \
+        if ((i) == kRing - 1) rec.advance(kRing);        \
+        if (p == p_end) {                                \
+            ph = ((i) + 1) % kRing;                      \
+            break;                                       \
+        }
+                        BSG_RING_SLOT(0)
+                        BSG_RING_SLOT(1)
+                        BSG_RING_SLOT(2)
+                        BSG_RING_SLOT(3)
+                        BSG_RING_SLOT(4)
+                        BSG_RING_SLOT(5)
+                        BSG_RING_SLOT(6)
+                        BSG_RING_SLOT(7)
+#undef BSG_RING_SLOT
+                        ph = 0;
                     }
-                    rec.load(4, off[3], wq[3]);
-                    rec.advance(1);
                 }
-                float4 sc = make_float4(0.f, 0.f, 0.f, 0.f), bi = sc;
-                if (KIND != 0) {
-                    sc = s_scale[r - r_lo];
-                    bi = s_bias[r - r_lo];
-                }
-                int red[8];
-                reduce_quads(lane, acc, red);
-                if (rs >= sa + ws0 && re <= sa + ws1) {
-                    store_token<KIND>(a, N, m0 + ta, r, red, sc, bi);
-                    store_token<KIND>(a, N, m0 + ta + 8, r, red + 4, sc, bi);
+                if (gs >= sa + ws0 && ge <= sa + ws1) {
+                    store_lane<KIND>(a, N, m0 + g, r, acc, sc, bi);
                 } else {
                     // Shared with other warps: sum into the slot of the first warp
-                    // boundary inside the block-row (the first b with s_wst[b] > s0);
-                    // the last warp to add finishes it.
-                    const int s0 = rs - sa, s1 = re - sa;  // the row's steps
+                    // boundary inside the group (the first b with s_wst[b] > s0);
+                    // the last warp to add finishes it.  Slot layout [i][c][lane]:
+                    // every warp's lane l holds the same (token, block-row, channel).
+                    const int s0 = gs - sa, s1 = ge - sa;  // the group's steps
                     int b = 1;
                     while (s_wst[b] <= s0) ++b;
-                    int* sl = slots + (b - 1) * SW;
+                    int* sl = slots + (b - 1) * SW + lane;
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) atomicAdd(sl + (ta + 8 * (j >> 2)) * 4 + (j & 3), red[j]);
+                    for (int j = 0; j < 32; ++j) atomicAdd(sl + 32 * j, acc[j]);
                     __syncwarp();
                     int arrived = 0;
                     if (lane == 0) {
@@ -517,20 +520,19 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                         arrived = atomicAdd(&s_cnt[b - 1], 1) + 1;
                     }
                     arrived = __shfl_sync(0xffffffffu, arrived, 0);
-                    int parts = 0;  // warps whose step range meets the row's
+                    int parts = 0;  // warps whose step range meets the group's
                     for (int wi = b - 1; wi < kWarps && s_wst[wi] < s1; ++wi)
                         parts += (s_wst[wi] < s_wst[wi + 1]) ? 1 : 0;
                     if (arrived == parts) {
                         __threadfence_block();
 #pragma unroll
-                        for (int j = 0; j < 8; ++j) red[j] = atomicExch(sl + (ta + 8 * (j >> 2)) * 4 + (j & 3), 0);
-                        store_token<KIND>(a, N, m0 + ta, r, red, sc, bi);
-                        store_token<KIND>(a, N, m0 + ta + 8, r, red + 4, sc, bi);
+                        for (int j = 0; j < 32; ++j) acc[j] = atomicExch(sl + 32 * j, 0);
+                        store_lane<KIND>(a, N, m0 + g, r, acc, sc, bi);
                         if (lane == 0) s_cnt[b - 1] = 0;
                     }
                 }
-                ++r;
-                while (r < r_hi && sp(r + 1) == sp(r)) ++r;  // skip block-rows without steps
+                ++gi;
+                while (gi < g_hi && gp(gi + 1) == gp(gi)) ++gi;  // skip groups without steps
             }
         }
         __syncthreads();  // the tile, window and slots may be reused
@@ -630,10 +632,8 @@ const void* kernel_for(int kind) {
 
 size_t smem_bytes(int K) {
     const size_t kpad = (static_cast<size_t>(K) + 15) & ~static_cast<size_t>(15);
-    // 128 bytes of slack to align the tile, the tile, the split-row slots,
-    // the window's scales and biases
-    return 128 + kpad * kTile + static_cast<size_t>(kSlots) * kTile * 4 * sizeof(int) +
-           2 * static_cast<size_t>(kRowWin) * sizeof(float4);
+    // 128 bytes of slack to align the tile, the tile, the split-group slots
+    return 128 + kpad * kTile + static_cast<size_t>(kSlots) * kTile * 16 * sizeof(int);
 }
 
 int max_k() {
