@@ -51,6 +51,12 @@ namespace {
 
 constexpr int kSmemOptin = 232448;  // sm_103 opt-in shared memory per block
 constexpr int kSlots = kWarps - 1;  // one per split point between warp ranges
+// Cost of a row group's end (epilogue, stores) in steps, for splitting a
+// window's work evenly between warps.
+#ifndef BSG_GROUP_END_COST
+#define BSG_GROUP_END_COST 6
+#endif
+constexpr int kGroupEndCost = BSG_GROUP_END_COST;
 
 // 4x4 byte transpose.  In: a/b/c/d = bytes (x0..x3) of rows 0..3.  Out:
 // t_i = (a_i, b_i, c_i, d_i).
@@ -282,6 +288,14 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, unsigned
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
                  ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
+// Programmatic dependent launch: both kernels are launched so that they may
+// start while the previous kernel of the stream finishes.  Before a kernel
+// reads its activations or writes any global memory, every thread waits
+// until the previous grid has completed and its writes are visible (a no-op
+// when there is none); early on it lets the next kernel launch.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+
 // Order this thread's earlier generic-proxy shared-memory accesses before
 // later asynchronous-proxy (bulk copy) writes.
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
@@ -342,7 +356,6 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int s_gp[kGroupWin + 1];                // step offsets of the current group window
     __shared__ __align__(8) unsigned long long s_bar;  // completion of the token tile's bulk copy
-    __shared__ int s_cnt[kSlots];                      // warps that have added into each slot
     __shared__ int s_wst[kWarps + 1];                  // first step of each warp in the window (relative)
 
     const int K = w.K, N = w.N;
@@ -357,17 +370,18 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     const uint32_t lb = 16u * static_cast<uint32_t>(lane >> 4);
     const long long ng = w.ngroups;
 
+    griddep_launch_dependents();
     const uint32_t bar = smem_addr(&s_bar);
     if (TMA && tid == 0) mbar_init(bar, 1);
-    // slots and their counters start at zero; whoever finishes a slot resets it
+    // slots start at zero; whoever finishes a slot resets it
     for (int i = tid; i < kSlots * SW; i += kThreads) slots[i] = 0;
-    if (tid < kSlots) s_cnt[tid] = 0;
     __syncthreads();
     unsigned phase = 0;
     long long u = sched.u[blockIdx.x];
     const long long u_end = sched.u[blockIdx.x + 1];
 
     long long staged = -1;  // token tile currently in shared memory
+    bool waited = false;    // the previous grid's writes are visible
     while (u < u_end) {
         // next window: one token tile, at most kGroupWin consecutive row groups
         const long long t = u / ng;
@@ -378,10 +392,9 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         auto gp = [&](int gi) { return s_gp[gi - g_lo]; };
 
         for (int i = tid; i <= g_hi - g_lo; i += kThreads) s_gp[i] = __ldg(w.gptr + g_lo + i);
-        if (tid <= kWarps) {
-            // warps take an even split of the window's steps
-            const long long nst = __ldg(w.gptr + g_hi) - __ldg(w.gptr + g_lo);
-            s_wst[tid] = static_cast<int>(nst * tid / kWarps);
+        if (!waited) {  // nothing above reads the activations or writes global memory
+            griddep_wait();
+            waited = true;
         }
         const bool stage = (t != staged);
         if (TMA && stage && tid == 0) {
@@ -394,14 +407,56 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 bulk_g2s(tb + off, src + off, min(65536u, bytes - off), bar);
         }
         __syncthreads();  // the group window is visible
+        const int sa = gp(g_lo);
+        if (tid <= kWarps) {
+            // Warps take an even split of the window's cost: a step costs 1,
+            // a group's end kGroupEndCost (charged after its last step).
+            // Group j of the window starts at cost s_gp[j] - sa + j * kGroupEndCost;
+            // warp tid starts at the step where the cost reaches tid / kWarps
+            // of the total, or at the next group if that falls on a group's end.
+            const int ngw = g_hi - g_lo;
+            const long long total = static_cast<long long>(s_gp[ngw] - sa) + static_cast<long long>(ngw) * kGroupEndCost;
+            const long long target = total * tid / kWarps;
+            int lo = 0, hi = ngw;  // the last group j with its start cost <= target
+            while (hi - lo > 1) {
+                const int mid = (lo + hi) >> 1;
+                if (static_cast<long long>(s_gp[mid] - sa) + static_cast<long long>(mid) * kGroupEndCost <= target) lo = mid;
+                else hi = mid;
+            }
+            const long long into = target - (static_cast<long long>(s_gp[lo] - sa) + static_cast<long long>(lo) * kGroupEndCost);
+            const int len = s_gp[lo + 1] - s_gp[lo];
+            s_wst[tid] = (tid == kWarps) ? s_gp[ngw] - sa : s_gp[lo] - sa + static_cast<int>(into < len ? into : len);
+        }
+        __syncthreads();  // the warps' step ranges are visible
         if (!TMA && stage) {  // gather the tile with per-thread loads
             stage_tile(tile, a, K, kpad, m0);
             __syncthreads();
             staged = t;
         }
 
-        const int sa = gp(g_lo);
         const int ws0 = s_wst[warp], ws1 = s_wst[warp + 1];
+
+        // Groups split between warps are finished after the window's last
+        // barrier: warp w takes boundary w + 1 if it is the first boundary
+        // inside its group (slot w then holds the group's sum).  Its block-row,
+        // scale and bias load now.
+        int fin_r = -1;
+        float4 fin_sc = make_float4(0.f, 0.f, 0.f, 0.f), fin_bi = fin_sc;
+        bool fin = false;
+        if (warp < kSlots) {
+            const int bnd = s_wst[warp + 1];
+            const int j = row_of(s_gp, 0, g_hi - g_lo, sa + min(bnd, s_wst[kWarps] - 1));
+            const int gs = s_gp[j] - sa;
+            fin = bnd > gs && bnd < s_gp[j + 1] - sa && s_wst[warp] <= gs;
+            if (fin) {
+                const int4 gr = __ldg(w.grow + g_lo + j);
+                fin_r = q == 0 ? gr.x : q == 1 ? gr.y : q == 2 ? gr.z : gr.w;
+                if (KIND != 0 && fin_r >= 0) {
+                    fin_sc = load_s4(w.scale, fin_r);
+                    fin_bi = load_s4(w.bias, fin_r);
+                }
+            }
+        }
 
         // The warp's first kRing step records load while the tile does; the
         // record of a step is loaded kRing steps before its use (the record
@@ -503,39 +558,34 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 if (gs >= sa + ws0 && ge <= sa + ws1) {
                     store_lane<KIND>(a, N, m0 + g, r, acc, sc, bi);
                 } else {
-                    // Shared with other warps: sum into the slot of the first warp
-                    // boundary inside the group (the first b with s_wst[b] > s0);
-                    // the last warp to add finishes it.  Slot layout [i][c][lane]:
-                    // every warp's lane l holds the same (token, block-row, channel).
-                    const int s0 = gs - sa, s1 = ge - sa;  // the group's steps
+                    // Shared with other warps: add into the slot of the first warp
+                    // boundary inside the group (the first b with s_wst[b] > the
+                    // group's first step); the group is finished after the window's
+                    // barrier.  Slot layout [j][lane]: every warp's lane l holds
+                    // the same (token, block-row, channel) in acc[j].
                     int b = 1;
-                    while (s_wst[b] <= s0) ++b;
+                    while (s_wst[b] <= gs - sa) ++b;
                     int* sl = slots + (b - 1) * SW + lane;
 #pragma unroll
                     for (int j = 0; j < 32; ++j) atomicAdd(sl + 32 * j, acc[j]);
-                    __syncwarp();
-                    int arrived = 0;
-                    if (lane == 0) {
-                        __threadfence_block();
-                        arrived = atomicAdd(&s_cnt[b - 1], 1) + 1;
-                    }
-                    arrived = __shfl_sync(0xffffffffu, arrived, 0);
-                    int parts = 0;  // warps whose step range meets the group's
-                    for (int wi = b - 1; wi < kWarps && s_wst[wi] < s1; ++wi)
-                        parts += (s_wst[wi] < s_wst[wi + 1]) ? 1 : 0;
-                    if (arrived == parts) {
-                        __threadfence_block();
-#pragma unroll
-                        for (int j = 0; j < 32; ++j) acc[j] = atomicExch(sl + 32 * j, 0);
-                        store_lane<KIND>(a, N, m0 + g, r, acc, sc, bi);
-                        if (lane == 0) s_cnt[b - 1] = 0;
-                    }
                 }
                 ++gi;
                 while (gi < g_hi && gp(gi + 1) == gp(gi)) ++gi;  // skip groups without steps
             }
         }
-        __syncthreads();  // the tile, window and slots may be reused
+        __syncthreads();  // every part of every split group is in its slot
+
+        if (fin) {  // the split group of boundary warp + 1 (see above)
+            int* sl = slots + warp * SW + lane;
+            int acc[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                acc[j] = sl[32 * j];
+                sl[32 * j] = 0;
+            }
+            store_lane<KIND>(a, N, m0 + g, fin_r, acc, fin_sc, fin_bi);
+        }
+        __syncthreads();  // the window's offsets, the slots' reset and the tile may be reused
     }
 }
 
@@ -582,6 +632,8 @@ pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __r
             }
         }
     };
+    griddep_launch_dependents();
+    griddep_wait();  // x may be the previous kernel's output
     uint4 v[NL];
     long long it = blockIdx.x;
     if (it < items) load_item(it, v);
@@ -656,10 +708,21 @@ cudaError_t prepare_kernels(int K, int* ctas_per_sm) {
 
 cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int grid, cudaStream_t s) {
     const size_t smem = smem_bytes(w.K);
-#define BSG_LAUNCH(KV)                                                                  \
-    do {                                                                                \
-        if (a.xb) bsgemm_kernel<KV, true><<<grid, kThreads, smem, s>>>(w, a, sched);    \
-        else bsgemm_kernel<KV, false><<<grid, kThreads, smem, s>>>(w, a, sched);        \
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaSuccess;
+#define BSG_LAUNCH(KV)                                                                                   \
+    do {                                                                                                 \
+        e = a.xb ? cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, true>, w, a, sched)                        \
+                 : cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, false>, w, a, sched);                      \
     } while (0)
     switch (a.kind) {
     case 0: BSG_LAUNCH(0); break;
@@ -669,7 +732,7 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
     default: BSG_LAUNCH(4); break;
     }
 #undef BSG_LAUNCH
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 size_t tiled_bytes(int K, long long M) {
@@ -683,8 +746,17 @@ cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, c
     const long long items = (static_cast<long long>(M) + kTile - 1) / kTile * ncb;
     const long long cap = 4LL * (sms > 0 ? sms : 1);  // 4 resident CTAs per SM (35 KB of shared memory each)
     const unsigned grid = static_cast<unsigned>(items < cap ? items : cap);
-    pretile_kernel<<<grid, 256, 0, s>>>(x, M, K, kpad, xb, items, ncb);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, pretile_kernel, x, M, K, kpad, xb, items, ncb);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace bsg
