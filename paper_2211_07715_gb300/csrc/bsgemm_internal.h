@@ -70,7 +70,10 @@ struct LaunchArgs {
 // registers a thread).
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
-constexpr int kRing = 8;            // step records a warp keeps in flight (registers)
+#ifndef BSG_RING
+#define BSG_RING 12
+#endif
+constexpr int kRing = BSG_RING;     // step records a warp keeps in flight (registers), 8..16
 constexpr int kStepPad = kRing;     // zero step records after the last one (the record prefetch runs ahead)
 constexpr int kGroupWin = 512;      // row groups whose step offsets a CTA keeps in shared memory
 constexpr int kStaticSmem = 2304;   // bytes of static shared memory the kernel may use

@@ -51,6 +51,7 @@ namespace {
 
 constexpr int kSmemOptin = 232448;  // sm_103 opt-in shared memory per block
 constexpr int kSlots = kWarps - 1;  // one per split point between warp ranges
+static_assert(kRing == 8 || kRing == 12 || kRing == 16, "the record ring's switch has 8, 12 or 16 slots");
 // Cost of a row group's end (epilogue, stores) in steps, for splitting a
 // window's work evenly between warps.
 #ifndef BSG_GROUP_END_COST
@@ -226,9 +227,12 @@ __device__ __forceinline__ void store_unit(unsigned char* xt, int g, int kc, con
 // Stage activation rows m0..m0+63, all kpad columns, into the swizzled tile
 // with per-thread loads.  Each thread keeps kStageBatch units' loads in
 // flight before transposing them.
+#ifndef BSG_STAGE_BATCH
+#define BSG_STAGE_BATCH 8
+#endif
 __device__ __forceinline__ void stage_tile(unsigned char* xt, const LaunchArgs& a, int K, int kpad, long long m0) {
     constexpr int G = kTile / 4;
-    constexpr int kStageBatch = 2;
+    constexpr int kStageBatch = BSG_STAGE_BATCH;
     const int total = G * (kpad >> 4);
     for (int base = threadIdx.x; base < total; base += kStageBatch * kThreads) {
         uint32_t rw[kStageBatch][4][4];
@@ -551,6 +555,18 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                         BSG_RING_SLOT(5)
                         BSG_RING_SLOT(6)
                         BSG_RING_SLOT(7)
+#if BSG_RING > 8
+                        BSG_RING_SLOT(8)
+                        BSG_RING_SLOT(9)
+                        BSG_RING_SLOT(10)
+                        BSG_RING_SLOT(11)
+#endif
+#if BSG_RING > 12
+                        BSG_RING_SLOT(12)
+                        BSG_RING_SLOT(13)
+                        BSG_RING_SLOT(14)
+                        BSG_RING_SLOT(15)
+#endif
 #undef BSG_RING_SLOT
                         ph = 0;
                     }
@@ -590,82 +606,82 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
 }
 
 // Token-tile relayout: x [M][K] -> swizzled tiles (tile t = tokens
-// 64t..64t+63, all kpad columns; zero past M or K).  A persistent CTA walks
-// items (tile t, block of 256 columns): 64 tokens x 256 columns (16 KB)
-// through shared memory -- 16-byte row loads, a 4x4 byte transpose per
-// thread, then each 16-token chunk of a column is one 16-byte store into its
-// slot of the swizzled tile (a block of 256 columns is 128 whole lines,
-// written contiguously).  The next item's loads are in flight (in
-// registers) while the current item is transposed and stored.
+// 64t..64t+63, all kpad columns; zero past M or K).  One warp takes one
+// unit -- 64 tokens x 32 columns -- at a time, with no block-wide barrier:
+//   * lane (g, h) = (lane / 2, lane % 2) loads tokens 4g..4g+3 x columns
+//     16h..16h+15 (four 16-byte loads; per load the warp reads 32
+//     contiguous bytes of each of 16 rows);
+//   * four 4x4 byte transposes turn them into words (4 tokens of one
+//     column), written to the warp's staging buffer in shared memory: 32
+//     column rows x 16 words, rows with bit 4 set stored at the partner
+//     row (bit 0 flipped) so that the two column halves of a store use
+//     different banks;
+//   * the warp copies the 32 rows out as 16-byte chunks (16 tokens of one
+//     column) to their slots of the swizzled tile: 8 lanes fill one
+//     128-byte line.
+// The next unit's loads are in flight while a unit is transposed.
 __global__ void __launch_bounds__(256)
-pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __restrict__ xb, long long items,
+pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __restrict__ xb, long long units,
                int ncb) {
-    constexpr int KC = 256;               // columns per item
-    constexpr int C16 = KC / 16;          // 16-byte chunks per raw row
-    constexpr int RW = KC / 4 + 4;        // raw row stride in words (rows shift by 4 banks)
-    constexpr int OS = kTile / 4 + 1;     // transposed row stride in words
-    constexpr int NL = (kTile * C16) / 256;  // row loads per thread and item
-    __shared__ __align__(16) uint32_t raw[kTile * RW];
-    __shared__ uint32_t tr[KC * OS];
+    constexpr int kW = 8;                        // warps per CTA
+    __shared__ __align__(16) uint32_t stage[kW][32 * 16];
+    griddep_launch_dependents();
+    griddep_wait();  // x may be the previous kernel's output
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = lane >> 1, h = lane & 1;
+    uint32_t* st = stage[warp];
     const bool vec16 = ((K & 15) == 0) && ((reinterpret_cast<uintptr_t>(x) & 15) == 0);
-    auto load_item = [&](long long it, uint4 (&v)[NL]) {
-        const long long m0 = (it / ncb) * kTile;
-        const int k0 = static_cast<int>(it % ncb) * KC;
+    const long long nw = static_cast<long long>(gridDim.x) * kW;
+
+    // rw[i][j] = bytes of token 4g+i at columns k0+16h+4j .. +3 of unit u (zero past M or K)
+    auto load_unit = [&](long long u, uint32_t (&rw)[4][4]) {
+        const long long t = u / ncb;
+        const int k = static_cast<int>(u % ncb) * 32 + 16 * h;
 #pragma unroll
-        for (int i = 0; i < NL; ++i) {
-            const int c = i * 256 + threadIdx.x;
-            const int rho = c / C16, c16 = c % C16;
-            const long long m = m0 + rho;
-            const int k = k0 + 16 * c16;
-            v[i] = make_uint4(0u, 0u, 0u, 0u);
+        for (int i = 0; i < 4; ++i) {
+            const long long m = t * kTile + 4 * g + i;
+            rw[i][0] = rw[i][1] = rw[i][2] = rw[i][3] = 0u;
             if (m < M && k < K) {
                 const int8_t* src = x + static_cast<size_t>(m) * K + k;
                 if (vec16) {
-                    v[i] = __ldg(reinterpret_cast<const uint4*>(src));
+                    const uint4 v = __ldg(reinterpret_cast<const uint4*>(src));
+                    rw[i][0] = v.x; rw[i][1] = v.y; rw[i][2] = v.z; rw[i][3] = v.w;
                 } else {
-                    uint32_t wv[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
                     for (int e = 0; e < 16; ++e)
-                        if (k + e < K) wv[e >> 2] |= static_cast<uint32_t>(static_cast<uint8_t>(src[e])) << (8 * (e & 3));
-                    v[i] = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                        if (k + e < K) rw[i][e >> 2] |= static_cast<uint32_t>(static_cast<uint8_t>(src[e])) << (8 * (e & 3));
                 }
             }
         }
     };
-    griddep_launch_dependents();
-    griddep_wait();  // x may be the previous kernel's output
-    uint4 v[NL];
-    long long it = blockIdx.x;
-    if (it < items) load_item(it, v);
-    for (; it < items; it += gridDim.x) {
-        const long long t = it / ncb;
-        const int k0 = static_cast<int>(it % ncb) * KC;
-        const int kc = min(KC, kpad - k0);  // a multiple of 16
+
+    long long u = static_cast<long long>(blockIdx.x) * kW + warp;
+    uint32_t rw[4][4];
+    if (u < units) load_unit(u, rw);
+    for (; u < units; u += nw) {
+        const long long t = u / ncb;
+        const int k0 = static_cast<int>(u % ncb) * 32;
 #pragma unroll
-        for (int i = 0; i < NL; ++i) {
-            const int c = i * 256 + threadIdx.x;
-            *reinterpret_cast<uint4*>(raw + (c / C16) * RW + 4 * (c % C16)) = v[i];
+        for (int j = 0; j < 4; ++j) {
+            uint32_t w4[4];
+            transpose4(rw[0][j], rw[1][j], rw[2][j], rw[3][j], w4[0], w4[1], w4[2], w4[3]);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) st[(16 * h + 4 * j + (e ^ h)) * 16 + g] = w4[e];
         }
-        __syncthreads();  // raw is complete; every thread is past the previous item's stores
-        if (it + gridDim.x < items) load_item(it + gridDim.x, v);
-        for (int i = threadIdx.x; i < (kTile / 4) * (KC / 4); i += 256) {
-            const int j = i % (KC / 4), g = i / (KC / 4);
-            uint32_t t0, t1, t2, t3;
-            transpose4(raw[(4 * g + 0) * RW + j], raw[(4 * g + 1) * RW + j], raw[(4 * g + 2) * RW + j],
-                       raw[(4 * g + 3) * RW + j], t0, t1, t2, t3);
-            tr[(4 * j + 0) * OS + g] = t0;
-            tr[(4 * j + 1) * OS + g] = t1;
-            tr[(4 * j + 2) * OS + g] = t2;
-            tr[(4 * j + 3) * OS + g] = t3;
-        }
-        __syncthreads();  // tr is complete; raw may be refilled
+        if (u + nw < units) load_unit(u + nw, rw);  // the next unit's loads fly while this one is stored
+        __syncwarp();
         int8_t* dst = xb + static_cast<size_t>(t) * kpad * kTile;
-        for (int i = threadIdx.x; i < kc * 4; i += 256) {
-            const int row = i >> 2, c = i & 3;
-            const uint32_t* srow = tr + row * OS + 4 * c;
-            *reinterpret_cast<uint4*>(dst + (row_off(k0 + row) ^ (static_cast<uint32_t>(c) << 4))) =
-                make_uint4(srow[0], srow[1], srow[2], srow[3]);
+#pragma unroll
+        for (int qq = 0; qq < 4; ++qq) {
+            const int ch = lane + 32 * qq;
+            const int row = ch >> 2, c = ch & 3;
+            const int k = k0 + row;
+            if (k < kpad) {
+                const uint4 v = *reinterpret_cast<const uint4*>(st + (row ^ (row >> 4)) * 16 + 4 * c);
+                *reinterpret_cast<uint4*>(dst + (row_off(k) ^ (static_cast<uint32_t>(c) << 4))) = v;
+            }
         }
+        __syncwarp();
     }
 }
 
@@ -742,10 +758,11 @@ size_t tiled_bytes(int K, long long M) {
 
 cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, cudaStream_t s) {
     const int kpad = (K + 15) & ~15;
-    const int ncb = (kpad + 255) / 256;
-    const long long items = (static_cast<long long>(M) + kTile - 1) / kTile * ncb;
-    const long long cap = 4LL * (sms > 0 ? sms : 1);  // 4 resident CTAs per SM (35 KB of shared memory each)
-    const unsigned grid = static_cast<unsigned>(items < cap ? items : cap);
+    const int ncb = (kpad + 31) / 32;  // units of 32 columns per token tile
+    const long long units = (static_cast<long long>(M) + kTile - 1) / kTile * ncb;
+    const long long cap = 8LL * (sms > 0 ? sms : 1);  // 8 resident CTAs of 8 warps per SM
+    const long long want = (units + 7) / 8;
+    const unsigned grid = static_cast<unsigned>(want < cap ? want : cap);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(256);
@@ -755,7 +772,7 @@ cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, c
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, pretile_kernel, x, M, K, kpad, xb, items, ncb);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, pretile_kernel, x, M, K, kpad, xb, units, ncb);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
