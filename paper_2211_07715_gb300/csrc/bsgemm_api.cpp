@@ -73,8 +73,14 @@ std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx
 // for 64 tokens: 32 dp4a per lane): every row group adds kGroupCost for its
 // epilogue, every token tile in a CTA's range adds kTileCost for its copy
 // into shared memory and the start-up around it.
-constexpr long long kGroupCost = 4;
-constexpr long long kTileCost = 250;
+#ifndef BSG_GROUP_COST
+#define BSG_GROUP_COST 4
+#endif
+#ifndef BSG_TILE_COST
+#define BSG_TILE_COST 250
+#endif
+constexpr long long kGroupCost = BSG_GROUP_COST;
+constexpr long long kTileCost = BSG_TILE_COST;
 
 // End of the greedy range that starts at unit u under the cost bound C: it
 // takes whole units while the cost (units' cost + tc per token tile

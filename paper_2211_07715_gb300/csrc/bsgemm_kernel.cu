@@ -115,11 +115,17 @@ __device__ __forceinline__ float gelu_f32_fast(float y) {
     return 0.5f * y * (1.0f + ((x < 0.0f) ? -e : e));
 }
 
-// fp32 -> int8: one fp32 multiply, round half to even, saturate.
-__device__ __forceinline__ uint32_t requant_s8(float v, float inv) {
-    int q = __float2int_rn(__fmul_rn(v, inv));
-    q = max(-128, min(127, q));
-    return static_cast<uint32_t>(q) & 0xffu;
+// fp32 -> int8 for 4 values: one fp32 multiply each, round half to even
+// (to int32, saturating), then saturate to [-128, 127] and pack v0 into
+// byte 0 .. v3 into byte 3 (cvt.pack.sat: b into the low byte, a into the
+// next, c's low half above).
+__device__ __forceinline__ uint32_t requant4_s8(float v0, float v1, float v2, float v3, float inv) {
+    const int q0 = __float2int_rn(__fmul_rn(v0, inv)), q1 = __float2int_rn(__fmul_rn(v1, inv));
+    const int q2 = __float2int_rn(__fmul_rn(v2, inv)), q3 = __float2int_rn(__fmul_rn(v3, inv));
+    uint32_t hi, d;
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(hi) : "r"(q3), "r"(q2), "r"(0));
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(q1), "r"(q0), "r"(hi));
+    return d;
 }
 
 // Epilogue for one token m (nothing past M): v = acc of the 4 channels of
@@ -151,10 +157,7 @@ __device__ __forceinline__ void store_token(const LaunchArgs& a, int N, long lon
     if (KIND == 1 || KIND == 2) {
         *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y0, y1, y2, y3);
     } else {
-        const float inv = a.inv_out_scale;
-        const uint32_t packed = requant_s8(y0, inv) | (requant_s8(y1, inv) << 8) | (requant_s8(y2, inv) << 16) |
-                                (requant_s8(y3, inv) << 24);
-        *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = packed;
+        *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = requant4_s8(y0, y1, y2, y3, a.inv_out_scale);
     }
 }
 
