@@ -70,17 +70,16 @@ std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx
 }
 
 // Schedule costs, in steps (one quad of each of a row group's 4 block-rows
-// for 64 tokens: 32 dp4a per lane): every row group adds kGroupCost for its
-// epilogue, every token tile in a CTA's range adds kTileCost for its copy
-// into shared memory and the start-up around it.
+// for 64 tokens: 32 dp4a per lane), from a least-squares fit of measured
+// CTA times on GB300 (FFN1/FFN2/QKV/attention-output shapes, M = 2K-8K):
+// a CTA spends about 19 cycles per step, 320 per row group (its epilogue)
+// and 6600 + 0.27 K per token tile it touches (the tile's copy into shared
+// memory, the warps' set-up and the spread of their finishing times).
 #ifndef BSG_GROUP_COST
-#define BSG_GROUP_COST 4
-#endif
-#ifndef BSG_TILE_COST
-#define BSG_TILE_COST 250
+#define BSG_GROUP_COST 17
 #endif
 constexpr long long kGroupCost = BSG_GROUP_COST;
-constexpr long long kTileCost = BSG_TILE_COST;
+long long tile_cost(int K) { return 350 + 11LL * K / 768; }
 
 // End of the greedy range that starts at unit u under the cost bound C: it
 // takes whole units while the cost (units' cost + tc per token tile
@@ -427,7 +426,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     {
         std::lock_guard<std::mutex> lock(h->sched_mu);
         if (h->sched_m != M) {
-            h->sched_grid = make_schedule(h->cost, upt, ntiles, static_cast<int>(cap), kTileCost, h->sched);
+            h->sched_grid = make_schedule(h->cost, upt, ntiles, static_cast<int>(cap), tile_cost(h->w.K), h->sched);
             h->sched_m = M;
         }
         grid = h->sched_grid;

@@ -58,6 +58,11 @@ static_assert(kRing == 8 || kRing == 12 || kRing == 16, "the record ring's switc
 #define BSG_GROUP_END_COST 6
 #endif
 constexpr int kGroupEndCost = BSG_GROUP_END_COST;
+// Bytes per bulk copy of a token tile into shared memory (a multiple of 16).
+#ifndef BSG_TMA_PIECE
+#define BSG_TMA_PIECE 65536
+#endif
+constexpr unsigned kTmaPiece = BSG_TMA_PIECE;
 
 // 4x4 byte transpose.  In: a/b/c/d = bytes (x0..x3) of rows 0..3.  Out:
 // t_i = (a_i, b_i, c_i, d_i).
@@ -314,11 +319,12 @@ __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.
 // column offset for row l % 16, lb = 16 (l / 16) selects the chunk (16
 // tokens) of matrix l / 16.  tb is 128-byte aligned, so XOR with 16 c moves
 // to chunk c of the same row.
-__device__ __forceinline__ void step16(uint32_t tb, uint32_t lb, int off, const int4& w, int (&acc)[32]) {
+__device__ __forceinline__ void gather16(uint32_t tb, uint32_t lb, int off, uint32_t (&t)[8]) {
     const uint32_t a0 = tb + (static_cast<uint32_t>(off) ^ lb);
-    uint32_t t[8];
     ldsm_x2_trans_b8(a0, t[0], t[1], t[2], t[3]);
     ldsm_x2_trans_b8(a0 ^ 32u, t[4], t[5], t[6], t[7]);
+}
+__device__ __forceinline__ void dot16(const uint32_t (&t)[8], const int4& w, int (&acc)[32]) {
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         acc[4 * i + 0] = __dp4a(static_cast<int>(t[i]), w.x, acc[4 * i + 0]);
@@ -326,6 +332,11 @@ __device__ __forceinline__ void step16(uint32_t tb, uint32_t lb, int off, const 
         acc[4 * i + 2] = __dp4a(static_cast<int>(t[i]), w.z, acc[4 * i + 2]);
         acc[4 * i + 3] = __dp4a(static_cast<int>(t[i]), w.w, acc[4 * i + 3]);
     }
+}
+__device__ __forceinline__ void step16(uint32_t tb, uint32_t lb, int off, const int4& w, int (&acc)[32]) {
+    uint32_t t[8];
+    gather16(tb, lb, off, t);
+    dot16(t, w, acc);
 }
 
 // This lane's view of the step records: ro points at the column offset of
@@ -404,14 +415,16 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             waited = true;
         }
         const bool stage = (t != staged);
-        if (TMA && stage && tid == 0) {
-            // one bulk copy of the token tile (already swizzled in a.xb)
+        if (TMA && stage && warp == 0) {
+            // the token tile (already swizzled in a.xb) in kTmaPiece-byte bulk
+            // copies, issued by the lanes of warp 0 (one completion barrier)
             const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
             const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * kTile;
             fence_proxy_async();
-            mbar_arrive_expect_tx(bar, bytes);
-            for (unsigned off = 0; off < bytes; off += 65536u)
-                bulk_g2s(tb + off, src + off, min(65536u, bytes - off), bar);
+            if (lane == 0) mbar_arrive_expect_tx(bar, bytes);
+            __syncwarp();
+            for (unsigned off = static_cast<unsigned>(lane) * kTmaPiece; off < bytes; off += 32u * kTmaPiece)
+                bulk_g2s(tb + off, src + off, min(static_cast<unsigned>(kTmaPiece), bytes - off), bar);
         }
         __syncthreads();  // the group window is visible
         const int sa = gp(g_lo);
