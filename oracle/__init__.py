@@ -63,6 +63,8 @@ def _load():
             lib.oracle_gelu_f64.restype = c_double
             lib.oracle_gelu_f32.argtypes = [c_float]
             lib.oracle_gelu_f32.restype = c_float
+            lib.oracle_recip_f32.argtypes = [c_float]
+            lib.oracle_recip_f32.restype = c_float
             lib.oracle_requant.argtypes = [c_float, c_float]
             lib.oracle_requant.restype = ctypes.c_int8
             lib.oracle_linear.argtypes = [c_int, c_int, c_int, i8p, i8p, f32p, f32p, c_int, c_float,
@@ -142,6 +144,12 @@ def dequant_f64(a: int, scale: float, bias: float) -> float:
 
 def gelu_f32(y: float) -> np.float32:
     return np.float32(_load().oracle_gelu_f32(float(np.float32(y))))
+
+
+def recip_f32(b: float) -> np.float32:
+    """1/b (1 <= b < 2^25) by the fixed Newton-Raphson fp32 sequence that
+    the int8 GELU uses."""
+    return np.float32(_load().oracle_recip_f32(float(np.float32(b))))
 
 
 def gelu_f64(y: float) -> float:

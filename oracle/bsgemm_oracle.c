@@ -143,6 +143,37 @@ double oracle_gelu_f64(double y) {
     return 0.5 * y * (1.0 + erf(y / sqrt(2.0)));
 }
 
+/* 1/b for 1 <= b < 2^25 by Newton's method for the reciprocal, as a fixed
+ * sequence of IEEE fp32 operations (round to nearest even), so that every
+ * machine gets the same bits:
+ *   b = m 2^E with 1 <= m < 2 (exact, from the bits of b)
+ *   y0 = fma(-8/17, m, 24/17)   (the minimax straight line for 1/m on [1, 2),
+ *                                relative error <= 1/17; both constants rounded
+ *                                to fp32: 0x1.e1e1e2p-2, 0x1.69696ap+0)
+ *   y_{i+1} = fma(y_i, fma(-m, y_i, 1), y_i),  i = 0, 1, 2
+ *                               (each step squares the relative error:
+ *                                1/17 -> 3.5e-3 -> 1.2e-5 -> 1.5e-10)
+ *   1/b = y3 * 2^-E             (exact: a power of two, result normal)
+ * The result is within about half an ulp of 1/b; it need not be the
+ * correctly rounded quotient. */
+float oracle_recip_f32(float b) {
+    uint32_t bits;
+    memcpy(&bits, &b, sizeof bits);
+    const int E = (int)((bits >> 23) & 0xffu) - 127;
+    const uint32_t mbits = (bits & 0x7fffffu) | (127u << 23);
+    float m;
+    memcpy(&m, &mbits, sizeof m);
+    float y = fmaf(-0x1.e1e1e2p-2f, m, 0x1.69696ap+0f);
+    for (int i = 0; i < 3; ++i) {
+        const float e = fmaf(-m, y, 1.0f);
+        y = fmaf(y, e, y);
+    }
+    const uint32_t sbits = (uint32_t)(127 - E) << 23;
+    float s2;
+    memcpy(&s2, &sbits, sizeof s2);
+    return y * s2;
+}
+
 /* erf-form GELU evaluated in fp32 by a fixed op sequence, so that an int8
  * result decided from it is reproducible on any IEEE machine.  erf comes from
  * Abramowitz & Stegun, Handbook of Mathematical Functions, formula 7.1.28:
@@ -154,7 +185,10 @@ double oracle_gelu_f64(double y) {
  *   h  = fma(ax, a6, a5); h = fma(ax, h, a4); h = fma(ax, h, a3);
  *   h  = fma(ax, h, a2);  h = fma(ax, h, a1); p = fma(ax, h, 1)
  *   p2 = p*p; p4 = p2*p2; p8 = p4*p4; p16 = p8*p8
- *   e  = 1 - 1/p16;   erf = (x < 0) ? -e : e
+ *   e  = 1 if p16 >= 2^25, else 1 - recip(p16)  (recip: Newton's method
+ *        above; from p16 = 2^25 on, 1 - 1/p16 rounds to 1 in fp32 for the
+ *        exact quotient too: 1 - 2^-25 is a tie, rounded to even)
+ *   erf = (x < 0) ? -e : e
  *   g  = (0.5 * y) * (1 + erf)                                            */
 float oracle_gelu_f32(float y) {
     const float a1 = 0.0705230784f, a2 = 0.0422820123f, a3 = 0.0092705272f;
@@ -171,8 +205,7 @@ float oracle_gelu_f32(float y) {
     float p4 = p2 * p2;
     float p8 = p4 * p4;
     float p16 = p8 * p8;
-    float rcp = 1.0f / p16;
-    float e = 1.0f - rcp;
+    float e = (p16 >= 0x1p25f) ? 1.0f : 1.0f - oracle_recip_f32(p16);
     float erfv = (x < 0.0f) ? -e : e;
     float half_y = 0.5f * y;
     float one_plus = 1.0f + erfv;

@@ -78,9 +78,29 @@ __device__ __forceinline__ void transpose4(uint32_t a, uint32_t b, uint32_t c, u
     t3 = __byte_perm(ab_hi, cd_hi, 0x7632);            // a3 b3 c3 d3
 }
 
+// 1/b for 1 <= b < 2^25 by Newton's method, as a fixed sequence of IEEE
+// round-to-nearest fp32 operations (no branch, no special function unit):
+// b = m 2^E (1 <= m < 2, from the bits), y0 = 24/17 - (8/17) m (the minimax
+// straight line for 1/m, relative error <= 1/17; both constants rounded to
+// fp32), three steps y <- y + y (1 - m y) (each squares the relative error,
+// 1/17 -> 3.5e-3 -> 1.2e-5 -> 1.5e-10), then the exact scaling by 2^-E.
+// Within about half an ulp of 1/b, the same bits on every IEEE machine.
+__device__ __forceinline__ float recip_nr_f32(float b) {
+    const uint32_t bits = __float_as_uint(b);
+    const uint32_t ex = (bits >> 23) & 0xffu;  // E + 127
+    const float m = __uint_as_float((bits & 0x7fffffu) | (127u << 23));
+    float y = __fmaf_rn(-0x1.e1e1e2p-2f, m, 0x1.69696ap+0f);
+#pragma unroll
+    for (int i = 0; i < 3; ++i) y = __fmaf_rn(y, __fmaf_rn(-m, y, 1.0f), y);
+    return __fmul_rn(y, __uint_as_float((254u - ex) << 23));  // 2^-E: biased exponent 127 - E
+}
+
 // erf-form GELU in fp32 by a fixed sequence of IEEE round-to-nearest ops.
 // erf(|x|) = 1 - p(|x|)^-16, p = 1 + a1 x + ... + a6 x^6 (Abramowitz &
-// Stegun 7.1.28, |error| <= 3e-7); p^16 by four squarings.
+// Stegun 7.1.28, |error| <= 3e-7); p^16 by four squarings; 1/p^16 by
+// recip_nr_f32 below 2^25, and erf = 1 from there on (where 1 - 1/p^16
+// rounds to 1 in fp32 whatever the quotient's last bits).  Branch-free, so
+// the 32 values of a lane's epilogue interleave.
 __device__ __forceinline__ float gelu_f32(float y) {
     const float x = __fmul_rn(y, 0.70710678f);
     const float ax = fabsf(x);
@@ -94,7 +114,8 @@ __device__ __forceinline__ float gelu_f32(float y) {
     const float p4 = __fmul_rn(p2, p2);
     const float p8 = __fmul_rn(p4, p4);
     const float p16 = __fmul_rn(p8, p8);
-    const float e = __fsub_rn(1.0f, __frcp_rn(p16));  // IEEE 1/p16, round to nearest
+    const float r = recip_nr_f32(fminf(p16, 0x1.fffffep24f));  // p16 below 2^25 unchanged; unused from there on
+    const float e = (p16 >= 0x1p25f) ? 1.0f : __fsub_rn(1.0f, r);
     const float erf_x = (x < 0.0f) ? -e : e;
     return __fmul_rn(__fmul_rn(0.5f, y), __fadd_rn(1.0f, erf_x));
 }

@@ -217,6 +217,25 @@ def test_gelu_f32_within_derived_bound():
         assert abs(float(oracle.gelu_f32(y)) - exact) <= 1.2e-6 * abs(float(y)) + 1e-12, y
 
 
+def test_recip_f32_within_an_ulp_of_the_quotient():
+    """Newton's method for 1/b (three steps from the 1/17 straight line)
+    lands within one ulp of the exact reciprocal over [1, 2^25)."""
+    rng = np.random.default_rng(7)
+    bs = np.concatenate([rng.uniform(1.0, 2.0, 20000), np.exp2(rng.uniform(0.0, 25.0, 20000)),
+                         [1.0, np.nextafter(np.float32(1), np.float32(2)), np.nextafter(np.float32(2), np.float32(1)),
+                          3.0, 7.5, 2.0 ** 24 + 2.0, np.nextafter(np.float32(2.0 ** 25), np.float32(0))]]).astype(np.float32)
+    for b in bs:
+        r = float(oracle.recip_f32(b))
+        exact = 1.0 / float(b)
+        ulp = float(np.spacing(np.float32(exact)))
+        assert abs(r - exact) <= ulp, (b, r, exact)
+
+
+def test_recip_f32_powers_of_two_exact():
+    for k in range(25):
+        assert float(oracle.recip_f32(np.float32(2.0 ** k))) == 2.0 ** -k
+
+
 def test_gelu_f32_special_values():
     assert float(oracle.gelu_f32(0.0)) == 0.0
     assert float(oracle.gelu_f32(1.0)) == pytest.approx(0.8413447460685429, abs=2e-7)
