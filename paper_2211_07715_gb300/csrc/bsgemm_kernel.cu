@@ -431,22 +431,23 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         auto gp = [&](int gi) { return s_gp[gi - g_lo]; };
 
         for (int i = tid; i <= g_hi - g_lo; i += kThreads) s_gp[i] = __ldg(w.gptr + g_lo + i);
-        if (!waited) {  // nothing above reads the activations or writes global memory
-            griddep_wait();
-            waited = true;
-        }
         const bool stage = (t != staged);
-        if (TMA && stage && warp == 0) {
-            // the token tile (already swizzled in a.xb) in kTmaPiece-byte bulk
-            // copies, issued by the lanes of warp 0 (one completion barrier)
-            const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
-            const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * kTile;
-            fence_proxy_async();
-            if (lane == 0) mbar_arrive_expect_tx(bar, bytes);
-            __syncwarp();
-            for (unsigned off = static_cast<unsigned>(lane) * kTmaPiece; off < bytes; off += 32u * kTmaPiece)
-                bulk_g2s(tb + off, src + off, min(static_cast<unsigned>(kTmaPiece), bytes - off), bar);
-        }
+        // the token tile (already swizzled in a.xb) in kTmaPiece-byte bulk
+        // copies, issued by the lanes of warp 0 (one completion barrier)
+        auto copy_tile = [&]() {
+            if (TMA && stage && warp == 0) {
+                const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
+                const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * kTile;
+                fence_proxy_async();
+                if (lane == 0) mbar_arrive_expect_tx(bar, bytes);
+                __syncwarp();
+                for (unsigned off = static_cast<unsigned>(lane) * kTmaPiece; off < bytes; off += 32u * kTmaPiece)
+                    bulk_g2s(tb + off, src + off, min(static_cast<unsigned>(kTmaPiece), bytes - off), bar);
+            }
+        };
+        // After the first window the previous grid is done: the copy starts
+        // at once and overlaps the window's set-up.
+        if (waited) copy_tile();
         __syncthreads();  // the group window is visible
         const int sa = gp(g_lo);
         if (tid <= kWarps) {
@@ -469,11 +470,6 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             s_wst[tid] = (tid == kWarps) ? s_gp[ngw] - sa : s_gp[lo] - sa + static_cast<int>(into < len ? into : len);
         }
         __syncthreads();  // the warps' step ranges are visible
-        if (!TMA && stage) {  // gather the tile with per-thread loads
-            stage_tile(tile, a, K, kpad, m0);
-            __syncthreads();
-            staged = t;
-        }
 
         const int ws0 = s_wst[warp], ws1 = s_wst[warp + 1];
 
@@ -510,6 +506,20 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             off[i] = 0;
             wq[i] = make_int4(0, 0, 0, 0);
             if (ws0 < ws1) rec.load(i, off[i], wq[i]);
+        }
+
+        // Everything above reads only the weights: in the first window it
+        // overlaps the end of the previous kernel.  The activations and any
+        // global write wait for that kernel's completion.
+        if (!waited) {
+            griddep_wait();
+            waited = true;
+            copy_tile();
+        }
+        if (!TMA && stage) {  // gather the tile with per-thread loads
+            stage_tile(tile, a, K, kpad, m0);
+            __syncthreads();
+            staged = t;
         }
 
         // Row groups without any stored block: acc = 0.
