@@ -413,7 +413,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     const uint32_t bar = smem_addr(&s_bar);
     if (TMA && tid == 0) mbar_init(bar, 1);
     // slots start at zero; whoever finishes a slot resets it
-    for (int i = tid; i < kSlots * SW; i += kThreads) slots[i] = 0;
+    for (int i = tid; i < kSlots * SW / 4; i += kThreads) reinterpret_cast<int4*>(slots)[i] = make_int4(0, 0, 0, 0);
     __syncthreads();
     unsigned phase = 0;
     long long u = sched.u[blockIdx.x];
@@ -648,7 +648,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             }
             store_lane<KIND>(a, N, m0 + g, fin_r, acc, fin_sc, fin_bi);
         }
-        __syncthreads();  // the window's offsets, the slots' reset and the tile may be reused
+        if (u < u_end) __syncthreads();  // the window's offsets, the slots' reset and the tile may be reused
     }
 }
 
