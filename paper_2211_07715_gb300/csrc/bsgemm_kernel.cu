@@ -257,7 +257,7 @@ __device__ __forceinline__ void store_unit(unsigned char* xt, int g, int kc, con
 // with per-thread loads.  Each thread keeps kStageBatch units' loads in
 // flight before transposing them.
 #ifndef BSG_STAGE_BATCH
-#define BSG_STAGE_BATCH 8
+#define BSG_STAGE_BATCH 4
 #endif
 __device__ __forceinline__ void stage_tile(unsigned char* xt, const LaunchArgs& a, int K, int kpad, long long m0) {
     constexpr int G = kTile / 4;
