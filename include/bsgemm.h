@@ -171,6 +171,32 @@ int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, v
                      void* stream);
 
 /*
+ * bsgemm_run_host -- the end-to-end call on HOST buffers: copy act in, run
+ * the layer (bsgemm_run_ws's two kernels), copy the result out, all
+ * enqueued on `stream`.  The paper's engine (Sec. 3) runs on the CPU and
+ * takes and returns tensors in host memory; this is that call on the GPU,
+ * with the transfers over the host link inside it.
+ *   act        HOST int8 [M][K] row-major.
+ *   out        HOST [M][N] row-major of the epilogue's type.
+ *              Both should be page-locked (cudaHostAlloc/cudaHostRegister):
+ *              then the two copies are asynchronous.  Pageable buffers
+ *              work, with CUDA's pageable-copy behaviour (the calling
+ *              thread blocks on the copies).
+ *   workspace  DEVICE, >= bsgemm_host_workspace_bytes(h, M, epi.kind)
+ *              bytes, 16-byte aligned: the activations' copy, their token
+ *              tiles and the device result, each at a 256-byte aligned
+ *              offset.  Scratch as for bsgemm_run_ws: two calls in flight
+ *              at the same time need two workspaces.
+ * Returns after enqueueing (two copies, two kernels); `out` holds the
+ * result once `stream` has completed, and `act` must not change before
+ * then.  Return codes as bsgemm_run_ws, plus BSGEMM_ERR_CUDA if a copy
+ * cannot be enqueued.
+ */
+size_t bsgemm_host_workspace_bytes(bsgemm_t h, int M, int32_t kind);
+int bsgemm_run_host(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* workspace,
+                    size_t workspace_bytes, void* stream);
+
+/*
  * bsgemm_device_status -- read (and with clear != 0, reset) the handle's
  * device status word.  0 means every wait in the kernels completed; bit 0
  * (BSGEMM_STATUS_TIMEOUT) means a bounded wait on an asynchronous copy gave

@@ -68,6 +68,10 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_tile_activations.restype = ctypes.c_int
     lib.bsgemm_run_tiled.argtypes = [vp, vp, ctypes.c_size_t, ctypes.c_int, vp, Epilogue, vp]
     lib.bsgemm_run_tiled.restype = ctypes.c_int
+    lib.bsgemm_host_workspace_bytes.argtypes = [vp, ctypes.c_int, ctypes.c_int32]
+    lib.bsgemm_host_workspace_bytes.restype = ctypes.c_size_t
+    lib.bsgemm_run_host.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp, ctypes.c_size_t, vp]
+    lib.bsgemm_run_host.restype = ctypes.c_int
     lib.bsgemm_device_status.argtypes = [vp, ctypes.c_int]
     lib.bsgemm_device_status.restype = ctypes.c_int
     return lib
@@ -76,7 +80,8 @@ def _load() -> ctypes.CDLL:
 _lib = _load()
 
 EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
-            "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
+            "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_host_workspace_bytes", "bsgemm_run_host",
+            "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
             "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
 
 
@@ -149,6 +154,19 @@ def bsgemm_run_tiled(h: int, tiles_ptr: int, tiles_bytes: int, m: int, out_ptr: 
                                stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_run_host(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float, ws_ptr: int,
+                    ws_bytes: int, stream: int = 0) -> None:
+    """Enqueue the end-to-end call: HOST act and out, a DEVICE workspace."""
+    rc = _lib.bsgemm_run_host(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), ws_ptr,
+                              int(ws_bytes), stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_host_workspace_bytes(h: int, m: int, kind: int) -> int:
+    return int(_lib.bsgemm_host_workspace_bytes(h, int(m), int(kind)))
 
 
 def bsgemm_workspace_bytes(h: int, m: int) -> int:
@@ -239,23 +257,45 @@ class SparseInt8Linear:
         bsgemm_run_ws(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, workspace.data_ptr(),
                       workspace.numel() * workspace.element_size(), s.cuda_stream)
 
-    def __call__(self, x, kind: int, out_scale: float = 1.0, stream=None):
-        """Allocate the output and run.  A CPU `x` is copied in and the result
-        copied back (the end-to-end path); a CUDA `x` stays on the device."""
+    def __call__(self, x, kind: int, out_scale: float = 1.0, stream=None, out=None, sync: bool = True):
+        """Allocate the output (unless `out` is given) and run.
+
+        A CUDA `x` stays on the device.  A CPU `x` takes the end-to-end path
+        (bsgemm_run_host): it is copied in, the layer runs, and the result is
+        copied back into `out` (a CPU tensor, pinned for an asynchronous
+        copy) or a new one.  With sync=False and pinned `x` and `out`, the
+        call only enqueues on `stream` (default: the current stream): the
+        caller synchronises that stream before reading `out`, and leaves `x`
+        unchanged until then.  The device workspace comes from PyTorch's
+        caching allocator on that stream.
+        """
         import torch
         dtype = getattr(torch, _OUT_DTYPES[kind])
+        s = torch.cuda.current_stream() if stream is None else stream
         if x.is_cuda:
-            out = torch.empty((x.shape[0], self.n_out), dtype=dtype, device=x.device)
-            self.run(x, out, kind, out_scale, stream)
+            if out is None:
+                out = torch.empty((x.shape[0], self.n_out), dtype=dtype, device=x.device)
+            self.run(x, out, kind, out_scale, s)
             return out
+        if x.dtype != torch.int8 or not x.is_contiguous() or x.dim() != 2 or x.shape[1] != self.k_in:
+            raise ValueError("x must be a contiguous int8 tensor [M][K]")
+        m = x.shape[0]
         pinned = x.is_pinned()
-        xd = x.to("cuda", non_blocking=pinned)
-        out = torch.empty((x.shape[0], self.n_out), dtype=dtype, device=xd.device)
-        self.run(xd, out, kind, out_scale, stream)
-        host = torch.empty(out.shape, dtype=dtype, pin_memory=pinned)
-        host.copy_(out, non_blocking=pinned)
-        (torch.cuda.current_stream() if stream is None else stream).synchronize()
-        return host
+        if out is None:
+            out = torch.empty((m, self.n_out), dtype=dtype, pin_memory=pinned)
+        elif out.is_cuda or out.dtype != dtype or tuple(out.shape) != (m, self.n_out) or not out.is_contiguous():
+            raise ValueError(f"out must be a contiguous CPU {dtype} tensor of shape {(m, self.n_out)}")
+        if not sync and not (pinned and out.is_pinned()):
+            raise ValueError("sync=False needs a pinned x and a pinned out")
+        if m == 0:
+            return out
+        need = bsgemm_host_workspace_bytes(self._h, m, kind)
+        with torch.cuda.stream(s):
+            ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+        bsgemm_run_host(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, ws.data_ptr(), need, s.cuda_stream)
+        if sync:
+            s.synchronize()
+        return out
 
     def close(self) -> None:
         if getattr(self, "_h", None):

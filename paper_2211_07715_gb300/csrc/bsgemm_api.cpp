@@ -507,6 +507,58 @@ size_t bsgemm_workspace_bytes(bsgemm_t h, int M) {
     return bsg::tiled_bytes(h->w.K, M);
 }
 
+// Workspace of bsgemm_run_host: [act copy | token tiles | device result],
+// each part at a 256-byte aligned offset.  Returns 0 for an unknown kind.
+static size_t host_parts(bsgemm_t h, int M, int32_t kind, size_t* off_tiles, size_t* off_out, size_t* out_bytes) {
+    static const size_t elem[5] = {4, 4, 4, 1, 1};
+    if (kind < BSGEMM_OUT_I32 || kind > BSGEMM_OUT_I8_GELU) return 0;
+    const size_t m = static_cast<size_t>(M);
+    *off_tiles = align_up(m * static_cast<size_t>(h->w.K), 256);
+    *off_out = *off_tiles + align_up(bsg::tiled_bytes(h->w.K, M), 256);
+    *out_bytes = m * static_cast<size_t>(h->w.N) * elem[kind];
+    return *off_out + *out_bytes;
+}
+
+size_t bsgemm_host_workspace_bytes(bsgemm_t h, int M, int32_t kind) {
+    if (!h || M <= 0) return 0;
+    size_t ot = 0, oo = 0, ob = 0;
+    return host_parts(h, M, kind, &ot, &oo, &ob);
+}
+
+int bsgemm_run_host(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* workspace,
+                    size_t workspace_bytes, void* stream) {
+    clear_error();
+    if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
+    if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
+    if (epi.kind < BSGEMM_OUT_I32 || epi.kind > BSGEMM_OUT_I8_GELU)
+        return fail(BSGEMM_ERR_INVALID, "unknown epilogue kind " + std::to_string(epi.kind));
+    if (M == 0) return BSGEMM_OK;
+    if (!act || !out) return fail(BSGEMM_ERR_INVALID, "act and out must not be NULL");
+    size_t off_tiles = 0, off_out = 0, out_bytes = 0;
+    const size_t need = host_parts(h, M, epi.kind, &off_tiles, &off_out, &out_bytes);
+    if (!workspace || workspace_bytes < need)
+        return fail(BSGEMM_ERR_INVALID, "workspace must hold bsgemm_host_workspace_bytes(h, M, kind) = " +
+                                            std::to_string(need) + " bytes");
+    if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0)
+        return fail(BSGEMM_ERR_INVALID, "workspace must be 16-byte aligned");
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
+    if (dev != h->device)
+        return fail(BSGEMM_ERR_INVALID, "current device " + std::to_string(dev) + " is not the handle's device " +
+                                            std::to_string(h->device));
+    char* ws = static_cast<char*>(workspace);
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    e = cudaMemcpyAsync(ws, act, static_cast<size_t>(M) * static_cast<size_t>(h->w.K), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("copy of act to the device", e));
+    const int rc = run_common(h, reinterpret_cast<const int8_t*>(ws), M, ws + off_out, epi, ws + off_tiles,
+                              off_out - off_tiles, 1, stream);
+    if (rc != BSGEMM_OK) return rc;
+    e = cudaMemcpyAsync(out, ws + off_out, out_bytes, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("copy of the result to the host", e));
+    return BSGEMM_OK;
+}
+
 int bsgemm_device_status(bsgemm_t h, int clear) {
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");

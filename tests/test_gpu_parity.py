@@ -299,6 +299,58 @@ def test_host_tensors_round_trip(bsg):
           synth.I8)
 
 
+def test_host_tensors_pipelined_on_two_streams(bsg):
+    """The asynchronous end-to-end call: pinned batches in, pinned results
+    out, steps alternating between two streams, read after a synchronize."""
+    import torch
+    rng = synth.rng_for(5710)
+    wt = synth.draw_weight(rng, 96, 1024, 0.9)
+    w = oracle.weight_dense(wt)
+    lin = make_linear(bsg, wt)
+    streams = [torch.cuda.Stream() for _ in range(2)]
+    xs = [synth.draw_x(rng, m, 1024, "u127") for m in (130, 64, 1, 257)]
+    hx = [torch.from_numpy(x).pin_memory() for x in xs]
+    hout = [torch.empty((x.shape[0], 96), dtype=torch.int8, pin_memory=True) for x in xs]
+    for i in range(len(xs)):
+        got = lin(hx[i], synth.I8_GELU, 0.03, stream=streams[i % 2], out=hout[i], sync=False)
+        assert got is hout[i]
+    for st in streams:
+        st.synchronize()
+    for x, out in zip(xs, hout):
+        check(out.numpy(), oracle.linear(x, w, wt.scales, wt.bias, synth.I8_GELU, out_scale=0.03), synth.I8_GELU)
+    with pytest.raises(ValueError):
+        lin(torch.from_numpy(xs[0]), synth.I8, 1.0, out=hout[0], sync=False)
+    with pytest.raises(ValueError):
+        lin(hx[0], synth.F32, 1.0, out=hout[0])
+
+
+def test_run_host_through_the_c_abi(bsg):
+    """bsgemm_run_host with raw pointers: pageable buffers (the copies block),
+    every epilogue kind, and its argument checks."""
+    import torch
+    rng = synth.rng_for(5720)
+    wt = synth.draw_weight(rng, 64, 520, 0.8)
+    w = oracle.weight_dense(wt)
+    lin = make_linear(bsg, wt)
+    x = synth.draw_x(rng, 77, 520, "u127")
+    for kind in KINDS:
+        need = bsg.bsgemm_host_workspace_bytes(lin._h, 77, kind)
+        elem = 1 if kind in (synth.I8, synth.I8_GELU) else 4
+        assert need >= 77 * 520 + bsg.bsgemm_workspace_bytes(lin._h, 77) + 77 * 64 * elem
+        ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+        out = np.zeros((77, 64), dtype={synth.I32: np.int32, synth.I8: np.int8, synth.I8_GELU: np.int8}.get(kind, np.float32))
+        bsg.bsgemm_run_host(lin._h, x.ctypes.data, 77, out.ctypes.data, kind, 0.04, ws.data_ptr(), need, 0)
+        torch.cuda.synchronize()
+        check(out, oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.04), kind)
+        with pytest.raises(bsg.BsgemmError) as e:
+            bsg.bsgemm_run_host(lin._h, x.ctypes.data, 77, out.ctypes.data, kind, 0.04, ws.data_ptr(), need - 1, 0)
+        assert e.value.code == bsg.ERR_INVALID
+    assert bsg.bsgemm_host_workspace_bytes(lin._h, 77, 7) == 0
+    bsg.bsgemm_run_host(lin._h, 0, 0, 0, synth.I8, 1.0, 0, 0, 0)  # M = 0: nothing to do
+    with pytest.raises(bsg.BsgemmError):
+        bsg.bsgemm_run_host(lin._h, 0, 77, 0, synth.I8, 1.0, ws.data_ptr(), need, 0)
+
+
 def test_from_dense(bsg):
     rng = synth.rng_for(5800)
     wt = synth.draw_weight(rng, 128, 768, 0.8)
