@@ -413,9 +413,39 @@ def cpu_baseline(case, rows: int | None, threads: int | None = None, reps: int =
 
 # -------------------------------------------------------- reference arm --
 
+def run_reference_prune(args) -> dict:
+    """The oracle's block pruning (double scores, qsort) on the prune
+    workload's weights, one whole weight per step."""
+    import oracle
+    n_out, k_in, sparsity = 768, 3072, 0.9
+    blocks = n_out // 4 * k_in
+    rng = synth.rng_for(synth.SEED_BASE + 50)
+    w_host = [rng.normal(0.0, 0.02, size=(n_out, k_in)).astype(np.float32) for _ in range(2)]
+    for i in range(args.warmup):
+        oracle.block_prune(w_host[i % 2], sparsity)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        oracle.block_prune(w_host[i % 2], sparsity)
+    dt = (time.perf_counter() - t0) / args.steps
+    value = blocks / dt
+    return {
+        "impl": "reference", "metric": "block pruning throughput (4x1 blocks scored and selected per second)",
+        "value": round(value, 1), "unit": "blocks/s", "n_gpus": 0, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(dt * 1e3, 3), "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "average-magnitude 4x1 block pruning of a 768 x 3072 fp32 weight to 90% sparsity",
+                   "n_out": n_out, "k_in": k_in, "sparsity": sparsity, "blocks": blocks},
+        "cpu_baseline": {"value": round(value, 1), "unit": "blocks/s", "cores": 1, "kind": "oracle",
+                         "sample": "the whole weight per step, one host thread"},
+        "e2e": {"value": round(value, 1), "unit": "blocks/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
 def run_reference(args, rank: int) -> dict | None:
     if rank != 0:
         return None
+    if args.workload == "prune":
+        return run_reference_prune(args)
     case = WORKLOADS[args.workload]()
     threads = os.cpu_count() or 1
     rows = min(case.m, args.ref_rows)
@@ -726,15 +756,122 @@ def run_stack(args) -> dict:
     }
 
 
+def run_prune(args) -> dict:
+    """Create-side block pruning (App. A.1) of an fp32 weight of the FFN2
+    shape (768 x 3072, normal(0, 0.02)) to 90% block sparsity: one step is
+    one bsgemm_block_prune call (score kernel, 8-pass radix select of the
+    threshold score, ordered tie count and mask write; it synchronises its
+    stream)."""
+    import torch
+    import paper_2211_07715_gb300 as bsg
+    import oracle
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    props = torch.cuda.get_device_properties(dev)
+    n_out, k_in, sparsity = 768, 3072, 0.9
+    blocks = n_out // 4 * k_in
+    w_bytes = n_out * k_in * 4
+    nsets = max(2, math.ceil(2 * int(getattr(props, "L2_cache_size", 128 << 20)) / w_bytes) + 1)
+    rng = synth.rng_for(synth.SEED_BASE + 50)
+    w_host = [rng.normal(0.0, 0.02, size=(n_out, k_in)).astype(np.float32) for _ in range(2)]
+    ws = [torch.from_numpy(w_host[i % 2]).to(dev) for i in range(nsets)]
+    keeps = [torch.empty((n_out // 4, k_in), dtype=torch.uint8, device=dev) for _ in range(nsets)]
+    stream = torch.cuda.current_stream(dev)
+    kept = []
+
+    def step(i: int):
+        kept.append(bsg.bsgemm_block_prune(n_out, k_in, ws[i % nsets].data_ptr(), sparsity,
+                                           keeps[i % nsets].data_ptr(), stream.cuda_stream))
+
+    for i in range(args.warmup):
+        step(i)
+    steps = args.steps
+    sampler = ClockSampler(str(getattr(props, "uuid", "")))
+    sampler.start()
+    time.sleep(0.3)
+    mark0 = sampler.mark()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(steps):
+        step(i)
+    end.record(stream)
+    end.synchronize()
+    mark1 = sampler.mark()
+    time.sleep(0.2)
+    sampler.stop()
+    clocks = sampler.summary(mark0, max(mark1, mark0 + 1))
+    ms = start.elapsed_time(end) / steps
+    assert all(k == blocks - int(np.floor(sparsity * blocks + 0.5)) for k in kept)
+
+    # end to end: the weight from pinned host memory, the mask back to it
+    hw = [torch.from_numpy(w_host[i]).pin_memory() for i in range(2)]
+    hk = [torch.empty((n_out // 4, k_in), dtype=torch.uint8, pin_memory=True) for _ in range(2)]
+    wd = torch.empty((n_out, k_in), dtype=torch.float32, device=dev)
+
+    def e2e_step(i: int):
+        wd.copy_(hw[i % 2], non_blocking=True)
+        keep = bsg.block_prune(wd, sparsity, stream)
+        hk[i % 2].copy_(keep, non_blocking=True)
+
+    for i in range(3):
+        e2e_step(i)
+    e_steps = min(steps, 200)
+    s2, t2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s2.record(stream)
+    for i in range(e_steps):
+        e2e_step(i)
+    t2.record(stream)
+    t2.synchronize()
+    e2e_ms = s2.elapsed_time(t2) / e_steps
+
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peaks = json.load(f)
+    except (OSError, ValueError):
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6683.8))
+    alg = w_bytes + blocks  # read W once, write the mask once
+    gbs = alg / (ms * 1e-3) / 1e9
+    result = {
+        "metric": "block pruning throughput (4x1 blocks scored and selected per second)",
+        "value": round(blocks / (ms * 1e-3), 1), "unit": "blocks/s", "n_gpus": 1, "steps": steps,
+        "warmup": args.warmup, "ms_per_step": round(ms, 6), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "average-magnitude 4x1 block pruning of a 768 x 3072 fp32 weight to 90% sparsity",
+                   "n_out": n_out, "k_in": k_in, "sparsity": sparsity, "blocks": blocks,
+                   "l2": f"rotating {nsets} weights ({nsets * w_bytes / 2**20:.0f} MiB > 2 x L2)",
+                   "launch": "one synchronous bsgemm_block_prune call per step (20 kernels)"},
+        "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
+                     "frac": round(gbs / hbm_peak, 4), "traffic": None, "kernel": "bsgemm_block_prune (whole call)",
+                     "bytes_basis": "algorithmic: fp32 weight read once + uint8 mask written once"},
+        "e2e": {"value": round(blocks / (e2e_ms * 1e-3), 1), "unit": "blocks/s", "h2d_bytes_per_step": w_bytes,
+                "d2h_bytes_per_step": blocks},
+        "gpu_launches": 20 * steps, "clocks": clocks,
+    }
+    if not args.no_cpu_baseline:
+        t0 = time.perf_counter()
+        reps = 0
+        while reps < 3 or time.perf_counter() - t0 < 2.0:
+            oracle.block_prune(w_host[reps % 2], sparsity)
+            reps += 1
+        dt = (time.perf_counter() - t0) / reps
+        result["cpu_baseline"] = {"value": round(blocks / dt, 1), "unit": "blocks/s", "cores": 1, "kind": "oracle",
+                                  "sample": f"the whole weight, {reps} passes, {dt * 1e3:.1f} ms per pass "
+                                            "(double scores, qsort of (score, index))"}
+    return result
+
+
 def main():
     p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=2000)
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "stack"], default="ffn2",
+    p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "stack", "prune"], default="ffn2",
                    help="ffn2/ffn1/single: one linear; layer: the encoder layer's four linears; stack: the "
-                        "six-layer stack sweep")
+                        "six-layer stack sweep; prune: create-side block pruning of an FFN2-shaped weight")
     p.add_argument("--ref-rows", type=int, default=512, help="tokens per reference step")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--soak-seconds", type=float, default=1.0, help="untimed load before the timed region")
@@ -747,6 +884,8 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
+        if args.workload in ("layer", "stack"):
+            p.error("--impl reference times the single-linear workloads and prune")
         res = run_reference(args, rank)
     else:
         if world > 1:
@@ -758,6 +897,8 @@ def main():
             res = run_layer(args) if rank == 0 else None
         elif args.workload == "stack":
             res = run_stack(args) if rank == 0 else None
+        elif args.workload == "prune":
+            res = run_prune(args) if rank == 0 else None
         else:
             res = run_ours(args, rank, world, local_rank)
         if world > 1:

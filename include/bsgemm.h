@@ -197,6 +197,26 @@ int bsgemm_run_host(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epil
                     size_t workspace_bytes, void* stream);
 
 /*
+ * bsgemm_block_prune -- the create-side pruning step (App. A.1): score each
+ * 4x1 block of a dense weight by the mean magnitude of its 4 values and
+ * prune the lowest-scoring ones until the sparsity ratio is reached.
+ *   N, K      weight shape; N a multiple of 4, N >= 4, K >= 1.
+ *   W         DEVICE float [N][K] row-major; every value finite.
+ *   sparsity  fraction of blocks pruned, 0 <= sparsity <= 1: the number
+ *             pruned is floor(sparsity * (N/4 * K) + 0.5).
+ *   keep      DEVICE uint8 [N/4][K]: written 1 for a kept block, 0 for a
+ *             pruned one.
+ * Scores are computed in double as (((|w0| + |w1|) + |w2|) + |w3|) / 4,
+ * w_i = W[4r + i][k], in that order; equal scores prune the lower block
+ * index r * K + k first, so the mask is unique.  Runs on `stream` on the
+ * current device with stream-ordered scratch (8 bytes per block) and
+ * synchronises `stream` before returning.  Returns the number of kept
+ * blocks, or BSGEMM_ERR_INVALID (bad shape, pointer or sparsity, or a
+ * non-finite weight; `keep` is then undefined) or BSGEMM_ERR_CUDA.
+ */
+int64_t bsgemm_block_prune(int N, int K, const float* W, double sparsity, uint8_t* keep, void* stream);
+
+/*
  * bsgemm_device_status -- read (and with clear != 0, reset) the handle's
  * device status word.  0 means every wait in the kernels completed; bit 0
  * (BSGEMM_STATUS_TIMEOUT) means a bounded wait on an asynchronous copy gave

@@ -72,6 +72,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_host_workspace_bytes.restype = ctypes.c_size_t
     lib.bsgemm_run_host.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp, ctypes.c_size_t, vp]
     lib.bsgemm_run_host.restype = ctypes.c_int
+    lib.bsgemm_block_prune.argtypes = [ctypes.c_int, ctypes.c_int, vp, ctypes.c_double, vp, vp]
+    lib.bsgemm_block_prune.restype = ctypes.c_int64
     lib.bsgemm_device_status.argtypes = [vp, ctypes.c_int]
     lib.bsgemm_device_status.restype = ctypes.c_int
     return lib
@@ -81,7 +83,7 @@ _lib = _load()
 
 EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
             "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_host_workspace_bytes", "bsgemm_run_host",
-            "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
+            "bsgemm_block_prune", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
             "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
 
 
@@ -169,6 +171,30 @@ def bsgemm_host_workspace_bytes(h: int, m: int, kind: int) -> int:
     return int(_lib.bsgemm_host_workspace_bytes(h, int(m), int(kind)))
 
 
+def bsgemm_block_prune(n_out: int, k_in: int, w_ptr: int, sparsity: float, keep_ptr: int, stream: int = 0) -> int:
+    """Average-magnitude 4x1 block pruning on the device (raw pointers);
+    returns the number of kept blocks, raises on failure."""
+    rc = _lib.bsgemm_block_prune(int(n_out), int(k_in), w_ptr, float(sparsity), keep_ptr, stream)
+    if rc < 0:
+        raise BsgemmError(int(rc), bsgemm_last_error())
+    return int(rc)
+
+
+def block_prune(w, sparsity: float, stream=None):
+    """Keep-mask [N/4][K] (uint8 CUDA tensor, 1 = kept) of the App. A.1
+    pruning of the fp32 CUDA weight `w` [N][K] to the given sparsity."""
+    import torch
+    if w.dtype != torch.float32 or not w.is_cuda or not w.is_contiguous() or w.dim() != 2:
+        raise ValueError("w must be a contiguous fp32 CUDA tensor [N][K]")
+    n_out, k_in = w.shape
+    if n_out % BLOCK:
+        raise ValueError("N must be a multiple of 4")
+    keep = torch.empty((n_out // BLOCK, k_in), dtype=torch.uint8, device=w.device)
+    s = torch.cuda.current_stream() if stream is None else stream
+    bsgemm_block_prune(n_out, k_in, w.data_ptr(), sparsity, keep.data_ptr(), s.cuda_stream)
+    return keep
+
+
 def bsgemm_workspace_bytes(h: int, m: int) -> int:
     return int(_lib.bsgemm_workspace_bytes(h, int(m)))
 
@@ -196,15 +222,22 @@ def bsgemm_info(h: int) -> dict:
 _OUT_DTYPES = {OUT_I32: "int32", OUT_F32: "float32", OUT_F32_GELU: "float32", OUT_I8: "int8", OUT_I8_GELU: "int8"}
 
 
-def dense_to_blocks(w: np.ndarray):
-    """Block-compress a dense int8 weight [N][K], keeping every 4x1 block that
-    holds a nonzero value.  Returns (indptr, colidx, values)."""
+def dense_to_blocks(w: np.ndarray, keep=None):
+    """Block-compress a dense int8 weight [N][K].  Stores the 4x1 blocks
+    where `keep` [N/4][K] is true (a mask from block_prune; its pruned
+    blocks are dropped whatever they hold), or without a mask every block
+    that holds a nonzero value.  Returns (indptr, colidx, values)."""
     w = _host_array(w, np.int8)
     n_out, k_in = w.shape
     if n_out % BLOCK:
         raise ValueError("N must be a multiple of 4")
     blocks = w.reshape(n_out // BLOCK, BLOCK, k_in)          # [r][i][k]
-    keep = (blocks != 0).any(axis=1)                          # [r][k]
+    if keep is None:
+        keep = (blocks != 0).any(axis=1)                      # [r][k]
+    else:
+        keep = _host_array(keep, np.uint8).astype(bool)
+        if keep.shape != (n_out // BLOCK, k_in):
+            raise ValueError(f"keep must have shape {(n_out // BLOCK, k_in)}")
     r_idx, k_idx = np.nonzero(keep)                           # row-major: sorted by r, then k
     indptr = np.zeros(n_out // BLOCK + 1, np.int32)
     np.cumsum(keep.sum(axis=1), out=indptr[1:])
@@ -222,9 +255,11 @@ class SparseInt8Linear:
         self.info = bsgemm_info(self._h)
 
     @classmethod
-    def from_dense(cls, w, scales, bias=None) -> "SparseInt8Linear":
+    def from_dense(cls, w, scales, bias=None, keep=None) -> "SparseInt8Linear":
+        """From a dense int8 weight [N][K]; `keep` [N/4][K] (e.g. from
+        block_prune) selects the stored blocks."""
         w = _host_array(w, np.int8)
-        indptr, colidx, values = dense_to_blocks(w)
+        indptr, colidx, values = dense_to_blocks(w, keep)
         return cls(w.shape[0], w.shape[1], indptr, colidx, values, scales, bias)
 
     def workspace_bytes(self, m: int) -> int:

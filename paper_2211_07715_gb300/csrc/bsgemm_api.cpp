@@ -559,6 +559,25 @@ int bsgemm_run_host(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epil
     return BSGEMM_OK;
 }
 
+int64_t bsgemm_block_prune(int N, int K, const float* W, double sparsity, uint8_t* keep, void* stream) {
+    clear_error();
+    if (N < 4 || N % 4 != 0 || K < 1) return fail(BSGEMM_ERR_INVALID, "N must be a positive multiple of 4 and K >= 1");
+    if (!W || !keep) return fail(BSGEMM_ERR_INVALID, "W and keep must not be NULL");
+    if (!(sparsity >= 0.0 && sparsity <= 1.0)) return fail(BSGEMM_ERR_INVALID, "sparsity must lie in [0, 1]");
+    const long long total = static_cast<long long>(N / 4) * K;
+    long long npruned = static_cast<long long>(std::floor(sparsity * static_cast<double>(total) + 0.5));
+    if (npruned > total) npruned = total;
+    int dev = -1, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("device query", e));
+    bool bad = false;
+    e = bsg::block_prune(W, N, K, npruned, keep, sms, static_cast<cudaStream_t>(stream), &bad);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("block pruning", e));
+    if (bad) return fail(BSGEMM_ERR_INVALID, "W holds a value that is not finite");
+    return total - npruned;
+}
+
 int bsgemm_device_status(bsgemm_t h, int clear) {
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");

@@ -93,6 +93,11 @@ cudaError_t prepare_kernels(int K, int* ctas_per_sm);  // set attributes, occupa
 cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int grid, cudaStream_t s);
 // x [M][K] -> swizzled token tiles in xb (the layout the kernel stages by TMA).
 cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, cudaStream_t s);
+// Average-magnitude block pruning of a dense fp32 W [N][K] (DEVICE) into
+// keep [N/4][K] (DEVICE): the `npruned` lowest-scoring blocks get 0.  Uses
+// stream-ordered scratch and synchronises `s`; *bad = a weight was not finite.
+cudaError_t block_prune(const float* W, int N, int K, long long npruned, uint8_t* keep, int sms, cudaStream_t s,
+                        bool* bad);
 // Address of the fixed token-tile scratch (BSGEMM_STATIC_SCRATCH_BYTES) on
 // `device`, which must be the current device; looked up on the first call
 // per device, then cached.

@@ -86,3 +86,19 @@ def test_dense_to_blocks(bsg):
             back[4 * r:4 * r + 4, colidx[j]] = values[j]
     assert np.array_equal(back, w)
     assert all((values[j] != 0).any() for j in range(len(colidx)))
+
+
+def test_block_prune_rejects_bad_arguments(bsg):
+    """Shape, pointer and sparsity checks come before any CUDA call."""
+    def code(*args):
+        with pytest.raises(bsg.BsgemmError) as e:
+            bsg.bsgemm_block_prune(*args)
+        return e.value.code
+    assert code(6, 8, 16, 0.5, 16) == bsg.ERR_INVALID      # N % 4
+    assert code(0, 8, 16, 0.5, 16) == bsg.ERR_INVALID      # N = 0
+    assert code(8, 0, 16, 0.5, 16) == bsg.ERR_INVALID      # K = 0
+    assert code(8, 8, 0, 0.5, 16) == bsg.ERR_INVALID       # W NULL
+    assert code(8, 8, 16, 0.5, 0) == bsg.ERR_INVALID       # keep NULL
+    assert code(8, 8, 16, 1.5, 16) == bsg.ERR_INVALID      # sparsity > 1
+    assert code(8, 8, 16, -0.1, 16) == bsg.ERR_INVALID     # sparsity < 0
+    assert code(8, 8, 16, float("nan"), 16) == bsg.ERR_INVALID
