@@ -55,7 +55,7 @@ static_assert(kRing == 8 || kRing == 12 || kRing == 16, "the record ring's switc
 // Cost of a row group's end (epilogue, stores) in steps, for splitting a
 // window's work evenly between warps.
 #ifndef BSG_GROUP_END_COST
-#define BSG_GROUP_END_COST 6
+#define BSG_GROUP_END_COST 14
 #endif
 constexpr int kGroupEndCost = BSG_GROUP_END_COST;
 // Bytes per bulk copy of a token tile into shared memory (a multiple of 16).
