@@ -4,8 +4,10 @@
 Default workload: the DistilBERT FFN2 linear, 3072 -> 768 at 90% block
 sparsity (4x1 blocks), M = 32 x 128 = 4096 tokens, int8 activations uniform
 in [0, 127], bias + requantise to int8 (scale 0.05).  One step = one pass of
-the layer over the whole batch: two kernel launches through the C ABI
-(bsgemm_tile_activations, then bsgemm_run_tiled).
+the layer over the whole batch: one kernel launch through the C ABI
+(bsgemm_run_ws), which stages the activations' token tiles itself by tensor
+copies.  The two-kernel path (relayout kernel + tiled layer kernel) is
+timed beside it for comparison.
 
 Metric: effective INT8 TOPS = 2 * M * nnzb * 4 / t (every stored block's
 MACs, padding excluded) and achieved HBM GB/s = algorithmic bytes / t, where
@@ -16,13 +18,11 @@ Timing: the --steps timed steps are captured once as one CUDA graph and
 replayed between CUDA events on the launching stream, after --warmup
 stream-launched steps and an untimed soak of about a second (so that the
 clock sampler sees the GPU under this load); barrier + synchronize on both
-sides, max over ranks.  The layer kernel's time (the roofline's) is its
-share of a step: the graph's time per step minus that of a graph of the
-same relayouts alone.  A stream-launched loop with events around each
-kernel gives the per-launch times with the stream's launch latency
-("stream_*").  Input/output buffer sets rotate so that the working set of
-consecutive launches exceeds twice the L2 (no launch finds its
-activations in L2).
+sides, max over ranks.  The layer kernel's time (the roofline's) is the
+graph's time per step.  A stream-launched loop gives the per-step time with
+the host's launch cost ("stream_ms_per_step").  Input/output buffer sets
+rotate so that the working set of consecutive launches exceeds twice the L2
+(no launch finds its activations in L2).
 
 --impl reference times the CPU oracle (plain C, the layer's definition) on
 the host cores on row samples of the same workload.
@@ -187,15 +187,12 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     ws_bytes = lin.workspace_bytes(case.m)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
 
-    # One step = the layer over the whole batch through the C ABI's two
-    # kernels: token-tile relayout of the activations, then the sparse layer.
-    def step(i: int, mid=None):
-        bsg.bsgemm_tile_activations(lin._h, xs[i % nsets].data_ptr(), case.m, ws.data_ptr(), ws_bytes,
-                                    stream.cuda_stream)
-        if mid is not None:
-            mid.record(stream)
-        bsg.bsgemm_run_tiled(lin._h, ws.data_ptr(), ws_bytes, case.m, outs[i % nsets].data_ptr(), case.kind,
-                             case.out_scale, stream.cuda_stream)
+    # One step = the layer over the whole batch through the C ABI's fast
+    # call, bsgemm_run_ws: one kernel that stages each token tile of the
+    # activations by tensor copies and computes the layer.
+    def step(i: int, s=None):
+        bsg.bsgemm_run_ws(lin._h, xs[i % nsets].data_ptr(), case.m, outs[i % nsets].data_ptr(), case.kind,
+                          case.out_scale, ws.data_ptr(), ws_bytes, (s or stream).cuda_stream)
 
     def barrier():
         if world > 1:
@@ -203,22 +200,23 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
             dist.barrier()
         torch.cuda.synchronize(dev)
 
-    # The timed region is one CUDA graph of exactly --steps steps (two
-    # launches each, cycling through the input/output sets), so the GPU runs
-    # them back to back without the host's per-launch cost.
+    def graph_of(body, n):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            for i in range(n):
+                body(i, side)
+        torch.cuda.synchronize(dev)
+        return g
+
+    # The timed region is one CUDA graph of exactly --steps steps (cycling
+    # through the input/output sets), so the GPU runs them back to back
+    # without the host's per-launch cost.
     for i in range(max(args.warmup, nsets)):
         step(i)  # warm-up; also computes (and caches) the schedule for this M outside capture
     torch.cuda.synchronize(dev)
     side = torch.cuda.Stream(dev)
     side.wait_stream(stream)
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph, stream=side):
-        for i in range(args.steps):
-            bsg.bsgemm_tile_activations(lin._h, xs[i % nsets].data_ptr(), case.m, ws.data_ptr(), ws_bytes,
-                                        side.cuda_stream)
-            bsg.bsgemm_run_tiled(lin._h, ws.data_ptr(), ws_bytes, case.m, outs[i % nsets].data_ptr(), case.kind,
-                                 case.out_scale, side.cuda_stream)
-    torch.cuda.synchronize(dev)
+    graph = graph_of(step, args.steps)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     graph.replay()
@@ -249,43 +247,43 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     clocks = sampler.summary(mark0, max(mark1, mark0 + 1)) if rank == 0 else {}
     del graph
 
-    # The layer kernel's time in the pipeline: the same --steps relayouts as
-    # one CUDA graph without the layer kernels; the difference per step is
-    # the layer kernel's share of a step (its launch inside the graph
-    # included).  An event pair around a single stream launch would add the
-    # stream's launch latency (several microseconds) to every kernel.
-    graph_r = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph_r, stream=side):
-        for i in range(args.steps):
-            bsg.bsgemm_tile_activations(lin._h, xs[i % nsets].data_ptr(), case.m, ws.data_ptr(), ws_bytes,
-                                        side.cuda_stream)
-    torch.cuda.synchronize(dev)
-    graph_r.replay()
-    barrier()
-    r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    r0.record(stream)
-    graph_r.replay()
-    r1.record(stream)
-    r1.synchronize()
-    relayout_graph_ms = r0.elapsed_time(r1) / args.steps
-    del graph_r
+    # For comparison, the two-kernel path of bsgemm_tile_activations +
+    # bsgemm_run_tiled (relayout kernel, then bulk copies of the relaid
+    # tiles), as a graph of --steps steps.
+    def two_kernel_step(i: int, s=None):
+        st = (s or stream).cuda_stream
+        bsg.bsgemm_tile_activations(lin._h, xs[i % nsets].data_ptr(), case.m, ws.data_ptr(), ws_bytes, st)
+        bsg.bsgemm_run_tiled(lin._h, ws.data_ptr(), ws_bytes, case.m, outs[i % nsets].data_ptr(), case.kind,
+                             case.out_scale, st)
 
-    # The kernels' times launched one by one from the stream, an event
-    # between the relayout and the layer kernel (this loop includes the
-    # host's and the stream's launch cost; its total is reported as
-    # "stream_ms_per_step").
+    def relayout_only(i: int, s=None):
+        bsg.bsgemm_tile_activations(lin._h, xs[i % nsets].data_ptr(), case.m, ws.data_ptr(), ws_bytes,
+                                    (s or stream).cuda_stream)
+
+    def graph_ms(body):
+        g = graph_of(body, args.steps)
+        g.replay()
+        barrier()
+        r0, r1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        r0.record(stream)
+        g.replay()
+        r1.record(stream)
+        r1.synchronize()
+        return r0.elapsed_time(r1) / args.steps
+
+    two_kernel_ms = graph_ms(two_kernel_step)
+    relayout_graph_ms = graph_ms(relayout_only)
+
+    # The same steps launched one by one from the stream (host launch cost
+    # included): "stream_ms_per_step".
     split_steps = min(args.steps, 500)
-    mids = [torch.cuda.Event(enable_timing=True) for _ in range(split_steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(split_steps)]
-    s0 = torch.cuda.Event(enable_timing=True)
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     s0.record(stream)
     for i in range(split_steps):
-        step(i, mids[i])
-        ends[i].record(stream)
-    ends[-1].synchronize()
-    stream_ms = s0.elapsed_time(ends[-1]) / split_steps
-    main_ms = [mids[i].elapsed_time(ends[i]) for i in range(split_steps)]
-    relayout_ms = [(s0 if i == 0 else ends[i - 1]).elapsed_time(mids[i]) for i in range(split_steps)]
+        step(i)
+    s1.record(stream)
+    s1.synchronize()
+    stream_ms = s0.elapsed_time(s1) / split_steps
 
     # end to end through the public call a user makes: a pinned host batch
     # in, the result back in pinned host memory (both copies of every step
@@ -333,9 +331,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     ms_per_step = elapsed_ms / args.steps
     ops = effective_ops(case)
     tops = world * ops / (ms_per_step * 1e-3) / 1e12
-    main_avg_ms = statistics.fmean(main_ms)
-    relayout_avg_ms = statistics.fmean(relayout_ms)
-    kernel_ms = ms_per_step - relayout_graph_ms
+    kernel_ms = ms_per_step  # one kernel per step
     tops_kernel = ops / (kernel_ms * 1e-3) / 1e12
     hbm_gbs = algorithmic_bytes(case) / (ms_per_step * 1e-3) / 1e9
     e2e_tops = world * ops / (e2e_ms / e2e_steps * 1e-3) / 1e12 if e2e_steps > 0 else None
@@ -368,25 +364,24 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
                    "epilogue": synth.KIND_NAMES[case.kind], "out_scale": case.out_scale,
                    "l2": f"rotating {nsets} activation/output sets ({nsets * set_bytes / 2**20:.0f} MiB > 2 x L2)",
                    "parallelism": f"replicas x{world}", "soak_replays": soak,
-                   "launch": "the timed steps are one CUDA graph of --steps steps (relayout + layer kernel each)"},
+                   "launch": "the timed steps are one CUDA graph of --steps steps (one bsgemm_run_ws kernel each)"},
         "stream_ms_per_step": round(stream_ms, 6),
         "hbm_gbs": round(hbm_gbs, 1),
         "hbm_frac": round(hbm_gbs / hbm_peak, 4),
         "roofline": {"bound": "alu", "achieved": round(tops_kernel, 3), "peak": round(peak, 2), "unit": "TOPS",
                      "frac": round(tops_kernel / peak, 4), "traffic": traffic, "kernel": "bsgemm_kernel",
                      "kernel_ms": round(kernel_ms, 6),
-                     "kernel_ms_basis": "graph of --steps (relayout + layer) steps minus graph of --steps relayouts, "
-                                        "per step",
-                     "stream_kernel_ms": round(main_avg_ms, 6),
+                     "kernel_ms_basis": "graph of --steps steps, per step (the step is this one kernel)",
                      "peak_basis": f"{props.multi_processor_count} SMs x {DP4A_LANES_PER_SM_CLK} dp4a lanes/clk x "
                                    f"{OPS_PER_DP4A} ops x {max_mhz:.0f} MHz (max SM clock)"},
         "e2e": {"value": None if e2e_tops is None else round(e2e_tops, 3), "unit": UNIT, "h2d_bytes_per_step": int(case.m * wt.k_in),
                 "d2h_bytes_per_step": int(case.m * wt.n_out * out_elem)},
-        "relayout": {"kernel": "pretile_kernel", "ms": round(relayout_graph_ms, 6),
-                     "ms_basis": "graph of --steps relayouts, per launch", "stream_ms": round(relayout_avg_ms, 6),
-                     "gbs": round(2 * case.m * wt.k_in / (relayout_graph_ms * 1e-3) / 1e9, 1),
-                     "hbm_frac": round(2 * case.m * wt.k_in / (relayout_graph_ms * 1e-3) / 1e9 / hbm_peak, 4)},
-        "gpu_launches": 2 * args.steps,
+        "two_kernel_path": {"ms_per_step": round(two_kernel_ms, 6),
+                            "value": round(ops / (two_kernel_ms * 1e-3) / 1e12, 3),
+                            "relayout_ms": round(relayout_graph_ms, 6),
+                            "basis": "bsgemm_tile_activations + bsgemm_run_tiled (pretile_kernel, then bulk copies of "
+                                     "the relaid tiles), graphs of --steps steps; not the timed path"},
+        "gpu_launches": args.steps,
         "clocks": clocks,
         "kernel_source_sha256": kernel_sha(),
     }
@@ -492,7 +487,7 @@ def _peak_tops(props, max_mhz) -> float:
 
 class _Chain:
     """One encoder layer's four linears on the device, back to back on one
-    stream through the C ABI (relayout + layer kernel each): QKV on the
+    stream through the C ABI (one bsgemm_run_ws kernel each): QKV on the
     layer input, the attention output on a context buffer (the attention
     step itself is outside the timed path), FFN1 + GELU on its result, FFN2
     on FFN1's.  int8 everywhere, frozen calibrated output scales."""
@@ -514,15 +509,12 @@ class _Chain:
                 "f1": t.empty((self.m, 3072), dtype=t.int8, device=dev),
                 "f2": t.empty((self.m, 768), dtype=t.int8, device=dev)}
 
-    def linear(self, i, x, out, stream, ev=None, layer=True):
-        bsg = self.bsg
+    def linear(self, i, x, out, stream, ev=None):
         lin = self.lins[i]
-        bsg.bsgemm_tile_activations(lin._h, x.data_ptr(), self.m, self.ws.data_ptr(), self.ws_bytes, stream)
         if ev is not None:
             ev[0].record()
-        if layer:
-            bsg.bsgemm_run_tiled(lin._h, self.ws.data_ptr(), self.ws_bytes, self.m, out.data_ptr(), self.kinds[i],
-                                 self.scales[i], stream)
+        self.bsg.bsgemm_run_ws(lin._h, x.data_ptr(), self.m, out.data_ptr(), self.kinds[i], self.scales[i],
+                               self.ws.data_ptr(), self.ws_bytes, stream)
         if ev is not None:
             ev[1].record()
 
@@ -565,7 +557,7 @@ def run_layer(args) -> dict:
     for i in range(nsets):
         chain.run(xs[i], ctxs[i], bufs[i], sh)
     torch.cuda.synchronize(dev)
-    # the timed passes are one CUDA graph of exactly --steps passes (8 launches each)
+    # the timed passes are one CUDA graph of exactly --steps passes (4 launches each)
     steps = args.steps
     side = torch.cuda.Stream(dev)
     side.wait_stream(stream)
@@ -590,19 +582,18 @@ def run_layer(args) -> dict:
     sampler.stop()
     clocks = sampler.summary(mark0, max(mark1, mark0 + 1))
     del graph
-    # Per-linear layer-kernel times, each its share of a graph step: a graph
-    # of `reps` (relayout + layer kernel) launches of that linear minus a
-    # graph of its `reps` relayouts alone.
+    # Per-linear layer-kernel times: a graph of `reps` launches of that
+    # linear alone, per launch.
     reps = min(steps, 200)
     inputs = [lambda i: xs[i % nsets], lambda i: ctxs[i % nsets], lambda i: bufs[i % nsets]["o"],
               lambda i: bufs[i % nsets]["f1"]]
     outputs = ["qkv", "o", "f1", "f2"]
 
-    def graph_ms(j, layer):
+    def graph_ms(j):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=side):
             for i in range(reps):
-                chain.linear(j, inputs[j](i), bufs[i % nsets][outputs[j]], side.cuda_stream, layer=layer)
+                chain.linear(j, inputs[j](i), bufs[i % nsets][outputs[j]], side.cuda_stream)
         torch.cuda.synchronize(dev)
         g.replay()
         torch.cuda.synchronize(dev)
@@ -614,7 +605,7 @@ def run_layer(args) -> dict:
         del g
         return e0.elapsed_time(e1) / reps
 
-    graph_kern_ms = [graph_ms(j, True) - graph_ms(j, False) for j in range(4)]
+    graph_kern_ms = [graph_ms(j) for j in range(4)]
     # per-linear stream-launched times: the passes launched one by one with events around each kernel
     split = min(steps, 200)
     evs = [[[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(4)] for _ in range(split)]
@@ -651,16 +642,16 @@ def run_layer(args) -> dict:
                      "frac": round(kernel_tops / peak, 4), "traffic": None, "kernel": "bsgemm_kernel (4 linears)",
                      "kernel_ms": round(sum(graph_kern_ms), 6)},
         "per_linear": per,
-        "per_linear_basis": "kernel_ms: graph of 200 (relayout + layer) launches of the linear minus graph of its "
-                            "200 relayouts, per launch; stream_kernel_ms: events around stream launches",
-        "gpu_launches": 8 * steps, "clocks": clocks, "kernel_source_sha256": kernel_sha(),
+        "per_linear_basis": "kernel_ms: graph of 200 launches of the linear, per launch; stream_kernel_ms: events "
+                            "around stream launches",
+        "gpu_launches": 4 * steps, "clocks": clocks, "kernel_source_sha256": kernel_sha(),
     }
 
 
 def run_stack(args) -> dict:
     """cfg 5: the six-layer stack of 24 sparse linears swept over batch
     {1, 8, 32, 128} x seq {128, 384} x sparsity {70, 80, 90}%.  One pass =
-    24 linears (48 launches) back to back on one stream, the attention step
+    24 linears (24 launches) back to back on one stream, the attention step
     replaced by a seeded int8 context buffer; also replayed as one CUDA
     graph.  Tokens/s = M / pass time."""
     import torch
@@ -751,7 +742,7 @@ def run_stack(args) -> dict:
         "config": {"workload": "six-layer stack of 24 sparse INT8 linears (QKV, attention output, FFN1 + GELU, FFN2 "
                                "per layer); value = the batch 8 x seq 384, 80% point; attention replaced in the "
                                "timed path by a seeded int8 context buffer", "points": len(points)},
-        "points": points, "gpu_launches": 48 * reps * len(points) * 2, "clocks": clocks,
+        "points": points, "gpu_launches": 24 * reps * len(points) * 2, "clocks": clocks,
         "kernel_source_sha256": kernel_sha(),
     }
 

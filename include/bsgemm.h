@@ -101,7 +101,10 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
  *   stream  a cudaStream_t (NULL = the legacy default stream).
  * Asynchronous: returns after enqueueing one kernel launch; allocates
  * nothing, does not synchronise and keeps no reference to act or out.  The
- * current device must be the one the handle was created on.
+ * current device must be the one the handle was created on.  When K is a
+ * multiple of 16 and act is 16-byte aligned (the fast path) the kernel
+ * brings each 64-token tile of act into shared memory by tensor copies and
+ * transposes it there; otherwise it gathers the tile with per-thread loads.
  * Returns BSGEMM_OK, BSGEMM_ERR_INVALID (NULL handle or pointers, M < 0,
  * bad kind, bad out_scale, misaligned out, wrong device) or
  * BSGEMM_ERR_CUDA (launch failure).
@@ -118,11 +121,12 @@ size_t bsgemm_workspace_bytes(bsgemm_t h, int M);
 
 /*
  * bsgemm_run_ws -- bsgemm_run with a caller-owned DEVICE workspace of at
- * least bsgemm_workspace_bytes(h, M) bytes, 16-byte aligned.  Enqueues two
- * kernels on `stream`: one rewrites act as token tiles into the workspace,
- * the second streams each tile into shared memory with one bulk (TMA) copy
- * and computes the layer.  This is the fast path; bsgemm_run (no
- * workspace) gathers the activations with per-thread loads instead.  The
+ * least bsgemm_workspace_bytes(h, M) bytes, 16-byte aligned.  On bsgemm_run's
+ * fast path (K % 16 == 0, act 16-byte aligned) it is that one kernel and the
+ * workspace is not touched.  Otherwise it enqueues two kernels on `stream`:
+ * one rewrites act as token tiles into the workspace, the second streams
+ * each tile into shared memory with one bulk (TMA) copy and computes the
+ * layer (faster than bsgemm_run's per-thread gather for those shapes).  The
  * workspace is scratch: its contents are undefined afterwards, and two runs
  * in flight at the same time need two workspaces.  Same results, return
  * codes and asynchrony as bsgemm_run; a workspace that is NULL, too small or
@@ -172,7 +176,7 @@ int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, v
 
 /*
  * bsgemm_run_host -- the end-to-end call on HOST buffers: copy act in, run
- * the layer (bsgemm_run_ws's two kernels), copy the result out, all
+ * the layer (as bsgemm_run_ws does), copy the result out, all
  * enqueued on `stream`.  The paper's engine (Sec. 3) runs on the CPU and
  * takes and returns tensors in host memory; this is that call on the GPU,
  * with the transfers over the host link inside it.
@@ -187,7 +191,7 @@ int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, v
  *              tiles and the device result, each at a 256-byte aligned
  *              offset.  Scratch as for bsgemm_run_ws: two calls in flight
  *              at the same time need two workspaces.
- * Returns after enqueueing (two copies, two kernels); `out` holds the
+ * Returns after enqueueing (two copies, one or two kernels); `out` holds the
  * result once `stream` has completed, and `act` must not change before
  * then.  Return codes as bsgemm_run_ws, plus BSGEMM_ERR_CUDA if a copy
  * cannot be enqueued.

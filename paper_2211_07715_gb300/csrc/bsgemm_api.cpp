@@ -409,9 +409,14 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
                                             std::to_string(h->device));
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
 
+    // With K a multiple of 16 and act 16-byte aligned the layer kernel stages
+    // its tiles from act itself (tensor copies); the relayout kernel and the
+    // workspace serve the other shapes and bsgemm_run_tiled.
+    const bool tensor = mode != 2 && bsg::tensor_staging(h->w.K, act);
     bsg::LaunchArgs a{};
     a.x = act;
-    a.xb = use_ws ? static_cast<const int8_t*>(workspace) : nullptr;
+    a.xb = use_ws && !tensor ? static_cast<const int8_t*>(workspace) : nullptr;
+    a.tensor = tensor;
     a.out = out;
     a.M = M;
     a.kind = epi.kind;
@@ -432,7 +437,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
         grid = h->sched_grid;
         std::memcpy(sched.u, h->sched.u, sizeof(long long) * (grid + 1));
     }
-    if (mode == 1) {
+    if (mode == 1 && !tensor) {
         e = bsg::launch_pretile(act, M, h->w.K, static_cast<int8_t*>(workspace), h->num_sms, s);
         if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("relayout launch", e));
     }

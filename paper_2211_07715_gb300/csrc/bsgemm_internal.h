@@ -64,6 +64,7 @@ struct LaunchArgs {
     int kind;
     float inv_out_scale;
     bool x_vec16;          // x 16-byte aligned and K % 16 == 0
+    bool tensor;           // stage tiles from x by tensor copies (xb unused; needs tensor_staging())
 };
 
 // Kernel configuration: 8 warps per CTA (2 per SM sub-partition, up to 255
@@ -75,7 +76,8 @@ constexpr int kThreads = kWarps * 32;
 #endif
 constexpr int kRing = BSG_RING;     // step records a warp keeps in flight (registers), 8..16
 constexpr int kStepPad = kRing;     // zero step records after the last one (the record prefetch runs ahead)
-constexpr int kGroupWin = 512;      // row groups whose step offsets a CTA keeps in shared memory
+constexpr int kGroupWin = 448;      // row groups whose step offsets a CTA keeps in shared memory
+constexpr int kMaxBoxes = 49;       // 64-column boxes of a token tile (K <= 3136)
 constexpr int kStaticSmem = 2304;   // bytes of static shared memory the kernel may use
 constexpr int kMaxGrid = 512;       // CTAs per launch at most
 
@@ -88,6 +90,9 @@ struct Schedule {
 
 size_t tiled_bytes(int K, long long M);    // bytes of the token-tile copy of x
 size_t smem_bytes(int K);                  // dynamic shared memory per CTA
+// Whether the layer kernel can stage x [M][K] itself by tensor copies (K a
+// multiple of 16, x 16-byte aligned, the driver's tensor-map encoder found).
+bool tensor_staging(int K, const void* x);
 int max_k();                               // largest K a tile supports
 cudaError_t prepare_kernels(int K, int* ctas_per_sm);  // set attributes, occupancy
 cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int grid, cudaStream_t s);

@@ -40,7 +40,10 @@
 //   and bias, optional GELU by a fixed fp32 op sequence (A&S 7.1.28 erf),
 //   optional requantise (fp32 multiply, round half to even, saturate).
 #include <cstdint>
+#include <cstring>
 #include <mutex>
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include "bsgemm.h"
@@ -321,6 +324,15 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, unsigned
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
                  ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
+// One 2-D box of a tensor map (x = innermost coordinate, y = row) into
+// shared memory, completing on an mbarrier.
+__device__ __forceinline__ void tensor_g2s(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n"
+                 ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar) : "memory");
+}
+__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
+    asm volatile("st.shared.u32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
+}
 // Programmatic dependent launch: both kernels are launched so that they may
 // start while the previous kernel of the stream finishes.  Before a kernel
 // reads its activations or writes any global memory, every thread waits
@@ -332,6 +344,48 @@ __device__ __forceinline__ void griddep_launch_dependents() { asm volatile("grid
 // Order this thread's earlier generic-proxy shared-memory accesses before
 // later asynchronous-proxy (bulk copy) writes.
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
+
+// Staging from the activations themselves (no relayout kernel): a tensor
+// copy brings box b of the token tile -- 64 tokens x columns 64b..64b+63,
+// row-major, 64 bytes a token -- into the tile's bytes [4096 b, 4096 b +
+// 4096), with the 64-byte swizzle: token r's 16-byte chunk c at 64 r + 16
+// (c ^ ((r >> 1) & 3)).  Those are the bytes the box's columns take in the
+// swizzled k-major tile, so one warp turns the box around in place: eight
+// transposed matrix loads (16 tokens x 16 columns each; lane l addresses
+// token row l of the two matrices) put the whole box in registers, and 32
+// word stores write lane (g, q)'s words -- 4 tokens of one column -- to
+// their column rows.  Both the loads (8 tokens of a phase on 8 distinct
+// 16-byte slots) and the stores (8 columns x 4 words on 32 banks) are free
+// of bank conflicts.
+__device__ __forceinline__ void transpose_box(uint32_t tb, int b, int lane) {
+    const uint32_t box = tb + 4096u * static_cast<uint32_t>(b);
+    uint32_t v[8][4];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const uint32_t r = 32u * h + static_cast<uint32_t>(lane);
+            ldsm_x2_trans_b8(box + 64u * r + 16u * (static_cast<uint32_t>(c) ^ ((r >> 1) & 3u)), v[4 * h + c][0],
+                             v[4 * h + c][1], v[4 * h + c][2], v[4 * h + c][3]);
+        }
+    }
+    __syncwarp();
+    const int g = lane >> 2;
+    const uint32_t wq4 = 4u * static_cast<uint32_t>(lane & 3);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int k = 64 * b + 16 * c + g;
+            const uint32_t o0 = row_off(k), o1 = row_off(k + 8);
+            const uint32_t j0 = 32u * h, j1 = 32u * h + 16u;  // chunks 2h, 2h + 1 (16 tokens each)
+            st_shared_u32(tb + (o0 ^ j0) + wq4, v[4 * h + c][0]);
+            st_shared_u32(tb + (o1 ^ j0) + wq4, v[4 * h + c][1]);
+            st_shared_u32(tb + (o0 ^ j1) + wq4, v[4 * h + c][2]);
+            st_shared_u32(tb + (o1 ^ j1) + wq4, v[4 * h + c][3]);
+        }
+    }
+}
 
 // One step for one lane: the step's 16 columns x the tile's 64 tokens come
 // in by two transposed gathers (tokens 0-31, then 32-63); lane l (g = l / 4,
@@ -388,21 +442,30 @@ __device__ __forceinline__ void store_lane(const LaunchArgs& a, int N, long long
     for (int i = 0; i < 8; ++i) store_token<KIND>(a, N, m_g + 8 * i, r, acc + 4 * i, sc, bi);
 }
 
-template <int KIND, bool TMA>
+// MODE: how a window's token tile reaches shared memory.
+constexpr int kStageGather = 0;  // per-thread loads from x [M][K], transposed in registers
+constexpr int kStageTiles = 1;   // one bulk copy of a tile the relayout kernel wrote
+constexpr int kStageTensor = 2;  // tensor copies of x's boxes, transposed in place (transpose_box)
+
+template <int KIND, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
-bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sched) {
+bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sched,
+              const __grid_constant__ CUtensorMap xmap) {
+    constexpr bool TMA = MODE == kStageTiles;
+    constexpr bool TENSOR = MODE == kStageTensor;
     constexpr int SW = kTile * 16;  // slot words: 64 tokens x 4 block-rows x 4 channels
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ int s_gp[kGroupWin + 1];                // step offsets of the current group window
-    __shared__ __align__(8) unsigned long long s_bar;  // completion of the token tile's bulk copy
-    __shared__ int s_wst[kWarps + 1];                  // first step of each warp in the window (relative)
+    __shared__ int s_gp[kGroupWin + 1];                          // step offsets of the current group window
+    __shared__ __align__(8) unsigned long long s_bar[kMaxBoxes];  // completion of the tile's copies
+    __shared__ int s_wst[kWarps + 1];                            // first step of each warp in the window (relative)
 
     const int K = w.K, N = w.N;
     const int kpad = (K + 15) & ~15;
+    const int nbox = (K + 63) >> 6;  // 64-column boxes of a tile
     const uint32_t sbase = smem_addr(smem);
-    const uint32_t tb = (sbase + 127u) & ~127u;  // the token tile, 128-byte aligned
+    const uint32_t tb = (sbase + 511u) & ~511u;  // the token tile, 512-byte aligned (the boxes' swizzle)
     unsigned char* tile = smem + (tb - sbase);
-    int* slots = reinterpret_cast<int*>(tile + static_cast<size_t>(kpad) * kTile);
+    int* slots = reinterpret_cast<int*>(tile + static_cast<size_t>(nbox) * 64 * kTile);
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int q = lane & 3, g = lane >> 2;  // block-row q of each group; tokens g + 8 i
@@ -410,8 +473,11 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     const long long ng = w.ngroups;
 
     griddep_launch_dependents();
-    const uint32_t bar = smem_addr(&s_bar);
+    const uint32_t bar = smem_addr(&s_bar[0]);  // box b's barrier at bar + 8 b (TMA: box 0 only)
     if (TMA && tid == 0) mbar_init(bar, 1);
+    if (TENSOR && tid < nbox) mbar_init(bar + 8u * tid, 1);
+    // this warp's boxes: [bx0, bx1)
+    const int bx0 = warp * nbox / kWarps, bx1 = (warp + 1) * nbox / kWarps;
     // slots start at zero; whoever finishes a slot resets it
     for (int i = tid; i < kSlots * SW / 4; i += kThreads) reinterpret_cast<int4*>(slots)[i] = make_int4(0, 0, 0, 0);
     __syncthreads();
@@ -435,6 +501,12 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         // the token tile (already swizzled in a.xb) in kTmaPiece-byte bulk
         // copies, issued by the lanes of warp 0 (one completion barrier)
         auto copy_tile = [&]() {
+            if (TENSOR && stage && lane < bx1 - bx0) {  // lane i of each warp: the warp's box bx0 + i
+                const int b = bx0 + lane;
+                fence_proxy_async();
+                mbar_arrive_expect_tx(bar + 8u * b, 64u * kTile);
+                tensor_g2s(tb + 4096u * b, &xmap, 64 * b, static_cast<int>(t * kTile), bar + 8u * b);
+            }
             if (TMA && stage && warp == 0) {
                 const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
                 const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * kTile;
@@ -516,7 +588,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             waited = true;
             copy_tile();
         }
-        if (!TMA && stage) {  // gather the tile with per-thread loads
+        if (MODE == kStageGather && stage) {  // gather the tile with per-thread loads
             stage_tile(tile, a, K, kpad, m0);
             __syncthreads();
             staged = t;
@@ -534,6 +606,24 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             }
         }
 
+        if (TENSOR && stage) {
+            // the warp turns its boxes around as they land
+            bool ok = true;
+            for (int b = bx0; b < bx1 && ok; ++b) {
+                ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * b, phase & 1u));
+                if (ok) transpose_box(tb, b, lane);
+            }
+            ++phase;
+            if (__syncthreads_or(!ok)) {
+                if (tid == 0) {
+                    atomicOr(w.status, kStatusTimeout);
+                    for (int b = 0; b < nbox; ++b) mbar_wait(bar + 8u * b, (phase - 1) & 1u);  // one more chance
+                }
+                __syncthreads();
+                return;
+            }
+            staged = t;
+        }
         if (TMA && stage) {
             const bool ok = mbar_wait(bar, phase & 1u);
             ++phase;
@@ -732,23 +822,48 @@ pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __r
     }
 }
 
-template <bool TMA>
+template <int MODE>
 const void* kernel_for(int kind) {
     switch (kind) {
-    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<0, TMA>);
-    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<1, TMA>);
-    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<2, TMA>);
-    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<3, TMA>);
-    default: return reinterpret_cast<const void*>(&bsgemm_kernel<4, TMA>);
+    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<0, MODE>);
+    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<1, MODE>);
+    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<2, MODE>);
+    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<3, MODE>);
+    default: return reinterpret_cast<const void*>(&bsgemm_kernel<4, MODE>);
     }
+}
+const void* kernel_for(int kind, int mode) {
+    return mode == kStageTensor ? kernel_for<kStageTensor>(kind)
+                                : mode == kStageTiles ? kernel_for<kStageTiles>(kind) : kernel_for<kStageGather>(kind);
+}
+
+// cuTensorMapEncodeTiled from the driver, looked up once.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
 }
 
 }  // namespace
 
+bool tensor_staging(int K, const void* x) {
+    return K % 16 == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0 && (K + 63) / 64 <= kMaxBoxes &&
+           tensor_map_encoder() != nullptr;
+}
+
 size_t smem_bytes(int K) {
-    const size_t kpad = (static_cast<size_t>(K) + 15) & ~static_cast<size_t>(15);
-    // 128 bytes of slack to align the tile, the tile, the split-group slots
-    return 128 + kpad * kTile + static_cast<size_t>(kSlots) * kTile * 16 * sizeof(int);
+    const size_t tpad = (static_cast<size_t>(K) + 63) & ~static_cast<size_t>(63);
+    // 512 bytes of slack to align the tile, the tile (whole 64-column boxes),
+    // the split-group slots
+    return 512 + tpad * kTile + static_cast<size_t>(kSlots) * kTile * 16 * sizeof(int);
 }
 
 int max_k() {
@@ -760,13 +875,13 @@ int max_k() {
 cudaError_t prepare_kernels(int K, int* ctas_per_sm) {
     const int smem = static_cast<int>(smem_bytes(K));
     for (int kind = 0; kind < 5; ++kind) {
-        for (int tma = 0; tma < 2; ++tma) {
-            cudaError_t e = cudaFuncSetAttribute(tma ? kernel_for<true>(kind) : kernel_for<false>(kind),
-                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemOptin - kStaticSmem);
+        for (int mode = 0; mode < 3; ++mode) {
+            cudaError_t e = cudaFuncSetAttribute(kernel_for(kind, mode), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 kSmemOptin - kStaticSmem);
             if (e != cudaSuccess) return e;
         }
     }
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_for<true>(0), kThreads, smem);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_for(0, kStageTensor), kThreads, smem);
 }
 
 cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int grid, cudaStream_t s) {
@@ -781,11 +896,31 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    // a.tensor: a tensor map over x [M][K] (int8, 64 x 64 boxes, 64-byte
+    // swizzle, zeros outside M x K); otherwise an unused all-zero map
+    CUtensorMap xmap;
+    std::memset(&xmap, 0, sizeof(xmap));
+    if (a.tensor) {
+        PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
+        if (!encode || (w.K + 63) / 64 > kMaxBoxes) return cudaErrorNotSupported;
+        const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(w.K), static_cast<cuuint64_t>(a.M)};
+        const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(w.K)};
+        const cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(kTile)};
+        const cuuint32_t estride[2] = {1u, 1u};
+        if (encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t*>(a.x), gdim, gstride, box, estride,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
     cudaError_t e = cudaSuccess;
 #define BSG_LAUNCH(KV)                                                                                   \
     do {                                                                                                 \
-        e = a.xb ? cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, true>, w, a, sched)                        \
-                 : cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, false>, w, a, sched);                      \
+        if (a.tensor)                                                                                    \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTensor>, w, a, sched, xmap);            \
+        else if (a.xb)                                                                                   \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTiles>, w, a, sched, xmap);             \
+        else                                                                                             \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageGather>, w, a, sched, xmap);            \
     } while (0)
     switch (a.kind) {
     case 0: BSG_LAUNCH(0); break;

@@ -351,6 +351,33 @@ def test_run_host_through_the_c_abi(bsg):
         bsg.bsgemm_run_host(lin._h, 0, 77, 0, synth.I8, 1.0, ws.data_ptr(), need, 0)
 
 
+@pytest.mark.parametrize("k", [768, 1001, 3072])
+def test_relayout_then_tiled_kernel(bsg, k):
+    """The two-kernel path: the relayout kernel writes the token tiles
+    (bsgemm_tile_activations) and the layer kernel copies them in
+    (bsgemm_run_tiled); the fast call stages tiles from x itself instead."""
+    import torch
+    rng = synth.rng_for(5900 + k)
+    wt = synth.draw_weight(rng, 96, k, 0.85)
+    w = oracle.weight_dense(wt)
+    lin = make_linear(bsg, wt)
+    m = 150
+    x = synth.draw_x(rng, m, k, "u127")
+    xd = torch.from_numpy(x).cuda()
+    need = lin.workspace_bytes(m)
+    ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+    for kind in KINDS:
+        dt = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+              synth.I8: torch.int8, synth.I8_GELU: torch.int8}[kind]
+        out = torch.empty((m, 96), dtype=dt, device="cuda")
+        torch.cuda.synchronize()
+        bsg.bsgemm_tile_activations(lin._h, xd.data_ptr(), m, ws.data_ptr(), need, 0)
+        bsg.bsgemm_run_tiled(lin._h, ws.data_ptr(), need, m, out.data_ptr(), kind, 0.05, 0)
+        torch.cuda.synchronize()
+        check(out.cpu().numpy(), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05), kind)
+    assert bsg.bsgemm_device_status(lin._h) == 0
+
+
 def test_from_dense(bsg):
     rng = synth.rng_for(5800)
     wt = synth.draw_weight(rng, 128, 768, 0.8)
