@@ -274,6 +274,22 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     two_kernel_ms = graph_ms(two_kernel_step)
     relayout_graph_ms = graph_ms(relayout_only)
 
+    # Also for comparison: the same batches held K-major (X^T [K][M], the
+    # input layout of Algorithm 1) through bsgemm_run_kmajor, whose tensor
+    # copies land the tiles in place with no transpose.
+    kmajor_ms = None
+    if case.m % 16 == 0:
+        xts = [x.t().contiguous() for x in xs]
+
+        def kmajor_step(i: int, s=None):
+            bsg.bsgemm_run_kmajor(lin._h, xts[i % nsets].data_ptr(), case.m, case.m, outs[i % nsets].data_ptr(),
+                                  case.kind, case.out_scale, (s or stream).cuda_stream)
+
+        for i in range(3):
+            kmajor_step(i)
+        kmajor_ms = graph_ms(kmajor_step)
+        del xts
+
     # The same steps launched one by one from the stream (host launch cost
     # included): "stream_ms_per_step".
     split_steps = min(args.steps, 500)
@@ -381,6 +397,10 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
                             "relayout_ms": round(relayout_graph_ms, 6),
                             "basis": "bsgemm_tile_activations + bsgemm_run_tiled (pretile_kernel, then bulk copies of "
                                      "the relaid tiles), graphs of --steps steps; not the timed path"},
+        "kmajor_path": None if kmajor_ms is None else {
+            "ms_per_step": round(kmajor_ms, 6), "value": round(ops / (kmajor_ms * 1e-3) / 1e12, 3),
+            "basis": "bsgemm_run_kmajor on the same batches stored K-major (X^T [K][M]), graph of --steps steps; "
+                     "not the timed path"},
         "gpu_launches": args.steps,
         "clocks": clocks,
         "kernel_source_sha256": kernel_sha(),

@@ -160,6 +160,20 @@ int bsgemm_run_ws(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilog
 int bsgemm_run_static(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream);
 
 /*
+ * bsgemm_run_kmajor -- bsgemm_run on activations stored K-major: act_t is
+ * X^T, int8 [K][M] with row stride ld bytes (row k = input feature k of the
+ * M tokens, tokens contiguous), the input layout of Algorithm 1, whose
+ * inner loop reads a k-block of input rows that each hold n-block
+ * consecutive tokens.  Each 64-token tile then comes into shared memory by
+ * tensor copies that land it directly in the kernel's layout: no transpose
+ * and no relayout, one kernel, no scratch.
+ *   act_t  DEVICE, 16-byte aligned; ld >= M and ld % 16 == 0.
+ *   out    DEVICE [M][N] row-major as for bsgemm_run.
+ * Results, asynchrony and the other return codes are bsgemm_run's.
+ */
+int bsgemm_run_kmajor(bsgemm_t h, const int8_t* act_t, int M, int ld, void* out, bsgemm_epilogue epi, void* stream);
+
+/*
  * The two steps of bsgemm_run_ws, for callers that keep activations in the
  * token-tiled layout between layers or time the steps apart:
  *   bsgemm_tile_activations -- act [M][K] (DEVICE) -> token tiles in

@@ -66,6 +66,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_run_static.restype = ctypes.c_int
     lib.bsgemm_tile_activations.argtypes = [vp, vp, ctypes.c_int, vp, ctypes.c_size_t, vp]
     lib.bsgemm_tile_activations.restype = ctypes.c_int
+    lib.bsgemm_run_kmajor.argtypes = [vp, vp, ctypes.c_int, ctypes.c_int, vp, Epilogue, vp]
+    lib.bsgemm_run_kmajor.restype = ctypes.c_int
     lib.bsgemm_run_tiled.argtypes = [vp, vp, ctypes.c_size_t, ctypes.c_int, vp, Epilogue, vp]
     lib.bsgemm_run_tiled.restype = ctypes.c_int
     lib.bsgemm_host_workspace_bytes.argtypes = [vp, ctypes.c_int, ctypes.c_int32]
@@ -82,9 +84,9 @@ def _load() -> ctypes.CDLL:
 _lib = _load()
 
 EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
-            "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_host_workspace_bytes", "bsgemm_run_host",
-            "bsgemm_block_prune", "bsgemm_destroy", "bsgemm_last_error", "bsgemm_last_status",
-            "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
+            "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_run_kmajor",
+            "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_destroy",
+            "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
 
 
 def bsgemm_last_error() -> str:
@@ -140,6 +142,14 @@ def bsgemm_run_static(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out
     """The fast path with the library's fixed device scratch: allocates
     nothing; calls overlapping in time on one device race (see the header)."""
     rc = _lib.bsgemm_run_static(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def bsgemm_run_kmajor(h: int, act_t_ptr: int, m: int, ld: int, out_ptr: int, kind: int, out_scale: float = 1.0,
+                      stream: int = 0) -> None:
+    """The layer on K-major activations X^T [K][M] (row stride ld bytes)."""
+    rc = _lib.bsgemm_run_kmajor(h, act_t_ptr, int(m), int(ld), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 
@@ -291,6 +301,21 @@ class SparseInt8Linear:
             raise ValueError(f"workspace must hold {need} bytes")
         bsgemm_run_ws(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, workspace.data_ptr(),
                       workspace.numel() * workspace.element_size(), s.cuda_stream)
+
+    def run_kmajor(self, xt, out, kind: int, out_scale: float = 1.0, stream=None) -> None:
+        """out[M][N] = epilogue(X W^T) from K-major activations: xt is a CUDA
+        int8 tensor [K][M] whose rows are 16-byte aligned (row stride a
+        multiple of 16 bytes, M <= stride); out a contiguous CUDA [M][N]."""
+        import torch
+        if (xt.dtype != torch.int8 or not xt.is_cuda or xt.dim() != 2 or xt.shape[0] != self.k_in
+                or xt.stride(1) != 1):
+            raise ValueError("xt must be a CUDA int8 tensor [K][M] with unit column stride")
+        m = xt.shape[1]
+        if (not out.is_cuda or not out.is_contiguous() or tuple(out.shape) != (m, self.n_out)
+                or str(out.dtype).split(".")[-1] != _OUT_DTYPES[kind]):
+            raise ValueError(f"out must be a contiguous CUDA {_OUT_DTYPES[kind]} tensor [M][N]")
+        s = torch.cuda.current_stream() if stream is None else stream
+        bsgemm_run_kmajor(self._h, xt.data_ptr(), m, xt.stride(0), out.data_ptr(), kind, out_scale, s.cuda_stream)
 
     def __call__(self, x, kind: int, out_scale: float = 1.0, stream=None, out=None, sync: bool = True):
         """Allocate the output (unless `out` is given) and run.

@@ -374,10 +374,12 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
 }
 
 // mode: 0 = gather from act (no scratch), 1 = relayout act into workspace
-// then stage tiles, 2 = stage tiles already in workspace (act unused).
+// then stage tiles, 2 = stage tiles already in workspace (act unused),
+// 3 = act is x^T [K][M] with row stride ld (no scratch).  Modes 0 and 1
+// stage from act by tensor copies instead when tensor_staging() allows.
 static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* workspace,
-                      size_t workspace_bytes, int mode, void* stream) {
-    const bool use_ws = mode != 0;
+                      size_t workspace_bytes, int mode, void* stream, int ld = 0) {
+    const bool use_ws = mode == 1 || mode == 2;
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
     if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
@@ -389,6 +391,10 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
             return fail(BSGEMM_ERR_INVALID, "out_scale must be finite and > 0 for int8 outputs");
         inv = 1.0f / epi.out_scale;
         if (!std::isfinite(inv)) return fail(BSGEMM_ERR_INVALID, "1 / out_scale overflows fp32");
+    }
+    if (mode == 3 && M > 0) {
+        if (ld < M || ld % 16 != 0) return fail(BSGEMM_ERR_INVALID, "ld must be >= M and a multiple of 16");
+        if (reinterpret_cast<uintptr_t>(act) % 16 != 0) return fail(BSGEMM_ERR_INVALID, "act must be 16-byte aligned");
     }
     if (M == 0) return BSGEMM_OK;
     if ((mode != 2 && !act) || !out) return fail(BSGEMM_ERR_INVALID, "act and out must not be NULL");
@@ -412,11 +418,13 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     // With K a multiple of 16 and act 16-byte aligned the layer kernel stages
     // its tiles from act itself (tensor copies); the relayout kernel and the
     // workspace serve the other shapes and bsgemm_run_tiled.
-    const bool tensor = mode != 2 && bsg::tensor_staging(h->w.K, act);
+    const bool tensor = (mode == 0 || mode == 1) && bsg::tensor_staging(h->w.K, act);
     bsg::LaunchArgs a{};
     a.x = act;
     a.xb = use_ws && !tensor ? static_cast<const int8_t*>(workspace) : nullptr;
     a.tensor = tensor;
+    a.kmajor = mode == 3;
+    a.ld = ld;
     a.out = out;
     a.M = M;
     a.kind = epi.kind;
@@ -453,6 +461,10 @@ int bsgemm_run(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue 
 int bsgemm_run_ws(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* workspace,
                   size_t workspace_bytes, void* stream) {
     return run_common(h, act, M, out, epi, workspace, workspace_bytes, 1, stream);
+}
+
+int bsgemm_run_kmajor(bsgemm_t h, const int8_t* act_t, int M, int ld, void* out, bsgemm_epilogue epi, void* stream) {
+    return run_common(h, act_t, M, out, epi, nullptr, 0, 3, stream, ld);
 }
 
 int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, void* out, bsgemm_epilogue epi,

@@ -14,14 +14,16 @@ constexpr int kTile = 64;
 // Shared-memory layout of one token tile ("swizzled k-major").  Column k of
 // the activations is a row of 64 bytes (the tile's 64 tokens), cut into 4
 // chunks of 16 tokens.  Rows 2i and 2i+1 share the 128-byte line i; chunk c
-// of row k sits in 16-byte slot ((4 (k & 1) + c) XOR (i & 7)) of its line.
+// of row k sits in 16-byte slot ((4 (k & 1) + c) XOR (i & 3)) of its line.
 // Row k's chunk 0 is therefore at byte tile_row_offset(k), and chunk c at
 // tile_row_offset(k) XOR 16 c.  The XOR spreads the chunks of different rows
 // over the 8 bank groups of shared memory, so a gather of 8 rows whose
-// "bank keys" (slot of chunk 0) differ reads in one pass.
+// "bank keys" (slot of chunk 0) differ reads in one pass.  It is also the
+// 64-byte swizzle of the tensor copies: a box of 64-byte rows k lands in
+// exactly this layout (row k at 64 k, chunk c at slot c XOR ((k >> 1) & 3)).
 inline uint32_t tile_row_offset(int k) {
     const uint32_t line = static_cast<uint32_t>(k) >> 1;
-    const uint32_t slot = ((static_cast<uint32_t>(k) & 1u) << 2) ^ (line & 7u);
+    const uint32_t slot = ((static_cast<uint32_t>(k) & 1u) << 2) ^ (line & 3u);
     return (line << 7) | (slot << 4);
 }
 inline int bank_key(int k) { return static_cast<int>((tile_row_offset(k) >> 4) & 7u); }
@@ -65,6 +67,8 @@ struct LaunchArgs {
     float inv_out_scale;
     bool x_vec16;          // x 16-byte aligned and K % 16 == 0
     bool tensor;           // stage tiles from x by tensor copies (xb unused; needs tensor_staging())
+    bool kmajor;           // x is x^T [K][M] with row stride ld: tensor copies, no transpose
+    int ld;                // row stride of x^T in bytes (kmajor only)
 };
 
 // Kernel configuration: 8 warps per CTA (2 per SM sub-partition, up to 255

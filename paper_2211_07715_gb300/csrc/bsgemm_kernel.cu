@@ -204,10 +204,10 @@ __device__ __forceinline__ int row_of(const int* sp, int lo, int hi, int q) {
 
 // Byte offset of chunk 0 of activation column k in a swizzled token tile
 // (rows 2i, 2i+1 share 128-byte line i; chunk c of row k in 16-byte slot
-// (4 (k & 1) + c) XOR (i & 7)); chunk c is at row_off(k) XOR 16 c.
+// (4 (k & 1) + c) XOR (i & 3)); chunk c is at row_off(k) XOR 16 c.
 __device__ __forceinline__ uint32_t row_off(int k) {
     const uint32_t line = static_cast<uint32_t>(k) >> 1;
-    return (line << 7) | ((((static_cast<uint32_t>(k) & 1u) << 2) ^ (line & 7u)) << 4);
+    return (line << 7) | ((((static_cast<uint32_t>(k) & 1u) << 2) ^ (line & 3u)) << 4);
 }
 
 // One staging unit: tokens 4g..4g+3 of the tile x columns 16kc..16kc+15.
@@ -446,13 +446,15 @@ __device__ __forceinline__ void store_lane(const LaunchArgs& a, int N, long long
 constexpr int kStageGather = 0;  // per-thread loads from x [M][K], transposed in registers
 constexpr int kStageTiles = 1;   // one bulk copy of a tile the relayout kernel wrote
 constexpr int kStageTensor = 2;  // tensor copies of x's boxes, transposed in place (transpose_box)
+constexpr int kStageKMajor = 3;  // tensor copies of x^T [K][M] boxes, already in the tile's layout
 
 template <int KIND, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
 bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sched,
               const __grid_constant__ CUtensorMap xmap) {
     constexpr bool TMA = MODE == kStageTiles;
-    constexpr bool TENSOR = MODE == kStageTensor;
+    constexpr bool KMAJOR = MODE == kStageKMajor;
+    constexpr bool TENSOR = MODE == kStageTensor || KMAJOR;
     constexpr int SW = kTile * 16;  // slot words: 64 tokens x 4 block-rows x 4 channels
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int s_gp[kGroupWin + 1];                          // step offsets of the current group window
@@ -463,7 +465,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     const int kpad = (K + 15) & ~15;
     const int nbox = (K + 63) >> 6;  // 64-column boxes of a tile
     const uint32_t sbase = smem_addr(smem);
-    const uint32_t tb = (sbase + 511u) & ~511u;  // the token tile, 512-byte aligned (the boxes' swizzle)
+    const uint32_t tb = (sbase + 511u) & ~511u;  // the token tile, 512-byte aligned (the boxes' 64-byte swizzle)
     unsigned char* tile = smem + (tb - sbase);
     int* slots = reinterpret_cast<int*>(tile + static_cast<size_t>(nbox) * 64 * kTile);
     const int tid = threadIdx.x;
@@ -505,7 +507,10 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 const int b = bx0 + lane;
                 fence_proxy_async();
                 mbar_arrive_expect_tx(bar + 8u * b, 64u * kTile);
-                tensor_g2s(tb + 4096u * b, &xmap, 64 * b, static_cast<int>(t * kTile), bar + 8u * b);
+                if (KMAJOR)  // rows 64b..64b+63 of x^T at tokens t*64.., landing as the tile's rows
+                    tensor_g2s(tb + 4096u * b, &xmap, static_cast<int>(t * kTile), 64 * b, bar + 8u * b);
+                else
+                    tensor_g2s(tb + 4096u * b, &xmap, 64 * b, static_cast<int>(t * kTile), bar + 8u * b);
             }
             if (TMA && stage && warp == 0) {
                 const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
@@ -609,9 +614,13 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         if (TENSOR && stage) {
             // the warp turns its boxes around as they land
             bool ok = true;
-            for (int b = bx0; b < bx1 && ok; ++b) {
-                ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * b, phase & 1u));
-                if (ok) transpose_box(tb, b, lane);
+            if (KMAJOR) {  // nothing to turn around: every thread sees every box land
+                for (int b = 0; b < nbox && ok; ++b) ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * b, phase & 1u));
+            } else {
+                for (int b = bx0; b < bx1 && ok; ++b) {
+                    ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * b, phase & 1u));
+                    if (ok) transpose_box(tb, b, lane);
+                }
             }
             ++phase;
             if (__syncthreads_or(!ok)) {
@@ -833,8 +842,12 @@ const void* kernel_for(int kind) {
     }
 }
 const void* kernel_for(int kind, int mode) {
-    return mode == kStageTensor ? kernel_for<kStageTensor>(kind)
-                                : mode == kStageTiles ? kernel_for<kStageTiles>(kind) : kernel_for<kStageGather>(kind);
+    switch (mode) {
+    case kStageKMajor: return kernel_for<kStageKMajor>(kind);
+    case kStageTensor: return kernel_for<kStageTensor>(kind);
+    case kStageTiles: return kernel_for<kStageTiles>(kind);
+    default: return kernel_for<kStageGather>(kind);
+    }
 }
 
 // cuTensorMapEncodeTiled from the driver, looked up once.
@@ -875,7 +888,7 @@ int max_k() {
 cudaError_t prepare_kernels(int K, int* ctas_per_sm) {
     const int smem = static_cast<int>(smem_bytes(K));
     for (int kind = 0; kind < 5; ++kind) {
-        for (int mode = 0; mode < 3; ++mode) {
+        for (int mode = 0; mode < 4; ++mode) {
             cudaError_t e = cudaFuncSetAttribute(kernel_for(kind, mode), cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  kSmemOptin - kStaticSmem);
             if (e != cudaSuccess) return e;
@@ -900,7 +913,20 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
     // swizzle, zeros outside M x K); otherwise an unused all-zero map
     CUtensorMap xmap;
     std::memset(&xmap, 0, sizeof(xmap));
-    if (a.tensor) {
+    if (a.kmajor) {
+        // x^T [K][M] (row stride a.ld bytes): 64 tokens x 64 rows a box; its
+        // 64-byte swizzle is the tile's layout (tile_row_offset)
+        PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
+        if (!encode || (w.K + 63) / 64 > kMaxBoxes) return cudaErrorNotSupported;
+        const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(a.M), static_cast<cuuint64_t>(w.K)};
+        const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(a.ld)};
+        const cuuint32_t box[2] = {static_cast<cuuint32_t>(kTile), 64u};
+        const cuuint32_t estride[2] = {1u, 1u};
+        if (encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t*>(a.x), gdim, gstride, box, estride,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    } else if (a.tensor) {
         PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
         if (!encode || (w.K + 63) / 64 > kMaxBoxes) return cudaErrorNotSupported;
         const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(w.K), static_cast<cuuint64_t>(a.M)};
@@ -915,7 +941,9 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
     cudaError_t e = cudaSuccess;
 #define BSG_LAUNCH(KV)                                                                                   \
     do {                                                                                                 \
-        if (a.tensor)                                                                                    \
+        if (a.kmajor)                                                                                    \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageKMajor>, w, a, sched, xmap);            \
+        else if (a.tensor)                                                                               \
             e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTensor>, w, a, sched, xmap);            \
         else if (a.xb)                                                                                   \
             e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTiles>, w, a, sched, xmap);             \

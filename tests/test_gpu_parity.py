@@ -378,6 +378,49 @@ def test_relayout_then_tiled_kernel(bsg, k):
     assert bsg.bsgemm_device_status(lin._h) == 0
 
 
+@pytest.mark.parametrize("n_out,k_in,m,pad", [(96, 768, 200, 0), (64, 3072, 130, 16), (48, 1001, 64, 0),
+                                              (32, 40, 1, 16), (16, 3072, 4096, 0), (16, 3136, 70, 0)])
+def test_kmajor_input(bsg, n_out, k_in, m, pad):
+    """bsgemm_run_kmajor: X^T [K][M] (row stride a multiple of 16, padded or
+    not) copied straight into the tile layout; every element, every kind."""
+    import torch
+    rng = synth.rng_for(6000 + n_out + k_in + m)
+    wt = synth.draw_weight(rng, n_out, k_in, 0.85)
+    w = oracle.weight_dense(wt)
+    lin = make_linear(bsg, wt)
+    x = synth.draw_x(rng, m, k_in, "u127")
+    ld = -(-m // 16) * 16 + pad
+    xt_full = torch.full((k_in, ld), 99, dtype=torch.int8, device="cuda")  # padding columns hold junk
+    xt_full[:, :m] = torch.from_numpy(np.ascontiguousarray(x.T)).cuda()
+    xt = xt_full[:, :m]
+    for kind in KINDS:
+        dt = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+              synth.I8: torch.int8, synth.I8_GELU: torch.int8}[kind]
+        out = torch.empty((m, n_out), dtype=dt, device="cuda")
+        lin.run_kmajor(xt, out, kind, 0.05)
+        torch.cuda.synchronize()
+        check(out.cpu().numpy(), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05), kind)
+    assert bsg.bsgemm_device_status(lin._h) == 0
+    lin.close()
+
+
+def test_kmajor_argument_checks(bsg):
+    import torch
+    rng = synth.rng_for(6050)
+    wt = synth.draw_weight(rng, 16, 64, 0.5)
+    lin = make_linear(bsg, wt)
+    xt = torch.zeros((64, 48), dtype=torch.int8, device="cuda")
+    out = torch.empty((40, 16), dtype=torch.int8, device="cuda")
+    with pytest.raises(bsg.BsgemmError) as e:  # ld not a multiple of 16
+        bsg.bsgemm_run_kmajor(lin._h, xt.data_ptr(), 40, 40, out.data_ptr(), synth.I8, 1.0, 0)
+    assert e.value.code == bsg.ERR_INVALID
+    with pytest.raises(bsg.BsgemmError):  # ld < M
+        bsg.bsgemm_run_kmajor(lin._h, xt.data_ptr(), 40, 32, out.data_ptr(), synth.I8, 1.0, 0)
+    with pytest.raises(bsg.BsgemmError):  # misaligned act
+        bsg.bsgemm_run_kmajor(lin._h, xt.data_ptr() + 4, 40, 48, out.data_ptr(), synth.I8, 1.0, 0)
+    lin.close()
+
+
 def test_from_dense(bsg):
     rng = synth.rng_for(5800)
     wt = synth.draw_weight(rng, 128, 768, 0.8)
