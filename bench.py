@@ -770,9 +770,9 @@ def run_stack(args) -> dict:
 def run_prune(args) -> dict:
     """Create-side block pruning (App. A.1) of an fp32 weight of the FFN2
     shape (768 x 3072, normal(0, 0.02)) to 90% block sparsity: one step is
-    one bsgemm_block_prune call (score kernel, 8-pass radix select of the
-    threshold score, ordered tie count and mask write; it synchronises its
-    stream)."""
+    one bsgemm_block_prune call (one cooperative kernel: scores, 8-pass
+    radix select of the threshold score, ordered tie count and mask write,
+    phases split by grid barriers; the call synchronises its stream)."""
     import torch
     import paper_2211_07715_gb300 as bsg
     import oracle
@@ -853,13 +853,14 @@ def run_prune(args) -> dict:
         "config": {"workload": "average-magnitude 4x1 block pruning of a 768 x 3072 fp32 weight to 90% sparsity",
                    "n_out": n_out, "k_in": k_in, "sparsity": sparsity, "blocks": blocks,
                    "l2": f"rotating {nsets} weights ({nsets * w_bytes / 2**20:.0f} MiB > 2 x L2)",
-                   "launch": "one synchronous bsgemm_block_prune call per step (20 kernels)"},
+                   "launch": "one synchronous bsgemm_block_prune call per step (a memset and one cooperative "
+                             "kernel)"},
         "roofline": {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                      "frac": round(gbs / hbm_peak, 4), "traffic": None, "kernel": "bsgemm_block_prune (whole call)",
                      "bytes_basis": "algorithmic: fp32 weight read once + uint8 mask written once"},
         "e2e": {"value": round(blocks / (e2e_ms * 1e-3), 1), "unit": "blocks/s", "h2d_bytes_per_step": w_bytes,
                 "d2h_bytes_per_step": blocks},
-        "gpu_launches": 20 * steps, "clocks": clocks,
+        "gpu_launches": steps, "clocks": clocks,
     }
     if not args.no_cpu_baseline:
         t0 = time.perf_counter()
