@@ -71,13 +71,16 @@ typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
  * Block-compressed layout (App. A.1 blocks; App. A.3.4 "the sparse weight is
  * compressed and the mask is used"), all HOST memory, read during the call
  * only (the caller keeps ownership and may free them on return):
- *   N        output features, a multiple of 4 (App. A.3.4: other N would
- *            need padding, which the paper leaves out; so does this build:
- *            N % 4 != 0 returns NULL with BSGEMM_ERR_UNSUPPORTED).
+ *   N        output features, N >= 1.  Block-row r holds rows 4r..4r+3;
+ *            when N % 4 != 0 the last block-row, r = ceil(N/4) - 1, holds
+ *            the N % 4 remaining rows and values[j][i] of its rows
+ *            4r + i >= N are ignored (App. A.3.4 notes that such N need
+ *            padding and leaves it out; here the block-row is zero-padded
+ *            at create time and only channels < N are stored).
  *   K        input features, 1 <= K <= bsgemm_max_k().
  *   block    must be 4.
- *   indices  int32: indptr[N/4 + 1] followed by colidx[nnzb], nnzb =
- *            indptr[N/4].  Block j of block-row r (indptr[r] <= j <
+ *   indices  int32: indptr[R + 1] followed by colidx[nnzb], R =
+ *            ceil(N/4), nnzb = indptr[R].  Block j of block-row r (indptr[r] <= j <
  *            indptr[r+1]) lies in column colidx[j]; columns strictly
  *            increase within a block-row; indptr[0] = 0.
  *   values   int8 [nnzb][4]: values[j][i] = W[4r + i][colidx[j]].  A stored

@@ -233,23 +233,26 @@ _OUT_DTYPES = {OUT_I32: "int32", OUT_F32: "float32", OUT_F32_GELU: "float32", OU
 
 
 def dense_to_blocks(w: np.ndarray, keep=None):
-    """Block-compress a dense int8 weight [N][K].  Stores the 4x1 blocks
-    where `keep` [N/4][K] is true (a mask from block_prune; its pruned
-    blocks are dropped whatever they hold), or without a mask every block
-    that holds a nonzero value.  Returns (indptr, colidx, values)."""
+    """Block-compress a dense int8 weight [N][K] (any N: the last block-row
+    takes the N % 4 remaining rows, its missing rows read as zeros).  Stores
+    the 4x1 blocks where `keep` [ceil(N/4)][K] is true (a mask from
+    block_prune; its pruned blocks are dropped whatever they hold), or
+    without a mask every block that holds a nonzero value.  Returns
+    (indptr, colidx, values)."""
     w = _host_array(w, np.int8)
     n_out, k_in = w.shape
+    nbr = -(-n_out // BLOCK)
     if n_out % BLOCK:
-        raise ValueError("N must be a multiple of 4")
-    blocks = w.reshape(n_out // BLOCK, BLOCK, k_in)          # [r][i][k]
+        w = np.concatenate([w, np.zeros((nbr * BLOCK - n_out, k_in), np.int8)])
+    blocks = w.reshape(nbr, BLOCK, k_in)                      # [r][i][k]
     if keep is None:
         keep = (blocks != 0).any(axis=1)                      # [r][k]
     else:
         keep = _host_array(keep, np.uint8).astype(bool)
-        if keep.shape != (n_out // BLOCK, k_in):
-            raise ValueError(f"keep must have shape {(n_out // BLOCK, k_in)}")
+        if keep.shape != (nbr, k_in):
+            raise ValueError(f"keep must have shape {(nbr, k_in)}")
     r_idx, k_idx = np.nonzero(keep)                           # row-major: sorted by r, then k
-    indptr = np.zeros(n_out // BLOCK + 1, np.int32)
+    indptr = np.zeros(nbr + 1, np.int32)
     np.cumsum(keep.sum(axis=1), out=indptr[1:])
     values = np.ascontiguousarray(blocks[r_idx, :, k_idx], dtype=np.int8)  # [nnzb][4]
     return indptr, k_idx.astype(np.int32), values

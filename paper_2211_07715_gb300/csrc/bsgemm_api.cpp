@@ -54,7 +54,7 @@ const int kZeroStatus = 0;
 
 // Check the block-compressed arrays; returns an empty string if valid.
 std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx) {
-    const int nbr = N / BSGEMM_BLOCK;
+    const int nbr = (N + BSGEMM_BLOCK - 1) / BSGEMM_BLOCK;
     if (indptr[0] != 0) return "indptr[0] must be 0";
     for (int r = 0; r < nbr; ++r) {
         if (indptr[r + 1] < indptr[r]) return "indptr must be non-decreasing (block-row " + std::to_string(r) + ")";
@@ -151,12 +151,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         fail(BSGEMM_ERR_UNSUPPORTED, "block must be 4 (4 output rows x 1 input column)");
         return nullptr;
     }
-    if (N < BSGEMM_BLOCK || K < 1) {
-        fail(BSGEMM_ERR_INVALID, "need N >= 4 and K >= 1");
-        return nullptr;
-    }
-    if (N % BSGEMM_BLOCK != 0) {
-        fail(BSGEMM_ERR_UNSUPPORTED, "N must be a multiple of 4 (padding is not implemented)");
+    if (N < 1 || K < 1) {
+        fail(BSGEMM_ERR_INVALID, "need N >= 1 and K >= 1");
         return nullptr;
     }
     if (K > bsg::max_k()) {
@@ -168,7 +164,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         fail(BSGEMM_ERR_INVALID, "indices and scales must not be NULL");
         return nullptr;
     }
-    const int nbr = N / BSGEMM_BLOCK;
+    const int nbr = (N + BSGEMM_BLOCK - 1) / BSGEMM_BLOCK;  // the last block-row may hold fewer than 4 rows
+    const int npad = BSGEMM_BLOCK * nbr;
     const int32_t* indptr = indices;
     const int64_t nnzb = indptr[nbr];
     if (indptr[0] != 0 || nnzb < 0 || nnzb > static_cast<int64_t>(nbr) * K) {
@@ -297,7 +294,10 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
             }
         }
     }
-    std::vector<float> bias_v(N, 0.0f);
+    // scales and biases padded with zeros to whole block-rows (the kernel
+    // reads 4 channels at a time and stores only channels < N)
+    std::vector<float> scale_v(npad, 0.0f), bias_v(npad, 0.0f);
+    std::memcpy(scale_v.data(), scales, sizeof(float) * N);
     if (bias) std::memcpy(bias_v.data(), bias, sizeof(float) * N);
 
     auto* h = new bsgemm_ctx();
@@ -331,8 +331,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     const size_t off_grow = align_up(off_gptr + sizeof(int32_t) * (ngroups + 1), 256);
     const size_t off_recs = align_up(off_grow + sizeof(int32_t) * grow.size(), 256);
     const size_t off_scale = align_up(off_recs + sizeof(int32_t) * recs.size(), 256);
-    const size_t off_bias = align_up(off_scale + sizeof(float) * N, 256);
-    const size_t off_status = align_up(off_bias + sizeof(float) * N, 256);
+    const size_t off_bias = align_up(off_scale + sizeof(float) * npad, 256);
+    const size_t off_status = align_up(off_bias + sizeof(float) * npad, 256);
     h->arena_bytes = align_up(off_status + sizeof(int), 256);
     e = cudaMalloc(&h->arena, h->arena_bytes);
     if (e != cudaSuccess) {
@@ -345,8 +345,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
         {off_gptr, gptr.data(), sizeof(int32_t) * gptr.size()},
         {off_grow, grow.data(), sizeof(int32_t) * grow.size()},
         {off_recs, recs.data(), sizeof(int32_t) * recs.size()},
-        {off_scale, scales, sizeof(float) * N},
-        {off_bias, bias_v.data(), sizeof(float) * N},
+        {off_scale, scale_v.data(), sizeof(float) * npad},
+        {off_bias, bias_v.data(), sizeof(float) * npad},
         {off_status, &kZeroStatus, sizeof(int)},
     };
     for (const Piece& p : pieces) {

@@ -164,29 +164,43 @@ __device__ __forceinline__ void store_token(const LaunchArgs& a, int N, long lon
                                             float4 b) {
     if (m >= a.M) return;
     const size_t o = static_cast<size_t>(m) * N + 4 * r;
+    // N % 4 != 0: rows of out are not 16-byte aligned and the last block-row
+    // has fewer than 4 channels -- one store a channel, channels < N only
+    const bool narrow = (N & 3) != 0;
+    const int nc = min(4, N - 4 * r);
     if (KIND == 0) {
-        *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(v[0], v[1], v[2], v[3]);
+        if (!narrow) {
+            *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(v[0], v[1], v[2], v[3]);
+        } else {
+            for (int c = 0; c < nc; ++c) static_cast<int32_t*>(a.out)[o + c] = v[c];
+        }
         return;
     }
-    float y0 = __fmaf_rn(__int2float_rn(v[0]), s.x, b.x);
-    float y1 = __fmaf_rn(__int2float_rn(v[1]), s.y, b.y);
-    float y2 = __fmaf_rn(__int2float_rn(v[2]), s.z, b.z);
-    float y3 = __fmaf_rn(__int2float_rn(v[3]), s.w, b.w);
+    float y[4];
+    y[0] = __fmaf_rn(__int2float_rn(v[0]), s.x, b.x);
+    y[1] = __fmaf_rn(__int2float_rn(v[1]), s.y, b.y);
+    y[2] = __fmaf_rn(__int2float_rn(v[2]), s.z, b.z);
+    y[3] = __fmaf_rn(__int2float_rn(v[3]), s.w, b.w);
     if (KIND == 2) {
-        y0 = gelu_f32_fast(y0);
-        y1 = gelu_f32_fast(y1);
-        y2 = gelu_f32_fast(y2);
-        y3 = gelu_f32_fast(y3);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) y[c] = gelu_f32_fast(y[c]);
     } else if (KIND == 4) {
-        y0 = gelu_f32(y0);
-        y1 = gelu_f32(y1);
-        y2 = gelu_f32(y2);
-        y3 = gelu_f32(y3);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) y[c] = gelu_f32(y[c]);
     }
     if (KIND == 1 || KIND == 2) {
-        *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y0, y1, y2, y3);
+        if (!narrow) {
+            *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y[0], y[1], y[2], y[3]);
+        } else {
+            for (int c = 0; c < nc; ++c) static_cast<float*>(a.out)[o + c] = y[c];
+        }
     } else {
-        *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = requant4_s8(y0, y1, y2, y3, a.inv_out_scale);
+        const uint32_t q = requant4_s8(y[0], y[1], y[2], y[3], a.inv_out_scale);
+        if (!narrow) {
+            *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = q;
+        } else {
+            for (int c = 0; c < nc; ++c) static_cast<int8_t*>(a.out)[o + c] = static_cast<int8_t>(q >> (8 * c));
+        }
     }
 }
 

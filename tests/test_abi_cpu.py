@@ -54,7 +54,7 @@ def _create(bsg, *args):
 
 def test_create_rejects_bad_arrays(bsg):
     ones = [1.0] * 8
-    assert _create(bsg, 6, 8, 4, [0, 0], [], [1.0] * 6) == bsg.ERR_UNSUPPORTED       # N % 4
+    assert _create(bsg, 6, 8, 4, [0, 1, 1, 8], [[1] * 4], [1.0] * 6) == bsg.ERR_INVALID  # N = 6 (2 block-rows): column = K
     assert _create(bsg, 8, 8, 2, [0, 0, 0], [], ones) == bsg.ERR_UNSUPPORTED         # block != 4
     assert _create(bsg, 8, 10**6, 4, [0, 0, 0], [], ones) == bsg.ERR_UNSUPPORTED     # K too large
     assert _create(bsg, 8, 8, 4, [1, 1, 1], [], ones) == bsg.ERR_INVALID             # indptr[0] != 0

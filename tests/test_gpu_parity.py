@@ -40,8 +40,9 @@ def make_linear(bsg, wt):
 
 
 def gpu_run(lin, x: np.ndarray, kind: int, out_scale: float, workspace=None) -> np.ndarray:
-    """workspace=None: the two-kernel path (token-tile relayout + bulk-copy
-    staging); workspace=False: the single kernel without scratch memory."""
+    """workspace=None: bsgemm_run_ws (with K % 16 == 0 the one kernel that
+    stages tiles by tensor copies, else relayout + bulk copies);
+    workspace=False: bsgemm_run (tensor copies, else per-thread gathers)."""
     xd = torch.from_numpy(x).cuda()
     dtype = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
              synth.I8: torch.int8, synth.I8_GELU: torch.int8}[kind]
@@ -418,6 +419,41 @@ def test_kmajor_argument_checks(bsg):
         bsg.bsgemm_run_kmajor(lin._h, xt.data_ptr(), 40, 32, out.data_ptr(), synth.I8, 1.0, 0)
     with pytest.raises(bsg.BsgemmError):  # misaligned act
         bsg.bsgemm_run_kmajor(lin._h, xt.data_ptr() + 4, 40, 48, out.data_ptr(), synth.I8, 1.0, 0)
+    lin.close()
+
+
+@pytest.mark.parametrize("n_out,k_in,m", [(6, 768, 130), (1, 64, 70), (18, 1001, 65), (770, 768, 200),
+                                          (3, 3072, 64)])
+def test_n_not_a_multiple_of_4(bsg, n_out, k_in, m):
+    """The last block-row holds N % 4 rows: zero-padded at create time, only
+    channels < N stored (rows of out are then not 16-byte aligned).  Every
+    staging path, every kind, every element."""
+    import torch
+    rng = synth.rng_for(6200 + n_out + k_in)
+    n4 = -(-n_out // 4) * 4
+    wt = synth.draw_weight(rng, n4, k_in, 0.8)
+    w = np.ascontiguousarray(oracle.weight_dense(wt)[:n_out])
+    scales, bias = wt.scales[:n_out].copy(), wt.bias[:n_out].copy()
+    lin = bsg.SparseInt8Linear.from_dense(w, scales, bias)
+    assert lin.n_out == n_out
+    x = synth.draw_x(rng, m, k_in, "u127")
+    for kind in KINDS:
+        want = oracle.linear(x, w, scales, bias, kind, out_scale=0.05)
+        for path in (None, False):
+            check(gpu_run(lin, x, kind, 0.05, workspace=path), want, kind, f"path {path}")
+        if m % 16 == 0:
+            dt = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+                  synth.I8: torch.int8, synth.I8_GELU: torch.int8}[kind]
+            out = torch.empty((m, n_out), dtype=dt, device="cuda")
+            lin.run_kmajor(torch.from_numpy(np.ascontiguousarray(x.T)).cuda(), out, kind, 0.05)
+            torch.cuda.synchronize()
+            check(out.cpu().numpy(), want, kind, "kmajor")
+    # a guard after the last row of out stays untouched
+    xd = torch.from_numpy(x).cuda()
+    buf = torch.full((m * n_out + 64,), 77, dtype=torch.int8, device="cuda")
+    lin.run(xd, buf[: m * n_out].view(m, n_out), synth.I8, 0.05)
+    torch.cuda.synchronize()
+    assert (buf[m * n_out:].cpu().numpy() == 77).all()
     lin.close()
 
 
