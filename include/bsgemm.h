@@ -61,7 +61,20 @@ typedef struct {
     int32_t kind;    /* a bsgemm_out_kind                                    */
     float out_scale; /* int8 kinds only: finite and > 0; the library         */
                      /* multiplies by 1.0f / out_scale (one fp32 division)   */
+    uint32_t flags;  /* 0 or BSGEMM_ACT_READY; other bits are invalid        */
 } bsgemm_epilogue;
+
+/*
+ * BSGEMM_ACT_READY: act was complete before the kernel that precedes this
+ * call on the stream began (an upload, or the output of work that has
+ * finished), so the layer kernel may start reading it while that kernel
+ * still runs (the kernels are launched with programmatic dependent launch).
+ * Without the flag act is read only after the preceding kernel has
+ * completed, which is right whenever that kernel writes act (a layer
+ * chain).  Outputs are written after the preceding kernel in either case.
+ * It changes nothing on the paths that stage relaid tiles.
+ */
+#define BSGEMM_ACT_READY 1u
 
 typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
 

@@ -35,8 +35,11 @@ class BsgemmError(RuntimeError):
         self.code = code
 
 
+ACT_READY = 1  # BSGEMM_ACT_READY: act may be read while the stream's previous kernel finishes
+
+
 class Epilogue(ctypes.Structure):
-    _fields_ = [("kind", ctypes.c_int32), ("out_scale", ctypes.c_float)]
+    _fields_ = [("kind", ctypes.c_int32), ("out_scale", ctypes.c_float), ("flags", ctypes.c_uint32)]
 
 
 def _load() -> ctypes.CDLL:
@@ -121,17 +124,18 @@ def bsgemm_create(n_out: int, k_in: int, block: int, indices, values, scales, bi
 
 
 def bsgemm_run(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float = 1.0,
-               stream: int = 0) -> None:
+               stream: int = 0, flags: int = 0) -> None:
     """Enqueue one run on `stream` (raw device pointers); raises on failure."""
-    rc = _lib.bsgemm_run(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
+    rc = _lib.bsgemm_run(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale), int(flags)), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 
 
 def bsgemm_run_ws(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float, ws_ptr: int,
-                  ws_bytes: int, stream: int = 0) -> None:
-    """Enqueue the two-kernel fast path with a device workspace; raises on failure."""
-    rc = _lib.bsgemm_run_ws(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), ws_ptr,
+                  ws_bytes: int, stream: int = 0, flags: int = 0) -> None:
+    """Enqueue a run with a device workspace (used only by the shapes that
+    need the relayout kernel); raises on failure."""
+    rc = _lib.bsgemm_run_ws(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale), int(flags)), ws_ptr,
                             int(ws_bytes), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
@@ -147,9 +151,10 @@ def bsgemm_run_static(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out
 
 
 def bsgemm_run_kmajor(h: int, act_t_ptr: int, m: int, ld: int, out_ptr: int, kind: int, out_scale: float = 1.0,
-                      stream: int = 0) -> None:
+                      stream: int = 0, flags: int = 0) -> None:
     """The layer on K-major activations X^T [K][M] (row stride ld bytes)."""
-    rc = _lib.bsgemm_run_kmajor(h, act_t_ptr, int(m), int(ld), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
+    rc = _lib.bsgemm_run_kmajor(h, act_t_ptr, int(m), int(ld), out_ptr,
+                                Epilogue(int(kind), float(out_scale), int(flags)), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 
@@ -278,13 +283,17 @@ class SparseInt8Linear:
     def workspace_bytes(self, m: int) -> int:
         return bsgemm_workspace_bytes(self._h, m)
 
-    def run(self, x, out, kind: int, out_scale: float = 1.0, stream=None, workspace=None) -> None:
+    def run(self, x, out, kind: int, out_scale: float = 1.0, stream=None, workspace=None,
+            act_ready: bool = False) -> None:
         """out[M][N] = epilogue(x[M][K] W^T); both CUDA tensors, contiguous.
 
-        Takes the fast two-kernel path with a workspace: the given uint8 CUDA
-        tensor, or (workspace=None) one drawn from PyTorch's caching
-        allocator on the same stream.  workspace=False forces the
-        single-kernel path without scratch memory."""
+        With K % 16 == 0 and x 16-byte aligned this is one kernel that stages
+        x itself (the workspace is then unused); otherwise the workspace --
+        the given uint8 CUDA tensor, or (workspace=None) one drawn from
+        PyTorch's caching allocator on the same stream -- takes the relaid
+        tiles, and workspace=False gathers them with per-thread loads
+        instead.  act_ready: x was complete
+        before the stream's previous kernel began (BSGEMM_ACT_READY)."""
         import torch
         if x.dtype != torch.int8 or not x.is_cuda or not x.is_contiguous() or x.dim() != 2 or x.shape[1] != self.k_in:
             raise ValueError("x must be a contiguous CUDA int8 tensor [M][K]")
@@ -293,8 +302,9 @@ class SparseInt8Linear:
             raise ValueError(f"out must be a contiguous CUDA {_OUT_DTYPES[kind]} tensor [M][N]")
         s = torch.cuda.current_stream() if stream is None else stream
         m = x.shape[0]
+        flags = ACT_READY if act_ready else 0
         if workspace is False or m == 0:
-            bsgemm_run(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, s.cuda_stream)
+            bsgemm_run(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, s.cuda_stream, flags)
             return
         need = self.workspace_bytes(m)
         if workspace is None:
@@ -303,7 +313,7 @@ class SparseInt8Linear:
         if workspace.numel() * workspace.element_size() < need:
             raise ValueError(f"workspace must hold {need} bytes")
         bsgemm_run_ws(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, workspace.data_ptr(),
-                      workspace.numel() * workspace.element_size(), s.cuda_stream)
+                      workspace.numel() * workspace.element_size(), s.cuda_stream, flags)
 
     def run_kmajor(self, xt, out, kind: int, out_scale: float = 1.0, stream=None) -> None:
         """out[M][N] = epilogue(X W^T) from K-major activations: xt is a CUDA

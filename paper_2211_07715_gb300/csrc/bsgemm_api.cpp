@@ -385,6 +385,8 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
     if (epi.kind < BSGEMM_OUT_I32 || epi.kind > BSGEMM_OUT_I8_GELU)
         return fail(BSGEMM_ERR_INVALID, "unknown epilogue kind " + std::to_string(epi.kind));
+    if (epi.flags & ~static_cast<uint32_t>(BSGEMM_ACT_READY))
+        return fail(BSGEMM_ERR_INVALID, "unknown bits in epi.flags");
     float inv = 0.0f;
     if (epi.kind == BSGEMM_OUT_I8 || epi.kind == BSGEMM_OUT_I8_GELU) {
         if (!(epi.out_scale > 0.0f) || !std::isfinite(epi.out_scale))
@@ -425,6 +427,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.tensor = tensor;
     a.kmajor = mode == 3;
     a.ld = ld;
+    a.act_ready = (epi.flags & BSGEMM_ACT_READY) != 0 && (tensor || mode == 3);
     a.out = out;
     a.M = M;
     a.kind = epi.kind;
@@ -568,7 +571,9 @@ int bsgemm_run_host(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epil
     const cudaStream_t s = static_cast<cudaStream_t>(stream);
     e = cudaMemcpyAsync(ws, act, static_cast<size_t>(M) * static_cast<size_t>(h->w.K), cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("copy of act to the device", e));
-    const int rc = run_common(h, reinterpret_cast<const int8_t*>(ws), M, ws + off_out, epi, ws + off_tiles,
+    bsgemm_epilogue e2 = epi;
+    e2.flags |= BSGEMM_ACT_READY;  // the copy above completes before the kernel starts (stream order)
+    const int rc = run_common(h, reinterpret_cast<const int8_t*>(ws), M, ws + off_out, e2, ws + off_tiles,
                               off_out - off_tiles, 1, stream);
     if (rc != BSGEMM_OK) return rc;
     e = cudaMemcpyAsync(out, ws + off_out, out_bytes, cudaMemcpyDeviceToHost, s);

@@ -68,6 +68,7 @@ struct LaunchArgs {
     bool x_vec16;          // x 16-byte aligned and K % 16 == 0
     bool tensor;           // stage tiles from x by tensor copies (xb unused; needs tensor_staging())
     bool kmajor;           // x is x^T [K][M] with row stride ld: tensor copies, no transpose
+    bool act_ready;        // x may be read before the previous kernel completes (BSGEMM_ACT_READY)
     int ld;                // row stride of x^T in bytes (kmajor only)
 };
 

@@ -159,47 +159,76 @@ __device__ __forceinline__ uint32_t requant4_s8(float v0, float v1, float v2, fl
 
 // Epilogue for one token m (nothing past M): v = acc of the 4 channels of
 // block-row r (scales s, bias b), written as out[m][4r .. 4r+3].
+// The epilogue value of channel c (c < 4) of one token: acc, or y =
+// fmaf((float)acc, s, b) with optional GELU.
+template <int KIND>
+__device__ __forceinline__ float epilogue_value(int v, float s, float b) {
+    float y = __fmaf_rn(__int2float_rn(v), s, b);
+    if (KIND == 2) y = gelu_f32_fast(y);
+    if (KIND == 4) y = gelu_f32(y);
+    return y;
+}
+
 template <int KIND>
 __device__ __forceinline__ void store_token(const LaunchArgs& a, int N, long long m, int r, const int* v, float4 s,
                                             float4 b) {
     if (m >= a.M) return;
     const size_t o = static_cast<size_t>(m) * N + 4 * r;
-    // N % 4 != 0: rows of out are not 16-byte aligned and the last block-row
-    // has fewer than 4 channels -- one store a channel, channels < N only
-    const bool narrow = (N & 3) != 0;
-    const int nc = min(4, N - 4 * r);
     if (KIND == 0) {
-        if (!narrow) {
-            *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(v[0], v[1], v[2], v[3]);
-        } else {
-            for (int c = 0; c < nc; ++c) static_cast<int32_t*>(a.out)[o + c] = v[c];
-        }
+        *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(v[0], v[1], v[2], v[3]);
         return;
     }
-    float y[4];
-    y[0] = __fmaf_rn(__int2float_rn(v[0]), s.x, b.x);
-    y[1] = __fmaf_rn(__int2float_rn(v[1]), s.y, b.y);
-    y[2] = __fmaf_rn(__int2float_rn(v[2]), s.z, b.z);
-    y[3] = __fmaf_rn(__int2float_rn(v[3]), s.w, b.w);
+    float y0 = __fmaf_rn(__int2float_rn(v[0]), s.x, b.x);
+    float y1 = __fmaf_rn(__int2float_rn(v[1]), s.y, b.y);
+    float y2 = __fmaf_rn(__int2float_rn(v[2]), s.z, b.z);
+    float y3 = __fmaf_rn(__int2float_rn(v[3]), s.w, b.w);
     if (KIND == 2) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c) y[c] = gelu_f32_fast(y[c]);
+        y0 = gelu_f32_fast(y0);
+        y1 = gelu_f32_fast(y1);
+        y2 = gelu_f32_fast(y2);
+        y3 = gelu_f32_fast(y3);
     } else if (KIND == 4) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c) y[c] = gelu_f32(y[c]);
+        y0 = gelu_f32(y0);
+        y1 = gelu_f32(y1);
+        y2 = gelu_f32(y2);
+        y3 = gelu_f32(y3);
     }
     if (KIND == 1 || KIND == 2) {
-        if (!narrow) {
-            *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y[0], y[1], y[2], y[3]);
-        } else {
-            for (int c = 0; c < nc; ++c) static_cast<float*>(a.out)[o + c] = y[c];
-        }
+        *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y0, y1, y2, y3);
     } else {
-        const uint32_t q = requant4_s8(y[0], y[1], y[2], y[3], a.inv_out_scale);
-        if (!narrow) {
-            *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = q;
+        *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = requant4_s8(y0, y1, y2, y3, a.inv_out_scale);
+    }
+}
+
+// N % 4 != 0: rows of out are not 16-byte aligned and the last block-row
+// has fewer than 4 channels -- one store a channel, channels < N only
+// (constant indices throughout, so acc stays in registers).
+template <int KIND>
+__device__ __forceinline__ void store_lane_narrow(const LaunchArgs& a, int N, long long m_g, int r,
+                                                  const int (&acc)[32], float4 sc, float4 bi) {
+    const int nc = min(4, N - 4 * r);
+    const float s4[4] = {sc.x, sc.y, sc.z, sc.w}, b4[4] = {bi.x, bi.y, bi.z, bi.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const long long m = m_g + 8 * i;
+        if (m >= a.M) continue;
+        const size_t o = static_cast<size_t>(m) * N + 4 * r;
+        if (KIND == 0) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < nc) static_cast<int32_t*>(a.out)[o + c] = acc[4 * i + c];
+        } else if (KIND == 1 || KIND == 2) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < nc) static_cast<float*>(a.out)[o + c] = epilogue_value<KIND>(acc[4 * i + c], s4[c], b4[c]);
         } else {
-            for (int c = 0; c < nc; ++c) static_cast<int8_t*>(a.out)[o + c] = static_cast<int8_t>(q >> (8 * c));
+            float y[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) y[c] = epilogue_value<KIND>(acc[4 * i + c], s4[c], b4[c]);
+            const uint32_t q = requant4_s8(y[0], y[1], y[2], y[3], a.inv_out_scale);
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < nc) static_cast<int8_t*>(a.out)[o + c] = static_cast<int8_t>(q >> (8 * c));
         }
     }
 }
@@ -452,6 +481,10 @@ template <int KIND>
 __device__ __forceinline__ void store_lane(const LaunchArgs& a, int N, long long m_g, int r, const int (&acc)[32],
                                            float4 sc, float4 bi) {
     if (r < 0) return;
+    if (N & 3) {
+        store_lane_narrow<KIND>(a, N, m_g, r, acc, sc, bi);
+        return;
+    }
 #pragma unroll
     for (int i = 0; i < 8; ++i) store_token<KIND>(a, N, m_g + 8 * i, r, acc + 4 * i, sc, bi);
 }
@@ -538,7 +571,11 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         };
         // After the first window the previous grid is done: the copy starts
         // at once and overlaps the window's set-up.
-        if (waited) copy_tile();
+        // With act_ready (x complete before the previous kernel started) the
+        // first window's tensor copies start at once too and overlap that
+        // kernel's end.
+        const bool issued = waited || (TENSOR && a.act_ready);
+        if (issued) copy_tile();
         __syncthreads();  // the group window is visible
         const int sa = gp(g_lo);
         if (tid <= kWarps) {
@@ -605,7 +642,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         if (!waited) {
             griddep_wait();
             waited = true;
-            copy_tile();
+            if (!issued) copy_tile();
         }
         if (MODE == kStageGather && stage) {  // gather the tile with per-thread loads
             stage_tile(tile, a, K, kpad, m0);

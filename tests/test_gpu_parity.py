@@ -457,6 +457,31 @@ def test_n_not_a_multiple_of_4(bsg, n_out, k_in, m):
     lin.close()
 
 
+def test_act_ready_back_to_back(bsg):
+    """BSGEMM_ACT_READY on independent batches launched back to back (the
+    tile copies may start while the previous launch ends): every result
+    equals the oracle's; an unknown flag bit is rejected."""
+    import torch
+    rng = synth.rng_for(6300)
+    wt = synth.draw_weight(rng, 128, 1024, 0.85)
+    w = oracle.weight_dense(wt)
+    lin = make_linear(bsg, wt)
+    xs = [synth.draw_x(rng, m, 1024, "u127") for m in (300, 64, 513, 129)]
+    xds = [torch.from_numpy(x).cuda() for x in xs]
+    outs = [torch.empty((x.shape[0], 128), dtype=torch.int8, device="cuda") for x in xs]
+    torch.cuda.synchronize()
+    for _ in range(3):
+        for xd, out in zip(xds, outs):
+            lin.run(xd, out, synth.I8_GELU, 0.04, act_ready=True)
+    torch.cuda.synchronize()
+    for x, out in zip(xs, outs):
+        check(out.cpu().numpy(), oracle.linear(x, w, wt.scales, wt.bias, synth.I8_GELU, out_scale=0.04), synth.I8_GELU)
+    with pytest.raises(bsg.BsgemmError) as e:
+        bsg.bsgemm_run(lin._h, xds[0].data_ptr(), 300, outs[0].data_ptr(), synth.I8, 1.0, 0, 2)
+    assert e.value.code == bsg.ERR_INVALID
+    lin.close()
+
+
 def test_from_dense(bsg):
     rng = synth.rng_for(5800)
     wt = synth.draw_weight(rng, 128, 768, 0.8)
