@@ -71,6 +71,12 @@ def _load():
                                           ctypes.c_void_p, c_int, c_int]
             lib.oracle_linear.restype = c_int
             lib.oracle_block_prune.argtypes = [c_int, c_int, f32p, c_double, u8p]
+            lib.oracle_linear_resid.argtypes = [c_int, c_int, c_int, i8p, i8p, f32p, f32p, i8p, c_float, f32p,
+                                                c_int, c_int]
+            lib.oracle_linear_resid.restype = c_int
+            lib.oracle_layernorm.argtypes = [c_int, c_int, f32p, f32p, f32p, c_double,
+                                             ctypes.POINTER(c_double)]
+            lib.oracle_layernorm.restype = None
             lib.oracle_block_prune.restype = ctypes.c_int64
             _lib = lib
     return _lib
@@ -202,6 +208,57 @@ def linear(x: np.ndarray, w: np.ndarray, scales, bias, kind: int, out_scale: flo
             raise OverflowError("accumulator leaves the int32 range")
         if rc:
             raise RuntimeError(f"oracle_linear failed ({rc})")
+    return out
+
+
+def linear_resid(x: np.ndarray, w: np.ndarray, scales, bias, residual: np.ndarray, res_scale: float,
+                 threads: int = 1) -> np.ndarray:
+    """z = fmaf((float)acc, scale, bias) + res_scale * (float)residual, in
+    fp32 op by op (the residual add before LayerNorm); float32 [M][N]."""
+    lib = _load()
+    w = _c(w, np.int8)
+    n_out, k_in = w.shape
+    x = _c(x, np.int8)
+    m = x.shape[0]
+    residual = _c(residual, np.int8)
+    if residual.shape != (m, n_out):
+        raise ValueError("residual must be [M][N]")
+    scales = _c(scales, np.float32)
+    bias_arr = None if bias is None else _c(bias, np.float32)
+    out = np.empty((m, n_out), dtype=np.float32)
+
+    def run(r0, r1):
+        return lib.oracle_linear_resid(m, n_out, k_in, _ptr(x, ctypes.c_int8), _ptr(w, ctypes.c_int8),
+                                       _ptr(scales, ctypes.c_float),
+                                       None if bias_arr is None else _ptr(bias_arr, ctypes.c_float),
+                                       _ptr(residual, ctypes.c_int8), float(np.float32(res_scale)),
+                                       _ptr(out, ctypes.c_float), r0, r1)
+
+    threads = max(1, min(int(threads), m))
+    bounds = [m * i // threads for i in range(threads + 1)]
+    if threads == 1:
+        rcs = [run(0, m)]
+    else:
+        with ThreadPoolExecutor(threads) as ex:
+            rcs = list(ex.map(lambda i: run(bounds[i], bounds[i + 1]), range(threads)))
+    for rc in rcs:
+        if rc == -2:
+            raise OverflowError("accumulator leaves the int32 range")
+        if rc:
+            raise RuntimeError(f"oracle_linear_resid failed ({rc})")
+    return out
+
+
+def layernorm(z: np.ndarray, gamma, beta, eps: float) -> np.ndarray:
+    """LayerNorm of each row of the fp32 z [M][N] in fp64 (float64 [M][N])."""
+    lib = _load()
+    z = _c(z, np.float32)
+    m, n = z.shape
+    gamma = _c(gamma, np.float32)
+    beta = _c(beta, np.float32)
+    out = np.empty((m, n), dtype=np.float64)
+    lib.oracle_layernorm(m, n, _ptr(z, ctypes.c_float), _ptr(gamma, ctypes.c_float), _ptr(beta, ctypes.c_float),
+                         float(eps), out.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
     return out
 
 

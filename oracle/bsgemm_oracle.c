@@ -267,6 +267,62 @@ int oracle_linear(int M, int N, int K, const int8_t* X, const int8_t* W, const f
 }
 
 /* ---------------------------------------------------------------------- */
+/* Residual add before LayerNorm (the post-operators the optimized INT8     */
+/* graph fuses after an InnerProduct, Sec. 3 "Graph optimization"; the     */
+/* encoder adds the sub-layer's input before its LayerNorm).  For rows      */
+/* [row0, row1) of the layer:                                               */
+/*   y = fmaf((float)acc, scale[n], bias[n])            (fp32, as above)    */
+/*   z = y + (res_scale * (float)r[m][n])               (two fp32 ops,     */
+/*                                                       multiply first)    */
+/* r is the int8 residual [M][N] (the sub-layer's input in the int8 chain)  */
+/* with its per-tensor scale.  Writes z (fp32) to out[M][N].                */
+/* Returns 0, -2 on accumulator overflow, -3 out of memory.                 */
+/* ---------------------------------------------------------------------- */
+int oracle_linear_resid(int M, int N, int K, const int8_t* X, const int8_t* W, const float* scales,
+                        const float* bias, const int8_t* R, float res_scale, float* out, int row0, int row1) {
+    int32_t* acc = (int32_t*)malloc(sizeof(int32_t) * (size_t)(N > 0 ? N : 1));
+    if (!acc) return -3;
+    for (int m = row0; m < row1; ++m) {
+        int rc = oracle_acc(M, N, K, X + (size_t)m * K, W, acc, 0, 1);
+        if (rc) { free(acc); return rc; }
+        for (int n = 0; n < N; ++n) {
+            size_t o = (size_t)m * N + n;
+            float y = oracle_dequant_f32(acc[n], scales[n], bias ? bias[n] : 0.0f);
+            float rs = res_scale * (float)R[o];
+            out[o] = y + rs;
+        }
+    }
+    free(acc);
+    return 0;
+}
+
+/* LayerNorm over the N channels of each row (the LayerNorm the optimized    */
+/* INT8 graph fuses, Sec. 3 "Graph optimization"):                          */
+/*   mu = (1/N) sum_n z[n],  var = (1/N) sum_n (z[n] - mu)^2,                */
+/*   out[n] = (z[n] - mu) / sqrt(var + eps) * gamma[n] + beta[n],            */
+/* in fp64 (the exact value the fp32 kernel approximates; the paper fixes    */
+/* no summation order).  Two passes over the row: the mean, then the         */
+/* centred squares.                                                         */
+void oracle_layernorm(int M, int N, const float* Z, const float* gamma, const float* beta, double eps,
+                      double* out) {
+    for (int m = 0; m < M; ++m) {
+        const float* z = Z + (size_t)m * N;
+        double sum = 0.0;
+        for (int n = 0; n < N; ++n) sum += (double)z[n];
+        double mu = sum / (double)N;
+        double sq = 0.0;
+        for (int n = 0; n < N; ++n) {
+            double d = (double)z[n] - mu;
+            sq += d * d;
+        }
+        double var = sq / (double)N;
+        double inv_sd = 1.0 / sqrt(var + eps);
+        for (int n = 0; n < N; ++n)
+            out[(size_t)m * N + n] = ((double)z[n] - mu) * inv_sd * (double)gamma[n] + (double)beta[n];
+    }
+}
+
+/* ---------------------------------------------------------------------- */
 /* Block-wise pruning with the average-magnitude heuristic (App. A.1): the  */
 /* score of a 4x1 block is the mean |w| of its four weights; the blocks     */
 /* with the lowest scores are pruned until the required sparsity ratio is   */

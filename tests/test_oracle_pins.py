@@ -310,3 +310,71 @@ def test_block_prune_brute_force():
         for r in range(n // 4):
             for c in range(k):
                 assert keep[r, c] == ((r * k + c) not in pruned)
+
+
+# ------------------------------------------------- residual add + LayerNorm --
+
+def test_layernorm_hand_case():
+    """z = [1, 2, 3, 4]: mean 2.5, variance 1.25, so the normalised row is
+    (z - 2.5) / sqrt(1.25) = [-3, -1, 1, 3] / sqrt(5)."""
+    z = np.array([[1, 2, 3, 4]], np.float32)
+    got = oracle.layernorm(z, np.ones(4, np.float32), np.zeros(4, np.float32), 0.0)
+    want = np.array([[-3, -1, 1, 3]]) / math.sqrt(5.0)
+    assert np.allclose(got, want, rtol=0, atol=1e-15)
+    # gamma and beta act per channel: 2 * norm + 3
+    got2 = oracle.layernorm(z, np.full(4, 2, np.float32), np.full(4, 3, np.float32), 0.0)
+    assert np.allclose(got2, 2 * want + 3, rtol=0, atol=1e-14)
+    # eps enters under the root: var + eps = 1.25 + 3.75 = 5 -> (z - 2.5) / sqrt(5)
+    got3 = oracle.layernorm(z, np.ones(4, np.float32), np.zeros(4, np.float32), 3.75)
+    assert np.allclose(got3, (z.astype(np.float64) - 2.5) / math.sqrt(5.0), rtol=0, atol=1e-15)
+
+
+def test_layernorm_invariants():
+    rng = np.random.default_rng(61)
+    # multiples of 2^-10 below 2^7: shifting by 64 and doubling stay exact in fp32
+    z = (np.round((rng.normal(size=(5, 768)) * 7 + 3) * 1024) / 1024).astype(np.float32)
+    g = rng.normal(size=768).astype(np.float32)
+    b = rng.normal(size=768).astype(np.float32)
+    ones, zeros = np.ones(768, np.float32), np.zeros(768, np.float32)
+    norm = oracle.layernorm(z, ones, zeros, 0.0)
+    assert np.allclose(norm.mean(axis=1), 0.0, atol=1e-12)             # zero mean
+    assert np.allclose((norm ** 2).mean(axis=1), 1.0, atol=1e-12)      # unit variance
+    # a constant row normalises to 0: the output is beta
+    const = np.full((1, 768), 4.25, np.float32)
+    assert np.array_equal(oracle.layernorm(const, g, b, 1e-5)[0], b.astype(np.float64))
+    # shifting a row (exactly representable shift) changes nothing
+    shifted = (z + np.float32(64.0)).astype(np.float32)
+    assert np.allclose(oracle.layernorm(shifted, g, b, 1e-5), oracle.layernorm(z, g, b, 1e-5), atol=1e-9)
+    # scaling a row by 2 (exact in fp32) changes nothing when eps = 0
+    assert np.allclose(oracle.layernorm(z * np.float32(2), g, b, 0.0), oracle.layernorm(z, g, b, 0.0), atol=1e-12)
+
+
+def test_linear_resid_hand_case_and_special_cases():
+    """The residual add: z = fmaf((float)acc, s, b) + res_scale * (float)r,
+    two fp32 operations."""
+    # W 4x2 holding one block [1, -2, 3, 127] in column 0; x = [[-127, 5]]:
+    # acc = [-127, 254, -381, -16129]
+    w = np.zeros((4, 2), np.int8)
+    w[:, 0] = [1, -2, 3, 127]
+    x = np.array([[-127, 5]], np.int8)
+    s = np.array([0.5, 0.25, 1.0, 0.125], np.float32)
+    b = np.array([1, -1, 0.5, 2], np.float32)
+    r = np.array([[4, -8, 0, 127]], np.int8)
+    z = oracle.linear_resid(x, w, s, b, r, 0.25)
+    # y = [-62.5, 62.5, -380.5, -2014.125]; 0.25 r = [1, -2, 0, 31.75]
+    assert z.tolist() == [[-61.5, 60.5, -380.5, -1982.375]]
+    rng = np.random.default_rng(62)
+    wt = synth.draw_weight(rng, 64, 200, 0.8)
+    wd = oracle.weight_dense(wt)
+    xx = synth.draw_x(rng, 30, 200, "u127")
+    zero = np.zeros((30, 64), np.int8)
+    y = oracle.linear(xx, wd, wt.scales, wt.bias, oracle.F32)
+    # r = 0: z is the fp32 dequantised value itself
+    assert np.array_equal(oracle.linear_resid(xx, wd, wt.scales, wt.bias, zero, 0.5), y.astype(np.float32))
+    # res_scale = 0: the same
+    rr = synth.draw_x(rng, 30, 64, "u127")
+    assert np.array_equal(oracle.linear_resid(xx, wd, wt.scales, wt.bias, rr, 0.0), y.astype(np.float32))
+    # otherwise the exact sum rounded once more (both terms are fp32)
+    z = oracle.linear_resid(xx, wd, wt.scales, wt.bias, rr, 0.03)
+    rs = (np.float32(0.03) * rr.astype(np.float32)).astype(np.float32)
+    assert np.array_equal(z, (y.astype(np.float32) + rs).astype(np.float32))
