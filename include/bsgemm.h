@@ -54,7 +54,8 @@ typedef enum {
     BSGEMM_OUT_F32 = 1,      /* float y = fmaf((float)acc, s[n], b[n])   */
     BSGEMM_OUT_F32_GELU = 2, /* float GELU(y)                           */
     BSGEMM_OUT_I8 = 3,       /* int8  q(y)                              */
-    BSGEMM_OUT_I8_GELU = 4   /* int8  q(GELU(y))                        */
+    BSGEMM_OUT_I8_GELU = 4,  /* int8  q(GELU(y))                        */
+    BSGEMM_OUT_F32_RESID = 5 /* float z = y + residual_scale * residual */
 } bsgemm_out_kind;
 
 typedef struct {
@@ -62,6 +63,10 @@ typedef struct {
     float out_scale; /* int8 kinds only: finite and > 0; the library         */
                      /* multiplies by 1.0f / out_scale (one fp32 division)   */
     uint32_t flags;  /* 0 or BSGEMM_ACT_READY; other bits are invalid        */
+    const int8_t* residual; /* BSGEMM_OUT_F32_RESID only: DEVICE int8 [M][N], */
+                            /* 4-byte aligned (the sub-layer's input that the */
+                            /* encoder adds before LayerNorm, Sec. 3)         */
+    float residual_scale;   /* its scale, finite                              */
 } bsgemm_epilogue;
 
 /*
@@ -249,6 +254,25 @@ int bsgemm_run_host(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epil
  * non-finite weight; `keep` is then undefined) or BSGEMM_ERR_CUDA.
  */
 int64_t bsgemm_block_prune(int N, int K, const float* W, double sparsity, uint8_t* keep, void* stream);
+
+/*
+ * bsgemm_layernorm -- LayerNorm of each row of z (the post-operator that
+ * Sec. 3's optimized INT8 graph fuses after the output projection and FFN2;
+ * with BSGEMM_OUT_F32_RESID the residual add before it happens in the
+ * linear's epilogue):
+ *   out[m][n] = (z[m][n] - mean_m) / sqrt(var_m + eps) * gamma[n] + beta[n]
+ * with the row mean and centred variance accumulated in double, the
+ * normalised value rounded to fp32 and combined by one fmaf with gamma and
+ * beta; for int8 output requantised as the linear's epilogue does.
+ *   z      DEVICE float [M][N];  gamma, beta DEVICE float [N].
+ *   out    DEVICE [M][N], float (epi.kind BSGEMM_OUT_F32) or int8
+ *          (BSGEMM_OUT_I8, epi.out_scale as for bsgemm_run); must not overlap z.
+ *   eps    >= 0, finite.
+ * One kernel (a warp a row) on `stream`, asynchronous; M = 0 is a no-op.
+ * Returns BSGEMM_OK, BSGEMM_ERR_INVALID or BSGEMM_ERR_CUDA.
+ */
+int bsgemm_layernorm(const float* z, int M, int N, const float* gamma, const float* beta, float eps, void* out,
+                     bsgemm_epilogue epi, void* stream);
 
 /*
  * bsgemm_device_status -- read (and with clear != 0, reset) the handle's

@@ -24,7 +24,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libbsgemm.so")
 
 BLOCK = 4
-OUT_I32, OUT_F32, OUT_F32_GELU, OUT_I8, OUT_I8_GELU = 0, 1, 2, 3, 4
+OUT_I32, OUT_F32, OUT_F32_GELU, OUT_I8, OUT_I8_GELU, OUT_F32_RESID = 0, 1, 2, 3, 4, 5
 ERR_INVALID, ERR_UNSUPPORTED, ERR_CUDA = -1, -2, -3
 STATIC_SCRATCH_BYTES = 16 << 20  # BSGEMM_STATIC_SCRATCH_BYTES: the token-tile scratch of bsgemm_run_static
 
@@ -39,7 +39,8 @@ ACT_READY = 1  # BSGEMM_ACT_READY: act may be read while the stream's previous k
 
 
 class Epilogue(ctypes.Structure):
-    _fields_ = [("kind", ctypes.c_int32), ("out_scale", ctypes.c_float), ("flags", ctypes.c_uint32)]
+    _fields_ = [("kind", ctypes.c_int32), ("out_scale", ctypes.c_float), ("flags", ctypes.c_uint32),
+                ("residual", ctypes.c_void_p), ("residual_scale", ctypes.c_float)]
 
 
 def _load() -> ctypes.CDLL:
@@ -79,6 +80,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_run_host.restype = ctypes.c_int
     lib.bsgemm_block_prune.argtypes = [ctypes.c_int, ctypes.c_int, vp, ctypes.c_double, vp, vp]
     lib.bsgemm_block_prune.restype = ctypes.c_int64
+    lib.bsgemm_layernorm.argtypes = [vp, ctypes.c_int, ctypes.c_int, vp, vp, ctypes.c_float, vp, Epilogue, vp]
+    lib.bsgemm_layernorm.restype = ctypes.c_int
     lib.bsgemm_device_status.argtypes = [vp, ctypes.c_int]
     lib.bsgemm_device_status.restype = ctypes.c_int
     return lib
@@ -88,8 +91,13 @@ _lib = _load()
 
 EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
             "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_run_kmajor",
-            "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_destroy",
+            "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_layernorm",
+            "bsgemm_destroy",
             "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
+
+
+def _epi(kind: int, out_scale: float, flags: int = 0, residual: int = 0, residual_scale: float = 1.0) -> Epilogue:
+    return Epilogue(int(kind), float(out_scale), int(flags), residual or None, float(residual_scale))
 
 
 def bsgemm_last_error() -> str:
@@ -124,19 +132,21 @@ def bsgemm_create(n_out: int, k_in: int, block: int, indices, values, scales, bi
 
 
 def bsgemm_run(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float = 1.0,
-               stream: int = 0, flags: int = 0) -> None:
+               stream: int = 0, flags: int = 0, residual_ptr: int = 0, residual_scale: float = 1.0) -> None:
     """Enqueue one run on `stream` (raw device pointers); raises on failure."""
-    rc = _lib.bsgemm_run(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale), int(flags)), stream)
+    rc = _lib.bsgemm_run(h, act_ptr, int(m), out_ptr, _epi(kind, out_scale, flags, residual_ptr, residual_scale),
+                         stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 
 
 def bsgemm_run_ws(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float, ws_ptr: int,
-                  ws_bytes: int, stream: int = 0, flags: int = 0) -> None:
+                  ws_bytes: int, stream: int = 0, flags: int = 0, residual_ptr: int = 0,
+                  residual_scale: float = 1.0) -> None:
     """Enqueue a run with a device workspace (used only by the shapes that
     need the relayout kernel); raises on failure."""
-    rc = _lib.bsgemm_run_ws(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale), int(flags)), ws_ptr,
-                            int(ws_bytes), stream)
+    rc = _lib.bsgemm_run_ws(h, act_ptr, int(m), out_ptr, _epi(kind, out_scale, flags, residual_ptr, residual_scale),
+                            ws_ptr, int(ws_bytes), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 
@@ -145,7 +155,7 @@ def bsgemm_run_static(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out
                       stream: int = 0) -> None:
     """The fast path with the library's fixed device scratch: allocates
     nothing; calls overlapping in time on one device race (see the header)."""
-    rc = _lib.bsgemm_run_static(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), stream)
+    rc = _lib.bsgemm_run_static(h, act_ptr, int(m), out_ptr, _epi(kind, out_scale), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 
@@ -154,7 +164,7 @@ def bsgemm_run_kmajor(h: int, act_t_ptr: int, m: int, ld: int, out_ptr: int, kin
                       stream: int = 0, flags: int = 0) -> None:
     """The layer on K-major activations X^T [K][M] (row stride ld bytes)."""
     rc = _lib.bsgemm_run_kmajor(h, act_t_ptr, int(m), int(ld), out_ptr,
-                                Epilogue(int(kind), float(out_scale), int(flags)), stream)
+                                _epi(kind, out_scale, flags), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 
@@ -167,7 +177,7 @@ def bsgemm_tile_activations(h: int, act_ptr: int, m: int, tiles_ptr: int, tiles_
 
 def bsgemm_run_tiled(h: int, tiles_ptr: int, tiles_bytes: int, m: int, out_ptr: int, kind: int, out_scale: float,
                      stream: int = 0) -> None:
-    rc = _lib.bsgemm_run_tiled(h, tiles_ptr, int(tiles_bytes), int(m), out_ptr, Epilogue(int(kind), float(out_scale)),
+    rc = _lib.bsgemm_run_tiled(h, tiles_ptr, int(tiles_bytes), int(m), out_ptr, _epi(kind, out_scale),
                                stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
@@ -176,7 +186,7 @@ def bsgemm_run_tiled(h: int, tiles_ptr: int, tiles_bytes: int, m: int, out_ptr: 
 def bsgemm_run_host(h: int, act_ptr: int, m: int, out_ptr: int, kind: int, out_scale: float, ws_ptr: int,
                     ws_bytes: int, stream: int = 0) -> None:
     """Enqueue the end-to-end call: HOST act and out, a DEVICE workspace."""
-    rc = _lib.bsgemm_run_host(h, act_ptr, int(m), out_ptr, Epilogue(int(kind), float(out_scale)), ws_ptr,
+    rc = _lib.bsgemm_run_host(h, act_ptr, int(m), out_ptr, _epi(kind, out_scale), ws_ptr,
                               int(ws_bytes), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
@@ -210,6 +220,32 @@ def block_prune(w, sparsity: float, stream=None):
     return keep
 
 
+def bsgemm_layernorm(z_ptr: int, m: int, n: int, gamma_ptr: int, beta_ptr: int, eps: float, out_ptr: int, kind: int,
+                     out_scale: float = 1.0, stream: int = 0) -> None:
+    """Enqueue the row-wise LayerNorm of z [M][N] fp32 (raw device pointers)."""
+    rc = _lib.bsgemm_layernorm(z_ptr, int(m), int(n), gamma_ptr, beta_ptr, float(eps), out_ptr, _epi(kind, out_scale),
+                               stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def layernorm(z, gamma, beta, eps: float, kind: int = OUT_F32, out_scale: float = 1.0, stream=None):
+    """LayerNorm of each row of the CUDA fp32 tensor z [M][N] (gamma, beta:
+    CUDA fp32 [N]); returns a new CUDA tensor, float32 or int8 by kind."""
+    import torch
+    for t, name in ((z, "z"), (gamma, "gamma"), (beta, "beta")):
+        if t.dtype != torch.float32 or not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA float32 tensor")
+    m, n = z.shape
+    if tuple(gamma.shape) != (n,) or tuple(beta.shape) != (n,):
+        raise ValueError("gamma and beta must be [N]")
+    out = torch.empty((m, n), dtype=torch.int8 if kind == OUT_I8 else torch.float32, device=z.device)
+    s = torch.cuda.current_stream() if stream is None else stream
+    bsgemm_layernorm(z.data_ptr(), m, n, gamma.data_ptr(), beta.data_ptr(), eps, out.data_ptr(), kind, out_scale,
+                     s.cuda_stream)
+    return out
+
+
 def bsgemm_workspace_bytes(h: int, m: int) -> int:
     return int(_lib.bsgemm_workspace_bytes(h, int(m)))
 
@@ -234,7 +270,8 @@ def bsgemm_info(h: int) -> dict:
     return dict(zip(keys, (int(v) for v in buf)))
 
 
-_OUT_DTYPES = {OUT_I32: "int32", OUT_F32: "float32", OUT_F32_GELU: "float32", OUT_I8: "int8", OUT_I8_GELU: "int8"}
+_OUT_DTYPES = {OUT_I32: "int32", OUT_F32: "float32", OUT_F32_GELU: "float32", OUT_I8: "int8", OUT_I8_GELU: "int8",
+               OUT_F32_RESID: "float32"}
 
 
 def dense_to_blocks(w: np.ndarray, keep=None):
@@ -284,7 +321,7 @@ class SparseInt8Linear:
         return bsgemm_workspace_bytes(self._h, m)
 
     def run(self, x, out, kind: int, out_scale: float = 1.0, stream=None, workspace=None,
-            act_ready: bool = False) -> None:
+            act_ready: bool = False, residual=None, residual_scale: float = 1.0) -> None:
         """out[M][N] = epilogue(x[M][K] W^T); both CUDA tensors, contiguous.
 
         With K % 16 == 0 and x 16-byte aligned this is one kernel that stages
@@ -292,8 +329,10 @@ class SparseInt8Linear:
         the given uint8 CUDA tensor, or (workspace=None) one drawn from
         PyTorch's caching allocator on the same stream -- takes the relaid
         tiles, and workspace=False gathers them with per-thread loads
-        instead.  act_ready: x was complete
-        before the stream's previous kernel began (BSGEMM_ACT_READY)."""
+        instead.  act_ready: x was complete before the stream's previous
+        kernel began (BSGEMM_ACT_READY).  OUT_F32_RESID adds residual_scale *
+        residual (a contiguous CUDA int8 [M][N] tensor) to the dequantised
+        value (the residual add before LayerNorm)."""
         import torch
         if x.dtype != torch.int8 or not x.is_cuda or not x.is_contiguous() or x.dim() != 2 or x.shape[1] != self.k_in:
             raise ValueError("x must be a contiguous CUDA int8 tensor [M][K]")
@@ -303,8 +342,15 @@ class SparseInt8Linear:
         s = torch.cuda.current_stream() if stream is None else stream
         m = x.shape[0]
         flags = ACT_READY if act_ready else 0
+        res_ptr = 0
+        if kind == OUT_F32_RESID:
+            if (residual is None or residual.dtype != torch.int8 or not residual.is_cuda
+                    or not residual.is_contiguous() or tuple(residual.shape) != (m, self.n_out)):
+                raise ValueError("OUT_F32_RESID needs a contiguous CUDA int8 residual [M][N]")
+            res_ptr = residual.data_ptr()
         if workspace is False or m == 0:
-            bsgemm_run(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, s.cuda_stream, flags)
+            bsgemm_run(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, s.cuda_stream, flags, res_ptr,
+                       residual_scale)
             return
         need = self.workspace_bytes(m)
         if workspace is None:
@@ -313,7 +359,7 @@ class SparseInt8Linear:
         if workspace.numel() * workspace.element_size() < need:
             raise ValueError(f"workspace must hold {need} bytes")
         bsgemm_run_ws(self._h, x.data_ptr(), m, out.data_ptr(), kind, out_scale, workspace.data_ptr(),
-                      workspace.numel() * workspace.element_size(), s.cuda_stream, flags)
+                      workspace.numel() * workspace.element_size(), s.cuda_stream, flags, res_ptr, residual_scale)
 
     def run_kmajor(self, xt, out, kind: int, out_scale: float = 1.0, stream=None) -> None:
         """out[M][N] = epilogue(X W^T) from K-major activations: xt is a CUDA

@@ -383,8 +383,13 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
     if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
-    if (epi.kind < BSGEMM_OUT_I32 || epi.kind > BSGEMM_OUT_I8_GELU)
+    if (epi.kind < BSGEMM_OUT_I32 || epi.kind > BSGEMM_OUT_F32_RESID)
         return fail(BSGEMM_ERR_INVALID, "unknown epilogue kind " + std::to_string(epi.kind));
+    if (epi.kind == BSGEMM_OUT_F32_RESID && M > 0) {
+        if (!epi.residual || reinterpret_cast<uintptr_t>(epi.residual) % 4 != 0)
+            return fail(BSGEMM_ERR_INVALID, "the residual must be a 4-byte aligned device array");
+        if (!std::isfinite(epi.residual_scale)) return fail(BSGEMM_ERR_INVALID, "residual_scale must be finite");
+    }
     if (epi.flags & ~static_cast<uint32_t>(BSGEMM_ACT_READY))
         return fail(BSGEMM_ERR_INVALID, "unknown bits in epi.flags");
     float inv = 0.0f;
@@ -428,6 +433,8 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.kmajor = mode == 3;
     a.ld = ld;
     a.act_ready = (epi.flags & BSGEMM_ACT_READY) != 0 && (tensor || mode == 3);
+    a.res = epi.residual;
+    a.res_scale = epi.residual_scale;
     a.out = out;
     a.M = M;
     a.kind = epi.kind;
@@ -530,8 +537,8 @@ size_t bsgemm_workspace_bytes(bsgemm_t h, int M) {
 // Workspace of bsgemm_run_host: [act copy | token tiles | device result],
 // each part at a 256-byte aligned offset.  Returns 0 for an unknown kind.
 static size_t host_parts(bsgemm_t h, int M, int32_t kind, size_t* off_tiles, size_t* off_out, size_t* out_bytes) {
-    static const size_t elem[5] = {4, 4, 4, 1, 1};
-    if (kind < BSGEMM_OUT_I32 || kind > BSGEMM_OUT_I8_GELU) return 0;
+    static const size_t elem[6] = {4, 4, 4, 1, 1, 4};
+    if (kind < BSGEMM_OUT_I32 || kind > BSGEMM_OUT_F32_RESID) return 0;
     const size_t m = static_cast<size_t>(M);
     *off_tiles = align_up(m * static_cast<size_t>(h->w.K), 256);
     *off_out = *off_tiles + align_up(bsg::tiled_bytes(h->w.K, M), 256);
@@ -550,7 +557,7 @@ int bsgemm_run_host(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epil
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
     if (M < 0) return fail(BSGEMM_ERR_INVALID, "M must be >= 0");
-    if (epi.kind < BSGEMM_OUT_I32 || epi.kind > BSGEMM_OUT_I8_GELU)
+    if (epi.kind < BSGEMM_OUT_I32 || epi.kind > BSGEMM_OUT_F32_RESID)
         return fail(BSGEMM_ERR_INVALID, "unknown epilogue kind " + std::to_string(epi.kind));
     if (M == 0) return BSGEMM_OK;
     if (!act || !out) return fail(BSGEMM_ERR_INVALID, "act and out must not be NULL");
@@ -598,6 +605,28 @@ int64_t bsgemm_block_prune(int N, int K, const float* W, double sparsity, uint8_
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("block pruning", e));
     if (bad) return fail(BSGEMM_ERR_INVALID, "W holds a value that is not finite");
     return total - npruned;
+}
+
+int bsgemm_layernorm(const float* z, int M, int N, const float* gamma, const float* beta, float eps, void* out,
+                     bsgemm_epilogue epi, void* stream) {
+    clear_error();
+    if (M < 0 || N < 1) return fail(BSGEMM_ERR_INVALID, "need M >= 0 and N >= 1");
+    if (epi.kind != BSGEMM_OUT_F32 && epi.kind != BSGEMM_OUT_I8)
+        return fail(BSGEMM_ERR_INVALID, "LayerNorm writes BSGEMM_OUT_F32 or BSGEMM_OUT_I8");
+    if (!(eps >= 0.0f) || !std::isfinite(eps)) return fail(BSGEMM_ERR_INVALID, "eps must be finite and >= 0");
+    float inv = 0.0f;
+    if (epi.kind == BSGEMM_OUT_I8) {
+        if (!(epi.out_scale > 0.0f) || !std::isfinite(epi.out_scale))
+            return fail(BSGEMM_ERR_INVALID, "out_scale must be finite and > 0 for int8 outputs");
+        inv = 1.0f / epi.out_scale;
+        if (!std::isfinite(inv)) return fail(BSGEMM_ERR_INVALID, "1 / out_scale overflows fp32");
+    }
+    if (M == 0) return BSGEMM_OK;
+    if (!z || !gamma || !beta || !out) return fail(BSGEMM_ERR_INVALID, "z, gamma, beta and out must not be NULL");
+    const cudaError_t e = bsg::launch_layernorm(z, M, N, gamma, beta, eps, epi.kind, inv, out,
+                                                static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("LayerNorm launch", e));
+    return BSGEMM_OK;
 }
 
 int bsgemm_device_status(bsgemm_t h, int clear) {

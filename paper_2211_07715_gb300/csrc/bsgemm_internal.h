@@ -69,6 +69,8 @@ struct LaunchArgs {
     bool tensor;           // stage tiles from x by tensor copies (xb unused; needs tensor_staging())
     bool kmajor;           // x is x^T [K][M] with row stride ld: tensor copies, no transpose
     bool act_ready;        // x may be read before the previous kernel completes (BSGEMM_ACT_READY)
+    const int8_t* res;     // kind 5: int8 residual [M][N]
+    float res_scale;       // kind 5: the residual's scale
     int ld;                // row stride of x^T in bytes (kmajor only)
 };
 
@@ -101,6 +103,9 @@ bool tensor_staging(int K, const void* x);
 int max_k();                               // largest K a tile supports
 cudaError_t prepare_kernels(int K, int* ctas_per_sm);  // set attributes, occupancy
 cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int grid, cudaStream_t s);
+// Row-wise LayerNorm of z [M][N] (kind 1: fp32 out, 3: int8 out).
+cudaError_t launch_layernorm(const float* z, int M, int N, const float* gamma, const float* beta, float eps, int kind,
+                             float inv_out_scale, void* out, cudaStream_t s);
 // x [M][K] -> swizzled token tiles in xb (the layout the kernel stages by TMA).
 cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, cudaStream_t s);
 // Average-magnitude block pruning of a dense fp32 W [N][K] (DEVICE) into

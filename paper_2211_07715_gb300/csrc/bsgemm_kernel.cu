@@ -193,7 +193,14 @@ __device__ __forceinline__ void store_token(const LaunchArgs& a, int N, long lon
         y2 = gelu_f32(y2);
         y3 = gelu_f32(y3);
     }
-    if (KIND == 1 || KIND == 2) {
+    if (KIND == 5) {  // residual add: z = y + res_scale * (float)r, two fp32 operations
+        const uint32_t r4 = __ldg(reinterpret_cast<const uint32_t*>(a.res + o));
+        y0 = __fadd_rn(y0, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4))));
+        y1 = __fadd_rn(y1, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4 >> 8))));
+        y2 = __fadd_rn(y2, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4 >> 16))));
+        y3 = __fadd_rn(y3, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4 >> 24))));
+    }
+    if (KIND == 1 || KIND == 2 || KIND == 5) {
         *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y0, y1, y2, y3);
     } else {
         *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = requant4_s8(y0, y1, y2, y3, a.inv_out_scale);
@@ -221,6 +228,13 @@ __device__ __forceinline__ void store_lane_narrow(const LaunchArgs& a, int N, lo
 #pragma unroll
             for (int c = 0; c < 4; ++c)
                 if (c < nc) static_cast<float*>(a.out)[o + c] = epilogue_value<KIND>(acc[4 * i + c], s4[c], b4[c]);
+        } else if (KIND == 5) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < nc)
+                    static_cast<float*>(a.out)[o + c] =
+                        __fadd_rn(epilogue_value<1>(acc[4 * i + c], s4[c], b4[c]),
+                                  __fmul_rn(a.res_scale, __int2float_rn(a.res[o + c])));
         } else {
             float y[4];
 #pragma unroll
@@ -889,7 +903,8 @@ const void* kernel_for(int kind) {
     case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<1, MODE>);
     case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<2, MODE>);
     case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<3, MODE>);
-    default: return reinterpret_cast<const void*>(&bsgemm_kernel<4, MODE>);
+    case 4: return reinterpret_cast<const void*>(&bsgemm_kernel<4, MODE>);
+    default: return reinterpret_cast<const void*>(&bsgemm_kernel<5, MODE>);
     }
 }
 const void* kernel_for(int kind, int mode) {
@@ -938,7 +953,7 @@ int max_k() {
 
 cudaError_t prepare_kernels(int K, int* ctas_per_sm) {
     const int smem = static_cast<int>(smem_bytes(K));
-    for (int kind = 0; kind < 5; ++kind) {
+    for (int kind = 0; kind < 6; ++kind) {
         for (int mode = 0; mode < 4; ++mode) {
             cudaError_t e = cudaFuncSetAttribute(kernel_for(kind, mode), cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  kSmemOptin - kStaticSmem);
@@ -1006,10 +1021,56 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
     case 1: BSG_LAUNCH(1); break;
     case 2: BSG_LAUNCH(2); break;
     case 3: BSG_LAUNCH(3); break;
-    default: BSG_LAUNCH(4); break;
+    case 4: BSG_LAUNCH(4); break;
+    default: BSG_LAUNCH(5); break;
     }
 #undef BSG_LAUNCH
     return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+// LayerNorm of each row of z [M][N] fp32 (the post-operator the optimized
+// INT8 graph fuses after the output projection and FFN2, Sec. 3 "Graph
+// optimization"): one warp a row.  Mean and centred variance accumulate in
+// double (the row is read three times, from L1 after the first), then
+// out = fmaf((float)((z - mean) * rstd), gamma, beta), fp32 or requantised
+// to int8 (kind 3: fp32 multiply by 1 / out_scale, round half even,
+// saturate).  Rows past M do nothing.
+__global__ void __launch_bounds__(256)
+layernorm_kernel(const float* __restrict__ z, int M, int N, const float* __restrict__ gamma,
+                 const float* __restrict__ beta, float eps, int kind, float inv_out_scale, void* __restrict__ out) {
+    const int lane = threadIdx.x & 31;
+    const long long m = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (m >= M) return;
+    const float* row = z + m * N;
+    double sum = 0.0;
+    for (int n = lane; n < N; n += 32) sum += static_cast<double>(__ldg(row + n));
+    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    const double mean = sum / N;
+    double sq = 0.0;
+    for (int n = lane; n < N; n += 32) {
+        const double d = static_cast<double>(__ldg(row + n)) - mean;
+        sq += d * d;
+    }
+    for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+    const double rstd = 1.0 / sqrt(sq / N + static_cast<double>(eps));
+    for (int n = lane; n < N; n += 32) {
+        const float t = static_cast<float>((static_cast<double>(__ldg(row + n)) - mean) * rstd);
+        const float v = __fmaf_rn(t, __ldg(gamma + n), __ldg(beta + n));
+        if (kind == 3) {
+            const int q = __float2int_rn(__fmul_rn(v, inv_out_scale));
+            static_cast<int8_t*>(out)[m * N + n] = static_cast<int8_t>(q > 127 ? 127 : (q < -128 ? -128 : q));
+        } else {
+            static_cast<float*>(out)[m * N + n] = v;
+        }
+    }
+}
+
+cudaError_t launch_layernorm(const float* z, int M, int N, const float* gamma, const float* beta, float eps, int kind,
+                             float inv_out_scale, void* out, cudaStream_t s) {
+    const int rows_per_block = 8;
+    const unsigned grid = static_cast<unsigned>((static_cast<long long>(M) + rows_per_block - 1) / rows_per_block);
+    layernorm_kernel<<<grid, 32 * rows_per_block, 0, s>>>(z, M, N, gamma, beta, eps, kind, inv_out_scale, out);
+    return cudaGetLastError();
 }
 
 size_t tiled_bytes(int K, long long M) {
