@@ -669,6 +669,130 @@ def run_layer(args) -> dict:
     }
 
 
+def run_encoder(args) -> dict:
+    """cfg 4 as an encoder layer with its sub-layer ends (Sec. 3's fused
+    post-operators): QKV -> [attention: a seeded int8 context buffer, outside
+    the timed path] -> attention output + residual (the layer input) ->
+    LayerNorm -> FFN1 + GELU -> FFN2 + residual (the first LayerNorm's
+    output) -> LayerNorm; int8 between.  The residual adds run in the
+    linears' epilogues (BSGEMM_OUT_F32_RESID), each LayerNorm is one kernel.
+    M = 8 x 384 tokens, 80% block sparsity.  Scales: the layer chain's
+    calibrated ones for QKV and FFN1; 0.02 for the input as a residual and
+    4/127 for the LayerNorm outputs (synthetic constants)."""
+    import torch
+    import paper_2211_07715_gb300 as bsg
+
+    dev = torch.device("cuda", 0)
+    props = torch.cuda.get_device_properties(dev)
+    with open(LAYER_SCALES) as f:
+        scales = json.load(f)["scales"]
+    weights, x0 = synth.encoder_layer()
+    m = x0.shape[0]
+    lins = _layer_linears(bsg, weights)
+    rng = synth.rng_for(synth.SEED_BASE + 80)
+    g1, b1, g2, b2 = (torch.from_numpy(a).to(dev) for a in (
+        rng.normal(1.0, 0.1, 768).astype(np.float32), rng.normal(0.0, 0.1, 768).astype(np.float32),
+        rng.normal(1.0, 0.1, 768).astype(np.float32), rng.normal(0.0, 0.1, 768).astype(np.float32)))
+    x_scale, ln_scale, eps = 0.02, 4.0 / 127.0, 1e-12
+    ctx_host = synth.draw_x(synth.rng_for(synth.SEED_BASE + 3 + 7), m, 768, "u127")
+    set_bytes = m * (768 * 2 + 2304 + 768 * 4 * 2 + 768 * 2 + 3072)
+    nsets = max(2, math.ceil(2 * int(getattr(props, "L2_cache_size", 128 << 20)) / set_bytes) + 1)
+    xs = [torch.from_numpy(x0).to(dev) for _ in range(nsets)]
+    ctxs = [torch.from_numpy(ctx_host).to(dev) for _ in range(nsets)]
+    t = torch
+    bufs = [{"qkv": t.empty((m, 2304), dtype=t.int8, device=dev), "z1": t.empty((m, 768), dtype=t.float32, device=dev),
+             "h1": t.empty((m, 768), dtype=t.int8, device=dev), "f1": t.empty((m, 3072), dtype=t.int8, device=dev),
+             "z2": t.empty((m, 768), dtype=t.float32, device=dev), "h2": t.empty((m, 768), dtype=t.int8, device=dev)}
+            for _ in range(nsets)]
+    ln_kernels = []
+
+    def layer(i, s):
+        b, sh = bufs[i % nsets], s.cuda_stream
+        x, ctx = xs[i % nsets], ctxs[i % nsets]
+        bsg.bsgemm_run(lins[0]._h, x.data_ptr(), m, b["qkv"].data_ptr(), synth.I8, scales["qkv"], sh)
+        bsg.bsgemm_run(lins[1]._h, ctx.data_ptr(), m, b["z1"].data_ptr(), bsg.OUT_F32_RESID, 1.0, sh, 0,
+                       x.data_ptr(), x_scale)
+        bsg.bsgemm_layernorm(b["z1"].data_ptr(), m, 768, g1.data_ptr(), b1.data_ptr(), eps, b["h1"].data_ptr(),
+                             bsg.OUT_I8, ln_scale, sh)
+        bsg.bsgemm_run(lins[2]._h, b["h1"].data_ptr(), m, b["f1"].data_ptr(), synth.I8_GELU, scales["ffn1"], sh)
+        bsg.bsgemm_run(lins[3]._h, b["f1"].data_ptr(), m, b["z2"].data_ptr(), bsg.OUT_F32_RESID, 1.0, sh, 0,
+                       b["h1"].data_ptr(), ln_scale)
+        bsg.bsgemm_layernorm(b["z2"].data_ptr(), m, 768, g2.data_ptr(), b2.data_ptr(), eps, b["h2"].data_ptr(),
+                             bsg.OUT_I8, ln_scale, sh)
+
+    stream = torch.cuda.current_stream(dev)
+    for i in range(nsets):
+        layer(i, stream)
+    torch.cuda.synchronize(dev)
+    steps = args.steps
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(stream)
+
+    def graph_ms(body, n):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            for i in range(n):
+                body(i, side)
+        torch.cuda.synchronize(dev)
+        g.replay()
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        e1.synchronize()
+        return e0.elapsed_time(e1) / n
+
+    sampler = ClockSampler(str(getattr(props, "uuid", "")))
+    sampler.start()
+    time.sleep(0.3)
+    mark0 = sampler.mark()
+    ms = graph_ms(layer, steps)
+    mark1 = sampler.mark()
+    time.sleep(0.2)
+    sampler.stop()
+    clocks = sampler.summary(mark0, max(mark1, mark0 + 1))
+    reps = min(steps, 200)
+
+    def ln_only(i, s):
+        b = bufs[i % nsets]
+        bsg.bsgemm_layernorm(b["z1"].data_ptr(), m, 768, g1.data_ptr(), b1.data_ptr(), eps, b["h1"].data_ptr(),
+                             bsg.OUT_I8, ln_scale, s.cuda_stream)
+
+    ln_ms = graph_ms(ln_only, reps)
+    ops = [2.0 * m * w.nnzb * 4 for w in weights]
+    peak = _peak_tops(props, clocks.get("sm_max_mhz") or 2070.0)
+    hbm_peak = 6683.8
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            hbm_peak = float(json.load(f).get("hbm_gbs", hbm_peak))
+    except (OSError, ValueError):
+        pass
+    ln_bytes = m * 768 * 4 + m * 768 + 2 * 768 * 4  # z read once, int8 out, gamma and beta
+    for lin in lins:
+        lin.close()
+    return {
+        "metric": METRIC, "value": round(sum(ops) / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "n_gpus": 1,
+        "steps": steps, "warmup": args.warmup, "ms_per_step": round(ms, 6), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "s8", "data": "synthetic",
+        "config": {"workload": "encoder layer with residual adds and LayerNorms: QKV, [attention: seeded int8 "
+                               "context], attention output + residual -> LayerNorm, FFN1 + GELU, FFN2 + residual "
+                               "-> LayerNorm; int8 between",
+                   "tokens": m, "batch": 8, "seq": 384, "sparsity": 0.8,
+                   "l2": f"rotating {nsets} sets ({nsets * set_bytes / 2**20:.0f} MiB > 2 x L2)",
+                   "launch": "the timed passes are one CUDA graph of --steps passes (6 launches each)"},
+        "tokens_per_s": round(m / (ms * 1e-3), 1),
+        "layernorm": {"kernel": "layernorm_kernel", "ms": round(ln_ms, 6),
+                      "gbs": round(ln_bytes / (ln_ms * 1e-3) / 1e9, 1),
+                      "hbm_frac": round(ln_bytes / (ln_ms * 1e-3) / 1e9 / hbm_peak, 4),
+                      "basis": "graph of 200 LayerNorm launches, per launch; bytes = fp32 z read once + int8 out"},
+        "roofline": {"bound": "alu", "achieved": round(sum(ops) / (ms * 1e-3) / 1e12, 3), "peak": round(peak, 2),
+                     "unit": "TOPS", "frac": round(sum(ops) / (ms * 1e-3) / 1e12 / peak, 4), "traffic": None,
+                     "kernel": "whole layer (4 linears + 2 LayerNorms)"},
+        "gpu_launches": 6 * steps, "clocks": clocks, "kernel_source_sha256": kernel_sha(),
+    }
+
+
 def run_stack(args) -> dict:
     """cfg 5: the six-layer stack of 24 sparse linears swept over batch
     {1, 8, 32, 128} x seq {128, 384} x sparsity {70, 80, 90}%.  One pass =
@@ -1004,9 +1128,11 @@ def main():
     p.add_argument("--steps", type=int, default=2000)
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "stack", "prune", "production"], default="ffn2",
+    p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "encoder", "stack", "prune", "production"],
+                   default="ffn2",
                    help="ffn2/ffn1/single: one linear; layer: the encoder layer's four linears; stack: the "
-                        "six-layer stack sweep; prune: create-side block pruning of an FFN2-shaped weight; "
+                        "six-layer stack sweep; encoder: the layer with residual adds and LayerNorms; "
+                        "prune: create-side block pruning of an FFN2-shaped weight; "
                         "production: maximum samples/s under 10 ms per batch")
     p.add_argument("--ref-rows", type=int, default=512, help="tokens per reference step")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -1020,7 +1146,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
-        if args.workload in ("layer", "stack", "production"):
+        if args.workload in ("layer", "encoder", "stack", "production"):
             p.error("--impl reference times the single-linear workloads and prune")
         res = run_reference(args, rank)
     else:
@@ -1031,6 +1157,8 @@ def main():
             dist.init_process_group("nccl")
         if args.workload == "layer":
             res = run_layer(args) if rank == 0 else None
+        elif args.workload == "encoder":
+            res = run_encoder(args) if rank == 0 else None
         elif args.workload == "stack":
             res = run_stack(args) if rank == 0 else None
         elif args.workload == "prune":

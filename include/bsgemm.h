@@ -261,9 +261,10 @@ int64_t bsgemm_block_prune(int N, int K, const float* W, double sparsity, uint8_
  * with BSGEMM_OUT_F32_RESID the residual add before it happens in the
  * linear's epilogue):
  *   out[m][n] = (z[m][n] - mean_m) / sqrt(var_m + eps) * gamma[n] + beta[n]
- * with the row mean and centred variance accumulated in double, the
- * normalised value rounded to fp32 and combined by one fmaf with gamma and
- * beta; for int8 output requantised as the linear's epilogue does.
+ * in fp32: the row mean as the first value plus the mean of the
+ * deviations from it, the variance from the centred squares, then one fmaf
+ * with gamma and beta; for int8 output requantised as the linear's
+ * epilogue does.
  *   z      DEVICE float [M][N];  gamma, beta DEVICE float [N].
  *   out    DEVICE [M][N], float (epi.kind BSGEMM_OUT_F32) or int8
  *          (BSGEMM_OUT_I8, epi.out_scale as for bsgemm_run); must not overlap z.

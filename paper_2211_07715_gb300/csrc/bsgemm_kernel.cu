@@ -1030,11 +1030,29 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
 
 // LayerNorm of each row of z [M][N] fp32 (the post-operator the optimized
 // INT8 graph fuses after the output projection and FFN2, Sec. 3 "Graph
-// optimization"): one warp a row.  Mean and centred variance accumulate in
-// double (the row is read three times, from L1 after the first), then
-// out = fmaf((float)((z - mean) * rstd), gamma, beta), fp32 or requantised
-// to int8 (kind 3: fp32 multiply by 1 / out_scale, round half even,
-// saturate).  Rows past M do nothing.
+// optimization"): one warp a row, fp32 throughout (GB300's fp64 rate is a
+// small fraction of its fp32 rate).  The mean is the row's first value c
+// plus the mean of (z - c) -- summing deviations from a value of the row
+// keeps the rounding small when the mean is large against the spread --
+// then the variance from the centred squares; out = fmaf((z - mean) *
+// rstd, gamma, beta), fp32 or requantised to int8 (kind 3: fp32 multiply
+// by 1 / out_scale, round half even, saturate).  With N % 4 == 0 and
+// 16-byte aligned arrays the row moves as float4 (and 4-byte int8 words).
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ void ln_store(int kind, void* out, long long idx, float v, float inv) {
+    if (kind == 3) {
+        const int q = __float2int_rn(__fmul_rn(v, inv));
+        static_cast<int8_t*>(out)[idx] = static_cast<int8_t>(q > 127 ? 127 : (q < -128 ? -128 : q));
+    } else {
+        static_cast<float*>(out)[idx] = v;
+    }
+}
+
 __global__ void __launch_bounds__(256)
 layernorm_kernel(const float* __restrict__ z, int M, int N, const float* __restrict__ gamma,
                  const float* __restrict__ beta, float eps, int kind, float inv_out_scale, void* __restrict__ out) {
@@ -1042,26 +1060,53 @@ layernorm_kernel(const float* __restrict__ z, int M, int N, const float* __restr
     const long long m = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (m >= M) return;
     const float* row = z + m * N;
-    double sum = 0.0;
-    for (int n = lane; n < N; n += 32) sum += static_cast<double>(__ldg(row + n));
-    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-    const double mean = sum / N;
-    double sq = 0.0;
-    for (int n = lane; n < N; n += 32) {
-        const double d = static_cast<double>(__ldg(row + n)) - mean;
-        sq += d * d;
-    }
-    for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
-    const double rstd = 1.0 / sqrt(sq / N + static_cast<double>(eps));
-    for (int n = lane; n < N; n += 32) {
-        const float t = static_cast<float>((static_cast<double>(__ldg(row + n)) - mean) * rstd);
-        const float v = __fmaf_rn(t, __ldg(gamma + n), __ldg(beta + n));
-        if (kind == 3) {
-            const int q = __float2int_rn(__fmul_rn(v, inv_out_scale));
-            static_cast<int8_t*>(out)[m * N + n] = static_cast<int8_t>(q > 127 ? 127 : (q < -128 ? -128 : q));
-        } else {
-            static_cast<float*>(out)[m * N + n] = v;
+    const float c = __ldg(row);
+    const bool vec = (N & 3) == 0 && (reinterpret_cast<uintptr_t>(z) & 15) == 0 &&
+                     (reinterpret_cast<uintptr_t>(gamma) & 15) == 0 && (reinterpret_cast<uintptr_t>(beta) & 15) == 0 &&
+                     (reinterpret_cast<uintptr_t>(out) & 15) == 0;
+    float s1 = 0.0f;
+    if (vec) {
+        for (int n = 4 * lane; n < N; n += 128) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(row + n));
+            s1 += ((v.x - c) + (v.y - c)) + ((v.z - c) + (v.w - c));
         }
+    } else {
+        for (int n = lane; n < N; n += 32) s1 += __ldg(row + n) - c;
+    }
+    const float mean = c + warp_sum(s1) / N;
+    float s2 = 0.0f;
+    if (vec) {
+        for (int n = 4 * lane; n < N; n += 128) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(row + n));
+            const float a = v.x - mean, b = v.y - mean, d = v.z - mean, e = v.w - mean;
+            s2 += (a * a + b * b) + (d * d + e * e);
+        }
+    } else {
+        for (int n = lane; n < N; n += 32) {
+            const float a = __ldg(row + n) - mean;
+            s2 += a * a;
+        }
+    }
+    const float rstd = rsqrtf(warp_sum(s2) / N + eps);
+    const long long base = m * N;
+    if (vec) {
+        for (int n = 4 * lane; n < N; n += 128) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(row + n));
+            const float4 g = __ldg(reinterpret_cast<const float4*>(gamma + n));
+            const float4 b = __ldg(reinterpret_cast<const float4*>(beta + n));
+            const float y0 = __fmaf_rn((v.x - mean) * rstd, g.x, b.x), y1 = __fmaf_rn((v.y - mean) * rstd, g.y, b.y);
+            const float y2 = __fmaf_rn((v.z - mean) * rstd, g.z, b.z), y3 = __fmaf_rn((v.w - mean) * rstd, g.w, b.w);
+            if (kind == 3) {
+                *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(out) + base + n) =
+                    requant4_s8(y0, y1, y2, y3, inv_out_scale);
+            } else {
+                *reinterpret_cast<float4*>(static_cast<float*>(out) + base + n) = make_float4(y0, y1, y2, y3);
+            }
+        }
+    } else {
+        for (int n = lane; n < N; n += 32)
+            ln_store(kind, out, base + n, __fmaf_rn((__ldg(row + n) - mean) * rstd, __ldg(gamma + n), __ldg(beta + n)),
+                     inv_out_scale);
     }
 }
 
