@@ -59,6 +59,34 @@ KERNEL_SOURCES = ("paper_2211_07715_gb300/csrc/bsgemm_kernel.cu", "paper_2211_07
 WORKLOADS = {"ffn2": synth.ffn2, "ffn1": synth.ffn1, "single": synth.single_768}
 
 
+# ------------------------------------------------- replicas on N GPUs --
+# The layer shards by tokens with no exchange step: every rank runs its own
+# batch of the same shape on its own GPU (weak scaling), the job's time is
+# the slowest rank's, and the job's throughput counts every rank's work.
+
+def rank_input_seed(seed: int, rank: int) -> int:
+    """Seed of rank `rank`'s batch (rank 0 keeps the workload's own)."""
+    return seed + 7919 * rank
+
+
+def max_over_ranks(values, device=None) -> list:
+    """Element-wise maximum of per-rank timings over the process group (the
+    values themselves with one process or no group)."""
+    import torch
+    import torch.distributed as dist
+    values = [float(v) for v in values]
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return values
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_tops(world: int, ops_per_step: float, ms_per_step: float) -> float:
+    """Whole-job throughput: every rank's ops per step over the step time."""
+    return world * ops_per_step / (ms_per_step * 1e-3) / 1e12
+
+
 def kernel_sha() -> str:
     h = hashlib.sha256()
     for rel in KERNEL_SOURCES:
@@ -170,7 +198,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     props = torch.cuda.get_device_properties(dev)
     case = WORKLOADS[args.workload]()
     if world > 1:  # weak scaling: every rank runs its own batch of the same shape
-        case.x = synth.draw_x(synth.rng_for(case.meta["seed"] + 7919 * rank), case.m, case.weight.k_in,
+        case.x = synth.draw_x(synth.rng_for(rank_input_seed(case.meta["seed"], rank)), case.m, case.weight.k_in,
                               case.meta["x_dist"])
     wt = case.weight
     lin = bsg.SparseInt8Linear(wt.n_out, wt.k_in, wt.indptr, wt.colidx, wt.values, wt.scales, wt.bias)
@@ -337,23 +365,19 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
         barrier()
         e2e_ms = s2.elapsed_time(t2)
 
-    # max over ranks
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([elapsed_ms, e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms, e2e_ms = float(t[0]), float(t[1])
+    # the job's time is the slowest rank's
+    elapsed_ms, e2e_ms = max_over_ranks([elapsed_ms, e2e_ms], dev)
     lin.close()
     if rank != 0:
         return None
 
     ms_per_step = elapsed_ms / args.steps
     ops = effective_ops(case)
-    tops = world * ops / (ms_per_step * 1e-3) / 1e12
+    tops = job_tops(world, ops, ms_per_step)
     kernel_ms = ms_per_step  # one kernel per step
     tops_kernel = ops / (kernel_ms * 1e-3) / 1e12
     hbm_gbs = algorithmic_bytes(case) / (ms_per_step * 1e-3) / 1e9
-    e2e_tops = world * ops / (e2e_ms / e2e_steps * 1e-3) / 1e12 if e2e_steps > 0 else None
+    e2e_tops = job_tops(world, ops, e2e_ms / e2e_steps) if e2e_steps > 0 else None
     max_mhz = clocks.get("sm_max_mhz") or 2070.0
     peak = props.multi_processor_count * DP4A_LANES_PER_SM_CLK * OPS_PER_DP4A * max_mhz * 1e6 / 1e12
     peaks = {}
