@@ -158,7 +158,8 @@ int bsgemm_run_ws(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilog
 
 /*
  * bsgemm_run_static -- bsgemm_run_ws without a caller workspace and without
- * any allocation: the token tiles go to a fixed scratch array of
+ * any allocation: on bsgemm_run's fast path nothing but that kernel runs;
+ * otherwise the token tiles go to a fixed scratch array of
  * BSGEMM_STATIC_SCRATCH_BYTES (16 MiB) that the library holds in device
  * memory, one per device.  The paper has no counterpart; this entry point
  * serves callers that must not allocate at run time.

@@ -14,10 +14,13 @@
 //   contiguous, cost-balanced range per CTA of a persistent grid (CTAs =
 //   SMs x resident CTAs).
 // * The CTA stages its token tile of the activations for ALL of K in shared
-//   memory once (one bulk TMA copy of a tile the relayout kernel has already
-//   swizzled); every row group of the tile then gathers from it.  This is
-//   the re-organisation of the input by the mask that Algorithm 1 does with
-//   vpermt2d/vpshufb, done once per tile instead of once per block.
+//   memory once, swizzled k-major; every row group of the tile then gathers
+//   from it.  This is the re-organisation of the input by the mask that
+//   Algorithm 1 does with vpermt2d/vpshufb, done once per tile instead of
+//   once per block.  The fast path copies 64 x 64-byte boxes of x [M][K] by
+//   tensor copies and each warp transposes its boxes in place; K-major x^T
+//   lands in the layout as it is; other shapes use tiles the relayout
+//   kernel wrote (one bulk copy) or per-thread gathers.
 // * One step of a warp takes one quad (4 stored columns) of each of the
 //   group's 4 block-rows: two transposed shared-memory gathers (ldmatrix
 //   .m16n16 .b8) give lane l (q = l % 4, g = l / 4) 8 dot-4 operands -- tokens
@@ -30,15 +33,17 @@
 //   swizzled tile, so a gather reads in one pass per 8 rows.
 // * A CTA's steps are split evenly between its 8 warps.  Each warp reads
 //   its contiguous range of 128-byte step records straight from global
-//   memory (L1/L2) into an 8-deep register ring.  A row group that
+//   memory (L1/L2) into a 12-deep register ring.  A row group that
 //   straddles a split between warps is summed in a shared-memory slot
-//   (int32 atomics); the last warp to add finishes it.
+//   (int32 atomics) and finished after the window's barrier.
 // * GB300 runs int8 dot products on dp4a at the rate of its int8 MMA paths
 //   (tcgen05 has no int8 kind on sm_103a), and a 4-channel block cannot fill
 //   an MMA tile, so the contraction stays on dp4a.
 // * The epilogue runs in registers: int32 -> fp32 (RNE), one fma with scale
 //   and bias, optional GELU by a fixed fp32 op sequence (A&S 7.1.28 erf),
-//   optional requantise (fp32 multiply, round half to even, saturate).
+//   optional requantise (fp32 multiply, round half to even, saturate), or
+//   the residual add before LayerNorm (the LayerNorm itself is a row-wise
+//   kernel at the end of this file).
 #include <cstdint>
 #include <cstring>
 #include <mutex>
