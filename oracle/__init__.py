@@ -78,6 +78,9 @@ def _load():
                                              ctypes.POINTER(c_double)]
             lib.oracle_layernorm.restype = None
             lib.oracle_block_prune.restype = ctypes.c_int64
+            lib.oracle_attention.argtypes = [c_int, c_int, c_int, c_int, i8p, c_int, c_float,
+                                             ctypes.POINTER(c_double)]
+            lib.oracle_attention.restype = c_int
             _lib = lib
     return _lib
 
@@ -313,6 +316,46 @@ def attention_f32(qkv: np.ndarray, qkv_scale, batch: int, seq: int, heads: int =
     p = p / p.sum(axis=-1, keepdims=True, dtype=np.float32)
     ctx = np.matmul(p, v)  # [batch][heads][seq][hd]
     return np.ascontiguousarray(ctx.transpose(0, 2, 1, 3).reshape(m, d)).astype(np.float32)
+
+
+def attention_f64(qkv: np.ndarray, qkv_scale, batch: int, seq: int, heads: int = HEADS, head_dim: int = None,
+                  threads: int = 1) -> np.ndarray:
+    """Multi-head self-attention in fp64 (the C oracle's oracle_attention):
+    the context [batch * seq][heads * head_dim] of the int8 QKV rows
+    [batch * seq][>= 3 * heads * head_dim] (q | k | v), dequantised by
+    qkv_scale.  head_dim defaults to a third of the row width / heads.
+    threads > 1 runs sequences on that many host threads."""
+    lib = _load()
+    qkv = _c(qkv, np.int8)
+    m, ld = qkv.shape
+    assert m == batch * seq
+    if head_dim is None:
+        assert ld % (3 * heads) == 0
+        head_dim = ld // (3 * heads)
+    d = heads * head_dim
+    out = np.empty((m, d), dtype=np.float64)
+    if m == 0:
+        return out
+    dp = ctypes.POINTER(ctypes.c_double)
+
+    def run(b0, b1):
+        if b1 <= b0:
+            return 0
+        q = qkv[b0 * seq:b1 * seq]
+        o = out[b0 * seq:b1 * seq]
+        return lib.oracle_attention(b1 - b0, seq, heads, head_dim, _ptr(q, ctypes.c_int8), ld,
+                                    float(np.float32(qkv_scale)), o.ctypes.data_as(dp))
+
+    threads = max(1, min(int(threads), batch))
+    bounds = [batch * i // threads for i in range(threads + 1)]
+    if threads == 1:
+        rcs = [run(0, batch)]
+    else:
+        with ThreadPoolExecutor(threads) as ex:
+            rcs = list(ex.map(lambda i: run(bounds[i], bounds[i + 1]), range(threads)))
+    if any(rcs):
+        raise ValueError("oracle_attention: bad sizes")
+    return out
 
 
 def attention(qkv: np.ndarray, qkv_scale, batch: int, seq: int, ctx_scale, heads: int = HEADS) -> np.ndarray:

@@ -361,3 +361,58 @@ int64_t oracle_block_prune(int N, int K, const float* W /* [N][K] */, double spa
     free(s);
     return total - npruned;
 }
+
+/* ---------------------------------------------------------------------- */
+/* Multi-head self-attention on the int8 QKV projection: the two Matmuls   */
+/* and the softmax between the QKV and output linears of the INT8 graph    */
+/* (Sec. 3 "Graph optimization" fuses post-operators into InnerProduct and */
+/* Matmul alike).  The paper does not write attention out; this is the     */
+/* standard scaled dot-product form over the heads of DistilBERT:          */
+/*   row m = b * seq + t of QKV holds q | k | v, each heads * hd wide,     */
+/*   int8 times qkv_scale;                                                 */
+/*   for sequence b, head h and query t (columns h*hd .. h*hd + hd - 1):   */
+/*     s_j   = (q_t . k_j) / sqrt(hd)                 j = 0 .. seq - 1     */
+/*     p_j   = exp(s_j - max_j s_j) / sum_j exp(s_j - max_j s_j)           */
+/*     out_t = sum_j p_j v_j                                               */
+/* in fp64; every position of a sequence is a token (no mask).  Rows of   */
+/* QKV are ld bytes apart; out is [batch * seq][heads * hd].  Returns 0,   */
+/* or -1 on bad sizes / allocation failure.                                */
+/* ---------------------------------------------------------------------- */
+int oracle_attention(int batch, int seq, int heads, int hd, const int8_t* QKV, int ld, float qkv_scale,
+                     double* out) {
+    const int d = heads * hd;
+    if (batch < 0 || seq < 1 || heads < 1 || hd < 1 || ld < 3 * d) return -1;
+    double* s = (double*)malloc(sizeof(double) * (size_t)seq);
+    if (!s) return -1;
+    const double scale = (double)qkv_scale;
+    const double inv_sqrt_hd = 1.0 / sqrt((double)hd);
+    for (int b = 0; b < batch; ++b)
+        for (int h = 0; h < heads; ++h)
+            for (int t = 0; t < seq; ++t) {
+                const int8_t* q = QKV + (size_t)(b * seq + t) * ld + h * hd;
+                double smax = -INFINITY;
+                for (int j = 0; j < seq; ++j) {
+                    const int8_t* k = QKV + (size_t)(b * seq + j) * ld + d + h * hd;
+                    double dot = 0.0;
+                    for (int c = 0; c < hd; ++c) dot += ((double)q[c] * scale) * ((double)k[c] * scale);
+                    s[j] = dot * inv_sqrt_hd;
+                    if (s[j] > smax) smax = s[j];
+                }
+                double sum = 0.0;
+                for (int j = 0; j < seq; ++j) {
+                    s[j] = exp(s[j] - smax);
+                    sum += s[j];
+                }
+                double* o = out + (size_t)(b * seq + t) * d + h * hd;
+                for (int c = 0; c < hd; ++c) {
+                    double acc = 0.0;
+                    for (int j = 0; j < seq; ++j) {
+                        const int8_t* v = QKV + (size_t)(b * seq + j) * ld + 2 * d + h * hd;
+                        acc += (s[j] / sum) * ((double)v[c] * scale);
+                    }
+                    o[c] = acc;
+                }
+            }
+    free(s);
+    return 0;
+}

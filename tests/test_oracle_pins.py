@@ -378,3 +378,94 @@ def test_linear_resid_hand_case_and_special_cases():
     z = oracle.linear_resid(xx, wd, wt.scales, wt.bias, rr, 0.03)
     rs = (np.float32(0.03) * rr.astype(np.float32)).astype(np.float32)
     assert np.array_equal(z, (y.astype(np.float32) + rs).astype(np.float32))
+
+
+# ------------------------------------------------------- multi-head attention --
+
+def _qkv_rows(q, k, v):
+    """Token rows q | k | v (int8) from per-token lists."""
+    return np.concatenate([np.asarray(q), np.asarray(k), np.asarray(v)], axis=1).astype(np.int8)
+
+
+def test_attention_closed_form_two_keys():
+    """One head of width 4, two tokens.  Token 0's query (1,1,1,1) meets keys
+    0 and (1,1,1,1): scores 0 and 4 s^2 / sqrt(4) = 2 s^2.  With s^2 =
+    ln(3) / 2 the weights are 1/4 and 3/4, so its context is
+    s (v0 + 3 v1) / 4 (this fixes the 1/sqrt(hd) factor, the sign of the
+    softmax and which values get mixed).  Token 1's query is 0: equal
+    scores, the context is the mean s (v0 + v1) / 2."""
+    s = np.float32(math.sqrt(math.log(3.0) / 2.0))
+    v0, v1 = np.array([10, 0, -5, 3]), np.array([2, 8, 1, -7])
+    qkv = _qkv_rows([[1, 1, 1, 1], [0, 0, 0, 0]], [[0, 0, 0, 0], [1, 1, 1, 1]], [v0, v1])
+    got = oracle.attention_f64(qkv, s, 1, 2, heads=1)
+    want0 = float(s) * (v0 + 3 * v1) / 4.0
+    want1 = float(s) * (v0 + v1) / 2.0
+    # the float rounding of s moves the weight 3 by ~1e-7 relative
+    assert np.allclose(got[0], want0, rtol=0, atol=1e-6)
+    assert np.allclose(got[1], want1, rtol=0, atol=1e-15)
+
+
+def test_attention_max_subtraction_and_dominant_key():
+    """hd = 64, scale 1: all queries and keys 127 give scores of 127^2 * 64
+    / 8 = 129032 (exp overflows unless the row maximum is subtracted): equal
+    scores, the context is the mean of the values.  A single key of +127
+    among keys of -127 wins by 258064: the context is that key's value
+    exactly (the other weights underflow to 0)."""
+    rng = np.random.default_rng(63)
+    seq = 5
+    v = rng.integers(-127, 128, size=(seq, 64))
+    qkv = _qkv_rows(np.full((seq, 64), 127), np.full((seq, 64), 127), v)
+    got = oracle.attention_f64(qkv, 1.0, 1, seq, heads=1)
+    assert np.all(np.isfinite(got))
+    assert np.allclose(got, np.broadcast_to(v.mean(axis=0), (seq, 64)), rtol=0, atol=1e-12)
+    k = np.full((seq, 64), -127)
+    k[3] = 127
+    qkv = _qkv_rows(np.full((seq, 64), 127), k, v)
+    got = oracle.attention_f64(qkv, 1.0, 1, seq, heads=1)
+    assert np.array_equal(got, np.broadcast_to(v[3].astype(np.float64), (seq, 64)))
+
+
+def test_attention_single_token_is_its_value():
+    rng = np.random.default_rng(64)
+    qkv = rng.integers(-127, 128, size=(3, 3 * 2 * 64)).astype(np.int8)  # 3 sequences of 1 token, 2 heads
+    got = oracle.attention_f64(qkv, 0.125, 3, 1, heads=2)
+    assert np.array_equal(got, qkv[:, 2 * 128:].astype(np.float64) * 0.125)
+
+
+def test_attention_permutation_equivariance_and_independence():
+    """Permuting the tokens of a sequence permutes its context rows the same
+    way; a head's context depends only on that head's columns of its own
+    sequence."""
+    rng = np.random.default_rng(65)
+    batch, seq, heads, hd = 2, 7, 3, 8
+    d = heads * hd
+    qkv = rng.integers(-127, 128, size=(batch * seq, 3 * d)).astype(np.int8)
+    base = oracle.attention_f64(qkv, 0.02, batch, seq, heads=heads)
+    perm = rng.permutation(seq)
+    pq = qkv.copy()
+    pq[:seq] = qkv[perm]
+    got = oracle.attention_f64(pq, 0.02, batch, seq, heads=heads)
+    assert np.allclose(got[:seq], base[perm], rtol=1e-12, atol=1e-14)
+    assert np.array_equal(got[seq:], base[seq:])
+    # change head 1's queries, keys or values in sequence 0 only
+    for part in range(3):
+        cq = qkv.copy()
+        cq[:seq, part * d + hd:part * d + 2 * hd] = rng.integers(-127, 128, size=(seq, hd))
+        got = oracle.attention_f64(cq, 0.02, batch, seq, heads=heads)
+        changed = np.abs(got - base) > 0
+        assert changed[:seq, hd:2 * hd].any(), part
+        changed[:seq, hd:2 * hd] = False
+        assert not changed.any(), part
+
+
+def test_attention_agrees_with_fp32_numpy_fixture():
+    """The fp32 numpy attention (matmul + exp through numpy/BLAS, another
+    implementation) lies within fp32 rounding of the fp64 oracle."""
+    rng = np.random.default_rng(66)
+    batch, seq = 2, 40
+    qkv = rng.integers(-127, 128, size=(batch * seq, 3 * 768)).astype(np.int8)
+    a = oracle.attention_f64(qkv, 0.01, batch, seq)
+    b = oracle.attention_f32(qkv, 0.01, batch, seq)
+    assert np.abs(a - b).max() <= 1e-5 * 127 * 0.01
+    c = oracle.attention_f64(qkv, 0.01, batch, seq, threads=2)
+    assert np.array_equal(a, c)
