@@ -693,16 +693,52 @@ def run_layer(args) -> dict:
     }
 
 
+MMA_SYNC_BF16_TFLOPS = 594.0  # mma.sync m16n8k16 bf16 -> fp32, measured on GB300 at 2070 MHz (legacy tensor path)
+SFU_EX2_PER_SM_CLK = 16        # exponentials per SM per clock (special-function unit)
+
+
+def attention_roofline(batch: int, seq: int, heads: int, ms: float, sms: int, max_mhz: float, hbm_gbs: float,
+                       bf16_tflops: float) -> dict:
+    """The attention kernel against its floors: the tensor work (q k^T once,
+    P v twice for the two bf16 parts of P: 6 x batch x heads x seq^2 x 64
+    flops) at the measured dense bf16 rate, one exponential per score on the
+    special-function units, and the int8 QKV read once from HBM.  The
+    largest floor is the bound; the tensor floor at the rate the kernel's
+    mma.sync path itself can reach is reported beside it."""
+    macs = float(batch) * heads * seq * seq * 64
+    clk = max_mhz * 1e6
+    floors = {"tensor": 6 * macs / (bf16_tflops * 1e12),
+              "exp": float(batch) * heads * seq * seq / (sms * SFU_EX2_PER_SM_CLK * clk),
+              "hbm": float(batch) * seq * 3 * heads * 64 / (hbm_gbs * 1e9)}
+    name = max(floors, key=floors.get)
+    t = ms * 1e-3
+    mma_floor = 6 * macs / (MMA_SYNC_BF16_TFLOPS * 1e12)
+    return {"kernel": "attention_kernel", "ms": round(ms, 6), "ops": 4 * macs,
+            "achieved_tops": round(4 * macs / t / 1e12, 3),
+            "floors_us": {k: round(v * 1e6, 3) for k, v in floors.items()},
+            "bound": {"tensor": "tensor", "exp": "alu", "hbm": "hbm"}[name], "floor": name,
+            "peak": bf16_tflops, "frac": round(floors[name] / t, 4),
+            "mma_sync_floor_us": round(mma_floor * 1e6, 3), "frac_of_mma_sync": round(mma_floor / t, 4),
+            "basis": "graph of 200 launches, per launch; ops = 2 x (q k^T + P v) multiply-adds; floors: tensor = "
+                     "6 x MACs (P v twice: two bf16 parts) at the measured dense bf16 rate (MEASURED_PEAKS, burst), "
+                     "exp = one SFU exponential per score (16 per SM per clock at the max SM clock), hbm = QKV "
+                     "bytes at the measured copy rate; mma_sync = the tensor floor at the measured mma.sync m16n8k16 "
+                     "bf16 rate (594 TFLOP/s), the unit this kernel uses"}
+
+
 def run_encoder(args) -> dict:
-    """cfg 4 as an encoder layer with its sub-layer ends (Sec. 3's fused
-    post-operators): QKV -> [attention: a seeded int8 context buffer, outside
-    the timed path] -> attention output + residual (the layer input) ->
-    LayerNorm -> FFN1 + GELU -> FFN2 + residual (the first LayerNorm's
-    output) -> LayerNorm; int8 between.  The residual adds run in the
-    linears' epilogues (BSGEMM_OUT_F32_RESID), each LayerNorm is one kernel.
+    """cfg 4 as a whole encoder layer on the device: QKV -> multi-head
+    attention (bsgemm_attention, 12 heads of 64) -> attention output +
+    residual (the layer input) -> LayerNorm -> FFN1 + GELU -> FFN2 +
+    residual (the first LayerNorm's output) -> LayerNorm; int8 between.
+    The residual adds run in the linears' epilogues (BSGEMM_OUT_F32_RESID),
+    each LayerNorm and the attention are one kernel each: 7 launches.
     M = 8 x 384 tokens, 80% block sparsity.  Scales: the layer chain's
-    calibrated ones for QKV and FFN1; 0.02 for the input as a residual and
-    4/127 for the LayerNorm outputs (synthetic constants)."""
+    calibrated ones for QKV, the attention context and FFN1; 0.02 for the
+    input as a residual and 4/127 for the LayerNorm outputs (synthetic
+    constants).  `value` is the four linears' effective ops over the whole
+    layer's time; the attention's own time and roofline are reported
+    beside it."""
     import torch
     import paper_2211_07715_gb300 as bsg
 
@@ -718,13 +754,13 @@ def run_encoder(args) -> dict:
         rng.normal(1.0, 0.1, 768).astype(np.float32), rng.normal(0.0, 0.1, 768).astype(np.float32),
         rng.normal(1.0, 0.1, 768).astype(np.float32), rng.normal(0.0, 0.1, 768).astype(np.float32)))
     x_scale, ln_scale, eps = 0.02, 4.0 / 127.0, 1e-12
-    ctx_host = synth.draw_x(synth.rng_for(synth.SEED_BASE + 3 + 7), m, 768, "u127")
+    batch, seq, heads = 8, 384, 12
     set_bytes = m * (768 * 2 + 2304 + 768 * 4 * 2 + 768 * 2 + 3072)
     nsets = max(2, math.ceil(2 * int(getattr(props, "L2_cache_size", 128 << 20)) / set_bytes) + 1)
     xs = [torch.from_numpy(x0).to(dev) for _ in range(nsets)]
-    ctxs = [torch.from_numpy(ctx_host).to(dev) for _ in range(nsets)]
     t = torch
-    bufs = [{"qkv": t.empty((m, 2304), dtype=t.int8, device=dev), "z1": t.empty((m, 768), dtype=t.float32, device=dev),
+    bufs = [{"qkv": t.empty((m, 2304), dtype=t.int8, device=dev), "ctx": t.empty((m, 768), dtype=t.int8, device=dev),
+             "z1": t.empty((m, 768), dtype=t.float32, device=dev),
              "h1": t.empty((m, 768), dtype=t.int8, device=dev), "f1": t.empty((m, 3072), dtype=t.int8, device=dev),
              "z2": t.empty((m, 768), dtype=t.float32, device=dev), "h2": t.empty((m, 768), dtype=t.int8, device=dev)}
             for _ in range(nsets)]
@@ -732,9 +768,11 @@ def run_encoder(args) -> dict:
 
     def layer(i, s):
         b, sh = bufs[i % nsets], s.cuda_stream
-        x, ctx = xs[i % nsets], ctxs[i % nsets]
+        x = xs[i % nsets]
         bsg.bsgemm_run(lins[0]._h, x.data_ptr(), m, b["qkv"].data_ptr(), synth.I8, scales["qkv"], sh)
-        bsg.bsgemm_run(lins[1]._h, ctx.data_ptr(), m, b["z1"].data_ptr(), bsg.OUT_F32_RESID, 1.0, sh, 0,
+        bsg.bsgemm_attention(b["qkv"].data_ptr(), batch, seq, heads, 64, 2304, scales["qkv"], b["ctx"].data_ptr(),
+                             bsg.OUT_I8, scales["ctx"], sh)
+        bsg.bsgemm_run(lins[1]._h, b["ctx"].data_ptr(), m, b["z1"].data_ptr(), bsg.OUT_F32_RESID, 1.0, sh, 0,
                        x.data_ptr(), x_scale)
         bsg.bsgemm_layernorm(b["z1"].data_ptr(), m, 768, g1.data_ptr(), b1.data_ptr(), eps, b["h1"].data_ptr(),
                              bsg.OUT_I8, ln_scale, sh)
@@ -784,36 +822,49 @@ def run_encoder(args) -> dict:
                              bsg.OUT_I8, ln_scale, s.cuda_stream)
 
     ln_ms = graph_ms(ln_only, reps)
+
+    def attn_only(i, s):
+        b = bufs[i % nsets]
+        bsg.bsgemm_attention(b["qkv"].data_ptr(), batch, seq, heads, 64, 2304, scales["qkv"], b["ctx"].data_ptr(),
+                             bsg.OUT_I8, scales["ctx"], s.cuda_stream)
+
+    attn_ms = graph_ms(attn_only, reps)
     ops = [2.0 * m * w.nnzb * 4 for w in weights]
     peak = _peak_tops(props, clocks.get("sm_max_mhz") or 2070.0)
-    hbm_peak = 6683.8
+    hbm_peak, bf16_peak = 6683.8, 1900.0
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
-            hbm_peak = float(json.load(f).get("hbm_gbs", hbm_peak))
+            peaks = json.load(f)
+        hbm_peak = float(peaks.get("hbm_gbs", hbm_peak))
+        bf16_peak = float(peaks.get("bf16_tflops", bf16_peak))
     except (OSError, ValueError):
         pass
     ln_bytes = m * 768 * 4 + m * 768 + 2 * 768 * 4  # z read once, int8 out, gamma and beta
+    attn = attention_roofline(batch, seq, heads, attn_ms, props.multi_processor_count,
+                              clocks.get("sm_max_mhz") or 2070.0, hbm_peak, bf16_peak)
     for lin in lins:
         lin.close()
     return {
         "metric": METRIC, "value": round(sum(ops) / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "n_gpus": 1,
         "steps": steps, "warmup": args.warmup, "ms_per_step": round(ms, 6), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "s8", "data": "synthetic",
-        "config": {"workload": "encoder layer with residual adds and LayerNorms: QKV, [attention: seeded int8 "
-                               "context], attention output + residual -> LayerNorm, FFN1 + GELU, FFN2 + residual "
-                               "-> LayerNorm; int8 between",
+        "config": {"workload": "encoder layer on the device: QKV, multi-head attention (12 x 64), attention "
+                               "output + residual -> LayerNorm, FFN1 + GELU, FFN2 + residual -> LayerNorm; int8 "
+                               "between",
                    "tokens": m, "batch": 8, "seq": 384, "sparsity": 0.8,
                    "l2": f"rotating {nsets} sets ({nsets * set_bytes / 2**20:.0f} MiB > 2 x L2)",
-                   "launch": "the timed passes are one CUDA graph of --steps passes (6 launches each)"},
+                   "launch": "the timed passes are one CUDA graph of --steps passes (7 launches each)",
+                   "value_basis": "the four linears' effective int8 ops / the whole layer's time"},
         "tokens_per_s": round(m / (ms * 1e-3), 1),
         "layernorm": {"kernel": "layernorm_kernel", "ms": round(ln_ms, 6),
                       "gbs": round(ln_bytes / (ln_ms * 1e-3) / 1e9, 1),
                       "hbm_frac": round(ln_bytes / (ln_ms * 1e-3) / 1e9 / hbm_peak, 4),
                       "basis": "graph of 200 LayerNorm launches, per launch; bytes = fp32 z read once + int8 out"},
+        "attention": attn,
         "roofline": {"bound": "alu", "achieved": round(sum(ops) / (ms * 1e-3) / 1e12, 3), "peak": round(peak, 2),
                      "unit": "TOPS", "frac": round(sum(ops) / (ms * 1e-3) / 1e12 / peak, 4), "traffic": None,
-                     "kernel": "whole layer (4 linears + 2 LayerNorms)"},
-        "gpu_launches": 6 * steps, "clocks": clocks, "kernel_source_sha256": kernel_sha(),
+                     "kernel": "whole layer (4 linears + attention + 2 LayerNorms)"},
+        "gpu_launches": 7 * steps, "clocks": clocks, "kernel_source_sha256": kernel_sha(),
     }
 
 

@@ -277,6 +277,36 @@ int bsgemm_layernorm(const float* z, int M, int N, const float* gamma, const flo
                      bsgemm_epilogue epi, void* stream);
 
 /*
+ * bsgemm_attention -- multi-head self-attention on the int8 output of the
+ * QKV linear: the two Matmuls and the softmax between the QKV and output
+ * projections of Sec. 3's optimized INT8 graph (the paper leaves their form
+ * implicit; this is scaled dot-product attention, no mask).  For sequence
+ * b, head h and query t:
+ *   s_j   = (q_t . k_j) * qkv_scale^2 / sqrt(head_dim)   (q . k exact, int32)
+ *   out_t = sum_j exp(s_j - max s) v_j * qkv_scale / sum_j exp(s_j - max s)
+ * in fp32 after the exact dot product; for int8 output requantised as the
+ * linear's epilogue does.
+ *   qkv    DEVICE int8, rows of ld bytes: token row m = b * seq + t holds
+ *          q (bytes 0 .. d-1), k (d .. 2d-1) and v (2d .. 3d-1), d = heads
+ *          * head_dim; head h is bytes h * head_dim .. of each third (the
+ *          QKV linear's int8 output, ld = 3d).  16-byte aligned.
+ *   ld     >= 3d, a multiple of 16.
+ *   qkv_scale  the int8 scale of q, k and v: finite, > 0, with
+ *          qkv_scale^2 / sqrt(head_dim) a normal fp32 number below 2^100.
+ *   out    DEVICE [batch * seq][d], float (epi.kind BSGEMM_OUT_F32) or
+ *          int8 (BSGEMM_OUT_I8, epi.out_scale as for bsgemm_run);
+ *          16-byte aligned; must not overlap qkv.  Other epi fields unused.
+ * head_dim must be 64 and seq <= BSGEMM_ATTN_MAX_SEQ (else
+ * BSGEMM_ERR_UNSUPPORTED); 1 <= heads <= 65535, 0 <= batch <= 65535, seq >=
+ * 1 unless batch = 0 (a no-op).  One kernel on `stream`, asynchronous.
+ * Returns BSGEMM_OK, BSGEMM_ERR_INVALID, BSGEMM_ERR_UNSUPPORTED or
+ * BSGEMM_ERR_CUDA.
+ */
+#define BSGEMM_ATTN_MAX_SEQ 512
+int bsgemm_attention(const int8_t* qkv, int batch, int seq, int heads, int head_dim, int ld, float qkv_scale,
+                     void* out, bsgemm_epilogue epi, void* stream);
+
+/*
  * bsgemm_device_status -- read (and with clear != 0, reset) the handle's
  * device status word.  0 means every wait in the kernels completed; bit 0
  * (BSGEMM_STATUS_TIMEOUT) means a bounded wait on an asynchronous copy gave

@@ -82,6 +82,9 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_block_prune.restype = ctypes.c_int64
     lib.bsgemm_layernorm.argtypes = [vp, ctypes.c_int, ctypes.c_int, vp, vp, ctypes.c_float, vp, Epilogue, vp]
     lib.bsgemm_layernorm.restype = ctypes.c_int
+    lib.bsgemm_attention.argtypes = [vp, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                     ctypes.c_float, vp, Epilogue, vp]
+    lib.bsgemm_attention.restype = ctypes.c_int
     lib.bsgemm_device_status.argtypes = [vp, ctypes.c_int]
     lib.bsgemm_device_status.restype = ctypes.c_int
     return lib
@@ -92,7 +95,7 @@ _lib = _load()
 EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
             "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_run_kmajor",
             "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_layernorm",
-            "bsgemm_destroy",
+            "bsgemm_attention", "bsgemm_destroy",
             "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
 
 
@@ -243,6 +246,46 @@ def layernorm(z, gamma, beta, eps: float, kind: int = OUT_F32, out_scale: float 
     s = torch.cuda.current_stream() if stream is None else stream
     bsgemm_layernorm(z.data_ptr(), m, n, gamma.data_ptr(), beta.data_ptr(), eps, out.data_ptr(), kind, out_scale,
                      s.cuda_stream)
+    return out
+
+
+ATTN_MAX_SEQ = 512  # BSGEMM_ATTN_MAX_SEQ
+ATTN_HEAD_DIM = 64
+
+
+def bsgemm_attention(qkv_ptr: int, batch: int, seq: int, heads: int, head_dim: int, ld: int, qkv_scale: float,
+                     out_ptr: int, kind: int, out_scale: float = 1.0, stream: int = 0) -> None:
+    """Enqueue multi-head self-attention on the int8 QKV rows (raw device
+    pointers; rows of ld bytes holding q | k | v)."""
+    rc = _lib.bsgemm_attention(qkv_ptr, int(batch), int(seq), int(heads), int(head_dim), int(ld), float(qkv_scale),
+                               out_ptr, _epi(kind, out_scale), stream)
+    if rc != 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+
+
+def attention(qkv, batch: int, seq: int, heads: int, qkv_scale: float, kind: int = OUT_F32, out_scale: float = 1.0,
+              out=None, stream=None):
+    """Multi-head self-attention (head width 64) on the CUDA int8 tensor qkv
+    [batch * seq][>= 3 * heads * 64] (the QKV linear's output, q | k | v;
+    its row stride may be padded to a multiple of 16).  Returns the context
+    [batch * seq][heads * 64], float32 or int8 by kind (or fills `out`)."""
+    import torch
+    if qkv.dtype != torch.int8 or not qkv.is_cuda or qkv.dim() != 2 or qkv.stride(1) != 1:
+        raise ValueError("qkv must be a CUDA int8 [M][row] tensor with unit column stride")
+    m = qkv.shape[0]
+    if m != batch * seq:
+        raise ValueError("qkv must have batch * seq rows")
+    d = heads * ATTN_HEAD_DIM
+    if qkv.shape[1] < 3 * d:
+        raise ValueError("qkv rows must hold q, k and v (3 * heads * 64 bytes)")
+    dtype = torch.int8 if kind == OUT_I8 else torch.float32
+    if out is None:
+        out = torch.empty((m, d), dtype=dtype, device=qkv.device)
+    elif out.dtype != dtype or tuple(out.shape) != (m, d) or not out.is_contiguous():
+        raise ValueError(f"out must be a contiguous {dtype} [{m}][{d}] tensor")
+    s = torch.cuda.current_stream() if stream is None else stream
+    bsgemm_attention(qkv.data_ptr(), batch, seq, heads, ATTN_HEAD_DIM, qkv.stride(0), qkv_scale, out.data_ptr(), kind,
+                     out_scale, s.cuda_stream)
     return out
 
 

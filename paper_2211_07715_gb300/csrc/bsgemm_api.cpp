@@ -5,6 +5,7 @@
 #include "bsgemm.h"
 
 #include <algorithm>
+#include <cfloat>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -626,6 +627,41 @@ int bsgemm_layernorm(const float* z, int M, int N, const float* gamma, const flo
     const cudaError_t e = bsg::launch_layernorm(z, M, N, gamma, beta, eps, epi.kind, inv, out,
                                                 static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("LayerNorm launch", e));
+    return BSGEMM_OK;
+}
+
+int bsgemm_attention(const int8_t* qkv, int batch, int seq, int heads, int head_dim, int ld, float qkv_scale,
+                     void* out, bsgemm_epilogue epi, void* stream) {
+    clear_error();
+    if (batch < 0 || batch > 65535 || heads < 1 || heads > 65535 || seq < 0)
+        return fail(BSGEMM_ERR_INVALID, "need 0 <= batch <= 65535, 1 <= heads <= 65535 and seq >= 0");
+    if (head_dim != 64) return fail(BSGEMM_ERR_UNSUPPORTED, "head_dim must be 64");
+    if (seq > BSGEMM_ATTN_MAX_SEQ)
+        return fail(BSGEMM_ERR_UNSUPPORTED, "seq exceeds BSGEMM_ATTN_MAX_SEQ = " + std::to_string(BSGEMM_ATTN_MAX_SEQ));
+    if (epi.kind != BSGEMM_OUT_F32 && epi.kind != BSGEMM_OUT_I8)
+        return fail(BSGEMM_ERR_INVALID, "attention writes BSGEMM_OUT_F32 or BSGEMM_OUT_I8");
+    const long long d = static_cast<long long>(heads) * head_dim;
+    if (ld < 3 * d || ld % 16 != 0) return fail(BSGEMM_ERR_INVALID, "ld must be >= 3 * heads * head_dim and a multiple of 16");
+    if (static_cast<long long>(batch) * seq > INT32_MAX) return fail(BSGEMM_ERR_INVALID, "batch * seq exceeds 2^31 - 1");
+    if (!(qkv_scale > 0.0f) || !std::isfinite(qkv_scale)) return fail(BSGEMM_ERR_INVALID, "qkv_scale must be finite and > 0");
+    const double c = static_cast<double>(qkv_scale) * qkv_scale / std::sqrt(static_cast<double>(head_dim));
+    if (!(c >= static_cast<double>(FLT_MIN)) || !(c < 0x1p100))
+        return fail(BSGEMM_ERR_INVALID, "qkv_scale^2 / sqrt(head_dim) must be a normal fp32 number below 2^100");
+    float inv = 0.0f;
+    if (epi.kind == BSGEMM_OUT_I8) {
+        if (!(epi.out_scale > 0.0f) || !std::isfinite(epi.out_scale))
+            return fail(BSGEMM_ERR_INVALID, "out_scale must be finite and > 0 for int8 outputs");
+        inv = 1.0f / epi.out_scale;
+        if (!std::isfinite(inv)) return fail(BSGEMM_ERR_INVALID, "1 / out_scale overflows fp32");
+    }
+    if (batch == 0) return BSGEMM_OK;
+    if (seq < 1) return fail(BSGEMM_ERR_INVALID, "seq must be >= 1");
+    if (!qkv || !out) return fail(BSGEMM_ERR_INVALID, "qkv and out must not be NULL");
+    if ((reinterpret_cast<uintptr_t>(qkv) & 15u) || (reinterpret_cast<uintptr_t>(out) & 15u))
+        return fail(BSGEMM_ERR_INVALID, "qkv and out must be 16-byte aligned");
+    const cudaError_t e = bsg::launch_attention(qkv, batch, seq, heads, ld, static_cast<float>(c), qkv_scale, epi.kind,
+                                                inv, out, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("attention launch", e));
     return BSGEMM_OK;
 }
 

@@ -106,6 +106,12 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
 // Row-wise LayerNorm of z [M][N] (kind 1: fp32 out, 3: int8 out).
 cudaError_t launch_layernorm(const float* z, int M, int N, const float* gamma, const float* beta, float eps, int kind,
                              float inv_out_scale, void* out, cudaStream_t s);
+// Multi-head self-attention (head width 64, 1 <= seq <= BSGEMM_ATTN_MAX_SEQ)
+// on the int8 QKV rows qkv [batch * seq][ld] into out [batch * seq][heads *
+// 64] (kind 1: fp32, 3: int8); score_scale = qkv_scale^2 / 8.
+size_t attention_smem_bytes(int seq);
+cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, int ld, float score_scale,
+                             float qkv_scale, int kind, float inv_out_scale, void* out, cudaStream_t s);
 // x [M][K] -> swizzled token tiles in xb (the layout the kernel stages by TMA).
 cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, cudaStream_t s);
 // Average-magnitude block pruning of a dense fp32 W [N][K] (DEVICE) into

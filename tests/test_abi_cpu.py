@@ -102,3 +102,35 @@ def test_block_prune_rejects_bad_arguments(bsg):
     assert code(8, 8, 16, 1.5, 16) == bsg.ERR_INVALID      # sparsity > 1
     assert code(8, 8, 16, -0.1, 16) == bsg.ERR_INVALID     # sparsity < 0
     assert code(8, 8, 16, float("nan"), 16) == bsg.ERR_INVALID
+
+
+def test_attention_rejects_bad_arguments(bsg):
+    """Shape, stride, scale, kind and pointer checks come before any CUDA
+    call; batch = 0 is a no-op."""
+    def code(batch=2, seq=8, heads=12, head_dim=64, ld=2304, scale=0.05, qkv=16, out=16, kind=None, out_scale=1.0):
+        with pytest.raises(bsg.BsgemmError) as e:
+            bsg.bsgemm_attention(qkv, batch, seq, heads, head_dim, ld, scale, out,
+                                 bsg.OUT_F32 if kind is None else kind, out_scale)
+        return e.value.code
+    assert code(head_dim=32) == bsg.ERR_UNSUPPORTED
+    assert code(seq=bsg.ATTN_MAX_SEQ + 1) == bsg.ERR_UNSUPPORTED
+    assert code(batch=-1) == bsg.ERR_INVALID
+    assert code(batch=65536) == bsg.ERR_INVALID
+    assert code(heads=0) == bsg.ERR_INVALID
+    assert code(seq=-1) == bsg.ERR_INVALID
+    assert code(seq=0) == bsg.ERR_INVALID
+    assert code(ld=2304 - 16) == bsg.ERR_INVALID            # ld < 3d
+    assert code(ld=2304 + 8) == bsg.ERR_INVALID             # ld % 16
+    assert code(scale=0.0) == bsg.ERR_INVALID
+    assert code(scale=float("nan")) == bsg.ERR_INVALID
+    assert code(scale=1e-20) == bsg.ERR_INVALID             # scale^2 / 8 not a normal fp32
+    assert code(scale=1e30) == bsg.ERR_INVALID              # scores would overflow
+    assert code(kind=bsg.OUT_I32) == bsg.ERR_INVALID
+    assert code(kind=bsg.OUT_F32_GELU) == bsg.ERR_INVALID
+    assert code(kind=bsg.OUT_I8, out_scale=0.0) == bsg.ERR_INVALID
+    assert code(qkv=0) == bsg.ERR_INVALID
+    assert code(out=0) == bsg.ERR_INVALID
+    assert code(qkv=24) == bsg.ERR_INVALID                  # not 16-byte aligned
+    assert code(out=8) == bsg.ERR_INVALID
+    assert "aligned" in bsg.bsgemm_last_error()
+    bsg.bsgemm_attention(0, 0, 8, 12, 64, 2304, 0.05, 0, bsg.OUT_F32)  # batch = 0: nothing to do

@@ -1,0 +1,152 @@
+"""Multi-head self-attention on device (bsgemm_attention) against the fp64
+oracle (oracle.attention_f64).
+
+Tolerance, derived from the kernel's arithmetic.  The scores are exact
+int32 dot products (bf16 tensor-core products of int8 values, partial sums
+below 2^24) times c = fl(qkv_scale^2 / 8), so each s_j carries a relative
+error of at most 2^-23; s_j - max s adds 2^-24 of |s_j - max s| and expf at
+most 2 ulp, so each weight e_j is within 2^-21 (S + 1) of its exact value
+(S = the largest |s_j|).  P enters the P v product as two bf16 parts, which
+drops at most 2^-16 of each weight.  The sums over the seq keys (of e_j in
+fp32 adds; of e_j v_j in the tensor cores' fp32 accumulation, counted with
+truncating adds) add at most seq 2^-24 and seq 2^-23 relative to their sums
+of magnitudes; the online softmax rescales the context and the sum by the
+same factors (one rounding each per block of 64 keys), and the final scale
+and product add 2 ulp.  In units of vmax = max |v| * qkv_scale that is at
+most
+    (3 seq 2^-24 + 2^-16 + 2^-21 (S + 1) + (2 ceil(seq / 64) + 4) 2^-24) vmax
+per element.  A dropped or repeated key (weight ~ 1 / seq), a wrong scale
+or head offset moves an element by orders of magnitude more.  int8 outputs
+must equal rne(exact * inv) saturated, except within that bound (times inv)
+of a rounding boundary, where the neighbour is allowed."""
+import numpy as np
+import pytest
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+HD = 64
+
+
+@pytest.fixture(scope="module")
+def bsg():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2211_07715_gb300
+    return paper_2211_07715_gb300
+
+
+def draw_qkv(rng, batch, seq, heads, pad=0, std=35.0):
+    """int8 QKV rows like a calibrated QKV linear's output: rounded normals,
+    clipped to [-127, 127]; `pad` extra bytes per row hold noise that the
+    kernel must not read into the result."""
+    d = heads * HD
+    q = np.clip(np.rint(rng.normal(0.0, std, size=(batch * seq, 3 * d))), -127, 127).astype(np.int8)
+    if pad:
+        q = np.concatenate([q, rng.integers(-128, 128, size=(batch * seq, pad)).astype(np.int8)], axis=1)
+    return np.ascontiguousarray(q)
+
+
+def bound(qkv, scale, batch, seq, heads):
+    d = heads * HD
+    x = qkv[:, :3 * d].astype(np.int64)
+    smax = 0.0
+    for b in range(batch):
+        rows = slice(b * seq, (b + 1) * seq)
+        for h in range(heads):
+            qh = x[rows, h * HD:(h + 1) * HD]
+            kh = x[rows, d + h * HD:d + (h + 1) * HD]
+            smax = max(smax, float(np.abs(qh @ kh.T).max()) * scale * scale / 8.0)
+    vmax = float(np.abs(x[:, 2 * d:3 * d]).max()) * scale
+    return (3 * seq * 2.0 ** -24 + 2.0 ** -16 + 2.0 ** -21 * (smax + 1) + (2 * -(-seq // 64) + 4) * 2.0 ** -24) * vmax
+
+
+def run_device(bsg, qkv, batch, seq, heads, scale, kind=None, out_scale=1.0, guard_rows=0, stream=None):
+    import torch
+    kind = bsg.OUT_F32 if kind is None else kind
+    d = heads * HD
+    dt = torch.int8 if kind == bsg.OUT_I8 else torch.float32
+    buf = torch.full((batch * seq + guard_rows, d), 90 if dt == torch.int8 else 1234.5, dtype=dt, device="cuda")
+    out = buf[:batch * seq]
+    bsg.attention(torch.from_numpy(qkv).cuda(), batch, seq, heads, scale, kind, out_scale, out=out, stream=stream)
+    torch.cuda.synchronize()
+    got = buf.cpu().numpy()
+    if guard_rows:
+        guard = got[batch * seq:]
+        assert (guard == (90 if dt == torch.int8 else np.float32(1234.5))).all(), "bytes after out were written"
+    return got[:batch * seq]
+
+
+@pytest.mark.parametrize("batch,seq,heads,pad,scale", [
+    (1, 1, 1, 0, 0.05), (2, 5, 2, 16, 0.05), (1, 64, 12, 0, 0.05), (3, 65, 4, 0, 0.08),
+    (2, 130, 3, 48, 0.02), (1, 512, 2, 0, 0.05), (2, 384, 12, 0, 0.12)])
+def test_attention_f32_parity(bsg, batch, seq, heads, pad, scale):
+    rng = np.random.default_rng(7000 + 7 * seq + heads)
+    qkv = draw_qkv(rng, batch, seq, heads, pad)
+    got = run_device(bsg, qkv, batch, seq, heads, scale, guard_rows=2)
+    want = oracle.attention_f64(qkv, scale, batch, seq, heads=heads, head_dim=HD, threads=8)
+    tol = bound(qkv, scale, batch, seq, heads)
+    err = np.abs(got.astype(np.float64) - want)
+    assert err.max() <= tol, f"max err {err.max():.3g} > bound {tol:.3g}"
+
+
+def test_attention_i8_full_layer_shape(bsg):
+    """The encoder layer's shape: 8 sequences x 384 tokens, 12 heads; int8
+    context with the scale a calibration would pick (max |ctx| / 127)."""
+    import torch
+    batch, seq, heads, scale = 8, 384, 12, 0.05
+    rng = np.random.default_rng(7100)
+    qkv = draw_qkv(rng, batch, seq, heads)
+    want = oracle.attention_f64(qkv, scale, batch, seq, heads=heads, head_dim=HD, threads=16)
+    out_scale = float(np.float32(np.abs(want).max()) / np.float32(127.0))
+    inv = float(np.float32(1.0) / np.float32(out_scale))
+    got = run_device(bsg, qkv, batch, seq, heads, scale, bsg.OUT_I8, out_scale, guard_rows=1)
+    tol = bound(qkv, scale, batch, seq, heads)
+    t = want * inv
+    ref = np.clip(np.rint(t), -128, 127).astype(np.int64)
+    g = got.astype(np.int64)
+    diff = g != ref
+    near = np.abs(np.abs(t - np.floor(t)) - 0.5) <= tol * inv + 1e-6
+    assert not (diff & ~(near & (np.abs(g - ref) == 1))).any(), \
+        f"{int((diff & ~near).sum())} int8 values differ away from a rounding boundary"
+    assert int(diff.sum()) <= g.size // 100
+    # the fp32 path on the same input, from a side stream
+    s = torch.cuda.Stream()
+    got32 = run_device(bsg, qkv, batch, seq, heads, scale, stream=s)
+    assert np.abs(got32.astype(np.float64) - want).max() <= tol
+
+
+def test_attention_special_cases(bsg):
+    rng = np.random.default_rng(7200)
+    seq, heads = 100, 2
+    d = heads * HD
+    v = rng.integers(-127, 128, size=(seq, d))
+    # one dominant key: every context row is that key's value times the scale (0.5: exact)
+    k = np.full((seq, d), -127)
+    k[37] = 127
+    qkv = np.concatenate([np.full((seq, d), 127), k, v], axis=1).astype(np.int8)
+    got = run_device(bsg, qkv, 1, seq, heads, 0.5)
+    assert np.array_equal(got, np.broadcast_to((v[37] * 0.5).astype(np.float32), (seq, d)))
+    # zero queries: every key weighs the same, the context is the mean value
+    qkv = np.concatenate([np.zeros((seq, d)), rng.integers(-127, 128, size=(seq, d)), v], axis=1).astype(np.int8)
+    got = run_device(bsg, qkv, 1, seq, heads, 0.05)
+    want = oracle.attention_f64(qkv, 0.05, 1, seq, heads=heads, head_dim=HD)
+    assert np.allclose(want, np.broadcast_to(v.mean(axis=0) * np.float64(np.float32(0.05)), (seq, d)), atol=1e-12)
+    assert np.abs(got - want).max() <= bound(qkv, 0.05, 1, seq, heads)
+
+
+def test_attention_checks_on_device(bsg):
+    import torch
+    qkv = torch.zeros((2 * 8, 3 * 64), dtype=torch.int8, device="cuda")
+    with pytest.raises(ValueError):
+        bsg.attention(qkv, 2, 9, 1, 0.05)                       # rows != batch * seq
+    with pytest.raises(ValueError):
+        bsg.attention(qkv[:, :100], 2, 8, 1, 0.05)              # rows too short for q | k | v
+    with pytest.raises(bsg.BsgemmError) as e:
+        bsg.attention(qkv, 2, 8, 1, -1.0)
+    assert e.value.code == bsg.ERR_INVALID
+    out = bsg.attention(qkv, 2, 8, 1, 0.05)                    # all zero: the context is 0
+    torch.cuda.synchronize()
+    assert out.abs().max().item() == 0.0
