@@ -81,6 +81,8 @@ def _load():
             lib.oracle_attention.argtypes = [c_int, c_int, c_int, c_int, i8p, c_int, c_float,
                                              ctypes.POINTER(c_double)]
             lib.oracle_attention.restype = c_int
+            lib.oracle_bsr1x4_to_dense.argtypes = [c_int, c_int, i32p, i32p, i8p, i8p]
+            lib.oracle_bsr1x4_to_dense.restype = c_int
             _lib = lib
     return _lib
 
@@ -104,6 +106,21 @@ def bsr_to_dense(n_out: int, k_in: int, indptr, colidx, values) -> np.ndarray:
                                  _ptr(values, ctypes.c_int8), _ptr(w, ctypes.c_int8))
     if rc:
         raise ValueError("invalid block-compressed arrays")
+    return w
+
+
+def bsr1x4_to_dense(n_out: int, k_in: int, indptr, colgrp, values) -> np.ndarray:
+    """Dense int8 W [N][K] of a weight sparse in 1 x 4 blocks (one output
+    row x 4 consecutive input columns; block e of row n covers columns
+    4 colgrp[e] .. 4 colgrp[e] + 3)."""
+    lib = _load()
+    indptr, colgrp = _c(indptr, np.int32), _c(colgrp, np.int32)
+    values = _c(values, np.int8).reshape(-1)
+    w = np.empty((n_out, k_in), dtype=np.int8)
+    rc = lib.oracle_bsr1x4_to_dense(n_out, k_in, _ptr(indptr, ctypes.c_int32), _ptr(colgrp, ctypes.c_int32),
+                                    _ptr(values, ctypes.c_int8), _ptr(w, ctypes.c_int8))
+    if rc:
+        raise ValueError("invalid 1x4 block arrays")
     return w
 
 

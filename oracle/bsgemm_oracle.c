@@ -416,3 +416,30 @@ int oracle_attention(int batch, int seq, int heads, int hd, const int8_t* QKV, i
     free(s);
     return 0;
 }
+
+/* ---------------------------------------------------------------------- */
+/* Weights sparse in 1 x 4 blocks (one output row x 4 consecutive input    */
+/* columns): the variant block shape along the reduction dimension, where  */
+/* one block is exactly one dot-4 (the k_block = 4 of Algorithm 1 within   */
+/* a single output row).  Row n holds blocks indptr[n] .. indptr[n+1]-1;   */
+/* block e covers columns 4 colgrp[e] .. 4 colgrp[e] + 3 with values       */
+/* values[e][0..3] in column order.  Decompresses into the dense W [N][K]  */
+/* (K a multiple of 4).  Returns 0, or -1 if the arrays are invalid        */
+/* (indptr not starting at 0 / decreasing, a group outside [0, K/4), or    */
+/* groups of a row not strictly increasing).                               */
+/* ---------------------------------------------------------------------- */
+int oracle_bsr1x4_to_dense(int N, int K, const int32_t* indptr, const int32_t* colgrp, const int8_t* values,
+                           int8_t* W) {
+    if (N < 1 || K < 4 || K % 4 != 0 || indptr[0] != 0) return -1;
+    memset(W, 0, (size_t)N * K);
+    for (int n = 0; n < N; ++n) {
+        if (indptr[n + 1] < indptr[n]) return -1;
+        for (int32_t e = indptr[n]; e < indptr[n + 1]; ++e) {
+            const int32_t j = colgrp[e];
+            if (j < 0 || j >= K / 4) return -1;
+            if (e > indptr[n] && colgrp[e - 1] >= j) return -1;
+            for (int i = 0; i < 4; ++i) W[(size_t)n * K + 4 * j + i] = values[4 * (size_t)e + i];
+        }
+    }
+    return 0;
+}

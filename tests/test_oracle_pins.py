@@ -469,3 +469,41 @@ def test_attention_agrees_with_fp32_numpy_fixture():
     assert np.abs(a - b).max() <= 1e-5 * 127 * 0.01
     c = oracle.attention_f64(qkv, 0.01, batch, seq, threads=2)
     assert np.array_equal(a, c)
+
+
+# ------------------------------------------------------------- 1 x 4 blocks --
+
+def test_bsr1x4_hand_case_and_rejects():
+    w = oracle.bsr1x4_to_dense(2, 8, [0, 1, 2], [1, 0], [[1, 2, 3, 4], [5, 6, 7, -8]])
+    assert w.tolist() == [[0, 0, 0, 0, 1, 2, 3, 4], [5, 6, 7, -8, 0, 0, 0, 0]]
+    ones = [[1, 1, 1, 1]] * 2
+    for args in (([1, 1, 2], [0, 1]),       # indptr[0] != 0
+                 ([0, 2, 1], [0, 1]),       # decreasing
+                 ([0, 1, 2], [0, 2]),       # group = K / 4
+                 ([0, 2, 2], [1, 1]),       # repeated group
+                 ([0, 2, 2], [1, 0])):      # unsorted
+        with pytest.raises(ValueError):
+            oracle.bsr1x4_to_dense(2, 8, args[0], args[1], ones)
+    with pytest.raises(ValueError):                       # K not a multiple of 4
+        oracle.bsr1x4_to_dense(2, 6, [0, 0, 0], [], np.zeros((0, 4)))
+
+
+def test_bsr1x4_is_the_transpose_of_4x1_blocks():
+    """A 1 x 4 block of W (row n, columns 4j .. 4j+3) is a 4 x 1 block of
+    W^T (rows 4j .. 4j+3, column n): re-indexed by group, the same arrays
+    through the 4 x 1 decompression give W^T."""
+    rng = np.random.default_rng(67)
+    n, k = 10, 24
+    keep = rng.random((n, k // 4)) < 0.4
+    rows, grps = np.nonzero(keep)                          # row-major: by n, then j
+    vals = rng.integers(-127, 128, size=(len(rows), 4)).astype(np.int8)
+    indptr = np.concatenate([[0], np.cumsum(keep.sum(axis=1))]).astype(np.int32)
+    w = oracle.bsr1x4_to_dense(n, k, indptr, grps.astype(np.int32), vals)
+    order = np.lexsort((rows, grps))                       # by j, then n
+    indptr_t = np.concatenate([[0], np.cumsum(np.bincount(grps, minlength=k // 4))]).astype(np.int32)
+    wt = oracle.bsr_to_dense(k, n, indptr_t, rows[order].astype(np.int32), vals[order])
+    assert np.array_equal(w, wt.T)
+    # and the linear through it is the library's integer matmul
+    x = rng.integers(-127, 128, size=(7, k)).astype(np.int8)
+    acc = oracle.linear(x, w, np.ones(n, np.float32), np.zeros(n, np.float32), oracle.I32)
+    assert np.array_equal(acc, x.astype(np.int64) @ w.astype(np.int64).T)
