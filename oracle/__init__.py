@@ -83,6 +83,8 @@ def _load():
             lib.oracle_attention.restype = c_int
             lib.oracle_bsr1x4_to_dense.argtypes = [c_int, c_int, i32p, i32p, i8p, i8p]
             lib.oracle_bsr1x4_to_dense.restype = c_int
+            lib.oracle_2to4_to_dense.argtypes = [c_int, c_int, i8p, u8p, i8p]
+            lib.oracle_2to4_to_dense.restype = c_int
             _lib = lib
     return _lib
 
@@ -121,6 +123,22 @@ def bsr1x4_to_dense(n_out: int, k_in: int, indptr, colgrp, values) -> np.ndarray
                                     _ptr(values, ctypes.c_int8), _ptr(w, ctypes.c_int8))
     if rc:
         raise ValueError("invalid 1x4 block arrays")
+    return w
+
+
+def sparse2to4_to_dense(values, idx) -> np.ndarray:
+    """Dense int8 W [N][K] of a 2:4-sparse weight: values and idx [N][K/2],
+    two values per group of 4 input columns at in-group positions idx
+    (strictly increasing per group)."""
+    lib = _load()
+    values, idx = _c(values, np.int8), _c(idx, np.uint8)
+    n_out, half = values.shape
+    if idx.shape != values.shape:
+        raise ValueError("values and idx must have the same shape")
+    w = np.empty((n_out, 2 * half), dtype=np.int8)
+    if lib.oracle_2to4_to_dense(n_out, 2 * half, _ptr(values, ctypes.c_int8), _ptr(idx, ctypes.c_uint8),
+                                _ptr(w, ctypes.c_int8)):
+        raise ValueError("invalid 2:4 arrays")
     return w
 
 

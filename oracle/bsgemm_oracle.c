@@ -443,3 +443,27 @@ int oracle_bsr1x4_to_dense(int N, int K, const int32_t* indptr, const int32_t* c
     }
     return 0;
 }
+
+/* ---------------------------------------------------------------------- */
+/* Weights with 2:4 structured sparsity along the input dimension: in each */
+/* output row, each group of 4 consecutive input columns holds at most 2   */
+/* nonzero weights (the pattern of sparse tensor cores the paper cites as  */
+/* related work, Sec. 1).  Compressed form per row n and group g: two      */
+/* values values[n][2g + t] at the in-group positions idx[n][2g + t]       */
+/* (t = 0, 1; 0 <= idx < 4, strictly increasing within the group).         */
+/* Decompresses into the dense W [N][K] (K a multiple of 4).  Returns 0,   */
+/* or -1 on an invalid index.                                              */
+/* ---------------------------------------------------------------------- */
+int oracle_2to4_to_dense(int N, int K, const int8_t* values, const uint8_t* idx, int8_t* W) {
+    if (N < 1 || K < 4 || K % 4 != 0) return -1;
+    memset(W, 0, (size_t)N * K);
+    const int half = K / 2;
+    for (int n = 0; n < N; ++n)
+        for (int g = 0; g < K / 4; ++g) {
+            const uint8_t i0 = idx[(size_t)n * half + 2 * g], i1 = idx[(size_t)n * half + 2 * g + 1];
+            if (i0 >= 4 || i1 >= 4 || i0 >= i1) return -1;
+            W[(size_t)n * K + 4 * g + i0] = values[(size_t)n * half + 2 * g];
+            W[(size_t)n * K + 4 * g + i1] = values[(size_t)n * half + 2 * g + 1];
+        }
+    return 0;
+}

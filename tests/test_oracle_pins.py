@@ -507,3 +507,36 @@ def test_bsr1x4_is_the_transpose_of_4x1_blocks():
     x = rng.integers(-127, 128, size=(7, k)).astype(np.int8)
     acc = oracle.linear(x, w, np.ones(n, np.float32), np.zeros(n, np.float32), oracle.I32)
     assert np.array_equal(acc, x.astype(np.int64) @ w.astype(np.int64).T)
+
+
+# ------------------------------------------------------------ 2:4 sparsity --
+
+def test_2to4_hand_case_and_rejects():
+    vals = np.array([[3, -4, 5, 6]], np.int8)
+    idx = np.array([[0, 3, 1, 2]], np.uint8)
+    w = oracle.sparse2to4_to_dense(vals, idx)
+    assert w.tolist() == [[3, 0, 0, -4, 0, 5, 6, 0]]
+    for bad in ([[1, 1, 0, 1]], [[2, 1, 0, 1]], [[0, 4, 0, 1]]):   # repeated, decreasing, out of range
+        with pytest.raises(ValueError):
+            oracle.sparse2to4_to_dense(vals, np.array(bad, np.uint8))
+
+
+def test_2to4_structure_and_linear():
+    """Every group of 4 columns holds at most 2 nonzeros and exactly the
+    stored values; the linear through it is the library's integer matmul."""
+    rng = np.random.default_rng(68)
+    n, k = 12, 40
+    pos = np.sort(np.stack([rng.choice(4, 2, replace=False) for _ in range(n * k // 4)]), axis=1)
+    idx = pos.reshape(n, k // 2).astype(np.uint8)
+    vals = rng.integers(-127, 128, size=(n, k // 2)).astype(np.int8)
+    w = oracle.sparse2to4_to_dense(vals, idx)
+    groups = w.reshape(n, k // 4, 4)
+    assert ((groups != 0).sum(axis=2) <= 2).all()
+    # the stored values sit at their positions
+    got = np.take_along_axis(groups, idx.reshape(n, k // 4, 2).astype(np.int64), axis=2)
+    assert np.array_equal(got.reshape(n, k // 2), vals)
+    # the other two positions of each group are zero
+    assert int(np.abs(groups.astype(np.int64)).sum()) == int(np.abs(vals.astype(np.int64)).sum())
+    x = rng.integers(-127, 128, size=(9, k)).astype(np.int8)
+    acc = oracle.linear(x, w, np.ones(n, np.float32), np.zeros(n, np.float32), oracle.I32)
+    assert np.array_equal(acc, x.astype(np.int64) @ w.astype(np.int64).T)
