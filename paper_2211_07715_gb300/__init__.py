@@ -343,6 +343,53 @@ def dense_to_blocks(w: np.ndarray, keep=None):
     return indptr, k_idx.astype(np.int32), values
 
 
+def dense_from_blocks_1x4(n_out: int, k_in: int, indptr, colgrp, values) -> np.ndarray:
+    """Dense int8 W [N][K] of a weight sparse in 1 x 4 blocks: one output row
+    x 4 consecutive input columns (K a multiple of 4).  Row n holds blocks
+    indptr[n] .. indptr[n+1]-1; block e covers columns 4 colgrp[e] ..
+    4 colgrp[e] + 3 with values[e][0..3].  Checks the arrays the way
+    bsgemm_create checks its own (ValueError)."""
+    indptr = _host_array(indptr, np.int32).reshape(-1)
+    colgrp = _host_array(colgrp, np.int32).reshape(-1)
+    values = _host_array(values, np.int8).reshape(-1, 4)
+    if n_out < 1 or k_in < 4 or k_in % 4:
+        raise ValueError("need N >= 1 and K a positive multiple of 4")
+    if indptr.shape != (n_out + 1,) or indptr[0] != 0 or (np.diff(indptr) < 0).any():
+        raise ValueError("indptr must hold N + 1 non-decreasing entries from 0")
+    nnz = int(indptr[-1])
+    if colgrp.shape != (nnz,) or values.shape != (nnz, 4):
+        raise ValueError("colgrp and values must hold indptr[N] blocks")
+    if nnz and (colgrp.min() < 0 or colgrp.max() >= k_in // 4):
+        raise ValueError("column groups must lie in [0, K / 4)")
+    rows = np.repeat(np.arange(n_out), np.diff(indptr))
+    if nnz > 1:
+        same_row = rows[1:] == rows[:-1]
+        if (same_row & (colgrp[1:] <= colgrp[:-1])).any():
+            raise ValueError("column groups must increase strictly within a row")
+    w = np.zeros((n_out, k_in), np.int8)
+    w[rows[:, None], 4 * colgrp[:, None] + np.arange(4)] = values
+    return w
+
+
+def dense_from_2to4(values, idx) -> np.ndarray:
+    """Dense int8 W [N][K] of a 2:4-sparse weight: values and idx [N][K/2]
+    hold, per output row and group g of 4 input columns, two values at the
+    in-group positions idx[n][2g], idx[n][2g+1] (0 <= idx < 4, strictly
+    increasing).  ValueError on bad indices."""
+    values = _host_array(values, np.int8)
+    idx = _host_array(idx, np.uint8)
+    if values.ndim != 2 or idx.shape != values.shape or values.shape[1] % 2:
+        raise ValueError("values and idx must be [N][K/2] with K a multiple of 4")
+    n_out, half = values.shape
+    pairs = idx.reshape(n_out, half // 2, 2)
+    if (idx >= 4).any() or (pairs[:, :, 0] >= pairs[:, :, 1]).any():
+        raise ValueError("in-group positions must lie in [0, 4) and increase within each group")
+    cols = 4 * (np.arange(half) // 2)[None, :] + idx.astype(np.int64)
+    w = np.zeros((n_out, 2 * half), np.int8)
+    w[np.arange(n_out)[:, None], cols] = values
+    return w
+
+
 class SparseInt8Linear:
     """One block-sparse int8 linear layer resident on the current CUDA device."""
 
@@ -359,6 +406,24 @@ class SparseInt8Linear:
         w = _host_array(w, np.int8)
         indptr, colidx, values = dense_to_blocks(w, keep)
         return cls(w.shape[0], w.shape[1], indptr, colidx, values, scales, bias)
+
+    @classmethod
+    def from_blocks_1x4(cls, n_out: int, k_in: int, indptr, colgrp, values, scales, bias=None) -> "SparseInt8Linear":
+        """A weight sparse in 1 x 4 blocks (one output row x 4 input
+        columns), run by the 4 x 1-block kernel: at create time its blocks
+        are regrouped into the 4 x 1 blocks that hold them (every column of
+        a block-row that one of its four rows uses), so results are exact
+        and the kernel does the union's work (at 90% sparsity ~3.4 stored
+        blocks per useful one)."""
+        return cls.from_dense(dense_from_blocks_1x4(n_out, k_in, indptr, colgrp, values), scales, bias)
+
+    @classmethod
+    def from_2to4(cls, values, idx, scales, bias=None) -> "SparseInt8Linear":
+        """A 2:4-sparse weight (values, idx [N][K/2]), run by the 4 x 1-block
+        kernel after the same regrouping as from_blocks_1x4: exact, with
+        the union of four rows' columns stored (~94% of all blocks for
+        random 2:4 patterns)."""
+        return cls.from_dense(dense_from_2to4(values, idx), scales, bias)
 
     def workspace_bytes(self, m: int) -> int:
         return bsgemm_workspace_bytes(self._h, m)

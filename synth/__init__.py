@@ -169,3 +169,66 @@ def stack_point(batch: int, seq: int, sparsity: float, point: int, n_layers: int
 
 
 STACK_POINTS = [(b, s, sp) for b in (1, 8, 32, 128) for s in (128, 384) for sp in (0.70, 0.80, 0.90)]
+
+
+# ----------------------------------------------------- variant block shapes --
+
+@dataclass
+class Blocks1x4:
+    """A weight sparse in 1 x 4 blocks (one output row x 4 consecutive input
+    columns): row n holds blocks indptr[n] .. indptr[n+1]-1, block e covers
+    columns 4 colgrp[e] .. 4 colgrp[e] + 3 with values[e][0..3]."""
+    n_out: int
+    k_in: int
+    indptr: np.ndarray  # int32 [N + 1]
+    colgrp: np.ndarray  # int32 [nnz]
+    values: np.ndarray  # int8  [nnz, 4]
+    scales: np.ndarray  # float32 [N]
+    bias: np.ndarray    # float32 [N]
+
+
+def draw_weight_1x4(rng: np.random.Generator, n_out: int, k_in: int, sparsity: float) -> Blocks1x4:
+    """round(sparsity * total) of the N x K/4 blocks zero, chosen uniformly
+    without replacement; values uniform in [-127, 127]; scales and bias as
+    draw_weight's.  Draw order: positions, values, scales, bias."""
+    if k_in % 4:
+        raise ValueError("k_in must be a multiple of 4")
+    total = n_out * (k_in // 4)
+    pruned = min(max(int(np.floor(sparsity * total + 0.5)), 0), total)
+    nnz = total - pruned
+    ids = np.arange(total, dtype=np.int64) if nnz == total else np.sort(rng.choice(total, size=nnz, replace=False))
+    rows = ids // (k_in // 4)
+    indptr = np.zeros(n_out + 1, dtype=np.int32)
+    np.cumsum(np.bincount(rows, minlength=n_out), out=indptr[1:])
+    colgrp = (ids % (k_in // 4)).astype(np.int32)
+    values = rng.integers(-127, 128, size=(nnz, 4)).astype(np.int8)
+    scales = rng.uniform(1e-3, 1e-2, size=n_out).astype(np.float32)
+    bias = rng.normal(0.0, 0.02, size=n_out).astype(np.float32)
+    return Blocks1x4(n_out, k_in, indptr, colgrp, values, scales, bias)
+
+
+@dataclass
+class Sparse2to4:
+    """A 2:4-sparse weight: per output row and group of 4 input columns, two
+    values at in-group positions idx (ascending)."""
+    n_out: int
+    k_in: int
+    values: np.ndarray  # int8  [N, K/2]
+    idx: np.ndarray     # uint8 [N, K/2]
+    scales: np.ndarray  # float32 [N]
+    bias: np.ndarray    # float32 [N]
+
+
+def draw_weight_2to4(rng: np.random.Generator, n_out: int, k_in: int) -> Sparse2to4:
+    """Each group's two positions uniform among the 6 pairs, values uniform
+    in [-127, 127]; scales and bias as draw_weight's.  Draw order:
+    positions, values, scales, bias."""
+    if k_in % 4:
+        raise ValueError("k_in must be a multiple of 4")
+    pairs = np.array([(a, b) for a in range(4) for b in range(a + 1, 4)], dtype=np.uint8)
+    pick = rng.integers(0, len(pairs), size=(n_out, k_in // 4))
+    idx = pairs[pick].reshape(n_out, k_in // 2)
+    values = rng.integers(-127, 128, size=(n_out, k_in // 2)).astype(np.int8)
+    scales = rng.uniform(1e-3, 1e-2, size=n_out).astype(np.float32)
+    bias = rng.normal(0.0, 0.02, size=n_out).astype(np.float32)
+    return Sparse2to4(n_out, k_in, values, idx, scales, bias)

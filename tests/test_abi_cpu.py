@@ -1,5 +1,6 @@
 """The C-ABI library builds, loads, exports every symbol include/bsgemm.h
-declares, and rejects bad arguments before touching a GPU.  CPU only."""
+declares, and rejects bad arguments before touching a GPU; the binding's
+create-time helpers agree with the oracle.  CPU only."""
 import ctypes
 import os
 import re
@@ -7,6 +8,9 @@ import shutil
 
 import numpy as np
 import pytest
+
+import oracle
+import synth
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "bsgemm.h")
@@ -134,3 +138,37 @@ def test_attention_rejects_bad_arguments(bsg):
     assert code(out=8) == bsg.ERR_INVALID
     assert "aligned" in bsg.bsgemm_last_error()
     bsg.bsgemm_attention(0, 0, 8, 12, 64, 2304, 0.05, 0, bsg.OUT_F32)  # batch = 0: nothing to do
+
+
+@pytest.mark.parametrize("n_out,k_in,sparsity", [(10, 24, 0.6), (30, 200, 0.5), (7, 8, 0.0), (5, 16, 1.0)])
+def test_variant_shapes_decompress_like_the_oracle(bsg, n_out, k_in, sparsity):
+    """The binding's 1 x 4 and 2:4 decompressions (create-time helpers)
+    give the oracle's dense weight; the regrouped 4 x 1 blocks hold it."""
+    rng = np.random.default_rng(90 + n_out)
+    w1 = synth.draw_weight_1x4(rng, n_out, k_in, sparsity)
+    a = bsg.dense_from_blocks_1x4(n_out, k_in, w1.indptr, w1.colgrp, w1.values)
+    assert np.array_equal(a, oracle.bsr1x4_to_dense(n_out, k_in, w1.indptr, w1.colgrp, w1.values))
+    indptr, colidx, values = bsg.dense_to_blocks(a)
+    assert np.array_equal(oracle.bsr_to_dense(-(-n_out // 4) * 4, k_in, indptr, colidx, values)[:n_out], a)
+    t = synth.draw_weight_2to4(rng, n_out, k_in)
+    b = bsg.dense_from_2to4(t.values, t.idx)
+    assert np.array_equal(b, oracle.sparse2to4_to_dense(t.values, t.idx))
+
+
+def test_variant_shapes_reject_bad_arrays(bsg):
+    ones = np.ones((2, 4), np.int8)
+    for n, k, ip, cg in ((2, 6, [0, 1, 2], [0, 0]),       # K % 4
+                         (2, 8, [1, 1, 2], [0, 1]),       # indptr[0] != 0
+                         (2, 8, [0, 2, 1], [0, 1]),       # decreasing
+                         (2, 8, [0, 1, 2], [0, 2]),       # group = K / 4
+                         (2, 8, [0, 2, 2], [1, 1]),       # repeated group in a row
+                         (2, 8, [0, 2, 2], [1, 0]),       # unsorted
+                         (2, 8, [0, 1, 3], [0, 1])):      # indptr[N] != number of blocks
+        with pytest.raises(ValueError):
+            bsg.dense_from_blocks_1x4(n, k, ip, cg, ones)
+    v = np.ones((1, 4), np.int8)
+    for bad in ([[1, 1, 0, 1]], [[2, 1, 0, 1]], [[0, 4, 0, 1]]):
+        with pytest.raises(ValueError):
+            bsg.dense_from_2to4(v, np.array(bad, np.uint8))
+    with pytest.raises(ValueError):
+        bsg.dense_from_2to4(np.ones((1, 3), np.int8), np.zeros((1, 3), np.uint8))   # K not a multiple of 4

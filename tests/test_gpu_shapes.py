@@ -1,0 +1,73 @@
+"""Variant block shapes through the layer kernel: weights sparse in 1 x 4
+blocks (one output row x 4 input columns) and 2:4-sparse weights, regrouped
+at create time into the 4 x 1 blocks that hold them
+(SparseInt8Linear.from_blocks_1x4 / from_2to4).  Every element against the
+oracle's linear on the oracle's own decompression of the same arrays:
+integer outputs bit for bit, fp32 within 1e-4 abs or 1e-5 rel."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+KINDS = (synth.I32, synth.F32, synth.F32_GELU, synth.I8, synth.I8_GELU)
+
+
+@pytest.fixture(scope="module")
+def bsg():
+    import paper_2211_07715_gb300
+    return paper_2211_07715_gb300
+
+
+def check(got: np.ndarray, want: np.ndarray, kind: int, what: str = ""):
+    assert got.shape == want.shape, what
+    if kind in (synth.F32, synth.F32_GELU):
+        err = np.abs(got.astype(np.float64) - want)
+        bad = ~((err <= 1e-4) | (err <= 1e-5 * np.abs(want)))
+        assert not bad.any(), f"{what}: {bad.sum()} fp32 elements out of tolerance, max abs err {err.max():.3g}"
+    else:
+        diff = got != want
+        assert not diff.any(), f"{what}: {diff.sum()} elements differ"
+
+
+def gpu_run(lin, x: np.ndarray, kind: int, out_scale: float, workspace=None) -> np.ndarray:
+    xd = torch.from_numpy(x).cuda()
+    dtype = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+             synth.I8: torch.int8, synth.I8_GELU: torch.int8}[kind]
+    out = torch.empty((x.shape[0], lin.n_out), dtype=dtype, device="cuda")
+    lin.run(xd, out, kind, out_scale, workspace=workspace)
+    torch.cuda.synchronize()
+    return out.cpu().numpy()
+
+
+@pytest.mark.parametrize("n_out,k_in,m,sparsity", [(96, 768, 130, 0.9), (30, 200, 70, 0.5), (768, 3072, 64, 0.9)])
+def test_blocks_1x4_through_the_layer(bsg, n_out, k_in, m, sparsity):
+    rng = synth.rng_for(8000 + n_out + k_in)
+    wt = synth.draw_weight_1x4(rng, n_out, k_in, sparsity)
+    w = oracle.bsr1x4_to_dense(n_out, k_in, wt.indptr, wt.colgrp, wt.values)
+    lin = bsg.SparseInt8Linear.from_blocks_1x4(n_out, k_in, wt.indptr, wt.colgrp, wt.values, wt.scales, wt.bias)
+    assert (lin.n_out, lin.k_in) == (n_out, k_in)
+    x = synth.draw_x(rng, m, k_in, "u127")
+    for kind in KINDS:
+        want = oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
+        for path in (None, False):
+            check(gpu_run(lin, x, kind, 0.05, workspace=path), want, kind, f"1x4 kind {kind} path {path}")
+    lin.close()
+
+
+@pytest.mark.parametrize("n_out,k_in,m", [(64, 768, 100), (30, 200, 70), (768, 3072, 64)])
+def test_2to4_through_the_layer(bsg, n_out, k_in, m):
+    rng = synth.rng_for(8100 + n_out + k_in)
+    wt = synth.draw_weight_2to4(rng, n_out, k_in)
+    w = oracle.sparse2to4_to_dense(wt.values, wt.idx)
+    lin = bsg.SparseInt8Linear.from_2to4(wt.values, wt.idx, wt.scales, wt.bias)
+    assert (lin.n_out, lin.k_in) == (n_out, k_in)
+    x = synth.draw_x(rng, m, k_in, "n30")
+    for kind in KINDS:
+        want = oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
+        check(gpu_run(lin, x, kind, 0.05), want, kind, f"2:4 kind {kind}")
+    lin.close()
