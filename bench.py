@@ -1206,7 +1206,8 @@ def main():
     p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "encoder", "stack", "prune", "production"],
                    default="ffn2",
                    help="ffn2/ffn1/single: one linear; layer: the encoder layer's four linears; stack: the "
-                        "six-layer stack sweep; encoder: the layer with residual adds and LayerNorms; "
+                        "six-layer stack sweep; encoder: the whole layer on the device (attention, residual adds, "
+                        "LayerNorms); "
                         "prune: create-side block pruning of an FFN2-shaped weight; "
                         "production: maximum samples/s under 10 ms per batch")
     p.add_argument("--ref-rows", type=int, default=512, help="tokens per reference step")
