@@ -108,6 +108,13 @@ typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
  *   bias     float [N], or NULL for zeros; must be finite.
  * The call allocates device memory on the CURRENT CUDA device, copies the
  * repacked weights there and synchronises.  Returns NULL on failure.
+ *
+ * Other block shapes enter as the 4 x 1 blocks that hold them: a weight
+ * sparse in 1 x 4 blocks (one row x 4 input columns) or with 2:4 sparsity
+ * along K is passed as every 4 x 1 block with a nonzero value (the union of
+ * the four rows' columns of each block-row).  Results are exact; the
+ * stored work grows by that union (the Python binding's from_blocks_1x4 /
+ * from_2to4 build these arrays).
  */
 bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const int8_t* values,
                        const float* scales, const float* bias);
