@@ -93,7 +93,12 @@ def test_encoder_layer_on_device(bsg):
     # calibration on the oracle (frozen constants for the device pass)
     s_qkv = scale_of(oracle.linear(x0, dense[0], wq.scales, wq.bias, oracle.F32, threads=8))
     qkv_ref = oracle.linear(x0, dense[0], wq.scales, wq.bias, oracle.I8, s_qkv, threads=8)
-    s_ctx = scale_of(oracle.attention_f64(qkv_ref, s_qkv, BATCH, SEQ, HEADS, threads=8))
+    att_ref = oracle.attention_f64(qkv_ref, s_qkv, BATCH, SEQ, HEADS, threads=8)
+    s_ctx = scale_of(att_ref)
+    z1_ref = oracle.linear_resid(oracle.requant_f32(att_ref.astype(np.float32), s_ctx), dense[1], wo.scales, wo.bias,
+                                 x0, x_scale, threads=8)
+    h1_ref = oracle.requant_f32(oracle.layernorm(z1_ref, g1, b1, eps).astype(np.float32), ln_scale)
+    s_f1 = scale_of(oracle.linear(h1_ref, dense[2], w1.scales, w1.bias, oracle.F32_GELU, threads=8))
     lins = [bsg.SparseInt8Linear(w.n_out, w.k_in, w.indptr, w.colidx, w.values, w.scales, w.bias) for w in weights]
 
     # one device pass, all on the current stream
@@ -105,7 +110,6 @@ def test_encoder_layer_on_device(bsg):
     bsg.attention(qkv, BATCH, SEQ, HEADS, s_qkv, bsg.OUT_I8, s_ctx, out=ctx)
     lins[1].run(ctx, z1, bsg.OUT_F32_RESID, residual=xd, residual_scale=x_scale)
     h1 = bsg.layernorm(z1, gd[0], gd[1], eps, bsg.OUT_I8, ln_scale)
-    s_f1 = scale_of(oracle.linear(host(h1), dense[2], w1.scales, w1.bias, oracle.F32_GELU, threads=8))
     lins[2].run(h1, f1, bsg.OUT_I8_GELU, s_f1)
     lins[3].run(f1, z2, bsg.OUT_F32_RESID, residual=h1, residual_scale=ln_scale)
     h2 = bsg.layernorm(z2, gd[2], gd[3], eps, bsg.OUT_I8, ln_scale)
