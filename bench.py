@@ -453,6 +453,37 @@ def cpu_baseline(case, rows: int | None, threads: int | None = None, reps: int =
                                         f"weight, {threads} host threads, {dt:.2f} s per pass"}
 
 
+def encoder_cpu_baseline(weights, x0, scales: dict, seq: int, g1, b1, g2, b2, x_scale: float, ln_scale: float,
+                         eps: float, threads: int | None = None, nseq: int = 4) -> dict:
+    """The oracle through one whole encoder layer on a bounded sample: the
+    first nseq sequences (seq tokens each) of the layer input, every stage as the
+    device runs it (QKV, attention, output projection + residual,
+    LayerNorm, FFN1 + GELU, FFN2 + residual, LayerNorm).  value = the four
+    linears' effective ops on the sample / the pass time (the unit of the
+    encoder line's value); tokens/s beside it."""
+    import oracle
+    threads = threads or os.cpu_count() or 1
+    wq, wo, w1, w2 = weights
+    dense = [oracle.weight_dense(w) for w in weights]
+    nseq = max(1, min(nseq, x0.shape[0] // seq))
+    x = np.ascontiguousarray(x0[:nseq * seq])
+    t0 = time.perf_counter()
+    qkv = oracle.linear(x, dense[0], wq.scales, wq.bias, oracle.I8, scales["qkv"], threads=threads)
+    ctx = oracle.requant_f32(oracle.attention_f64(qkv, scales["qkv"], nseq, seq, threads=threads).astype(np.float32),
+                             scales["ctx"])
+    z1 = oracle.linear_resid(ctx, dense[1], wo.scales, wo.bias, x, x_scale, threads=threads)
+    h1 = oracle.requant_f32(oracle.layernorm(z1, g1, b1, eps).astype(np.float32), ln_scale)
+    f1 = oracle.linear(h1, dense[2], w1.scales, w1.bias, oracle.I8_GELU, scales["ffn1"], threads=threads)
+    z2 = oracle.linear_resid(f1, dense[3], w2.scales, w2.bias, h1, ln_scale, threads=threads)
+    oracle.requant_f32(oracle.layernorm(z2, g2, b2, eps).astype(np.float32), ln_scale)
+    dt = time.perf_counter() - t0
+    ops = sum(2.0 * nseq * seq * w.nnzb * 4 for w in weights)
+    return {"value": round(ops / dt / 1e12, 6), "unit": UNIT, "cores": threads, "kind": "oracle",
+            "tokens_per_s": round(nseq * seq / dt, 1),
+            "sample": f"{nseq} sequences of {seq} tokens through the whole layer (dense triple loops over the "
+                      f"decompressed weights, fp64 attention, LayerNorms), {threads} host threads, {dt:.2f} s"}
+
+
 # -------------------------------------------------------- reference arm --
 
 def run_reference_prune(args) -> dict:
@@ -842,6 +873,10 @@ def run_encoder(args) -> dict:
     ln_bytes = m * 768 * 4 + m * 768 + 2 * 768 * 4  # z read once, int8 out, gamma and beta
     attn = attention_roofline(batch, seq, heads, attn_ms, props.multi_processor_count,
                               clocks.get("sm_max_mhz") or 2070.0, hbm_peak, bf16_peak)
+    cpu = None
+    if not args.no_cpu_baseline:
+        cpu = encoder_cpu_baseline(weights, x0, scales, seq, *(t.cpu().numpy() for t in (g1, b1, g2, b2)),
+                                   x_scale, ln_scale, eps)
     for lin in lins:
         lin.close()
     return {
@@ -861,6 +896,7 @@ def run_encoder(args) -> dict:
                       "hbm_frac": round(ln_bytes / (ln_ms * 1e-3) / 1e9 / hbm_peak, 4),
                       "basis": "graph of 200 LayerNorm launches, per launch; bytes = fp32 z read once + int8 out"},
         "attention": attn,
+        "cpu_baseline": cpu,
         "roofline": {"bound": "alu", "achieved": round(sum(ops) / (ms * 1e-3) / 1e12, 3), "peak": round(peak, 2),
                      "unit": "TOPS", "frac": round(sum(ops) / (ms * 1e-3) / 1e12 / peak, 4), "traffic": None,
                      "kernel": "whole layer (4 linears + attention + 2 LayerNorms)"},

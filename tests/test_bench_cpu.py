@@ -44,3 +44,23 @@ def test_profile_traffic_follows_the_kernel_source(tmp_path, monkeypatch):
     assert bench.profile_traffic("x") is None
     assert bench.profile_traffic("y") == 7
     assert bench.profile_traffic("missing") is None
+
+
+def test_encoder_cpu_baseline_runs_the_oracle_layer():
+    """One sequence through the oracle's whole layer: the value counts the
+    four linears' effective ops over the measured time."""
+    import json
+
+    import numpy as np
+
+    import synth
+    with open(bench.LAYER_SCALES) as f:
+        scales = json.load(f)["scales"]
+    weights, x0 = synth.encoder_layer()
+    g = np.ones(768, np.float32)
+    z = np.zeros(768, np.float32)
+    r = bench.encoder_cpu_baseline(weights, x0, scales, 384, g, z, g, z, 0.02, 4.0 / 127.0, 1e-12, threads=4, nseq=1)
+    assert r["kind"] == "oracle" and r["cores"] == 4 and r["unit"] == bench.UNIT
+    ops = sum(2.0 * 384 * w.nnzb * 4 for w in weights)
+    dt = 384 / r["tokens_per_s"]
+    assert abs(r["value"] - ops / dt / 1e12) <= 1e-3 * r["value"] + 1e-6
