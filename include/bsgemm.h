@@ -170,10 +170,12 @@ int bsgemm_run_ws(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilog
  * BSGEMM_STATIC_SCRATCH_BYTES (16 MiB) that the library holds in device
  * memory, one per device.  The paper has no counterpart; this entry point
  * serves callers that must not allocate at run time.
- *   Limit: bsgemm_workspace_bytes(h, M) <= BSGEMM_STATIC_SCRATCH_BYTES,
+ *   Limit, only where the scratch is used (K % 16 != 0, or act not 16-byte
+ *   aligned): bsgemm_workspace_bytes(h, M) <= BSGEMM_STATIC_SCRATCH_BYTES,
  *   i.e. M <= floor(16 MiB / (round_up(K, 16) * T)) * T tokens
- *   (T = bsgemm_info()[4]; M <= 5440 at K = 3072, M <= 21760 at K = 768).
- *   A larger M returns BSGEMM_ERR_INVALID (use bsgemm_run_ws).
+ *   (T = bsgemm_info()[4]; M <= 5440 at K = 3072, M <= 21824 at K = 768).
+ *   A larger M there returns BSGEMM_ERR_INVALID (use bsgemm_run_ws); on the
+ *   fast path any M is accepted.
  *   Set-up: the first call on each device looks up the scratch array's
  *   address (cudaGetSymbolAddress) with that device current and caches it;
  *   make that first call before any stream capture.
@@ -322,6 +324,26 @@ int bsgemm_attention(const int8_t* qkv, int batch, int seq, int heads, int head_
  */
 #define BSGEMM_STATUS_TIMEOUT 1
 int bsgemm_device_status(bsgemm_t h, int clear);
+
+/*
+ * bsgemm_set_test_hooks -- make the bounded waits give up on purpose, so
+ * that a test can check the failure path without faulting or hanging a GPU
+ * (the paper has no counterpart; its engine runs on a CPU).  The bits apply
+ * to every later launch in the process until they are set back to 0:
+ *   BSGEMM_TEST_SKIP_TILE_COPY: the layer kernel issues no copy of a token
+ *     tile and gives each wait on one up after 64 polls.  No copy is then in
+ *     flight when a CTA leaves; the run's output is undefined and the
+ *     handle's device status gets BSGEMM_STATUS_TIMEOUT.  Staging by
+ *     per-thread loads (no copies) is unaffected.
+ *   BSGEMM_TEST_STALL_PRUNE_CTA: CTA 0 of the pruning kernel leaves before
+ *     its first grid barrier and the other CTAs give that barrier up after
+ *     4096 polls; every CTA returns and bsgemm_block_prune returns
+ *     BSGEMM_ERR_CUDA (keep is undefined).
+ * Not for production use.  Returns the previous bits.
+ */
+#define BSGEMM_TEST_SKIP_TILE_COPY 1u
+#define BSGEMM_TEST_STALL_PRUNE_CTA 2u
+uint32_t bsgemm_set_test_hooks(uint32_t bits);
 
 /*
  * bsgemm_destroy -- free the handle and its device memory.  The caller must

@@ -5,6 +5,7 @@
 #include "bsgemm.h"
 
 #include <algorithm>
+#include <atomic>
 #include <cfloat>
 #include <cmath>
 #include <cstring>
@@ -31,6 +32,7 @@ struct bsgemm_ctx {
 
 namespace {
 
+std::atomic<uint32_t> g_test_hooks{0};  // bsgemm_set_test_hooks
 thread_local std::string g_error;
 thread_local int g_status = BSGEMM_OK;
 
@@ -137,7 +139,11 @@ int make_schedule(const std::vector<int32_t>& cost, long long upt, long long nti
 
 }  // namespace
 
+unsigned bsg::test_hooks() { return g_test_hooks.load(); }
+
 extern "C" {
+
+uint32_t bsgemm_set_test_hooks(uint32_t bits) { return g_test_hooks.exchange(bits); }
 
 const char* bsgemm_last_error(void) { return g_error.c_str(); }
 
@@ -441,6 +447,8 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.kind = epi.kind;
     a.inv_out_scale = inv;
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
+    a.skip_copy = (g_test_hooks.load() & BSGEMM_TEST_SKIP_TILE_COPY) != 0;
+    a.wait_limit = a.skip_copy ? 64u : 0u;
     const long long ntiles = (static_cast<long long>(M) + bsg::kTile - 1) / bsg::kTile;
     const long long upt = h->w.ngroups;  // units per token tile
     long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
@@ -486,7 +494,9 @@ int bsgemm_run_tiled(bsgemm_t h, const void* tiles, size_t tiles_bytes, int M, v
 int bsgemm_run_static(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_epilogue epi, void* stream) {
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
-    if (M > 0) {
+    // With K % 16 == 0 and act 16-byte aligned the layer kernel stages its
+    // tiles itself and the scratch is not touched: no limit on M then.
+    if (M > 0 && !bsg::tensor_staging(h->w.K, act)) {
         const size_t need = bsg::tiled_bytes(h->w.K, M);
         if (need > BSGEMM_STATIC_SCRATCH_BYTES) {
             const size_t per_tile = bsg::tiled_bytes(h->w.K, bsg::kTile);
