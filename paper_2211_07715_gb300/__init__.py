@@ -26,6 +26,7 @@ LIB_PATH = os.path.join(_PKG, "libbsgemm.so")
 BLOCK = 4
 OUT_I32, OUT_F32, OUT_F32_GELU, OUT_I8, OUT_I8_GELU, OUT_F32_RESID = 0, 1, 2, 3, 4, 5
 ERR_INVALID, ERR_UNSUPPORTED, ERR_CUDA = -1, -2, -3
+STATUS_TIMEOUT = 1  # BSGEMM_STATUS_TIMEOUT: a bounded wait on an asynchronous copy gave up
 STATIC_SCRATCH_BYTES = 16 << 20  # BSGEMM_STATIC_SCRATCH_BYTES: the token-tile scratch of bsgemm_run_static
 
 
@@ -87,6 +88,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_attention.restype = ctypes.c_int
     lib.bsgemm_device_status.argtypes = [vp, ctypes.c_int]
     lib.bsgemm_device_status.restype = ctypes.c_int
+    lib.bsgemm_set_test_hooks.argtypes = [ctypes.c_uint32]
+    lib.bsgemm_set_test_hooks.restype = ctypes.c_uint32
     return lib
 
 
@@ -96,7 +99,8 @@ EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static",
             "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_run_kmajor",
             "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_layernorm",
             "bsgemm_attention", "bsgemm_destroy",
-            "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info")
+            "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info",
+            "bsgemm_set_test_hooks")
 
 
 def _epi(kind: int, out_scale: float, flags: int = 0, residual: int = 0, residual_scale: float = 1.0) -> Epilogue:
@@ -298,6 +302,16 @@ def bsgemm_device_status(h: int, clear: bool = False) -> int:
     if rc < 0:
         raise BsgemmError(rc, bsgemm_last_error())
     return rc
+
+
+TEST_SKIP_TILE_COPY = 1  # BSGEMM_TEST_SKIP_TILE_COPY
+TEST_STALL_PRUNE_CTA = 2  # BSGEMM_TEST_STALL_PRUNE_CTA
+
+
+def bsgemm_set_test_hooks(bits: int) -> int:
+    """Make the kernels' bounded waits give up on purpose (tests of the
+    failure path only); returns the previous bits."""
+    return int(_lib.bsgemm_set_test_hooks(int(bits)))
 
 
 def bsgemm_destroy(h: int) -> None:

@@ -72,6 +72,8 @@ struct LaunchArgs {
     const int8_t* res;     // kind 5: int8 residual [M][N]
     float res_scale;       // kind 5: the residual's scale
     int ld;                // row stride of x^T in bytes (kmajor only)
+    unsigned wait_limit;   // polls of a wait on a tile copy before it gives up (0: the default)
+    bool skip_copy;        // test hook: issue no tile copy, so that every such wait gives up
 };
 
 // Kernel configuration: 8 warps per CTA (2 per SM sub-partition, up to 255
@@ -119,6 +121,9 @@ cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, c
 // stream-ordered scratch and synchronises `s`; *bad = a weight was not finite.
 cudaError_t block_prune(const float* W, int N, int K, long long npruned, uint8_t* keep, int sms, cudaStream_t s,
                         bool* bad);
+// Test hooks for the bounded waits (BSGEMM_TEST_* bits of
+// bsgemm_set_test_hooks), read at each launch.
+unsigned test_hooks();
 // Address of the fixed token-tile scratch (BSGEMM_STATIC_SCRATCH_BYTES) on
 // `device`, which must be the current device; looked up on the first call
 // per device, then cached.

@@ -17,6 +17,7 @@
 #include <cstdint>
 #include <mutex>
 
+#include "bsgemm.h"
 #include "bsgemm_internal.h"
 
 namespace bsg {
@@ -41,7 +42,7 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
 
 // Grid barrier number `n` (0, 1, ...): every CTA arrives once; returns false
 // (in every thread of the CTA) if the wait gave up.
-__device__ bool grid_barrier(PruneScratch* st, unsigned n) {
+__device__ bool grid_barrier(PruneScratch* st, unsigned n, unsigned limit) {
     __shared__ int s_ok;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -49,8 +50,8 @@ __device__ bool grid_barrier(PruneScratch* st, unsigned n) {
         atomicAdd(&st->barrier, 1u);
         const unsigned target = (n + 1) * gridDim.x;
         unsigned i = 0;
-        while (ld_acquire(&st->barrier) < target && i < kBarrierLimit) ++i;
-        s_ok = i < kBarrierLimit;
+        while (ld_acquire(&st->barrier) < target && i < limit) ++i;
+        s_ok = i < limit;
         if (!s_ok) atomicOr(&st->bad, 2);
         __threadfence();
     }
@@ -90,7 +91,7 @@ __device__ void select_byte(const unsigned long long* hist, int pass, unsigned l
 __global__ void __launch_bounds__(kPruneThreads)
 prune_kernel(const float* __restrict__ W, int nbr, int K, unsigned long long npruned,
              unsigned long long* __restrict__ key, unsigned int* __restrict__ cnt, PruneScratch* st,
-             uint8_t* __restrict__ keep) {
+             uint8_t* __restrict__ keep, unsigned barrier_limit, int leave_cta) {
     __shared__ unsigned int h[256];
     __shared__ unsigned int ws[kPruneThreads / 32];
     __shared__ unsigned long long s_base;
@@ -135,7 +136,8 @@ prune_kernel(const float* __restrict__ W, int nbr, int K, unsigned long long npr
     for (int i = threadIdx.x; i < 256; i += blockDim.x)
         if (h[i]) atomicAdd(&st->hist[0][i], static_cast<unsigned long long>(h[i]));
     unsigned nb = 0;
-    if (!grid_barrier(st, nb++)) return;
+    if (static_cast<int>(blockIdx.x) == leave_cta) return;  // test hook: the others' first barrier gives up
+    if (!grid_barrier(st, nb++, barrier_limit)) return;
 
     // Radix select of the key at rank npruned (0 < npruned < total).
     unsigned long long prefix = 0, rank = npruned;
@@ -159,7 +161,7 @@ prune_kernel(const float* __restrict__ W, int nbr, int K, unsigned long long npr
         __syncthreads();
         for (int i = threadIdx.x; i < 256; i += blockDim.x)
             if (h[i]) atomicAdd(&st->hist[pass][i], static_cast<unsigned long long>(h[i]));
-        if (!grid_barrier(st, nb++)) return;
+        if (!grid_barrier(st, nb++, barrier_limit)) return;
     }
     select_byte(st->hist[7], 7, prefix, rank);
     const unsigned long long T = prefix, need = rank;
@@ -188,7 +190,7 @@ prune_kernel(const float* __restrict__ W, int nbr, int K, unsigned long long npr
         for (int w = 0; w < kPruneThreads / 32; ++w) s += ws[w];
         cnt[blockIdx.x] = s;
     }
-    if (!grid_barrier(st, nb++)) return;
+    if (!grid_barrier(st, nb++, barrier_limit)) return;
 
     // equal keys in the chunks before this one
     unsigned long long b = 0;
@@ -303,7 +305,12 @@ cudaError_t block_prune(const float* W, int N, int K, long long npruned, uint8_t
             e = cudaGetLastError();
         } else {
             unsigned long long np = static_cast<unsigned long long>(npruned);
-            void* args[] = {const_cast<float**>(&W), const_cast<int*>(&nbr), &K, &np, &key, &cnt, &st, &keep};
+            // test hook: CTA 0 leaves before the first grid barrier, the others give up after a few polls
+            const bool stall = (test_hooks() & BSGEMM_TEST_STALL_PRUNE_CTA) != 0;
+            unsigned limit = stall ? 4096u : kBarrierLimit;
+            int leave = stall ? 0 : -1;
+            void* args[] = {const_cast<float**>(&W), const_cast<int*>(&nbr), &K, &np, &key, &cnt, &st, &keep,
+                            &limit, &leave};
             e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(prune_kernel), dim3(grid),
                                             dim3(kPruneThreads), args, 0, s);
         }
