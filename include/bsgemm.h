@@ -89,7 +89,7 @@ typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
  * Block-compressed layout (App. A.1 blocks; App. A.3.4 "the sparse weight is
  * compressed and the mask is used"), all HOST memory, read during the call
  * only (the caller keeps ownership and may free them on return):
- *   N        output features, N >= 1.  Block-row r holds rows 4r..4r+3;
+ *   N        output features, 1 <= N <= BSGEMM_MAX_N.  Block-row r holds rows 4r..4r+3;
  *            when N % 4 != 0 the last block-row, r = ceil(N/4) - 1, holds
  *            the N % 4 remaining rows and values[j][i] of its rows
  *            4r + i >= N are ignored (App. A.3.4 notes that such N need
@@ -116,6 +116,7 @@ typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
  * stored work grows by that union (the Python binding's from_blocks_1x4 /
  * from_2to4 build these arrays).
  */
+#define BSGEMM_MAX_N (4 * 65535) /* block-row indices are 16-bit inside the kernel */
 bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const int8_t* values,
                        const float* scales, const float* bias);
 

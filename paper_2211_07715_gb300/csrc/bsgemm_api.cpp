@@ -137,6 +137,100 @@ int make_schedule(const std::vector<int32_t>& cost, long long upt, long long nti
     return n;
 }
 
+// Column order of every step of every row group (create time).  Each half
+// of a step (8 columns: one quad of block-row 2h, one of block-row 2h + 1,
+// one pass of the kernel's shared-memory gather) takes its columns from
+// distinct bank groups of the swizzled token tile where it can: pick by
+// pick, the block-row whose fullest bucket of an unused bank key is largest
+// takes a column from it; a block-row whose remaining columns all sit on
+// used keys takes one anyway (a conflict, never an extra step); a block-row
+// with no columns left is padded with a zero-weight entry on an unused key
+// (columns 0..7 cover all 8 keys and are rows of every tile).  ent[16 s + e] = the stored-block index j of entry e of step s, or
+// -1 - (pad column).
+void order_steps(const int32_t* indptr, const int32_t* colidx, int ngroups, const std::vector<int32_t>& grow,
+                 const std::vector<int32_t>& gptr, int (*bank_key)(int), std::vector<int32_t>& ent) {
+    ent.assign(static_cast<size_t>(gptr[ngroups]) * 16, 0);
+    int pad_col[8];
+    for (int k = 0; k < 8; ++k) pad_col[bank_key(k)] = k;
+    std::vector<int> bucket[4][8];  // stored-block indices j of each block-row, by bank key
+    int left[4];
+    for (int gi = 0; gi < ngroups; ++gi) {
+        for (int q = 0; q < 4; ++q) {
+            for (auto& bk : bucket[q]) bk.clear();
+            left[q] = 0;
+            const int r = grow[4 * gi + q];
+            if (r < 0) continue;
+            for (int j = indptr[r + 1] - 1; j >= indptr[r]; --j) bucket[q][bank_key(colidx[j])].push_back(j);
+            left[q] = indptr[r + 1] - indptr[r];
+        }
+        for (int s = gptr[gi]; s < gptr[gi + 1]; ++s) {
+            int32_t* es = &ent[static_cast<size_t>(s) * 16];
+            for (int h = 0; h < 2; ++h) {
+                bool used[8] = {false, false, false, false, false, false, false, false};
+                int placed[2] = {0, 0};
+                for (int n = 0; n < 8; ++n) {
+                    // candidate of each of the two block-rows still short of 4 entries:
+                    // the size of its fullest bucket on an unused key (-1: none)
+                    int best_x = -1, best_key = -1, best_size = -2;
+                    for (int x = 0; x < 2; ++x) {
+                        const int q = 2 * h + x;
+                        if (placed[x] == 4) continue;
+                        int key = -1, size = -1;
+                        for (int kk = 0; kk < 8; ++kk)
+                            if (!used[kk] && static_cast<int>(bucket[q][kk].size()) > size && !bucket[q][kk].empty()) {
+                                key = kk;
+                                size = static_cast<int>(bucket[q][kk].size());
+                            }
+                        if (size > best_size || (size == best_size && left[q] > left[2 * h + best_x])) {
+                            best_x = x;
+                            best_key = key;
+                            best_size = size;
+                        }
+                    }
+                    const int q = 2 * h + best_x;
+                    const int e = 4 * q + placed[best_x];
+                    int j = -1, key = best_key;
+                    if (key < 0 && left[q] > 0) {  // its columns sit on used keys only: take a conflict
+                        for (int kk = 0; kk < 8; ++kk)
+                            if (key < 0 || bucket[q][kk].size() > bucket[q][key].size()) key = kk;
+                    }
+                    if (key >= 0 && left[q] > 0) {
+                        j = bucket[q][key].back();
+                        bucket[q][key].pop_back();
+                        --left[q];
+                    } else {  // padding on an unused key (any key if all are used)
+                        key = 0;
+                        for (int kk = 7; kk >= 0; --kk)
+                            if (!used[kk]) key = kk;
+                    }
+                    used[key] = true;
+                    ++placed[best_x];
+                    es[e] = j >= 0 ? j : -1 - pad_col[key];
+                }
+            }
+        }
+    }
+}
+
+// One step's 16 entries: off[e] = the tile offset of its column (row_off of
+// the layout), w[q][c] byte e % 4 = W[4 r_q + c][column of entry 4q + e % 4]
+// (0 for padding).
+void step_entries(const int32_t* es, const int32_t* colidx, const int8_t* values, uint32_t (*row_off)(int),
+                  int32_t* off, uint32_t (&w)[4][4]) {
+    for (int e = 0; e < 16; ++e) {
+        const int j = es[e];
+        const int q = e / 4;
+        if (j >= 0) {
+            off[e] = static_cast<int32_t>(row_off(colidx[j]));
+            for (int c = 0; c < 4; ++c)
+                w[q][c] |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(j) * 4 + c]))
+                           << (8 * (e % 4));
+        } else {
+            off[e] = static_cast<int32_t>(row_off(-1 - j));
+        }
+    }
+}
+
 }  // namespace
 
 unsigned bsg::test_hooks() { return g_test_hooks.load(); }
@@ -160,6 +254,10 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
     }
     if (N < 1 || K < 1) {
         fail(BSGEMM_ERR_INVALID, "need N >= 1 and K >= 1");
+        return nullptr;
+    }
+    if (N > BSGEMM_MAX_N) {  // block-row indices are 16-bit fields in the kernel's group window
+        fail(BSGEMM_ERR_UNSUPPORTED, "N = " + std::to_string(N) + " exceeds " + std::to_string(BSGEMM_MAX_N));
         return nullptr;
     }
     if (K > bsg::max_k()) {
@@ -198,16 +296,8 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
 
     // Repack into row groups and steps.  Block-rows sorted by stored-block
     // count (longest first, ties by index) are taken 4 at a time, so a
-    // group's block-rows need about the same number of quads.  Each half of
-    // a step (8 columns: one quad of block-row 2h, one of block-row 2h + 1,
-    // one pass of the kernel's shared-memory gather) takes its columns from
-    // distinct bank groups of the swizzled token tile where it can: pick by
-    // pick, the block-row whose fullest bucket of an unused bank key is
-    // largest takes a column from it; a block-row whose remaining columns
-    // all sit on used keys takes one anyway (a conflict, never an extra
-    // step); a block-row with no columns left is padded with a zero-weight
-    // entry on an unused key (columns 0..7 cover all 8 keys and are rows of
-    // every tile, which has round_up(K, 16) >= 16 rows).
+    // group's block-rows need about the same number of quads; the columns
+    // of each step are ordered by order_steps.
     const int ngroups = (nbr + 3) / 4;
     std::vector<int> rows_sorted(nbr);
     for (int r = 0; r < nbr; ++r) rows_sorted[r] = r;
@@ -223,82 +313,23 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
             grow[4 * gi + q] = r;
             quads = std::max(quads, (indptr[r + 1] - indptr[r] + 3) / 4);
         }
+        quads = (quads + bsg::kBlock - 1) / bsg::kBlock * bsg::kBlock;  // whole blocks of the kernel's ring
         gptr[gi + 1] = gptr[gi] + quads;
         cost[gi + 1] = static_cast<int32_t>(cost[gi] + quads + (quads > 0 ? kGroupCost : 0));
     }
     const int S = gptr[ngroups];
+    // 128-byte step records: each step's columns in the order order_steps
+    // gives, its channel words beside them.
     std::vector<int32_t> recs(static_cast<size_t>(S + bsg::kStepPad) * 32, 0);
-    int pad_col[8];
-    for (int k = 0; k < 8; ++k) pad_col[bsg::bank_key(k)] = k;
     {
-        std::vector<int> bucket[4][8];  // stored-block indices j of each block-row, by bank key
-        int left[4];
-        for (int gi = 0; gi < ngroups; ++gi) {
-            for (int q = 0; q < 4; ++q) {
-                for (auto& bk : bucket[q]) bk.clear();
-                left[q] = 0;
-                const int r = grow[4 * gi + q];
-                if (r < 0) continue;
-                for (int j = indptr[r + 1] - 1; j >= indptr[r]; --j) bucket[q][bsg::bank_key(colidx[j])].push_back(j);
-                left[q] = indptr[r + 1] - indptr[r];
-            }
-            for (int s = gptr[gi]; s < gptr[gi + 1]; ++s) {
-                int32_t* rec = &recs[static_cast<size_t>(s) * 32];
-                uint32_t wwords[4][4] = {};
-                for (int h = 0; h < 2; ++h) {
-                    bool used[8] = {false, false, false, false, false, false, false, false};
-                    int placed[2] = {0, 0};
-                    for (int n = 0; n < 8; ++n) {
-                        // candidate of each of the two block-rows still short of 4 entries:
-                        // the size of its fullest bucket on an unused key (-1: none)
-                        int best_x = -1, best_key = -1, best_size = -2;
-                        for (int x = 0; x < 2; ++x) {
-                            const int q = 2 * h + x;
-                            if (placed[x] == 4) continue;
-                            int key = -1, size = -1;
-                            for (int kk = 0; kk < 8; ++kk)
-                                if (!used[kk] && static_cast<int>(bucket[q][kk].size()) > size &&
-                                    !bucket[q][kk].empty()) {
-                                    key = kk;
-                                    size = static_cast<int>(bucket[q][kk].size());
-                                }
-                            if (size > best_size || (size == best_size && left[q] > left[2 * h + best_x])) {
-                                best_x = x;
-                                best_key = key;
-                                best_size = size;
-                            }
-                        }
-                        const int q = 2 * h + best_x;
-                        const int e = 4 * q + placed[best_x];
-                        int j = -1, key = best_key;
-                        if (key < 0 && left[q] > 0) {  // its columns sit on used keys only: take a conflict
-                            for (int kk = 0; kk < 8; ++kk)
-                                if (key < 0 || bucket[q][kk].size() > bucket[q][key].size()) key = kk;
-                        }
-                        if (key >= 0 && left[q] > 0) {
-                            j = bucket[q][key].back();
-                            bucket[q][key].pop_back();
-                            --left[q];
-                        } else {  // padding on an unused key (any key if all are used)
-                            key = 0;
-                            for (int kk = 7; kk >= 0; --kk)
-                                if (!used[kk]) key = kk;
-                        }
-                        used[key] = true;
-                        ++placed[best_x];
-                        if (j >= 0) {
-                            rec[e] = static_cast<int32_t>(bsg::tile_row_offset(colidx[j]));
-                            for (int c = 0; c < 4; ++c)
-                                wwords[q][c] |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(j) * 4 + c]))
-                                                << (8 * (e % 4));
-                        } else {
-                            rec[e] = static_cast<int32_t>(bsg::tile_row_offset(pad_col[key]));
-                        }
-                    }
-                }
-                for (int q = 0; q < 4; ++q)
-                    for (int c = 0; c < 4; ++c) rec[16 + 4 * q + c] = static_cast<int32_t>(wwords[q][c]);
-            }
+        std::vector<int32_t> ent;
+        order_steps(indptr, colidx, ngroups, grow, gptr, bsg::bank_key, ent);
+        for (int s = 0; s < S; ++s) {
+            int32_t* rec = &recs[static_cast<size_t>(s) * 32];
+            uint32_t wwords[4][4] = {};
+            step_entries(ent.data() + 16 * static_cast<size_t>(s), colidx, values, bsg::tile_row_offset, rec, wwords);
+            for (int q = 0; q < 4; ++q)
+                for (int c = 0; c < 4; ++c) rec[16 + 4 * q + c] = static_cast<int32_t>(wwords[q][c]);
         }
     }
     // scales and biases padded with zeros to whole block-rows (the kernel
@@ -495,8 +526,10 @@ int bsgemm_run_static(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");
     // With K % 16 == 0 and act 16-byte aligned the layer kernel stages its
-    // tiles itself and the scratch is not touched: no limit on M then.
-    if (M > 0 && !bsg::tensor_staging(h->w.K, act)) {
+    // tiles itself and the scratch is not touched: bsgemm_run's one kernel,
+    // with no limit on M.
+    if (bsg::tensor_staging(h->w.K, act)) return run_common(h, act, M, out, epi, nullptr, 0, 0, stream);
+    if (M > 0) {
         const size_t need = bsg::tiled_bytes(h->w.K, M);
         if (need > BSGEMM_STATIC_SCRATCH_BYTES) {
             const size_t per_tile = bsg::tiled_bytes(h->w.K, bsg::kTile);

@@ -41,9 +41,9 @@ inline int bank_key(int k) { return static_cast<int>((tile_row_offset(k) >> 4) &
 //                    belong to the group's block-row q
 //   uint32 w[4][4] : w[q][c] = bytes W[4 r_q + c][k_{4q}] .. W[4 r_q + c][k_{4q+3}],
 //                    one dot-4 operand per output channel c of block-row q
-// A group has as many steps as its longest block-row has quads; shorter
-// block-rows are padded with zero-weight entries whose columns are valid
-// tile rows.  Within each half of a step (columns 0-7, 8-15) the columns'
+// A group has as many steps as its longest block-row has quads, rounded up
+// to a multiple of kBlock; shorter block-rows and the extra steps are padded
+// with zero-weight entries whose columns are valid tile rows.  Within each half of a step (columns 0-7, 8-15) the columns'
 // bank keys differ wherever the two block-rows' columns allow it.
 struct DeviceWeights {
     const int32_t* gptr;   // [ngroups + 1]
@@ -83,9 +83,10 @@ constexpr int kThreads = kWarps * 32;
 #ifndef BSG_RING
 #define BSG_RING 12
 #endif
-constexpr int kRing = BSG_RING;     // step records a warp keeps in flight (registers), 8..16
+constexpr int kRing = BSG_RING;     // step records a warp keeps in flight (registers): 3 blocks
+constexpr int kBlock = kRing / 3;   // every row group holds a multiple of kBlock steps (zero-weight padding)
 constexpr int kStepPad = kRing;     // zero step records after the last one (the record prefetch runs ahead)
-constexpr int kGroupWin = 448;      // row groups whose step offsets a CTA keeps in shared memory
+constexpr int kGroupWin = 128;      // row groups whose step offsets and block-rows a CTA keeps in shared memory
 constexpr int kMaxBoxes = 49;       // 64-column boxes of a token tile (K <= 3136)
 constexpr int kStaticSmem = 2304;   // bytes of static shared memory the kernel may use
 constexpr int kMaxGrid = 512;       // CTAs per launch at most

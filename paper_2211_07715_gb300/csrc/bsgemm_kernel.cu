@@ -52,6 +52,7 @@
 #include <cuda_runtime.h>
 
 #include "bsgemm.h"
+#include "bsgemm_device.cuh"
 #include "bsgemm_internal.h"
 
 namespace bsg {
@@ -59,7 +60,7 @@ namespace {
 
 constexpr int kSmemOptin = 232448;  // sm_103 opt-in shared memory per block
 constexpr int kSlots = kWarps - 1;  // one per split point between warp ranges
-static_assert(kRing == 8 || kRing == 12 || kRing == 16, "the record ring's switch has 8, 12 or 16 slots");
+static_assert(kRing == 3 * kBlock, "a ring round is three blocks of steps");
 // Cost of a row group's end (epilogue, stores) in steps, for splitting a
 // window's work evenly between warps.
 #ifndef BSG_GROUP_END_COST
@@ -86,183 +87,6 @@ __device__ __forceinline__ void transpose4(uint32_t a, uint32_t b, uint32_t c, u
     t3 = __byte_perm(ab_hi, cd_hi, 0x7632);            // a3 b3 c3 d3
 }
 
-// 1/b for 1 <= b < 2^25 by Newton's method, as a fixed sequence of IEEE
-// round-to-nearest fp32 operations (no branch, no special function unit):
-// b = m 2^E (1 <= m < 2, from the bits), y0 = 24/17 - (8/17) m (the minimax
-// straight line for 1/m, relative error <= 1/17; both constants rounded to
-// fp32), three steps y <- y + y (1 - m y) (each squares the relative error,
-// 1/17 -> 3.5e-3 -> 1.2e-5 -> 1.5e-10), then the exact scaling by 2^-E.
-// Within about half an ulp of 1/b, the same bits on every IEEE machine.
-__device__ __forceinline__ float recip_nr_f32(float b) {
-    const uint32_t bits = __float_as_uint(b);
-    const uint32_t ex = (bits >> 23) & 0xffu;  // E + 127
-    const float m = __uint_as_float((bits & 0x7fffffu) | (127u << 23));
-    float y = __fmaf_rn(-0x1.e1e1e2p-2f, m, 0x1.69696ap+0f);
-#pragma unroll
-    for (int i = 0; i < 3; ++i) y = __fmaf_rn(y, __fmaf_rn(-m, y, 1.0f), y);
-    return __fmul_rn(y, __uint_as_float((254u - ex) << 23));  // 2^-E: biased exponent 127 - E
-}
-
-// erf-form GELU in fp32 by a fixed sequence of IEEE round-to-nearest ops.
-// erf(|x|) = 1 - p(|x|)^-16, p = 1 + a1 x + ... + a6 x^6 (Abramowitz &
-// Stegun 7.1.28, |error| <= 3e-7); p^16 by four squarings; 1/p^16 by
-// recip_nr_f32 below 2^25, and erf = 1 from there on (where 1 - 1/p^16
-// rounds to 1 in fp32 whatever the quotient's last bits).  Branch-free, so
-// the 32 values of a lane's epilogue interleave.
-__device__ __forceinline__ float gelu_f32(float y) {
-    const float x = __fmul_rn(y, 0.70710678f);
-    const float ax = fabsf(x);
-    float h = __fmaf_rn(ax, 0.0000430638f, 0.0002765672f);
-    h = __fmaf_rn(ax, h, 0.0001520143f);
-    h = __fmaf_rn(ax, h, 0.0092705272f);
-    h = __fmaf_rn(ax, h, 0.0422820123f);
-    h = __fmaf_rn(ax, h, 0.0705230784f);
-    const float p = __fmaf_rn(ax, h, 1.0f);
-    const float p2 = __fmul_rn(p, p);
-    const float p4 = __fmul_rn(p2, p2);
-    const float p8 = __fmul_rn(p4, p4);
-    const float p16 = __fmul_rn(p8, p8);
-    const float r = recip_nr_f32(fminf(p16, 0x1.fffffep24f));  // p16 below 2^25 unchanged; unused from there on
-    const float e = (p16 >= 0x1p25f) ? 1.0f : __fsub_rn(1.0f, r);
-    const float erf_x = (x < 0.0f) ? -e : e;
-    return __fmul_rn(__fmul_rn(0.5f, y), __fadd_rn(1.0f, erf_x));
-}
-
-// The same erf-form GELU for fp32 outputs, with the hardware's approximate
-// reciprocal (relative error <= 2^-22) in place of the IEEE one: fp32
-// outputs are checked against a tolerance, not bit for bit, and the extra
-// error stays below 2e-7 |y|.  int8 outputs use gelu_f32, which an int8
-// decision must reproduce exactly.
-__device__ __forceinline__ float gelu_f32_fast(float y) {
-    const float x = y * 0.70710678f;
-    const float ax = fabsf(x);
-    float h = fmaf(ax, 0.0000430638f, 0.0002765672f);
-    h = fmaf(ax, h, 0.0001520143f);
-    h = fmaf(ax, h, 0.0092705272f);
-    h = fmaf(ax, h, 0.0422820123f);
-    h = fmaf(ax, h, 0.0705230784f);
-    const float p = fmaf(ax, h, 1.0f);
-    const float p2 = p * p, p4 = p2 * p2, p8 = p4 * p4, p16 = p8 * p8;
-    float rcp;
-    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(rcp) : "f"(p16));
-    const float e = 1.0f - rcp;
-    return 0.5f * y * (1.0f + ((x < 0.0f) ? -e : e));
-}
-
-// fp32 -> int8 for 4 values: one fp32 multiply each, round half to even
-// (to int32, saturating), then saturate to [-128, 127] and pack v0 into
-// byte 0 .. v3 into byte 3 (cvt.pack.sat: b into the low byte, a into the
-// next, c's low half above).
-__device__ __forceinline__ uint32_t requant4_s8(float v0, float v1, float v2, float v3, float inv) {
-    const int q0 = __float2int_rn(__fmul_rn(v0, inv)), q1 = __float2int_rn(__fmul_rn(v1, inv));
-    const int q2 = __float2int_rn(__fmul_rn(v2, inv)), q3 = __float2int_rn(__fmul_rn(v3, inv));
-    uint32_t hi, d;
-    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(hi) : "r"(q3), "r"(q2), "r"(0));
-    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(q1), "r"(q0), "r"(hi));
-    return d;
-}
-
-// Epilogue for one token m (nothing past M): v = acc of the 4 channels of
-// block-row r (scales s, bias b), written as out[m][4r .. 4r+3].
-// The epilogue value of channel c (c < 4) of one token: acc, or y =
-// fmaf((float)acc, s, b) with optional GELU.
-template <int KIND>
-__device__ __forceinline__ float epilogue_value(int v, float s, float b) {
-    float y = __fmaf_rn(__int2float_rn(v), s, b);
-    if (KIND == 2) y = gelu_f32_fast(y);
-    if (KIND == 4) y = gelu_f32(y);
-    return y;
-}
-
-template <int KIND>
-__device__ __forceinline__ void store_token(const LaunchArgs& a, int N, long long m, int r, const int* v, float4 s,
-                                            float4 b) {
-    if (m >= a.M) return;
-    const size_t o = static_cast<size_t>(m) * N + 4 * r;
-    if (KIND == 0) {
-        *reinterpret_cast<int4*>(static_cast<int32_t*>(a.out) + o) = make_int4(v[0], v[1], v[2], v[3]);
-        return;
-    }
-    float y0 = __fmaf_rn(__int2float_rn(v[0]), s.x, b.x);
-    float y1 = __fmaf_rn(__int2float_rn(v[1]), s.y, b.y);
-    float y2 = __fmaf_rn(__int2float_rn(v[2]), s.z, b.z);
-    float y3 = __fmaf_rn(__int2float_rn(v[3]), s.w, b.w);
-    if (KIND == 2) {
-        y0 = gelu_f32_fast(y0);
-        y1 = gelu_f32_fast(y1);
-        y2 = gelu_f32_fast(y2);
-        y3 = gelu_f32_fast(y3);
-    } else if (KIND == 4) {
-        y0 = gelu_f32(y0);
-        y1 = gelu_f32(y1);
-        y2 = gelu_f32(y2);
-        y3 = gelu_f32(y3);
-    }
-    if (KIND == 5) {  // residual add: z = y + res_scale * (float)r, two fp32 operations
-        const uint32_t r4 = __ldg(reinterpret_cast<const uint32_t*>(a.res + o));
-        y0 = __fadd_rn(y0, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4))));
-        y1 = __fadd_rn(y1, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4 >> 8))));
-        y2 = __fadd_rn(y2, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4 >> 16))));
-        y3 = __fadd_rn(y3, __fmul_rn(a.res_scale, __int2float_rn(static_cast<int8_t>(r4 >> 24))));
-    }
-    if (KIND == 1 || KIND == 2 || KIND == 5) {
-        *reinterpret_cast<float4*>(static_cast<float*>(a.out) + o) = make_float4(y0, y1, y2, y3);
-    } else {
-        *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(a.out) + o) = requant4_s8(y0, y1, y2, y3, a.inv_out_scale);
-    }
-}
-
-// N % 4 != 0: rows of out are not 16-byte aligned and the last block-row
-// has fewer than 4 channels -- one store a channel, channels < N only
-// (constant indices throughout, so acc stays in registers).
-template <int KIND>
-__device__ __forceinline__ void store_lane_narrow(const LaunchArgs& a, int N, long long m_g, int r,
-                                                  const int (&acc)[32], float4 sc, float4 bi) {
-    const int nc = min(4, N - 4 * r);
-    const float s4[4] = {sc.x, sc.y, sc.z, sc.w}, b4[4] = {bi.x, bi.y, bi.z, bi.w};
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const long long m = m_g + 8 * i;
-        if (m >= a.M) continue;
-        const size_t o = static_cast<size_t>(m) * N + 4 * r;
-        if (KIND == 0) {
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < nc) static_cast<int32_t*>(a.out)[o + c] = acc[4 * i + c];
-        } else if (KIND == 1 || KIND == 2) {
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < nc) static_cast<float*>(a.out)[o + c] = epilogue_value<KIND>(acc[4 * i + c], s4[c], b4[c]);
-        } else if (KIND == 5) {
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < nc)
-                    static_cast<float*>(a.out)[o + c] =
-                        __fadd_rn(epilogue_value<1>(acc[4 * i + c], s4[c], b4[c]),
-                                  __fmul_rn(a.res_scale, __int2float_rn(a.res[o + c])));
-        } else {
-            float y[4];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) y[c] = epilogue_value<KIND>(acc[4 * i + c], s4[c], b4[c]);
-            const uint32_t q = requant4_s8(y[0], y[1], y[2], y[3], a.inv_out_scale);
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < nc) static_cast<int8_t*>(a.out)[o + c] = static_cast<int8_t>(q >> (8 * c));
-        }
-    }
-}
-
-__device__ __forceinline__ float4 load_s4(const float* p, int r) { return __ldg(reinterpret_cast<const float4*>(p) + r); }
-
-// Last index r in [lo, hi) with sp[r] <= q, given sp[lo] <= q < sp[hi]
-// (sp: the shared-memory window of row-group step offsets).
-__device__ __forceinline__ int row_of(const int* sp, int lo, int hi, int q) {
-    while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (sp[mid] <= q) lo = mid; else hi = mid;
-    }
-    return lo;
-}
 
 // Byte offset of chunk 0 of activation column k in a swizzled token tile
 // (rows 2i, 2i+1 share 128-byte line i; chunk c of row k in 16-byte slot
@@ -343,69 +167,6 @@ __device__ __forceinline__ void stage_tile(unsigned char* xt, const LaunchArgs& 
     }
 }
 
-// 32-bit shared-window address of a shared-memory pointer.
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-// Gather two 16 x 16 byte matrices from shared memory, transposed: lane i
-// gives the address of row (i % 16) of matrix i / 16 (16 bytes, 16-byte
-// aligned); lane l receives, for matrix 0 (r0, r1) and matrix 1 (r2, r3),
-// the bytes of rows 4 (l % 4) .. 4 (l % 4) + 3 at column l / 4 (r0, r2) and
-// column l / 4 + 8 (r1, r3), row 4 (l % 4) in the lowest byte.
-__device__ __forceinline__ void ldsm_x2_trans_b8(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                                 uint32_t& r3) {
-    asm volatile("ldmatrix.sync.aligned.m16n16.x2.trans.shared.b8 {%0, %1, %2, %3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
-}
-
-// mbarrier + bulk-copy (TMA) helpers.  Waits are bounded: a wait that
-// gives up reports false and the caller records kStatusTimeout.
-constexpr unsigned kWaitLimit = 1u << 20;
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, unsigned count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
-    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, unsigned bytes) {
-    asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}\n"
-                 ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, unsigned parity, unsigned limit) {
-    for (unsigned i = 0; i < limit; ++i) {
-        unsigned done;
-        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-                     " selp.u32 %0, 1, 0, p;\n}\n"
-                     : "=r"(done) : "r"(bar), "r"(parity) : "memory");
-        if (done) return true;
-    }
-    return false;
-}
-// Global -> shared bulk copy completing on an mbarrier (16-byte aligned, size % 16 == 0).
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, unsigned bytes, uint32_t bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
-                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
-}
-// One 2-D box of a tensor map (x = innermost coordinate, y = row) into
-// shared memory, completing on an mbarrier.
-__device__ __forceinline__ void tensor_g2s(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
-    asm volatile("cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n"
-                 ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar) : "memory");
-}
-__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
-    asm volatile("st.shared.u32 [%0], %1;\n" ::"r"(addr), "r"(v) : "memory");
-}
-// Programmatic dependent launch: both kernels are launched so that they may
-// start while the previous kernel of the stream finishes.  Before a kernel
-// reads its activations or writes any global memory, every thread waits
-// until the previous grid has completed and its writes are visible (a no-op
-// when there is none); early on it lets the next kernel launch.
-__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
-__device__ __forceinline__ void griddep_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
-
-// Order this thread's earlier generic-proxy shared-memory accesses before
-// later asynchronous-proxy (bulk copy) writes.
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }
 
 // Staging from the activations themselves (no relayout kernel): a tensor
 // copy brings box b of the token tile -- 64 tokens x columns 64b..64b+63,
@@ -484,9 +245,9 @@ struct RecPtr {
     const int4* rw;
     __device__ __forceinline__ RecPtr(const int4* recs, long long s, int lane, int q)
         : ro(reinterpret_cast<const int*>(recs + s * 8) + (lane & 15)), rw(recs + s * 8 + 4 + q) {}
-    __device__ __forceinline__ void load(int i, int& off, int4& w) const {
-        off = __ldg(ro + 32 * i);
-        w = __ldg(rw + 8 * i);
+    __device__ __forceinline__ void load(int i, int& off, int4& w, uint64_t pol) const {
+        off = ldg_hint(ro + 32 * i, pol);
+        w = ldg_hint(rw + 8 * i, pol);
     }
     __device__ __forceinline__ void advance(int steps) {
         ro += 32 * steps;
@@ -501,11 +262,22 @@ __device__ __forceinline__ void store_lane(const LaunchArgs& a, int N, long long
                                            float4 sc, float4 bi) {
     if (r < 0) return;
     if (N & 3) {
-        store_lane_narrow<KIND>(a, N, m_g, r, acc, sc, bi);
+        store_lane_narrow<KIND, 8>(a, N, m_g, r, acc, sc, bi);
         return;
     }
 #pragma unroll
     for (int i = 0; i < 8; ++i) store_token<KIND>(a, N, m_g + 8 * i, r, acc + 4 * i, sc, bi);
+}
+
+// Block-row q of a row group whose 4 block-rows are packed as 16-bit
+// fields (0xffff: none).
+__device__ __forceinline__ int block_row16(unsigned long long gr, int q) {
+    const int v = static_cast<int>((gr >> (16 * q)) & 0xffffu);
+    return v == 0xffff ? -1 : v;
+}
+__device__ __forceinline__ unsigned long long pack_rows16(int4 gr) {
+    auto f = [](int r) { return static_cast<unsigned long long>(r < 0 ? 0xffff : r); };
+    return f(gr.x) | f(gr.y) << 16 | f(gr.z) << 32 | f(gr.w) << 48;
 }
 
 // MODE: how a window's token tile reaches shared memory.
@@ -522,8 +294,10 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     constexpr bool KMAJOR = MODE == kStageKMajor;
     constexpr bool TENSOR = MODE == kStageTensor || KMAJOR;
     constexpr int SW = kTile * 16;  // slot words: 64 tokens x 4 block-rows x 4 channels
+    static_assert(kGroupWin < kThreads, "one thread loads each group of a window");
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int s_gp[kGroupWin + 1];                          // step offsets of the current group window
+    __shared__ unsigned long long s_grow[kGroupWin];             // their block-rows (block_row16)
     __shared__ __align__(8) unsigned long long s_bar[kMaxBoxes];  // completion of the tile's copies
     __shared__ int s_wst[kWarps + 1];                            // first step of each warp in the window (relative)
 
@@ -540,7 +314,11 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     const uint32_t lb = 16u * static_cast<uint32_t>(lane >> 4);
     const long long ng = w.ngroups;
     const unsigned wlim = a.wait_limit ? a.wait_limit : kWaitLimit;
+    const uint64_t pol_w = l2_policy_evict_last(), pol_x = l2_policy_evict_first();
 
+    // the tensor map's descriptor comes into the TMA unit's cache while the
+    // CTA sets up, ahead of the first tensor copy
+    if (TENSOR && tid == 0) asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(&xmap)) : "memory");
     griddep_launch_dependents();
     const uint32_t bar = smem_addr(&s_bar[0]);  // box b's barrier at bar + 8 b (TMA: box 0 only)
     if (TMA && tid == 0) mbar_init(bar, 1);
@@ -555,7 +333,13 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     const long long u_end = sched.u[blockIdx.x + 1];
 
     long long staged = -1;  // token tile currently in shared memory
-    bool waited = false;    // the previous grid's writes are visible
+    bool waited = false;    // the previous grid has completed and its writes are visible
+    auto wait_prev = [&]() {  // before this thread's global writes
+        if (!waited) {
+            griddep_wait();
+            waited = true;
+        }
+    };
     while (u < u_end) {
         // next window: one token tile, at most kGroupWin consecutive row groups
         const long long t = u / ng;
@@ -565,7 +349,15 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         const long long m0 = t * kTile;
         auto gp = [&](int gi) { return s_gp[gi - g_lo]; };
 
-        for (int i = tid; i <= g_hi - g_lo; i += kThreads) s_gp[i] = __ldg(w.gptr + g_lo + i);
+        // The window's step offsets and block-rows load before the tile's
+        // copies go out, so that they do not queue behind the tile's bytes
+        // (every CTA of a launch stages at once).
+        int gp_v = 0;
+        unsigned long long gr_v = ~0ull;
+        if (tid <= g_hi - g_lo) {
+            gp_v = ldg_hint(w.gptr + g_lo + tid, pol_w);
+            if (tid < g_hi - g_lo) gr_v = pack_rows16(ldg_hint(w.grow + g_lo + tid, pol_w));
+        }
         const bool stage = (t != staged);
         // the token tile (already swizzled in a.xb) in kTmaPiece-byte bulk
         // copies, issued by the lanes of warp 0 (one completion barrier)
@@ -576,9 +368,9 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 fence_proxy_async();
                 mbar_arrive_expect_tx(bar + 8u * b, 64u * kTile);
                 if (KMAJOR)  // rows 64b..64b+63 of x^T at tokens t*64.., landing as the tile's rows
-                    tensor_g2s(tb + 4096u * b, &xmap, static_cast<int>(t * kTile), 64 * b, bar + 8u * b);
+                    tensor_g2s_hint(tb + 4096u * b, &xmap, static_cast<int>(t * kTile), 64 * b, bar + 8u * b, pol_x);
                 else
-                    tensor_g2s(tb + 4096u * b, &xmap, 64 * b, static_cast<int>(t * kTile), bar + 8u * b);
+                    tensor_g2s_hint(tb + 4096u * b, &xmap, 64 * b, static_cast<int>(t * kTile), bar + 8u * b, pol_x);
             }
             if (TMA && stage && warp == 0) {
                 const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
@@ -597,6 +389,8 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         // kernel's end.
         const bool issued = waited || (TENSOR && a.act_ready);
         if (issued) copy_tile();
+        if (tid <= g_hi - g_lo) s_gp[tid] = gp_v;     // g_hi - g_lo + 1 <= kGroupWin + 1 entries
+        if (tid < g_hi - g_lo) s_grow[tid] = gr_v;    // g_hi - g_lo <= kGroupWin entries
         __syncthreads();  // the group window is visible
         const int sa = gp(g_lo);
         if (tid <= kWarps) {
@@ -615,8 +409,9 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 else hi = mid;
             }
             const long long into = target - (static_cast<long long>(s_gp[lo] - sa) + static_cast<long long>(lo) * kGroupEndCost);
-            const int len = s_gp[lo + 1] - s_gp[lo];
-            s_wst[tid] = (tid == kWarps) ? s_gp[ngw] - sa : s_gp[lo] - sa + static_cast<int>(into < len ? into : len);
+            const int len = s_gp[lo + 1] - s_gp[lo];  // a multiple of kBlock
+            const int in_grp = static_cast<int>(into < len ? into : len) & ~(kBlock - 1);
+            s_wst[tid] = (tid == kWarps) ? s_gp[ngw] - sa : s_gp[lo] - sa + in_grp;
         }
         __syncthreads();  // the warps' step ranges are visible
 
@@ -635,11 +430,10 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             const int gs = s_gp[j] - sa;
             fin = bnd > gs && bnd < s_gp[j + 1] - sa && s_wst[warp] <= gs;
             if (fin) {
-                const int4 gr = __ldg(w.grow + g_lo + j);
-                fin_r = q == 0 ? gr.x : q == 1 ? gr.y : q == 2 ? gr.z : gr.w;
-                if (KIND != 0 && fin_r >= 0) {
-                    fin_sc = load_s4(w.scale, fin_r);
-                    fin_bi = load_s4(w.bias, fin_r);
+                fin_r = block_row16(s_grow[j], q);
+                if (KIND != 0) {  // needed after the window; no wait here
+                    fin_sc = ldg_hint(reinterpret_cast<const float4*>(w.scale) + max(fin_r, 0), pol_w);
+                    fin_bi = ldg_hint(reinterpret_cast<const float4*>(w.bias) + max(fin_r, 0), pol_w);
                 }
             }
         }
@@ -654,13 +448,15 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         for (int i = 0; i < kRing; ++i) {
             off[i] = 0;
             wq[i] = make_int4(0, 0, 0, 0);
-            if (ws0 < ws1) rec.load(i, off[i], wq[i]);
+            if (ws0 < ws1) rec.load(i, off[i], wq[i], pol_w);
         }
 
         // Everything above reads only the weights: in the first window it
-        // overlaps the end of the previous kernel.  The activations and any
-        // global write wait for that kernel's completion.
-        if (!waited) {
+        // overlaps the end of the previous kernel.  The activations wait for
+        // that kernel's completion -- unless act_ready says they were complete
+        // before it began: then only this thread's first global write waits
+        // (wait_prev), and the steps overlap that kernel's end.
+        if (!waited && !(TENSOR && a.act_ready)) {
             griddep_wait();
             waited = true;
             if (!issued) copy_tile();
@@ -674,11 +470,11 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         // Row groups without any stored block: acc = 0.
         for (int gi = g_lo + warp; gi < g_hi; gi += kWarps) {
             if (gp(gi) == gp(gi + 1)) {
-                const int4 gr = __ldg(w.grow + gi);
-                const int r = q == 0 ? gr.x : q == 1 ? gr.y : q == 2 ? gr.z : gr.w;
+                const int r = block_row16(s_grow[gi - g_lo], q);
                 int zero[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) zero[i] = 0;
+                wait_prev();
                 if (r >= 0) store_lane<KIND>(a, N, m0 + g, r, zero, load_s4(w.scale, r), load_s4(w.bias, r));
             }
         }
@@ -697,6 +493,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             ++phase;
             if (__syncthreads_or(!ok)) {
                 if (tid == 0) {
+                    wait_prev();
                     atomicOr(w.status, kStatusTimeout);
                     for (int b = 0; b < nbox; ++b) mbar_wait(bar + 8u * b, (phase - 1) & 1u, wlim);  // one more chance
                 }
@@ -710,6 +507,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             ++phase;
             if (__syncthreads_or(!ok)) {
                 if (tid == 0) {
+                    wait_prev();
                     atomicOr(w.status, kStatusTimeout);
                     mbar_wait(bar, (phase - 1) & 1u, wlim);  // give the copy one more bounded chance to land
                 }
@@ -722,74 +520,60 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         if (ws0 < ws1) {
             int gi = g_lo + row_of(s_gp, 0, g_hi - g_lo, sa + ws0);
             int p = ws0;  // step index relative to sa
-            int ph = 0;   // ring slot holding step p
+            int blk = 0;  // ring block (slots 4 blk .. 4 blk + 3) holding step p
             while (p < ws1) {
                 const int gs = gp(gi), ge = gp(gi + 1);
                 const int p_end = min(ws1, ge - sa);
-                const int4 gr = __ldg(w.grow + gi);
-                const int r = q == 0 ? gr.x : q == 1 ? gr.y : q == 2 ? gr.z : gr.w;
+                const int r = block_row16(s_grow[gi - g_lo], q);
                 float4 sc = make_float4(0.f, 0.f, 0.f, 0.f), bi = sc;
-                if (KIND != 0 && r >= 0) {  // needed at the group's end; load it now
-                    sc = load_s4(w.scale, r);
-                    bi = load_s4(w.bias, r);
+                if (KIND != 0) {  // used at the group's end: the loads fly during its steps
+                    sc = ldg_hint(reinterpret_cast<const float4*>(w.scale) + max(r, 0), pol_w);
+                    bi = ldg_hint(reinterpret_cast<const float4*>(w.bias) + max(r, 0), pol_w);
                 }
                 int acc[32];
 #pragma unroll
                 for (int i = 0; i < 32; ++i) acc[i] = 0;
                 // Steps p .. p_end - 1.  Ring slot i holds step (ring base + i);
                 // after its step it loads step (base + kRing + i), and after
-                // slot kRing - 1 the base moves on by kRing.  Whole rounds of
-                // the ring run as one straight block (the compiler overlaps
-                // one step's gathers with the previous step's dp4a); the
-                // switch enters at the slot of step p, so a group may start
-                // or end at any slot.
+                // slot kRing - 1 the base moves on by kRing.  Groups hold a
+                // multiple of kBlock steps and warp ranges start at such a
+                // multiple, so a group starts and ends at a block boundary:
+                // whole rounds run as one straight block of kRing steps (the
+                // compiler overlaps one step's gathers with the previous
+                // step's dp4a), and a round that a group enters or leaves in
+                // the middle runs block by block (kBlock straight steps each).
                 while (p < p_end) {
-                    if (ph == 0 && p + kRing <= p_end) {
+                    if (blk == 0 && p + kRing <= p_end) {
 #pragma unroll
                         for (int i = 0; i < kRing; ++i) {
                             step16(tb, lb, off[i], wq[i], acc);
-                            rec.load(kRing + i, off[i], wq[i]);
+                            rec.load(kRing + i, off[i], wq[i], pol_w);
                         }
                         rec.advance(kRing);
                         p += kRing;
                         continue;
                     }
-                    switch (ph) {
-#define BSG_RING_SLOT(i)                                 \
-    case i:                                              \
-        step16(tb, lb, off[i], wq[i], acc);              \
-        rec.load(kRing + (i), off[i], wq[i]);            \
-        ++p;                                             \
-        if ((i) == kRing - 1) rec.advance(kRing);        \
-        if (p == p_end) {                                \
-            ph = ((i) + 1) % kRing;                      \
-            break;                                       \
-        }
-                        BSG_RING_SLOT(0)
-                        BSG_RING_SLOT(1)
-                        BSG_RING_SLOT(2)
-                        BSG_RING_SLOT(3)
-                        BSG_RING_SLOT(4)
-                        BSG_RING_SLOT(5)
-                        BSG_RING_SLOT(6)
-                        BSG_RING_SLOT(7)
-#if BSG_RING > 8
-                        BSG_RING_SLOT(8)
-                        BSG_RING_SLOT(9)
-                        BSG_RING_SLOT(10)
-                        BSG_RING_SLOT(11)
-#endif
-#if BSG_RING > 12
-                        BSG_RING_SLOT(12)
-                        BSG_RING_SLOT(13)
-                        BSG_RING_SLOT(14)
-                        BSG_RING_SLOT(15)
-#endif
-#undef BSG_RING_SLOT
-                        ph = 0;
+#define BSG_RING_BLOCK(j)                                                   \
+    _Pragma("unroll") for (int i = kBlock * (j); i < kBlock * ((j) + 1); ++i) { \
+        step16(tb, lb, off[i], wq[i], acc);                                  \
+        rec.load(kRing + i, off[i], wq[i], pol_w);                           \
+    }
+                    if (blk == 0) {
+                        BSG_RING_BLOCK(0)
+                        blk = 1;
+                    } else if (blk == 1) {
+                        BSG_RING_BLOCK(1)
+                        blk = 2;
+                    } else {
+                        BSG_RING_BLOCK(2)
+                        rec.advance(kRing);
+                        blk = 0;
                     }
+#undef BSG_RING_BLOCK
+                    p += kBlock;
                 }
                 if (gs >= sa + ws0 && ge <= sa + ws1) {
+                    wait_prev();
                     store_lane<KIND>(a, N, m0 + g, r, acc, sc, bi);
                 } else {
                     // Shared with other warps: add into the slot of the first warp
@@ -817,6 +601,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 acc[j] = sl[32 * j];
                 sl[32 * j] = 0;
             }
+            wait_prev();
             store_lane<KIND>(a, N, m0 + g, fin_r, acc, fin_sc, fin_bi);
         }
         if (u < u_end) __syncthreads();  // the window's offsets, the slots' reset and the tile may be reused
