@@ -73,16 +73,24 @@ std::string check_bsr(int N, int K, const int32_t* indptr, const int32_t* colidx
 }
 
 // Schedule costs, in steps (one quad of each of a row group's 4 block-rows
-// for 64 tokens: 32 dp4a per lane), from a least-squares fit of measured
-// CTA times on GB300 (FFN1/FFN2/QKV/attention-output shapes, M = 2K-8K):
-// a CTA spends about 19 cycles per step, 320 per row group (its epilogue)
-// and 6600 + 0.27 K per token tile it touches (the tile's copy into shared
-// memory, the warps' set-up and the spread of their finishing times).
+// for 64 tokens: 32 dp4a per lane), from per-CTA clock traces of the
+// kernel on GB300 (FFN1/FFN2/QKV/attention-output shapes, M = 3072-4096):
+// a CTA spends about 19 cycles per step and 17 steps' worth per row group
+// (its epilogue); a CTA that touches a second token tile runs 1.6K-5K
+// cycles longer than the first tile's cost predicts (the tile's copy into
+// shared memory, its transpose, the warps' set-up and finishing spread),
+// which puts a tile at 450 + 300 K / 3072 steps (tuned on the four shapes).
 #ifndef BSG_GROUP_COST
 #define BSG_GROUP_COST 17
 #endif
 constexpr long long kGroupCost = BSG_GROUP_COST;
-long long tile_cost(int K) { return 350 + 11LL * K / 768; }
+#ifndef BSG_TILE_COST_A
+#define BSG_TILE_COST_A 450
+#endif
+#ifndef BSG_TILE_COST_B
+#define BSG_TILE_COST_B 300
+#endif
+long long tile_cost(int K) { return BSG_TILE_COST_A + BSG_TILE_COST_B * static_cast<long long>(K) / 3072; }
 
 // End of the greedy range that starts at unit u under the cost bound C: it
 // takes whole units while the cost (units' cost + tc per token tile

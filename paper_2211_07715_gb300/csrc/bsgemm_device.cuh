@@ -217,6 +217,13 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, unsigned count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
 }
+// n consecutive barriers (8 bytes apart) with one arrival each, then one
+// fence that makes all the initialisations visible to the async proxy.
+__device__ __forceinline__ void mbar_init_n(uint32_t bar, int n) {
+    for (int i = 0; i < n; ++i)
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(bar + 8u * static_cast<uint32_t>(i)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+}
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, unsigned bytes) {
     asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}\n"
                  ::"r"(bar), "r"(bytes) : "memory");

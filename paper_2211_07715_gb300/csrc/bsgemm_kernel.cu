@@ -321,12 +321,9 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     if (TENSOR && tid == 0) asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(&xmap)) : "memory");
     griddep_launch_dependents();
     const uint32_t bar = smem_addr(&s_bar[0]);  // box b's barrier at bar + 8 b (TMA: box 0 only)
-    if (TMA && tid == 0) mbar_init(bar, 1);
-    if (TENSOR && tid < nbox) mbar_init(bar + 8u * tid, 1);
+    if ((TMA || TENSOR) && tid == 0) mbar_init_n(bar, TENSOR ? nbox : 1);
     // this warp's boxes: [bx0, bx1)
     const int bx0 = warp * nbox / kWarps, bx1 = (warp + 1) * nbox / kWarps;
-    // slots start at zero; whoever finishes a slot resets it
-    for (int i = tid; i < kSlots * SW / 4; i += kThreads) reinterpret_cast<int4*>(slots)[i] = make_int4(0, 0, 0, 0);
     __syncthreads();
     unsigned phase = 0;
     long long u = sched.u[blockIdx.x];
@@ -365,7 +362,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             if (a.skip_copy) return;  // test hook: the waits below give up
             if (TENSOR && stage && lane < bx1 - bx0) {  // lane i of each warp: the warp's box bx0 + i
                 const int b = bx0 + lane;
-                fence_proxy_async();
+                if (staged >= 0) fence_proxy_async();  // the previous tile's reads come first
                 mbar_arrive_expect_tx(bar + 8u * b, 64u * kTile);
                 if (KMAJOR)  // rows 64b..64b+63 of x^T at tokens t*64.., landing as the tile's rows
                     tensor_g2s_hint(tb + 4096u * b, &xmap, static_cast<int>(t * kTile), 64 * b, bar + 8u * b, pol_x);
@@ -375,7 +372,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             if (TMA && stage && warp == 0) {
                 const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
                 const int8_t* src = a.xb + static_cast<size_t>(t) * kpad * kTile;
-                fence_proxy_async();
+                if (staged >= 0) fence_proxy_async();
                 if (lane == 0) mbar_arrive_expect_tx(bar, bytes);
                 __syncwarp();
                 for (unsigned off = static_cast<unsigned>(lane) * kTmaPiece; off < bytes; off += 32u * kTmaPiece)
@@ -389,6 +386,9 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         // kernel's end.
         const bool issued = waited || (TENSOR && a.act_ready);
         if (issued) copy_tile();
+        if (staged < 0) {  // the split-group slots start at zero; whoever finishes a slot resets it
+            for (int i = tid; i < kSlots * SW / 4; i += kThreads) reinterpret_cast<int4*>(slots)[i] = make_int4(0, 0, 0, 0);
+        }
         if (tid <= g_hi - g_lo) s_gp[tid] = gp_v;     // g_hi - g_lo + 1 <= kGroupWin + 1 entries
         if (tid < g_hi - g_lo) s_grow[tid] = gr_v;    // g_hi - g_lo <= kGroupWin entries
         __syncthreads();  // the group window is visible
