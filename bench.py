@@ -54,9 +54,10 @@ UNIT = "TOPS"
 DP4A_LANES_PER_SM_CLK = 64   # int8 dot-4 lanes per SM per clock (half rate on sm_103)
 OPS_PER_DP4A = 8             # 4 multiply-adds
 KERNEL_SOURCES = ("paper_2211_07715_gb300/csrc/bsgemm_kernel.cu", "paper_2211_07715_gb300/csrc/bsgemm_internal.h",
-                  "paper_2211_07715_gb300/csrc/bsgemm_api.cpp")
+                  "paper_2211_07715_gb300/csrc/bsgemm_api.cpp", "paper_2211_07715_gb300/csrc/bsgemm_device.cuh")
 
 WORKLOADS = {"ffn2": synth.ffn2, "ffn1": synth.ffn1, "single": synth.single_768}
+REPEATS = 7  # timed replays of the --steps graph; the value is their median
 
 
 # ------------------------------------------------- replicas on N GPUs --
@@ -263,15 +264,21 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
     mark0 = sampler.mark()
     for i in range(soak):
         graph.replay()
-    barrier()
-    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    start.record(stream)
-    graph.replay()
-    end.record(stream)
-    end.synchronize()
-    barrier()
+    # The timed region: REPEATS replays of the graph of exactly --steps
+    # steps, each bracketed by a barrier and a synchronize; the median
+    # replay is the value, min and max are reported beside it.
+    replay_ms = []
+    for _ in range(REPEATS):
+        barrier()
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        start.record(stream)
+        graph.replay()
+        end.record(stream)
+        end.synchronize()
+        barrier()
+        replay_ms.append(start.elapsed_time(end))
     mark1 = sampler.mark()
-    elapsed_ms = start.elapsed_time(end)
+    elapsed_ms = statistics.median(replay_ms)
     if rank == 0:
         time.sleep(0.2)
         sampler.stop()
@@ -366,7 +373,7 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
         e2e_ms = s2.elapsed_time(t2)
 
     # the job's time is the slowest rank's
-    elapsed_ms, e2e_ms = max_over_ranks([elapsed_ms, e2e_ms], dev)
+    elapsed_ms, e2e_ms, min_ms, max_ms = max_over_ranks([elapsed_ms, e2e_ms, min(replay_ms), max(replay_ms)], dev)
     lin.close()
     if rank != 0:
         return None
@@ -408,6 +415,10 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
                    "l2": f"rotating {nsets} activation/output sets ({nsets * set_bytes / 2**20:.0f} MiB > 2 x L2)",
                    "parallelism": f"replicas x{world}", "soak_replays": soak,
                    "launch": "the timed steps are one CUDA graph of --steps steps (one bsgemm_run_ws kernel each)"},
+        "repeats": {"n": REPEATS, "median_ms_per_step": round(ms_per_step, 6),
+                    "min_ms_per_step": round(min_ms / args.steps, 6), "max_ms_per_step": round(max_ms / args.steps, 6),
+                    "basis": "replays of the one graph of --steps steps, each timed alone between barriers; value "
+                             "and ms_per_step are the median replay"},
         "stream_ms_per_step": round(stream_ms, 6),
         "hbm_gbs": round(hbm_gbs, 1),
         "hbm_frac": round(hbm_gbs / hbm_peak, 4),
@@ -428,13 +439,131 @@ def run_ours(args, rank: int, world: int, local_rank: int) -> dict | None:
             "ms_per_step": round(kmajor_ms, 6), "value": round(ops / (kmajor_ms * 1e-3) / 1e12, 3),
             "basis": "bsgemm_run_kmajor on the same batches stored K-major (X^T [K][M]), graph of --steps steps; "
                      "not the timed path"},
-        "gpu_launches": args.steps,
+        "gpu_launches": args.steps * REPEATS,
+        "gpu_launches_basis": f"{args.steps} bsgemm_kernel launches per timed replay x {REPEATS} replays",
         "clocks": clocks,
         "kernel_source_sha256": kernel_sha(),
     }
+    if world == 1:
+        meas = measure_int8_peaks(bsg, torch, dev)
+        result["roofline"]["peak_measured"] = meas
+        result["roofline"]["frac_of_measured_dp4a"] = round(tops_kernel / meas["dp4a"], 4)
+    if world == 1 and not args.no_configs:
+        result["configs"] = run_configs(args)
     if world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline(case, rows=None)
     return result
+
+
+def measure_int8_peaks(bsg, torch, dev) -> dict:
+    """Peak rates of the int8 units that could carry the layer, measured
+    live: dp4a and mma.sync m16n8k32 s8 (probe kernels of the library), and
+    cuBLASLt's int8 GEMM (torch._int_mm, 8192^3, best of 3)."""
+    out = {"dp4a": round(bsg.bsgemm_int8_peak(0), 1), "mma_sync_s8": round(bsg.bsgemm_int8_peak(1), 1)}
+    n = 8192
+    a = torch.randint(-128, 128, (n, n), dtype=torch.int8, device=dev)
+    b = torch.randint(-128, 128, (n, n), dtype=torch.int8, device=dev).t().contiguous().t()
+    torch._int_mm(a, b)
+    torch.cuda.synchronize(dev)
+    best = float("inf")
+    for _ in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        torch._int_mm(a, b)
+        e1.record()
+        e1.synchronize()
+        best = min(best, e0.elapsed_time(e1))
+    out["cublaslt_int8"] = round(2.0 * n ** 3 / (best * 1e-3) / 1e12, 1)
+    out["tcgen05_kind_i8"] = "refused by ptxas for sm_103a (tests/test_toolchain_cpu.py)"
+    out["basis"] = "TOPS = 2 ops per int8 multiply-add; probe kernels on every SM, best of 3 timed launches"
+    del a, b
+    torch.cuda.empty_cache()
+    return out
+
+
+def linear_config(bsg, torch, dev, case, steps: int) -> dict:
+    """One linear timed as the default workload times FFN2: rotating input
+    and output sets (> 2 x L2), ACT_READY launches of bsgemm_run_ws, one
+    CUDA graph of `steps` launches replayed REPEATS times, median."""
+    props = torch.cuda.get_device_properties(dev)
+    wt = case.weight
+    lin = bsg.SparseInt8Linear(wt.n_out, wt.k_in, wt.indptr, wt.colidx, wt.values, wt.scales, wt.bias)
+    out_dtype = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+                 synth.I8: torch.int8, synth.I8_GELU: torch.int8}[case.kind]
+    set_bytes = case.m * wt.k_in + case.m * wt.n_out * torch.empty((), dtype=out_dtype).element_size()
+    nsets = max(2, math.ceil(2 * int(getattr(props, "L2_cache_size", 128 << 20)) / set_bytes) + 1)
+    xs = [torch.from_numpy(case.x).to(dev) for _ in range(nsets)]
+    outs = [torch.empty((case.m, wt.n_out), dtype=out_dtype, device=dev) for _ in range(nsets)]
+    ws_bytes = lin.workspace_bytes(case.m)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i, s):
+        bsg.bsgemm_run_ws(lin._h, xs[i % nsets].data_ptr(), case.m, outs[i % nsets].data_ptr(), case.kind,
+                          case.out_scale, ws.data_ptr(), ws_bytes, s.cuda_stream, bsg.ACT_READY)
+
+    for i in range(nsets):
+        step(i, stream)
+    torch.cuda.synchronize(dev)
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(stream)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        for i in range(steps):
+            step(i, side)
+    torch.cuda.synchronize(dev)
+    for _ in range(3):
+        g.replay()
+    ts = []
+    for _ in range(REPEATS):
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        e1.synchronize()
+        ts.append(e0.elapsed_time(e1) / steps)
+    del g
+    lin.close()
+    ms = statistics.median(ts)
+    tops = effective_ops(case) / (ms * 1e-3) / 1e12
+    peak = _peak_tops(props, 2070.0)
+    return {"workload": case.name, "ms_per_step": round(ms, 6), "min_ms_per_step": round(min(ts), 6),
+            "max_ms_per_step": round(max(ts), 6), "value": round(tops, 3), "unit": UNIT,
+            "roofline_frac": round(tops / peak, 4), "hbm_gbs": round(algorithmic_bytes(case) / (ms * 1e-3) / 1e9, 1),
+            "basis": f"graph of {steps} bsgemm_run_ws launches (ACT_READY, {nsets} rotating sets), median of "
+                     f"{REPEATS} replays; frac of the nominal dp4a peak"}
+
+
+def run_configs(args) -> dict:
+    """The metric's other configurations, measured in the same run as the
+    headline: FFN1 (768 -> 3072 + GELU, M = 4096), the encoder layer's four
+    linears chained (8 x 384, 80%), and one point of the six-layer stack
+    (batch 32 x seq 128, 80%: tokens/s and per-linear roofline fractions)."""
+    import torch
+    import paper_2211_07715_gb300 as bsg
+
+    dev = torch.device("cuda", 0)
+    steps = max(5, min(args.steps, 50))
+    out = {"ffn1": linear_config(bsg, torch, dev, synth.ffn1(), steps)}
+    sub = argparse.Namespace(**vars(args))
+    sub.steps = steps
+    lay = run_layer(sub)
+    out["layer_chain_8x384_s80"] = {
+        "ms_per_step": lay["ms_per_step"], "value": lay["value"], "unit": UNIT, "tokens_per_s": lay["tokens_per_s"],
+        "roofline_frac": lay["roofline"]["frac"],
+        "per_linear_frac": {n: v["frac"] for n, v in lay["per_linear"].items()},
+        "basis": f"graph of {steps} passes of the four linears (one kernel each), one timed replay; per-linear "
+                 "fractions from graphs of one linear's launches"}
+    st = run_stack(sub, only=[(32, 128, 0.8)])
+    pt = st["points"][0]
+    out["stack_32x128_s80"] = {
+        "tokens_per_s": pt["tokens_per_s"], "tokens_per_s_graph": pt["tokens_per_s_graph"],
+        "ms_per_pass": pt["ms"], "ms_per_pass_graph": pt["ms_graph"], "value": pt["tops"], "unit": UNIT,
+        "roofline_frac_per_linear": pt["roofline_frac_per_linear"],
+        "basis": "six layers x 4 linears = 24 launches per pass on one stream (and as one CUDA graph), "
+                 f"{st['steps']} passes"}
+    return out
 
 
 def cpu_baseline(case, rows: int | None, threads: int | None = None, reps: int = 1) -> dict:
@@ -711,7 +840,7 @@ def run_layer(args) -> dict:
                                "timed path by a seeded int8 context buffer",
                    "tokens": m, "batch": 8, "seq": 384, "sparsity": 0.8,
                    "l2": f"rotating {nsets} input/output sets ({nsets * set_bytes / 2**20:.0f} MiB > 2 x L2)",
-                   "launch": "the timed passes are one CUDA graph of --steps passes (the chain's 8 kernels each)"},
+                   "launch": "the timed passes are one CUDA graph of --steps passes (the chain's 4 kernels each)"},
         "tokens_per_s": round(m / (ms * 1e-3), 1),
         "stream_ms_per_step": round(stream_ms, 6),
         "roofline": {"bound": "alu", "achieved": round(kernel_tops, 3), "peak": round(peak, 2), "unit": "TOPS",
@@ -904,7 +1033,7 @@ def run_encoder(args) -> dict:
     }
 
 
-def run_stack(args) -> dict:
+def run_stack(args, only=None) -> dict:
     """cfg 5: the six-layer stack of 24 sparse linears swept over batch
     {1, 8, 32, 128} x seq {128, 384} x sparsity {70, 80, 90}%.  One pass =
     24 linears (24 launches) back to back on one stream, the attention step
@@ -925,6 +1054,8 @@ def run_stack(args) -> dict:
     time.sleep(0.3)
     mark0 = sampler.mark()
     for pi, (batch, seq, sp) in enumerate(synth.STACK_POINTS):
+        if only is not None and (batch, seq, sp) not in only:
+            continue
         layers, x0, ctx0 = synth.stack_point(batch, seq, sp, pi)
         m = batch * seq
         chains = [_Chain(bsg, torch, dev, w, m, scales) for w in layers]
@@ -990,7 +1121,7 @@ def run_stack(args) -> dict:
     time.sleep(0.2)
     sampler.stop()
     clocks = sampler.summary(mark0, max(mark1, mark0 + 1))
-    ref = next(pt for pt in points if (pt["batch"], pt["seq"], pt["sparsity"]) == (8, 384, 0.8))
+    ref = next((pt for pt in points if (pt["batch"], pt["seq"], pt["sparsity"]) == (8, 384, 0.8)), points[0])
     return {
         "metric": METRIC, "value": ref["tokens_per_s"], "unit": "tokens/s", "n_gpus": 1, "steps": reps,
         "warmup": 3, "ms_per_step": ref["ms"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -1248,6 +1379,7 @@ def main():
                         "production: maximum samples/s under 10 ms per batch")
     p.add_argument("--ref-rows", type=int, default=512, help="tokens per reference step")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-configs", action="store_true", help="skip the other configurations' sub-objects")
     p.add_argument("--soak-seconds", type=float, default=1.0, help="untimed load before the timed region")
     p.add_argument("--e2e-steps", type=int, default=200, help="steps of the end-to-end (host buffers) timing")
     args = p.parse_args()

@@ -353,6 +353,21 @@ uint32_t bsgemm_set_test_hooks(uint32_t bits);
  */
 void bsgemm_destroy(bsgemm_t h);
 
+/*
+ * bsgemm_int8_peak -- measure the peak rate of one int8 dot-product unit of
+ * the current device, the denominator of the layer's roofline (the layer is
+ * Algorithm 1's int8 dot-4 contraction; the paper has no counterpart of
+ * this measurement).  unit 0: dp4a (4 int8 multiply-adds into int32 per lane,
+ * the unit the layer kernel runs on); unit 1: mma.sync m16n8k32 s8 x s8 ->
+ * s32 (the warp-level tensor-core instruction).  A probe kernel runs `iters`
+ * loop iterations on every SM, four times; *tops receives the best of the
+ * last three as 10^12 ops/s (2 ops per multiply-add).  Allocates a few bytes
+ * of device memory and synchronises the device: a measurement helper, not
+ * for use while other work runs.  Returns BSGEMM_OK, BSGEMM_ERR_INVALID
+ * (unit not 0 or 1, iters < 1, tops NULL) or BSGEMM_ERR_CUDA.
+ */
+int bsgemm_int8_peak(int unit, int iters, double* tops);
+
 /* Message for the last failure on the calling thread ("" if none).  The
  * string stays valid until the next bsgemm_* call on this thread. */
 const char* bsgemm_last_error(void);

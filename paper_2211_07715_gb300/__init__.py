@@ -90,6 +90,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_device_status.restype = ctypes.c_int
     lib.bsgemm_set_test_hooks.argtypes = [ctypes.c_uint32]
     lib.bsgemm_set_test_hooks.restype = ctypes.c_uint32
+    lib.bsgemm_int8_peak.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
+    lib.bsgemm_int8_peak.restype = ctypes.c_int
     return lib
 
 
@@ -100,7 +102,7 @@ EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static",
             "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_layernorm",
             "bsgemm_attention", "bsgemm_destroy",
             "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info",
-            "bsgemm_set_test_hooks")
+            "bsgemm_set_test_hooks", "bsgemm_int8_peak")
 
 
 def _epi(kind: int, out_scale: float, flags: int = 0, residual: int = 0, residual_scale: float = 1.0) -> Epilogue:
@@ -312,6 +314,16 @@ def bsgemm_set_test_hooks(bits: int) -> int:
     """Make the kernels' bounded waits give up on purpose (tests of the
     failure path only); returns the previous bits."""
     return int(_lib.bsgemm_set_test_hooks(int(bits)))
+
+
+def bsgemm_int8_peak(unit: int, iters: int = 4000) -> float:
+    """Measured peak of an int8 dot-product unit in TOPS: unit 0 = dp4a,
+    1 = mma.sync m16n8k32 s8 (synchronises the device)."""
+    v = ctypes.c_double(0.0)
+    rc = _lib.bsgemm_int8_peak(int(unit), int(iters), ctypes.byref(v))
+    if rc != 0:
+        raise BsgemmError(rc, "int8 peak probe failed")
+    return float(v.value)
 
 
 def bsgemm_destroy(h: int) -> None:
