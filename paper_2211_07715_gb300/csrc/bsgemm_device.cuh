@@ -305,6 +305,15 @@ __device__ __forceinline__ void tensor_g2s_hint(uint32_t dst, const CUtensorMap*
                  ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(pol) : "memory");
 }
 
+// One 3-D box (x innermost, then y, then z) with an L2 eviction policy.
+__device__ __forceinline__ void tensor_g2s_3d_hint(uint32_t dst, const CUtensorMap* map, int x, int y, int z,
+                                                   uint32_t bar, uint64_t pol) {
+    asm volatile("cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+                 " [%0], [%1, {%2, %3, %4}], [%5], %6;\n"
+                 ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(bar), "l"(pol)
+                 : "memory");
+}
+
 // Order this thread's earlier generic-proxy shared-memory accesses before
 // later asynchronous-proxy (bulk copy) writes.
 __device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory"); }

@@ -72,6 +72,12 @@ constexpr int kGroupEndCost = BSG_GROUP_END_COST;
 #define BSG_TMA_PIECE 65536
 #endif
 constexpr unsigned kTmaPiece = BSG_TMA_PIECE;
+// Fewest tensor copies of a token tile when x is copied as a 3-D view
+// (each copy then brings box_d of its 64-column boxes).
+#ifndef BSG_MIN_COPIES
+#define BSG_MIN_COPIES 8
+#endif
+constexpr int kMinCopies = BSG_MIN_COPIES;
 
 // 4x4 byte transpose.  In: a/b/c/d = bytes (x0..x3) of rows 0..3.  Out:
 // t_i = (a_i, b_i, c_i, d_i).
@@ -321,9 +327,13 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
     if (TENSOR && tid == 0) asm volatile("prefetch.tensormap [%0];\n" ::"l"(reinterpret_cast<uint64_t>(&xmap)) : "memory");
     griddep_launch_dependents();
     const uint32_t bar = smem_addr(&s_bar[0]);  // box b's barrier at bar + 8 b (TMA: box 0 only)
-    if ((TMA || TENSOR) && tid == 0) mbar_init_n(bar, TENSOR ? nbox : 1);
-    // this warp's boxes: [bx0, bx1)
-    const int bx0 = warp * nbox / kWarps, bx1 = (warp + 1) * nbox / kWarps;
+    // A tensor copy brings box_d consecutive 64-column boxes (one barrier
+    // each copy); this warp issues copies [op0, op1) and turns their boxes
+    // around.
+    const int box_d = TENSOR ? a.box_d : 1;  // > 1 exactly when xmap is the 3-D view of x
+    const int nops = nbox / box_d;
+    if ((TMA || TENSOR) && tid == 0) mbar_init_n(bar, TENSOR ? nops : 1);
+    const int op0 = warp * nops / kWarps, op1 = (warp + 1) * nops / kWarps;
     __syncthreads();
     unsigned phase = 0;
     long long u = sched.u[blockIdx.x];
@@ -346,28 +356,22 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         const long long m0 = t * kTile;
         auto gp = [&](int gi) { return s_gp[gi - g_lo]; };
 
-        // The window's step offsets and block-rows load before the tile's
-        // copies go out, so that they do not queue behind the tile's bytes
-        // (every CTA of a launch stages at once).
-        int gp_v = 0;
-        unsigned long long gr_v = ~0ull;
-        if (tid <= g_hi - g_lo) {
-            gp_v = ldg_hint(w.gptr + g_lo + tid, pol_w);
-            if (tid < g_hi - g_lo) gr_v = pack_rows16(ldg_hint(w.grow + g_lo + tid, pol_w));
-        }
         const bool stage = (t != staged);
         // the token tile (already swizzled in a.xb) in kTmaPiece-byte bulk
         // copies, issued by the lanes of warp 0 (one completion barrier)
         auto copy_tile = [&]() {
             if (a.skip_copy) return;  // test hook: the waits below give up
-            if (TENSOR && stage && lane < bx1 - bx0) {  // lane i of each warp: the warp's box bx0 + i
-                const int b = bx0 + lane;
+            if (TENSOR && stage && lane < op1 - op0) {  // lane i of each warp: the warp's copy op0 + i
+                const int o = op0 + lane;
                 if (staged >= 0) fence_proxy_async();  // the previous tile's reads come first
-                mbar_arrive_expect_tx(bar + 8u * b, 64u * kTile);
-                if (KMAJOR)  // rows 64b..64b+63 of x^T at tokens t*64.., landing as the tile's rows
-                    tensor_g2s_hint(tb + 4096u * b, &xmap, static_cast<int>(t * kTile), 64 * b, bar + 8u * b, pol_x);
+                mbar_arrive_expect_tx(bar + 8u * o, 64u * kTile * box_d);
+                if (KMAJOR)  // rows 64o..64o+63 of x^T at tokens t*64.., landing as the tile's rows
+                    tensor_g2s_hint(tb + 4096u * o, &xmap, static_cast<int>(t * kTile), 64 * o, bar + 8u * o, pol_x);
+                else if (box_d > 1)  // x viewed as [K/64][M][64]: boxes o*box_d.. of tokens t*64..
+                    tensor_g2s_3d_hint(tb + 4096u * box_d * o, &xmap, 0, static_cast<int>(t * kTile), o * box_d,
+                                       bar + 8u * o, pol_x);
                 else
-                    tensor_g2s_hint(tb + 4096u * b, &xmap, 64 * b, static_cast<int>(t * kTile), bar + 8u * b, pol_x);
+                    tensor_g2s_hint(tb + 4096u * o, &xmap, 64 * o, static_cast<int>(t * kTile), bar + 8u * o, pol_x);
             }
             if (TMA && stage && warp == 0) {
                 const unsigned bytes = static_cast<unsigned>(kpad) * kTile;
@@ -379,13 +383,20 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                     bulk_g2s(tb + off, src + off, min(static_cast<unsigned>(kTmaPiece), bytes - off), bar);
             }
         };
-        // After the first window the previous grid is done: the copy starts
-        // at once and overlaps the window's set-up.
-        // With act_ready (x complete before the previous kernel started) the
-        // first window's tensor copies start at once too and overlap that
-        // kernel's end.
+        // The tile's copies go out first: after the first window the previous
+        // grid is done, and with act_ready (x complete before the previous
+        // kernel started) the first window's copies may start at once too;
+        // the window's set-up and the previous kernel's end overlap them.
         const bool issued = waited || (TENSOR && a.act_ready);
         if (issued) copy_tile();
+        // The window's step offsets and block-rows (the weights stay in L2:
+        // these loads hit it even while the tile's bytes stream in).
+        int gp_v = 0;
+        unsigned long long gr_v = ~0ull;
+        if (tid <= g_hi - g_lo) {
+            gp_v = ldg_hint(w.gptr + g_lo + tid, pol_w);
+            if (tid < g_hi - g_lo) gr_v = pack_rows16(ldg_hint(w.grow + g_lo + tid, pol_w));
+        }
         if (staged < 0) {  // the split-group slots start at zero; whoever finishes a slot resets it
             for (int i = tid; i < kSlots * SW / 4; i += kThreads) reinterpret_cast<int4*>(slots)[i] = make_int4(0, 0, 0, 0);
         }
@@ -483,11 +494,11 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             // the warp turns its boxes around as they land
             bool ok = true;
             if (KMAJOR) {  // nothing to turn around: every thread sees every box land
-                for (int b = 0; b < nbox && ok; ++b) ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * b, phase & 1u, wlim));
+                for (int o = 0; o < nops && ok; ++o) ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * o, phase & 1u, wlim));
             } else {
-                for (int b = bx0; b < bx1 && ok; ++b) {
-                    ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * b, phase & 1u, wlim));
-                    if (ok) transpose_box(tb, b, lane);
+                for (int o = op0; o < op1 && ok; ++o) {
+                    ok = __all_sync(0xffffffffu, mbar_wait(bar + 8u * o, phase & 1u, wlim));
+                    for (int j = 0; j < box_d && ok; ++j) transpose_box(tb, o * box_d + j, lane);
                 }
             }
             ++phase;
@@ -495,7 +506,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 if (tid == 0) {
                     wait_prev();
                     atomicOr(w.status, kStatusTimeout);
-                    for (int b = 0; b < nbox; ++b) mbar_wait(bar + 8u * b, (phase - 1) & 1u, wlim);  // one more chance
+                    for (int o = 0; o < nops; ++o) mbar_wait(bar + 8u * o, (phase - 1) & 1u, wlim);  // one more chance
                 }
                 __syncthreads();
                 return;
@@ -755,7 +766,9 @@ cudaError_t prepare_kernels(int K, int* ctas_per_sm) {
     return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_for(0, kStageTensor), kThreads, smem);
 }
 
-cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& sched, int grid, cudaStream_t s) {
+cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a_in, const Schedule& sched, int grid, cudaStream_t s) {
+    LaunchArgs a = a_in;
+    a.box_d = 1;
     const size_t smem = smem_bytes(w.K);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(grid));
@@ -786,15 +799,39 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a, const Schedule& 
             return cudaErrorInvalidValue;
     } else if (a.tensor) {
         PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
-        if (!encode || (w.K + 63) / 64 > kMaxBoxes) return cudaErrorNotSupported;
-        const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(w.K), static_cast<cuuint64_t>(a.M)};
-        const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(w.K)};
-        const cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(kTile)};
-        const cuuint32_t estride[2] = {1u, 1u};
-        if (encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t*>(a.x), gdim, gstride, box, estride,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-            return cudaErrorInvalidValue;
+        const int nbox = (w.K + 63) / 64;
+        if (!encode || nbox > kMaxBoxes) return cudaErrorNotSupported;
+        // box_d: the largest divisor of nbox that leaves at least kMinCopies
+        // copies (1: the 2-D boxes below)
+        int d = 1;
+        for (int c = 2; c <= nbox / kMinCopies; ++c)
+            if (nbox % c == 0) d = c;
+        if (w.K % 64 == 0 && d > 1) {  // box_d > 1 <=> the 3-D map (and copy)
+            // x viewed as [K/64 blocks][M tokens][64 columns] (the block
+            // stride is 64 bytes), boxes of box_d blocks x 64 tokens x 64
+            // columns: the 64-byte rows land as the 2-D boxes below would, box
+            // after box.  The tensor-copy unit takes and completes copies one
+            // by one, so 8 large copies (one a warp) finish a tile sooner
+            // than 48 small ones.
+            a.box_d = d;
+            const cuuint64_t gdim[3] = {64u, static_cast<cuuint64_t>(a.M), static_cast<cuuint64_t>(nbox)};
+            const cuuint64_t gstride[2] = {static_cast<cuuint64_t>(w.K), 64u};
+            const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(kTile), static_cast<cuuint32_t>(a.box_d)};
+            const cuuint32_t estride[3] = {1u, 1u, 1u};
+            if (encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<int8_t*>(a.x), gdim, gstride, box, estride,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+                return cudaErrorInvalidValue;
+        } else {
+            const cuuint64_t gdim[2] = {static_cast<cuuint64_t>(w.K), static_cast<cuuint64_t>(a.M)};
+            const cuuint64_t gstride[1] = {static_cast<cuuint64_t>(w.K)};
+            const cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(kTile)};
+            const cuuint32_t estride[2] = {1u, 1u};
+            if (encode(&xmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t*>(a.x), gdim, gstride, box, estride,
+                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+                return cudaErrorInvalidValue;
+        }
     }
     cudaError_t e = cudaSuccess;
 #define BSG_LAUNCH(KV)                                                                                   \

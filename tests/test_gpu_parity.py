@@ -107,6 +107,22 @@ def test_ragged_k(bsg, k, path):
               kind, f"k={k}")
 
 
+@pytest.mark.parametrize("k", [512, 1024, 2048, 2560, 3072])
+def test_k_multiple_of_64_tile_copies(bsg, k):
+    """K a multiple of 64: the one-kernel path copies the token tile in
+    boxes of 64 columns, one 3-D copy of K / 512 boxes per warp where that
+    is more than one box (K = 1024, 2048, 2560, 3072), 2-D boxes otherwise
+    (K = 512); tokens span three tiles and a ragged tail."""
+    rng = synth.rng_for(3100 + k)
+    wt = synth.draw_weight(rng, 80, k, 0.7)
+    x = synth.draw_x(rng, 150, k, "u127")
+    lin = make_linear(bsg, wt)
+    w = oracle.weight_dense(wt)
+    for kind in (synth.I32, synth.I8):
+        check(gpu_run(lin, x, kind, 0.07, False), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.07),
+              kind, f"k={k}")
+
+
 def test_max_k_and_int32_extremes(bsg):
     """Largest supported K with the largest-magnitude values."""
     k = bsg.bsgemm_max_k()
