@@ -535,6 +535,105 @@ def linear_config(bsg, torch, dev, case, steps: int) -> dict:
                      f"{REPEATS} replays; frac of the nominal dp4a peak"}
 
 
+def time_handle(bsg, torch, dev, lin, x_np, kind: int, out_scale: float, steps: int) -> tuple:
+    """(median, min, max) ms per launch of a handle on rotating input and
+    output sets (> 2 x L2): a CUDA graph of `steps` ACT_READY launches of
+    bsgemm_run_ws, replayed REPEATS times."""
+    props = torch.cuda.get_device_properties(dev)
+    m, k = x_np.shape
+    out_dtype = {synth.I32: torch.int32, synth.F32: torch.float32, synth.F32_GELU: torch.float32,
+                 synth.I8: torch.int8, synth.I8_GELU: torch.int8}[kind]
+    set_bytes = m * k + m * lin.n_out * torch.empty((), dtype=out_dtype).element_size()
+    nsets = max(2, math.ceil(2 * int(getattr(props, "L2_cache_size", 128 << 20)) / set_bytes) + 1)
+    xs = [torch.from_numpy(x_np).to(dev) for _ in range(nsets)]
+    outs = [torch.empty((m, lin.n_out), dtype=out_dtype, device=dev) for _ in range(nsets)]
+    ws_bytes = lin.workspace_bytes(m)
+    ws = torch.empty(max(ws_bytes, 16), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(i, s):
+        bsg.bsgemm_run_ws(lin._h, xs[i % nsets].data_ptr(), m, outs[i % nsets].data_ptr(), kind, out_scale,
+                          ws.data_ptr(), ws_bytes, s.cuda_stream, bsg.ACT_READY)
+
+    for i in range(nsets):
+        step(i, stream)
+    torch.cuda.synchronize(dev)
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(stream)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        for i in range(steps):
+            step(i, side)
+    torch.cuda.synchronize(dev)
+    for _ in range(3):
+        g.replay()
+    ts = []
+    for _ in range(REPEATS):
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        e1.synchronize()
+        ts.append(e0.elapsed_time(e1) / steps)
+    del g
+    return statistics.median(ts), min(ts), max(ts)
+
+
+def run_shapes(args) -> dict:
+    """Other block shapes on the FFN2 shape (768 <- 3072, M = 4096): a
+    weight sparse in 1 x 4 blocks at 90%, run natively by the kernel's 1 x 4
+    form and, for comparison, as the 4 x 1 blocks that hold it; and a 2:4
+    weight (run as its 4 x 1 blocks).  value = effective TOPS of the useful
+    multiply-adds (2 ops each) of the native 1 x 4 path."""
+    import torch
+    import paper_2211_07715_gb300 as bsg
+
+    dev = torch.device("cuda", 0)
+    props = torch.cuda.get_device_properties(dev)
+    steps = max(5, min(args.steps, 50))
+    n_out, k_in, m = 768, 3072, 4096
+    rng = synth.rng_for(synth.SEED_BASE + 40)
+    w14 = synth.draw_weight_1x4(rng, n_out, k_in, 0.9)
+    x = synth.draw_x(rng, m, k_in, "u0_127")
+    useful14 = 2.0 * m * w14.indptr[-1] * 4
+    peak = _peak_tops(props, 2070.0)
+    res = {}
+    lin = bsg.SparseInt8Linear.from_blocks_1x4(n_out, k_in, w14.indptr, w14.colgrp, w14.values, w14.scales, w14.bias)
+    ms, lo, hi = time_handle(bsg, torch, dev, lin, x, synth.I8, 0.05, steps)
+    res["blocks_1x4_native"] = {"ms_per_step": round(ms, 6), "min_ms": round(lo, 6), "max_ms": round(hi, 6),
+                                "value": round(useful14 / (ms * 1e-3) / 1e12, 3), "unit": UNIT,
+                                "stored_macs_per_useful": round(lin.info["quads"] * 4 * 1.0 / w14.indptr[-1] / 4, 3),
+                                "roofline_frac": round(useful14 / (ms * 1e-3) / 1e12 / peak, 4)}
+    lin.close()
+    dense = bsg.dense_from_blocks_1x4(n_out, k_in, w14.indptr, w14.colgrp, w14.values)
+    lin = bsg.SparseInt8Linear.from_dense(dense, w14.scales, w14.bias)
+    ms, lo, hi = time_handle(bsg, torch, dev, lin, x, synth.I8, 0.05, steps)
+    res["blocks_1x4_as_4x1"] = {"ms_per_step": round(ms, 6), "min_ms": round(lo, 6), "max_ms": round(hi, 6),
+                                "value": round(useful14 / (ms * 1e-3) / 1e12, 3), "unit": UNIT,
+                                "stored_macs_per_useful": round(lin.info["nnzb"] * 4 / (w14.indptr[-1] * 4), 3),
+                                "roofline_frac": round(useful14 / (ms * 1e-3) / 1e12 / peak, 4)}
+    lin.close()
+    w24 = synth.draw_weight_2to4(rng, n_out, k_in)
+    useful24 = 2.0 * m * n_out * k_in / 2
+    lin = bsg.SparseInt8Linear.from_2to4(w24.values, w24.idx, w24.scales, w24.bias)
+    ms, lo, hi = time_handle(bsg, torch, dev, lin, x, synth.I8, 0.05, steps)
+    res["sparse_2to4_as_4x1"] = {"ms_per_step": round(ms, 6), "min_ms": round(lo, 6), "max_ms": round(hi, 6),
+                                 "value": round(useful24 / (ms * 1e-3) / 1e12, 3), "unit": UNIT,
+                                 "stored_macs_per_useful": round(lin.info["nnzb"] * 4 / (n_out * k_in / 2), 3),
+                                 "roofline_frac": round(useful24 / (ms * 1e-3) / 1e12 / peak, 4)}
+    lin.close()
+    nat = res["blocks_1x4_native"]
+    return {"metric": METRIC, "value": nat["value"], "unit": UNIT, "n_gpus": 1, "steps": steps, "warmup": 3,
+            "ms_per_step": nat["ms_per_step"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "s8", "data": "synthetic",
+            "config": {"workload": "other block shapes on 768 <- 3072, M = 4096, int8 out: 1 x 4 blocks at 90% "
+                                   "(native / regrouped into 4 x 1), 2:4 (regrouped into 4 x 1)",
+                       "basis": f"graph of {steps} bsgemm_run_ws launches (ACT_READY, rotating sets), median of "
+                                f"{REPEATS} replays; value = useful multiply-adds x 2 / time"},
+            "shapes": res, "gpu_launches": 3 * steps * REPEATS, "kernel_source_sha256": kernel_sha()}
+
+
 def run_configs(args) -> dict:
     """The metric's other configurations, measured in the same run as the
     headline: FFN1 (768 -> 3072 + GELU, M = 4096), the encoder layer's four
@@ -1370,13 +1469,15 @@ def main():
     p.add_argument("--steps", type=int, default=2000)
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "encoder", "stack", "prune", "production"],
+    p.add_argument("--workload", choices=sorted(WORKLOADS) + ["layer", "encoder", "stack", "prune", "production",
+                                                              "shapes"],
                    default="ffn2",
                    help="ffn2/ffn1/single: one linear; layer: the encoder layer's four linears; stack: the "
                         "six-layer stack sweep; encoder: the whole layer on the device (attention, residual adds, "
                         "LayerNorms); "
                         "prune: create-side block pruning of an FFN2-shaped weight; "
-                        "production: maximum samples/s under 10 ms per batch")
+                        "production: maximum samples/s under 10 ms per batch; shapes: 1 x 4 blocks (native and "
+                        "regrouped) and 2:4 on the FFN2 shape")
     p.add_argument("--ref-rows", type=int, default=512, help="tokens per reference step")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-configs", action="store_true", help="skip the other configurations' sub-objects")
@@ -1390,7 +1491,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
-        if args.workload in ("layer", "encoder", "stack", "production"):
+        if args.workload in ("layer", "encoder", "stack", "production", "shapes"):
             p.error("--impl reference times the single-linear workloads and prune")
         res = run_reference(args, rank)
     else:
@@ -1409,6 +1510,8 @@ def main():
             res = run_prune(args) if rank == 0 else None
         elif args.workload == "production":
             res = run_production(args) if rank == 0 else None
+        elif args.workload == "shapes":
+            res = run_shapes(args) if rank == 0 else None
         else:
             res = run_ours(args, rank, world, local_rank)
         if world > 1:

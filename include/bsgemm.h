@@ -109,16 +109,48 @@ typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
  * The call allocates device memory on the CURRENT CUDA device, copies the
  * repacked weights there and synchronises.  Returns NULL on failure.
  *
- * Other block shapes enter as the 4 x 1 blocks that hold them: a weight
- * sparse in 1 x 4 blocks (one row x 4 input columns) or with 2:4 sparsity
- * along K is passed as every 4 x 1 block with a nonzero value (the union of
- * the four rows' columns of each block-row).  Results are exact; the
- * stored work grows by that union (the Python binding's from_blocks_1x4 /
- * from_2to4 build these arrays).
+ * Other block shapes: bsgemm_create_1x4 and bsgemm_create_2to4 below.
  */
 #define BSGEMM_MAX_N (4 * 65535) /* block-row indices are 16-bit inside the kernel */
 bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const int8_t* values,
                        const float* scales, const float* bias);
+
+/*
+ * bsgemm_create_1x4 -- a weight sparse in 1 x 4 blocks: one output row x 4
+ * consecutive input columns (the paper's 4 x 1 blocks turned along K; its
+ * App. A.3.4 leaves other block shapes to padding and regrouping).  The
+ * layer kernel runs them natively: each block is one dot-4 of a token's 4
+ * consecutive activations with the block's 4 weights, with no zero padding
+ * of the block's work.  HOST arrays, read during the call only:
+ *   N        output features, 1 <= N <= 65535 (any N; rows are independent).
+ *   K        input features, a multiple of 4, 4 <= K <= bsgemm_max_k().
+ *   indices  int32: indptr[N + 1] followed by colgrp[nnz], nnz = indptr[N]:
+ *            block e of row n (indptr[n] <= e < indptr[n + 1]) covers
+ *            columns 4 colgrp[e] .. 4 colgrp[e] + 3; colgrp strictly
+ *            increases within a row and lies in [0, K/4).
+ *   values   int8 [nnz][4]: values[e][i] = W[n][4 colgrp[e] + i].
+ *   scales, bias  as for bsgemm_create.
+ * Runs take every bsgemm_run* call and epilogue kind except
+ * BSGEMM_OUT_F32_RESID (BSGEMM_ERR_UNSUPPORTED).  bsgemm_info()[2] is nnz.
+ * Returns NULL on failure (bsgemm_last_error / bsgemm_last_status).
+ */
+bsgemm_t bsgemm_create_1x4(int N, int K, const int32_t* indices, const int8_t* values, const float* scales,
+                           const float* bias);
+
+/*
+ * bsgemm_create_2to4 -- a weight with 2:4 structured sparsity along K (two
+ * values in every group of 4 consecutive input columns of every row, the
+ * pattern of sparse tensor cores that Sec. 1 cites as related work).  HOST
+ * arrays [N][K/2], read during the call only: values int8 and idx uint8,
+ * where values[n][2j + t] is W[n][4j + idx[n][2j + t]]; idx[n][2j] <
+ * idx[n][2j + 1] <= 3 (a value may be 0).  K a multiple of 4.  The weight
+ * is run as the 4 x 1 blocks that hold its values (block (r, k) stored when
+ * one of rows 4r..4r+3 is nonzero in column k; about 1.9x the multiply-adds
+ * of the 2:4 values for random patterns).  scales, bias and the result as
+ * for bsgemm_create.
+ */
+bsgemm_t bsgemm_create_2to4(int N, int K, const int8_t* values, const uint8_t* idx, const float* scales,
+                            const float* bias);
 
 /*
  * bsgemm_run -- out = epilogue(X * W^T) on `stream`.

@@ -51,6 +51,10 @@ def _load() -> ctypes.CDLL:
     vp = ctypes.c_void_p
     lib.bsgemm_create.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]
     lib.bsgemm_create.restype = vp
+    lib.bsgemm_create_1x4.argtypes = [ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]
+    lib.bsgemm_create_1x4.restype = vp
+    lib.bsgemm_create_2to4.argtypes = [ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]
+    lib.bsgemm_create_2to4.restype = vp
     lib.bsgemm_run.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp]
     lib.bsgemm_run.restype = ctypes.c_int
     lib.bsgemm_destroy.argtypes = [vp]
@@ -97,7 +101,7 @@ def _load() -> ctypes.CDLL:
 
 _lib = _load()
 
-EXPORTED = ("bsgemm_create", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
+EXPORTED = ("bsgemm_create", "bsgemm_create_1x4", "bsgemm_create_2to4", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
             "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_run_kmajor",
             "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_layernorm",
             "bsgemm_attention", "bsgemm_destroy",
@@ -135,6 +139,33 @@ def bsgemm_create(n_out: int, k_in: int, block: int, indices, values, scales, bi
     bias = None if bias is None else _host_array(bias, np.float32)
     h = _lib.bsgemm_create(int(n_out), int(k_in), int(block), indices.ctypes.data, values.ctypes.data,
                            scales.ctypes.data, None if bias is None else bias.ctypes.data)
+    if not h:
+        raise BsgemmError(bsgemm_last_status(), bsgemm_last_error())
+    return h
+
+
+def bsgemm_create_1x4(n_out: int, k_in: int, indices, values, scales, bias=None) -> int:
+    """Handle of a weight sparse in 1 x 4 blocks: indices = indptr [N + 1]
+    then colgrp [nnz]; values int8 [nnz][4] (see include/bsgemm.h)."""
+    indices = _host_array(indices, np.int32)
+    values = _host_array(values, np.int8)
+    scales = _host_array(scales, np.float32)
+    bias = None if bias is None else _host_array(bias, np.float32)
+    h = _lib.bsgemm_create_1x4(int(n_out), int(k_in), indices.ctypes.data, values.ctypes.data, scales.ctypes.data,
+                               None if bias is None else bias.ctypes.data)
+    if not h:
+        raise BsgemmError(bsgemm_last_status(), bsgemm_last_error())
+    return h
+
+
+def bsgemm_create_2to4(n_out: int, k_in: int, values, idx, scales, bias=None) -> int:
+    """Handle of a 2:4-sparse weight: values int8 and idx uint8 [N][K/2]."""
+    values = _host_array(values, np.int8)
+    idx = _host_array(idx, np.uint8)
+    scales = _host_array(scales, np.float32)
+    bias = None if bias is None else _host_array(bias, np.float32)
+    h = _lib.bsgemm_create_2to4(int(n_out), int(k_in), values.ctypes.data, idx.ctypes.data, scales.ctypes.data,
+                                None if bias is None else bias.ctypes.data)
     if not h:
         raise BsgemmError(bsgemm_last_status(), bsgemm_last_error())
     return h
@@ -434,22 +465,30 @@ class SparseInt8Linear:
         return cls(w.shape[0], w.shape[1], indptr, colidx, values, scales, bias)
 
     @classmethod
+    def _of_handle(cls, h: int, n_out: int, k_in: int) -> "SparseInt8Linear":
+        self = cls.__new__(cls)
+        self.n_out, self.k_in = int(n_out), int(k_in)
+        self._h = h
+        self.info = bsgemm_info(h)
+        return self
+
+    @classmethod
     def from_blocks_1x4(cls, n_out: int, k_in: int, indptr, colgrp, values, scales, bias=None) -> "SparseInt8Linear":
-        """A weight sparse in 1 x 4 blocks (one output row x 4 input
-        columns), run by the 4 x 1-block kernel: at create time its blocks
-        are regrouped into the 4 x 1 blocks that hold them (every column of
-        a block-row that one of its four rows uses), so results are exact
-        and the kernel does the union's work (at 90% sparsity ~3.4 stored
-        blocks per useful one)."""
-        return cls.from_dense(dense_from_blocks_1x4(n_out, k_in, indptr, colgrp, values), scales, bias)
+        """A weight sparse in 1 x 4 blocks (one output row x 4 consecutive
+        input columns; block e of row n covers columns 4 colgrp[e] ..
+        4 colgrp[e] + 3), run natively by the layer kernel's 1 x 4 form
+        (bsgemm_create_1x4): one dot-4 per block and token."""
+        indices = np.concatenate([_host_array(indptr, np.int32), _host_array(colgrp, np.int32)])
+        return cls._of_handle(bsgemm_create_1x4(n_out, k_in, indices, values, scales, bias), n_out, k_in)
 
     @classmethod
     def from_2to4(cls, values, idx, scales, bias=None) -> "SparseInt8Linear":
-        """A 2:4-sparse weight (values, idx [N][K/2]), run by the 4 x 1-block
-        kernel after the same regrouping as from_blocks_1x4: exact, with
-        the union of four rows' columns stored (~94% of all blocks for
-        random 2:4 patterns)."""
-        return cls.from_dense(dense_from_2to4(values, idx), scales, bias)
+        """A 2:4-sparse weight (values, idx [N][K/2]) through
+        bsgemm_create_2to4: run as the 4 x 1 blocks that hold its values
+        (~94% of all blocks for random 2:4 patterns)."""
+        values = np.asarray(values)
+        n_out, k_in = values.shape[0], 2 * values.shape[1]
+        return cls._of_handle(bsgemm_create_2to4(n_out, k_in, values, idx, scales, bias), n_out, k_in)
 
     def workspace_bytes(self, m: int) -> int:
         return bsgemm_workspace_bytes(self._h, m)

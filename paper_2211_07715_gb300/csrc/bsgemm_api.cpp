@@ -15,8 +15,12 @@
 
 #include "bsgemm_internal.h"
 
+constexpr int kShape4x1 = 0;  // 4 consecutive output rows x 1 input column
+constexpr int kShape1x4 = 1;  // 1 output row x 4 consecutive input columns
+
 struct bsgemm_ctx {
     int device = -1;
+    int shape = kShape4x1;      // block shape of the stored weight
     int num_sms = 0;
     int ctas_per_sm = 0;
     int64_t nnzb = 0;
@@ -239,6 +243,101 @@ void step_entries(const int32_t* es, const int32_t* colidx, const int8_t* values
     }
 }
 
+// A weight repacked into row groups and step records (either block shape).
+struct Repacked {
+    int shape = kShape4x1;
+    int N = 0, K = 0;
+    int64_t nnzb = 0;
+    int ngroups = 0, S = 0;
+    std::vector<int32_t> grow, gptr, cost, recs;
+};
+
+// Device upload of a repacked weight into one arena; the kernels are set up
+// for K on the current device.  Returns NULL (with the error recorded) on
+// failure.
+bsgemm_t upload(const Repacked& rp, const float* scales, const float* bias) {
+    const int N = rp.N, K = rp.K, ngroups = rp.ngroups;
+    // scales and biases padded with zeros to a multiple of 4 channels (the
+    // 4 x 1 kernel reads 4 channels at a time and stores only channels < N)
+    const int npad = (N + 3) / 4 * 4;
+    std::vector<float> scale_v(npad, 0.0f), bias_v(npad, 0.0f);
+    std::memcpy(scale_v.data(), scales, sizeof(float) * N);
+    if (bias) std::memcpy(bias_v.data(), bias, sizeof(float) * N);
+
+    auto* h = new bsgemm_ctx();
+    cudaError_t e = cudaGetDevice(&h->device);
+    if (e != cudaSuccess) {
+        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
+        delete h;
+        return nullptr;
+    }
+    int optin = 0;
+    e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
+    if (e != cudaSuccess) {
+        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaDeviceGetAttribute", e));
+        delete h;
+        return nullptr;
+    }
+    if (bsg::smem_bytes(K) + bsg::kStaticSmem > static_cast<size_t>(optin)) {
+        fail(BSGEMM_ERR_UNSUPPORTED, "this device has too little shared memory per block for K = " + std::to_string(K));
+        delete h;
+        return nullptr;
+    }
+    e = bsg::prepare_kernels(K, &h->ctas_per_sm);
+    if (e != cudaSuccess || h->ctas_per_sm < 1) {
+        fail(BSGEMM_ERR_CUDA, e != cudaSuccess ? cuda_msg("kernel setup", e) : "kernel cannot be resident on an SM");
+        delete h;
+        return nullptr;
+    }
+
+    const size_t off_gptr = 0;
+    const size_t off_grow = align_up(off_gptr + sizeof(int32_t) * (ngroups + 1), 256);
+    const size_t off_recs = align_up(off_grow + sizeof(int32_t) * rp.grow.size(), 256);
+    const size_t off_scale = align_up(off_recs + sizeof(int32_t) * rp.recs.size(), 256);
+    const size_t off_bias = align_up(off_scale + sizeof(float) * npad, 256);
+    const size_t off_status = align_up(off_bias + sizeof(float) * npad, 256);
+    h->arena_bytes = align_up(off_status + sizeof(int), 256);
+    e = cudaMalloc(&h->arena, h->arena_bytes);
+    if (e != cudaSuccess) {
+        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaMalloc", e));
+        delete h;
+        return nullptr;
+    }
+    char* base = static_cast<char*>(h->arena);
+    struct Piece { size_t off; const void* src; size_t bytes; } pieces[] = {
+        {off_gptr, rp.gptr.data(), sizeof(int32_t) * rp.gptr.size()},
+        {off_grow, rp.grow.data(), sizeof(int32_t) * rp.grow.size()},
+        {off_recs, rp.recs.data(), sizeof(int32_t) * rp.recs.size()},
+        {off_scale, scale_v.data(), sizeof(float) * npad},
+        {off_bias, bias_v.data(), sizeof(float) * npad},
+        {off_status, &kZeroStatus, sizeof(int)},
+    };
+    for (const Piece& p : pieces) {
+        e = cudaMemcpy(base + p.off, p.src, p.bytes, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) {
+            fail(BSGEMM_ERR_CUDA, cuda_msg("cudaMemcpy", e));
+            cudaFree(h->arena);
+            delete h;
+            return nullptr;
+        }
+    }
+    h->nnzb = rp.nnzb;
+    h->cost = rp.cost;
+    h->shape = rp.shape;
+    h->w.gptr = reinterpret_cast<const int32_t*>(base + off_gptr);
+    h->w.grow = reinterpret_cast<const int4*>(base + off_grow);
+    h->w.recs = reinterpret_cast<const int4*>(base + off_recs);
+    h->w.scale = reinterpret_cast<const float*>(base + off_scale);
+    h->w.bias = reinterpret_cast<const float*>(base + off_bias);
+    h->w.status = reinterpret_cast<int*>(base + off_status);
+    h->w.N = N;
+    h->w.K = K;
+    h->w.ngroups = ngroups;
+    h->w.S = rp.S;
+    return h;
+}
+
 }  // namespace
 
 unsigned bsg::test_hooks() { return g_test_hooks.load(); }
@@ -340,83 +439,199 @@ bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const in
                 for (int c = 0; c < 4; ++c) rec[16 + 4 * q + c] = static_cast<int32_t>(wwords[q][c]);
         }
     }
-    // scales and biases padded with zeros to whole block-rows (the kernel
-    // reads 4 channels at a time and stores only channels < N)
-    std::vector<float> scale_v(npad, 0.0f), bias_v(npad, 0.0f);
-    std::memcpy(scale_v.data(), scales, sizeof(float) * N);
-    if (bias) std::memcpy(bias_v.data(), bias, sizeof(float) * N);
+    Repacked rp;
+    rp.shape = kShape4x1;
+    rp.N = N;
+    rp.K = K;
+    rp.nnzb = nnzb;
+    rp.ngroups = ngroups;
+    rp.S = S;
+    rp.grow = std::move(grow);
+    rp.gptr = std::move(gptr);
+    rp.cost = std::move(cost);
+    rp.recs = std::move(recs);
+    return upload(rp, scales, bias);
+}
 
-    auto* h = new bsgemm_ctx();
-    cudaError_t e = cudaGetDevice(&h->device);
-    if (e != cudaSuccess) {
-        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaGetDevice", e));
-        delete h;
+// Weights sparse in 1 x 4 blocks (one output row x 4 consecutive input
+// columns), repacked for the layer kernel's 1 x 4 form: rows sorted by block
+// count (longest first, ties by index) are taken 4 at a time into a group;
+// a step holds one block of each of the group's 4 rows (a "quad" = the
+// block's 4 columns, its one weight word), and a group has as many steps as
+// its longest row has blocks, rounded up to a multiple of kBlock.  In each
+// half of a step (the blocks of rows 2h and 2h + 1: one pass of the
+// shared-memory gather) one block has an even and one an odd column group
+// where the rows allow it: the 4 columns of an even group sit on bank keys
+// {0, 1, 4, 5} of the swizzled tile, of an odd group on {2, 3, 6, 7}.
+bsgemm_t bsgemm_create_1x4(int N, int K, const int32_t* indices, const int8_t* values, const float* scales,
+                           const float* bias) {
+    clear_error();
+    if (N < 1 || N > 65535 || K < 4 || K % 4 != 0) {
+        fail(BSGEMM_ERR_INVALID, "need 1 <= N <= 65535 and K >= 4 a multiple of 4");
         return nullptr;
     }
-    int optin = 0;
-    e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device);
-    if (e != cudaSuccess) {
-        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaDeviceGetAttribute", e));
-        delete h;
+    if (K > bsg::max_k()) {
+        fail(BSGEMM_ERR_UNSUPPORTED, "K = " + std::to_string(K) + " exceeds bsgemm_max_k() = " +
+                                         std::to_string(bsg::max_k()));
         return nullptr;
     }
-    if (bsg::smem_bytes(K) + bsg::kStaticSmem > static_cast<size_t>(optin)) {
-        fail(BSGEMM_ERR_UNSUPPORTED, "this device has too little shared memory per block for K = " + std::to_string(K));
-        delete h;
+    if (!indices || !scales) {
+        fail(BSGEMM_ERR_INVALID, "indices and scales must not be NULL");
         return nullptr;
     }
-    e = bsg::prepare_kernels(K, &h->ctas_per_sm);
-    if (e != cudaSuccess || h->ctas_per_sm < 1) {
-        fail(BSGEMM_ERR_CUDA, e != cudaSuccess ? cuda_msg("kernel setup", e) : "kernel cannot be resident on an SM");
-        delete h;
+    const int ng4 = K / 4;  // column groups
+    const int32_t* indptr = indices;
+    const int32_t* colgrp = indices + N + 1;
+    const int64_t nnz = indptr[N];
+    if (indptr[0] != 0 || nnz < 0 || nnz > static_cast<int64_t>(N) * ng4) {
+        fail(BSGEMM_ERR_INVALID, "indptr[0] must be 0 and 0 <= indptr[N] <= N * K / 4");
         return nullptr;
     }
-
-    const size_t off_gptr = 0;
-    const size_t off_grow = align_up(off_gptr + sizeof(int32_t) * (ngroups + 1), 256);
-    const size_t off_recs = align_up(off_grow + sizeof(int32_t) * grow.size(), 256);
-    const size_t off_scale = align_up(off_recs + sizeof(int32_t) * recs.size(), 256);
-    const size_t off_bias = align_up(off_scale + sizeof(float) * npad, 256);
-    const size_t off_status = align_up(off_bias + sizeof(float) * npad, 256);
-    h->arena_bytes = align_up(off_status + sizeof(int), 256);
-    e = cudaMalloc(&h->arena, h->arena_bytes);
-    if (e != cudaSuccess) {
-        fail(BSGEMM_ERR_CUDA, cuda_msg("cudaMalloc", e));
-        delete h;
+    if (nnz > 0 && !values) {
+        fail(BSGEMM_ERR_INVALID, "values must not be NULL when blocks are stored");
         return nullptr;
     }
-    char* base = static_cast<char*>(h->arena);
-    struct Piece { size_t off; const void* src; size_t bytes; } pieces[] = {
-        {off_gptr, gptr.data(), sizeof(int32_t) * gptr.size()},
-        {off_grow, grow.data(), sizeof(int32_t) * grow.size()},
-        {off_recs, recs.data(), sizeof(int32_t) * recs.size()},
-        {off_scale, scale_v.data(), sizeof(float) * npad},
-        {off_bias, bias_v.data(), sizeof(float) * npad},
-        {off_status, &kZeroStatus, sizeof(int)},
-    };
-    for (const Piece& p : pieces) {
-        e = cudaMemcpy(base + p.off, p.src, p.bytes, cudaMemcpyHostToDevice);
-        if (e != cudaSuccess) {
-            fail(BSGEMM_ERR_CUDA, cuda_msg("cudaMemcpy", e));
-            cudaFree(h->arena);
-            delete h;
+    for (int n = 0; n < N; ++n) {
+        if (indptr[n + 1] < indptr[n]) {
+            fail(BSGEMM_ERR_INVALID, "indptr must be non-decreasing (row " + std::to_string(n) + ")");
+            return nullptr;
+        }
+        for (int e = indptr[n]; e < indptr[n + 1]; ++e) {
+            if (colgrp[e] < 0 || colgrp[e] >= ng4 || (e > indptr[n] && colgrp[e - 1] >= colgrp[e])) {
+                fail(BSGEMM_ERR_INVALID, "column groups must lie in [0, K/4) and strictly increase within row " +
+                                             std::to_string(n));
+                return nullptr;
+            }
+        }
+        if (!std::isfinite(scales[n]) || (bias && !std::isfinite(bias[n]))) {
+            fail(BSGEMM_ERR_INVALID, "scales and bias must be finite (channel " + std::to_string(n) + ")");
             return nullptr;
         }
     }
-    h->nnzb = nnzb;
-    h->cost = cost;
-    h->w.gptr = reinterpret_cast<const int32_t*>(base + off_gptr);
-    h->w.grow = reinterpret_cast<const int4*>(base + off_grow);
-    h->w.recs = reinterpret_cast<const int4*>(base + off_recs);
-    h->w.scale = reinterpret_cast<const float*>(base + off_scale);
-    h->w.bias = reinterpret_cast<const float*>(base + off_bias);
-    h->w.status = reinterpret_cast<int*>(base + off_status);
-    h->w.N = N;
-    h->w.K = K;
-    h->w.ngroups = ngroups;
-    h->w.S = S;
-    return h;
+    Repacked rp;
+    rp.shape = kShape1x4;
+    rp.N = N;
+    rp.K = K;
+    rp.nnzb = nnz;
+    rp.ngroups = (N + 3) / 4;
+    std::vector<int> rows(N);
+    for (int n = 0; n < N; ++n) rows[n] = n;
+    std::stable_sort(rows.begin(), rows.end(),
+                     [&](int x, int y) { return indptr[x + 1] - indptr[x] > indptr[y + 1] - indptr[y]; });
+    rp.grow.assign(static_cast<size_t>(rp.ngroups) * 4, -1);
+    rp.gptr.assign(rp.ngroups + 1, 0);
+    rp.cost.assign(rp.ngroups + 1, 0);
+    for (int gi = 0; gi < rp.ngroups; ++gi) {
+        int steps = 0;
+        for (int q = 0; q < 4 && 4 * gi + q < N; ++q) {
+            rp.grow[4 * gi + q] = rows[4 * gi + q];
+            steps = std::max(steps, indptr[rows[4 * gi + q] + 1] - indptr[rows[4 * gi + q]]);
+        }
+        steps = (steps + bsg::kBlock - 1) / bsg::kBlock * bsg::kBlock;
+        rp.gptr[gi + 1] = rp.gptr[gi] + steps;
+        rp.cost[gi + 1] = static_cast<int32_t>(rp.cost[gi] + steps + (steps > 0 ? kGroupCost : 0));
+    }
+    rp.S = rp.gptr[rp.ngroups];
+    rp.recs.assign(static_cast<size_t>(rp.S + bsg::kStepPad) * 32, 0);
+    const int pad_grp[2] = {0, ng4 > 1 ? 1 : 0};  // padding blocks: column group 0 (even) or 1 (odd)
+    std::vector<int> left[4][2];                   // a row's remaining blocks by column-group parity
+    for (int gi = 0; gi < rp.ngroups; ++gi) {
+        for (int q = 0; q < 4; ++q) {
+            left[q][0].clear();
+            left[q][1].clear();
+            const int n = rp.grow[4 * gi + q];
+            if (n < 0) continue;
+            for (int e = indptr[n + 1] - 1; e >= indptr[n]; --e) left[q][colgrp[e] & 1].push_back(e);
+        }
+        for (int st = rp.gptr[gi]; st < rp.gptr[gi + 1]; ++st) {
+            int32_t* rec = &rp.recs[static_cast<size_t>(st) * 32];
+            for (int h = 0; h < 2; ++h) {
+                const int qa = 2 * h, qb = 2 * h + 1;
+                // parity of row qa's block this step: the pairing (pa, 1 - pa)
+                // that both rows can serve, from the fuller lists first
+                auto have = [&](int q, int par) { return !left[q][par].empty(); };
+                int pa;
+                const bool ok0 = have(qa, 0) && have(qb, 1), ok1 = have(qa, 1) && have(qb, 0);
+                if (ok0 && ok1)
+                    pa = left[qa][0].size() + left[qb][1].size() >= left[qa][1].size() + left[qb][0].size() ? 0 : 1;
+                else if (ok0 || ok1)
+                    pa = ok0 ? 0 : 1;
+                else  // one row (or neither) has blocks left: it takes its fuller list, the other pads opposite
+                    pa = have(qa, 0) || have(qa, 1) ? (left[qa][0].size() >= left[qa][1].size() ? 0 : 1)
+                                                     : (have(qb, 0) || have(qb, 1)
+                                                            ? 1 - (left[qb][0].size() >= left[qb][1].size() ? 0 : 1)
+                                                            : 0);
+                for (int x = 0; x < 2; ++x) {
+                    const int q = x == 0 ? qa : qb;
+                    const int par = x == 0 ? pa : 1 - pa;
+                    int blk = -1;
+                    if (have(q, par)) {
+                        blk = left[q][par].back();
+                        left[q][par].pop_back();
+                    } else if (have(q, 1 - par)) {  // a conflict rather than an extra step
+                        blk = left[q][1 - par].back();
+                        left[q][1 - par].pop_back();
+                    }
+                    const int j = blk >= 0 ? colgrp[blk] : pad_grp[par];
+                    uint32_t word = 0;
+                    if (blk >= 0)
+                        for (int e = 0; e < 4; ++e)
+                            word |= static_cast<uint32_t>(static_cast<uint8_t>(values[static_cast<size_t>(blk) * 4 + e]))
+                                    << (8 * e);
+                    for (int e = 0; e < 4; ++e) rec[4 * q + e] = static_cast<int32_t>(bsg::tile_row_offset(4 * j + e));
+                    rec[16 + 4 * q] = static_cast<int32_t>(word);  // w[q][0]; w[q][1..3] stay 0
+                }
+            }
+        }
+    }
+    return upload(rp, scales, bias);
+}
+
+// 2:4-sparse weights: run as the 4 x 1 blocks that hold their values (a
+// block (r, k) is stored when one of rows 4r..4r+3 has a nonzero value in
+// column k), through the 4 x 1 path.
+bsgemm_t bsgemm_create_2to4(int N, int K, const int8_t* values, const uint8_t* idx, const float* scales,
+                            const float* bias) {
+    clear_error();
+    if (N < 1 || K < 4 || K % 4 != 0 || !values || !idx) {
+        fail(BSGEMM_ERR_INVALID, "need N >= 1, K >= 4 a multiple of 4, and values and idx");
+        return nullptr;
+    }
+    const int half = K / 2;
+    const int nbr = (N + 3) / 4;
+    std::vector<int8_t> dense(static_cast<size_t>(nbr) * 4 * K, 0);
+    for (int n = 0; n < N; ++n) {
+        for (int gj = 0; gj < K / 4; ++gj) {
+            const size_t p = static_cast<size_t>(n) * half + 2 * gj;
+            const int i0 = idx[p], i1 = idx[p + 1];
+            if (i0 >= i1 || i1 > 3) {
+                fail(BSGEMM_ERR_INVALID, "2:4 positions must strictly increase within [0, 4) (row " +
+                                             std::to_string(n) + ", group " + std::to_string(gj) + ")");
+                return nullptr;
+            }
+            dense[static_cast<size_t>(n) * K + 4 * gj + i0] = values[p];
+            dense[static_cast<size_t>(n) * K + 4 * gj + i1] = values[p + 1];
+        }
+    }
+    std::vector<int32_t> indices(nbr + 1, 0);
+    std::vector<int8_t> vals;
+    std::vector<int32_t> cols;
+    for (int r = 0; r < nbr; ++r) {
+        for (int k = 0; k < K; ++k) {
+            int8_t v[4];
+            bool any = false;
+            for (int c = 0; c < 4; ++c) {
+                v[c] = dense[static_cast<size_t>(4 * r + c) * K + k];
+                any = any || v[c] != 0;
+            }
+            if (!any) continue;
+            cols.push_back(k);
+            vals.insert(vals.end(), v, v + 4);
+        }
+        indices[r + 1] = static_cast<int32_t>(cols.size());
+    }
+    indices.insert(indices.end(), cols.begin(), cols.end());
+    return bsgemm_create(N, K, BSGEMM_BLOCK, indices.data(), vals.empty() ? nullptr : vals.data(), scales, bias);
 }
 
 // mode: 0 = gather from act (no scratch), 1 = relayout act into workspace
@@ -436,6 +651,8 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
             return fail(BSGEMM_ERR_INVALID, "the residual must be a 4-byte aligned device array");
         if (!std::isfinite(epi.residual_scale)) return fail(BSGEMM_ERR_INVALID, "residual_scale must be finite");
     }
+    if (h->shape == kShape1x4 && epi.kind == BSGEMM_OUT_F32_RESID)
+        return fail(BSGEMM_ERR_UNSUPPORTED, "the residual epilogue takes 4 x 1-block weights");
     if (epi.flags & ~static_cast<uint32_t>(BSGEMM_ACT_READY))
         return fail(BSGEMM_ERR_INVALID, "unknown bits in epi.flags");
     float inv = 0.0f;
@@ -484,6 +701,7 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.out = out;
     a.M = M;
     a.kind = epi.kind;
+    a.shape = h->shape;
     a.inv_out_scale = inv;
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
     a.skip_copy = (g_test_hooks.load() & BSGEMM_TEST_SKIP_TILE_COPY) != 0;

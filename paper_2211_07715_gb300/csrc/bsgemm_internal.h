@@ -72,6 +72,7 @@ struct LaunchArgs {
     const int8_t* res;     // kind 5: int8 residual [M][N]
     float res_scale;       // kind 5: the residual's scale
     int ld;                // row stride of x^T in bytes (kmajor only)
+    int shape;             // block shape of the weight: 0 = 4 x 1 blocks, 1 = 1 x 4 blocks
     int box_d;             // 64-column boxes per tensor copy (set by launch: >1 with a 3-D map of x)
     unsigned wait_limit;   // polls of a wait on a tile copy before it gives up (0: the default)
     bool skip_copy;        // test hook: issue no tile copy, so that every such wait gives up

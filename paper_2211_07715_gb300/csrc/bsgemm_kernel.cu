@@ -237,11 +237,6 @@ __device__ __forceinline__ void dot16(const uint32_t (&t)[8], const int4& w, int
         acc[4 * i + 3] = __dp4a(static_cast<int>(t[i]), w.w, acc[4 * i + 3]);
     }
 }
-__device__ __forceinline__ void step16(uint32_t tb, uint32_t lb, int off, const int4& w, int (&acc)[32]) {
-    uint32_t t[8];
-    gather16(tb, lb, off, t);
-    dot16(t, w, acc);
-}
 
 // This lane's view of the step records: ro points at the column offset of
 // row (lane % 16) of a step, rw at quad q's 4 channel words of the same
@@ -286,20 +281,84 @@ __device__ __forceinline__ unsigned long long pack_rows16(int4 gr) {
     return f(gr.x) | f(gr.y) << 16 | f(gr.z) << 32 | f(gr.w) << 48;
 }
 
+// Block shapes of the stored weight.  A step's gather gives lane (g, q)
+// the dot-4 words of tokens g + 8 i (i < 8) for the 4 columns of quad q;
+// what a quad holds differs:
+//   kShape4x1: 4 stored 4 x 1 blocks of block-row q (4 columns, 4 output
+//     channels each): 32 dp4a against the quad's 4 channel words, 32
+//     accumulators a lane (8 tokens x 4 channels);
+//   kShape1x4: one 1 x 4 block (one output row x 4 consecutive columns) of
+//     the group's row q: 8 dp4a against its one weight word, 8 accumulators
+//     a lane (8 tokens x 1 row).
+constexpr int kShape4x1 = 0;
+constexpr int kShape1x4 = 1;
+
+template <int SHAPE>
+struct BlockShape {
+    static constexpr int kAcc = 32;
+    __device__ static __forceinline__ void dot(const uint32_t (&t)[8], const int4& w, int (&acc)[kAcc]) {
+        dot16(t, w, acc);
+    }
+    // scale and bias of block-row r's 4 channels (r < 0: an unused float4)
+    __device__ static __forceinline__ float4 load_sb(const float* p, int r, uint64_t pol) {
+        return ldg_hint(reinterpret_cast<const float4*>(p) + max(r, 0), pol);
+    }
+    template <int KIND>
+    __device__ static __forceinline__ void store(const LaunchArgs& a, int N, long long m_g, int r,
+                                                 const int (&acc)[kAcc], float4 sc, float4 bi) {
+        store_lane<KIND>(a, N, m_g, r, acc, sc, bi);
+    }
+};
+
+template <>
+struct BlockShape<kShape1x4> {
+    static constexpr int kAcc = 8;
+    __device__ static __forceinline__ void dot(const uint32_t (&t)[8], const int4& w, int (&acc)[kAcc]) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] = __dp4a(static_cast<int>(t[i]), w.x, acc[i]);
+    }
+    // scale and bias of row n in .x
+    __device__ static __forceinline__ float4 load_sb(const float* p, int n, uint64_t pol) {
+        return make_float4(__int_as_float(ldg_hint(reinterpret_cast<const int*>(p) + max(n, 0), pol)), 0.f, 0.f, 0.f);
+    }
+    // Epilogue of row n at tokens m_g + 8 i: one value a token (no residual kind).
+    template <int KIND>
+    __device__ static __forceinline__ void store(const LaunchArgs& a, int N, long long m_g, int n,
+                                                 const int (&acc)[kAcc], float4 sc, float4 bi) {
+        if (n < 0) return;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const long long m = m_g + 8 * i;
+            if (m >= a.M) continue;
+            const size_t o = static_cast<size_t>(m) * N + n;
+            if (KIND == 0) {
+                static_cast<int32_t*>(a.out)[o] = acc[i];
+            } else if (KIND == 1 || KIND == 2) {
+                static_cast<float*>(a.out)[o] = epilogue_value<KIND>(acc[i], sc.x, bi.x);
+            } else if (KIND == 3 || KIND == 4) {
+                const int q = __float2int_rn(__fmul_rn(epilogue_value<KIND>(acc[i], sc.x, bi.x), a.inv_out_scale));
+                static_cast<int8_t*>(a.out)[o] = static_cast<int8_t>(q > 127 ? 127 : (q < -128 ? -128 : q));
+            }
+        }
+    }
+};
+
 // MODE: how a window's token tile reaches shared memory.
 constexpr int kStageGather = 0;  // per-thread loads from x [M][K], transposed in registers
 constexpr int kStageTiles = 1;   // one bulk copy of a tile the relayout kernel wrote
 constexpr int kStageTensor = 2;  // tensor copies of x's boxes, transposed in place (transpose_box)
 constexpr int kStageKMajor = 3;  // tensor copies of x^T [K][M] boxes, already in the tile's layout
 
-template <int KIND, int MODE>
+template <int KIND, int MODE, int SHAPE>
 __global__ void __launch_bounds__(kThreads, 1)
 bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sched,
               const __grid_constant__ CUtensorMap xmap) {
     constexpr bool TMA = MODE == kStageTiles;
     constexpr bool KMAJOR = MODE == kStageKMajor;
     constexpr bool TENSOR = MODE == kStageTensor || KMAJOR;
-    constexpr int SW = kTile * 16;  // slot words: 64 tokens x 4 block-rows x 4 channels
+    using BS = BlockShape<SHAPE>;
+    constexpr int NA = BS::kAcc;    // accumulators a lane
+    constexpr int SW = 32 * NA;     // slot words: a warp's accumulators
     static_assert(kGroupWin < kThreads, "one thread loads each group of a window");
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int s_gp[kGroupWin + 1];                          // step offsets of the current group window
@@ -421,7 +480,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             }
             const long long into = target - (static_cast<long long>(s_gp[lo] - sa) + static_cast<long long>(lo) * kGroupEndCost);
             const int len = s_gp[lo + 1] - s_gp[lo];  // a multiple of kBlock
-            const int in_grp = static_cast<int>(into < len ? into : len) & ~(kBlock - 1);
+            const int in_grp = static_cast<int>(into < len ? into : len) / kBlock * kBlock;
             s_wst[tid] = (tid == kWarps) ? s_gp[ngw] - sa : s_gp[lo] - sa + in_grp;
         }
         __syncthreads();  // the warps' step ranges are visible
@@ -443,8 +502,8 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             if (fin) {
                 fin_r = block_row16(s_grow[j], q);
                 if (KIND != 0) {  // needed after the window; no wait here
-                    fin_sc = ldg_hint(reinterpret_cast<const float4*>(w.scale) + max(fin_r, 0), pol_w);
-                    fin_bi = ldg_hint(reinterpret_cast<const float4*>(w.bias) + max(fin_r, 0), pol_w);
+                    fin_sc = BS::load_sb(w.scale, fin_r, pol_w);
+                    fin_bi = BS::load_sb(w.bias, fin_r, pol_w);
                 }
             }
         }
@@ -482,11 +541,13 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
         for (int gi = g_lo + warp; gi < g_hi; gi += kWarps) {
             if (gp(gi) == gp(gi + 1)) {
                 const int r = block_row16(s_grow[gi - g_lo], q);
-                int zero[32];
+                int zero[NA];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) zero[i] = 0;
+                for (int i = 0; i < NA; ++i) zero[i] = 0;
                 wait_prev();
-                if (r >= 0) store_lane<KIND>(a, N, m0 + g, r, zero, load_s4(w.scale, r), load_s4(w.bias, r));
+                if (r >= 0)
+                    BS::template store<KIND>(a, N, m0 + g, r, zero, BS::load_sb(w.scale, r, pol_w),
+                                             BS::load_sb(w.bias, r, pol_w));
             }
         }
 
@@ -528,6 +589,12 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
             staged = t;
         }
 
+        // one step: the gathers, then the block shape's dot products
+        auto bsg_step = [&](int off_i, const int4& w_i, int (&acc_r)[NA]) {
+            uint32_t t[8];
+            gather16(tb, lb, off_i, t);
+            BS::dot(t, w_i, acc_r);
+        };
         if (ws0 < ws1) {
             int gi = g_lo + row_of(s_gp, 0, g_hi - g_lo, sa + ws0);
             int p = ws0;  // step index relative to sa
@@ -538,12 +605,12 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 const int r = block_row16(s_grow[gi - g_lo], q);
                 float4 sc = make_float4(0.f, 0.f, 0.f, 0.f), bi = sc;
                 if (KIND != 0) {  // used at the group's end: the loads fly during its steps
-                    sc = ldg_hint(reinterpret_cast<const float4*>(w.scale) + max(r, 0), pol_w);
-                    bi = ldg_hint(reinterpret_cast<const float4*>(w.bias) + max(r, 0), pol_w);
+                    sc = BS::load_sb(w.scale, r, pol_w);
+                    bi = BS::load_sb(w.bias, r, pol_w);
                 }
-                int acc[32];
+                int acc[NA];
 #pragma unroll
-                for (int i = 0; i < 32; ++i) acc[i] = 0;
+                for (int i = 0; i < NA; ++i) acc[i] = 0;
                 // Steps p .. p_end - 1.  Ring slot i holds step (ring base + i);
                 // after its step it loads step (base + kRing + i), and after
                 // slot kRing - 1 the base moves on by kRing.  Groups hold a
@@ -557,7 +624,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                     if (blk == 0 && p + kRing <= p_end) {
 #pragma unroll
                         for (int i = 0; i < kRing; ++i) {
-                            step16(tb, lb, off[i], wq[i], acc);
+                            bsg_step(off[i], wq[i], acc);
                             rec.load(kRing + i, off[i], wq[i], pol_w);
                         }
                         rec.advance(kRing);
@@ -566,7 +633,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                     }
 #define BSG_RING_BLOCK(j)                                                   \
     _Pragma("unroll") for (int i = kBlock * (j); i < kBlock * ((j) + 1); ++i) { \
-        step16(tb, lb, off[i], wq[i], acc);                                  \
+        bsg_step(off[i], wq[i], acc);                                  \
         rec.load(kRing + i, off[i], wq[i], pol_w);                           \
     }
                     if (blk == 0) {
@@ -585,7 +652,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                 }
                 if (gs >= sa + ws0 && ge <= sa + ws1) {
                     wait_prev();
-                    store_lane<KIND>(a, N, m0 + g, r, acc, sc, bi);
+                    BS::template store<KIND>(a, N, m0 + g, r, acc, sc, bi);
                 } else {
                     // Shared with other warps: add into the slot of the first warp
                     // boundary inside the group (the first b with s_wst[b] > the
@@ -596,7 +663,7 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
                     while (s_wst[b] <= gs - sa) ++b;
                     int* sl = slots + (b - 1) * SW + lane;
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) atomicAdd(sl + 32 * j, acc[j]);
+                    for (int j = 0; j < NA; ++j) atomicAdd(sl + 32 * j, acc[j]);
                 }
                 ++gi;
                 while (gi < g_hi && gp(gi + 1) == gp(gi)) ++gi;  // skip groups without steps
@@ -606,14 +673,14 @@ bsgemm_kernel(DeviceWeights w, LaunchArgs a, const __grid_constant__ Schedule sc
 
         if (fin) {  // the split group of boundary warp + 1 (see above)
             int* sl = slots + warp * SW + lane;
-            int acc[32];
+            int acc[NA];
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
+            for (int j = 0; j < NA; ++j) {
                 acc[j] = sl[32 * j];
                 sl[32 * j] = 0;
             }
             wait_prev();
-            store_lane<KIND>(a, N, m0 + g, fin_r, acc, fin_sc, fin_bi);
+            BS::template store<KIND>(a, N, m0 + g, fin_r, acc, fin_sc, fin_bi);
         }
         if (u < u_end) __syncthreads();  // the window's offsets, the slots' reset and the tile may be reused
     }
@@ -699,24 +766,30 @@ pretile_kernel(const int8_t* __restrict__ x, int M, int K, int kpad, int8_t* __r
     }
 }
 
-template <int MODE>
+template <int MODE, int SHAPE>
 const void* kernel_for(int kind) {
     switch (kind) {
-    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<0, MODE>);
-    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<1, MODE>);
-    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<2, MODE>);
-    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<3, MODE>);
-    case 4: return reinterpret_cast<const void*>(&bsgemm_kernel<4, MODE>);
-    default: return reinterpret_cast<const void*>(&bsgemm_kernel<5, MODE>);
+    case 0: return reinterpret_cast<const void*>(&bsgemm_kernel<0, MODE, SHAPE>);
+    case 1: return reinterpret_cast<const void*>(&bsgemm_kernel<1, MODE, SHAPE>);
+    case 2: return reinterpret_cast<const void*>(&bsgemm_kernel<2, MODE, SHAPE>);
+    case 3: return reinterpret_cast<const void*>(&bsgemm_kernel<3, MODE, SHAPE>);
+    case 4: return reinterpret_cast<const void*>(&bsgemm_kernel<4, MODE, SHAPE>);
+    default: return SHAPE == kShape4x1 ? reinterpret_cast<const void*>(&bsgemm_kernel<5, MODE, kShape4x1>) : nullptr;
     }
 }
-const void* kernel_for(int kind, int mode) {
+template <int SHAPE>
+const void* kernel_for_mode(int kind, int mode) {
     switch (mode) {
-    case kStageKMajor: return kernel_for<kStageKMajor>(kind);
-    case kStageTensor: return kernel_for<kStageTensor>(kind);
-    case kStageTiles: return kernel_for<kStageTiles>(kind);
-    default: return kernel_for<kStageGather>(kind);
+    case kStageKMajor: return kernel_for<kStageKMajor, SHAPE>(kind);
+    case kStageTensor: return kernel_for<kStageTensor, SHAPE>(kind);
+    case kStageTiles: return kernel_for<kStageTiles, SHAPE>(kind);
+    default: return kernel_for<kStageGather, SHAPE>(kind);
     }
+}
+// The layer kernel for an epilogue kind, staging mode and block shape (NULL
+// for the residual kind with 1 x 4 blocks, which is not built).
+const void* kernel_for(int kind, int mode, int shape) {
+    return shape == kShape1x4 ? kernel_for_mode<kShape1x4>(kind, mode) : kernel_for_mode<kShape4x1>(kind, mode);
 }
 
 // cuTensorMapEncodeTiled from the driver, looked up once.
@@ -756,14 +829,19 @@ int max_k() {
 
 cudaError_t prepare_kernels(int K, int* ctas_per_sm) {
     const int smem = static_cast<int>(smem_bytes(K));
-    for (int kind = 0; kind < 6; ++kind) {
-        for (int mode = 0; mode < 4; ++mode) {
-            cudaError_t e = cudaFuncSetAttribute(kernel_for(kind, mode), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 kSmemOptin - kStaticSmem);
-            if (e != cudaSuccess) return e;
+    for (int shape = 0; shape < 2; ++shape) {
+        for (int kind = 0; kind < 6; ++kind) {
+            for (int mode = 0; mode < 4; ++mode) {
+                const void* k = kernel_for(kind, mode, shape);
+                if (!k) continue;
+                cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                     kSmemOptin - kStaticSmem);
+                if (e != cudaSuccess) return e;
+            }
         }
     }
-    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_for(0, kStageTensor), kThreads, smem);
+    return cudaOccupancyMaxActiveBlocksPerMultiprocessor(ctas_per_sm, kernel_for(0, kStageTensor, kShape4x1), kThreads,
+                                                         smem);
 }
 
 cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a_in, const Schedule& sched, int grid, cudaStream_t s) {
@@ -834,25 +912,36 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a_in, const Schedul
         }
     }
     cudaError_t e = cudaSuccess;
-#define BSG_LAUNCH(KV)                                                                                   \
+#define BSG_LAUNCH(KV, SH)                                                                               \
     do {                                                                                                 \
         if (a.kmajor)                                                                                    \
-            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageKMajor>, w, a, sched, xmap);            \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageKMajor, SH>, w, a, sched, xmap);        \
         else if (a.tensor)                                                                               \
-            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTensor>, w, a, sched, xmap);            \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTensor, SH>, w, a, sched, xmap);        \
         else if (a.xb)                                                                                   \
-            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTiles>, w, a, sched, xmap);             \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageTiles, SH>, w, a, sched, xmap);         \
         else                                                                                             \
-            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageGather>, w, a, sched, xmap);            \
+            e = cudaLaunchKernelEx(&cfg, bsgemm_kernel<KV, kStageGather, SH>, w, a, sched, xmap);        \
+    } while (0)
+#define BSG_LAUNCH_KIND(KV)                       \
+    do {                                          \
+        if (a.shape == kShape1x4)                 \
+            BSG_LAUNCH(KV, kShape1x4);            \
+        else                                      \
+            BSG_LAUNCH(KV, kShape4x1);            \
     } while (0)
     switch (a.kind) {
-    case 0: BSG_LAUNCH(0); break;
-    case 1: BSG_LAUNCH(1); break;
-    case 2: BSG_LAUNCH(2); break;
-    case 3: BSG_LAUNCH(3); break;
-    case 4: BSG_LAUNCH(4); break;
-    default: BSG_LAUNCH(5); break;
+    case 0: BSG_LAUNCH_KIND(0); break;
+    case 1: BSG_LAUNCH_KIND(1); break;
+    case 2: BSG_LAUNCH_KIND(2); break;
+    case 3: BSG_LAUNCH_KIND(3); break;
+    case 4: BSG_LAUNCH_KIND(4); break;
+    default:
+        if (a.shape == kShape1x4) return cudaErrorNotSupported;
+        BSG_LAUNCH(5, kShape4x1);
+        break;
     }
+#undef BSG_LAUNCH_KIND
 #undef BSG_LAUNCH
     return e != cudaSuccess ? e : cudaGetLastError();
 }

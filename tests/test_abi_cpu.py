@@ -172,3 +172,31 @@ def test_variant_shapes_reject_bad_arrays(bsg):
             bsg.dense_from_2to4(v, np.array(bad, np.uint8))
     with pytest.raises(ValueError):
         bsg.dense_from_2to4(np.ones((1, 3), np.int8), np.zeros((1, 3), np.uint8))   # K not a multiple of 4
+
+
+def test_create_1x4_and_2to4_reject_bad_arrays_before_the_device(bsg):
+    """bsgemm_create_1x4 / bsgemm_create_2to4 check their host arrays before
+    any device call (so this runs without a GPU)."""
+    ones = np.ones((2, 4), np.int8)
+    sc = np.ones(2, np.float32)
+    for n, k, ip, cg in ((2, 6, [0, 1, 2], [0, 0]),       # K % 4
+                         (2, 8, [1, 1, 2], [0, 1]),       # indptr[0] != 0
+                         (2, 8, [0, 2, 1], [0, 1]),       # decreasing
+                         (2, 8, [0, 1, 2], [0, 2]),       # group = K / 4
+                         (2, 8, [0, 2, 2], [1, 1]),       # repeated group in a row
+                         (2, 8, [0, 2, 2], [1, 0]),       # unsorted
+                         (0, 8, [0], [])):                # N = 0
+        with pytest.raises(bsg.BsgemmError) as e:
+            bsg.bsgemm_create_1x4(n, k, np.array(ip + cg, np.int32), ones, sc)
+        assert e.value.code == bsg.ERR_INVALID
+    with pytest.raises(bsg.BsgemmError) as e:  # a NaN scale
+        bsg.bsgemm_create_1x4(2, 8, np.array([0, 1, 2, 0, 1], np.int32), ones, np.array([1, np.nan], np.float32))
+    assert e.value.code == bsg.ERR_INVALID
+    with pytest.raises(bsg.BsgemmError) as e:  # K beyond the tile
+        bsg.bsgemm_create_1x4(1, 4 * (bsg.bsgemm_max_k() // 4 + 1), np.array([0, 0], np.int32), ones, sc[:1])
+    assert e.value.code == bsg.ERR_UNSUPPORTED
+    v = np.ones((1, 2), np.int8)
+    for bad in ([[1, 1]], [[2, 1]], [[0, 4]]):  # positions must strictly increase within [0, 4)
+        with pytest.raises(bsg.BsgemmError) as e:
+            bsg.bsgemm_create_2to4(1, 4, v, np.array(bad, np.uint8), sc[:1])
+        assert e.value.code == bsg.ERR_INVALID

@@ -1,9 +1,12 @@
-"""Variant block shapes through the layer kernel: weights sparse in 1 x 4
-blocks (one output row x 4 input columns) and 2:4-sparse weights, regrouped
-at create time into the 4 x 1 blocks that hold them
-(SparseInt8Linear.from_blocks_1x4 / from_2to4).  Every element against the
-oracle's linear on the oracle's own decompression of the same arrays:
-integer outputs bit for bit, fp32 within 1e-4 abs or 1e-5 rel."""
+"""Other block shapes through the layer kernel, every element against the
+oracle's linear on the oracle's own decompression of the same arrays
+(integer outputs bit for bit, fp32 within 1e-4 abs or 1e-5 rel):
+  * weights sparse in 1 x 4 blocks (one output row x 4 input columns), run
+    natively by the kernel's 1 x 4 form (bsgemm_create_1x4): every kind but
+    the residual, both staging paths, ragged K (relayout path), K = 4,
+    N not a multiple of 4, rows without blocks, one token;
+  * 2:4-sparse weights (bsgemm_create_2to4: the 4 x 1 blocks that hold
+    them)."""
 import numpy as np
 import pytest
 
@@ -44,7 +47,8 @@ def gpu_run(lin, x: np.ndarray, kind: int, out_scale: float, workspace=None) -> 
     return out.cpu().numpy()
 
 
-@pytest.mark.parametrize("n_out,k_in,m,sparsity", [(96, 768, 130, 0.9), (30, 200, 70, 0.5), (768, 3072, 64, 0.9)])
+@pytest.mark.parametrize("n_out,k_in,m,sparsity", [(96, 768, 130, 0.9), (30, 200, 70, 0.5), (768, 3072, 64, 0.9),
+                                                    (7, 4, 65, 0.0), (130, 100, 1, 0.6), (64, 3072, 200, 0.97)])
 def test_blocks_1x4_through_the_layer(bsg, n_out, k_in, m, sparsity):
     rng = synth.rng_for(8000 + n_out + k_in)
     wt = synth.draw_weight_1x4(rng, n_out, k_in, sparsity)
@@ -70,4 +74,31 @@ def test_2to4_through_the_layer(bsg, n_out, k_in, m):
     for kind in KINDS:
         want = oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
         check(gpu_run(lin, x, kind, 0.05), want, kind, f"2:4 kind {kind}")
+    lin.close()
+
+
+def test_blocks_1x4_empty_rows_and_residual_rejected(bsg):
+    rng = synth.rng_for(8050)
+    n_out, k_in = 40, 256
+    wt = synth.draw_weight_1x4(rng, n_out, k_in, 0.8)
+    # rows 0, 5 and 39 without blocks
+    keep = np.ones(wt.indptr[-1], bool)
+    for r in (0, 5, 39):
+        keep[wt.indptr[r]:wt.indptr[r + 1]] = False
+    counts = np.diff(wt.indptr).copy()
+    for r in (0, 5, 39):
+        counts[r] = 0
+    indptr = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    colgrp, values = wt.colgrp[keep], wt.values[keep]
+    w = oracle.bsr1x4_to_dense(n_out, k_in, indptr, colgrp, values)
+    lin = bsg.SparseInt8Linear.from_blocks_1x4(n_out, k_in, indptr, colgrp, values, wt.scales, wt.bias)
+    assert lin.info["nnzb"] == int(indptr[-1])
+    x = synth.draw_x(rng, 99, k_in, "u127")
+    for kind in (synth.I32, synth.F32, synth.I8):
+        check(gpu_run(lin, x, kind, 0.05), oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05), kind)
+    out = torch.empty((99, n_out), dtype=torch.float32, device="cuda")
+    r8 = torch.zeros((99, n_out), dtype=torch.int8, device="cuda")
+    with pytest.raises(bsg.BsgemmError) as e:
+        lin.run(torch.from_numpy(x).cuda(), out, bsg.OUT_F32_RESID, residual=r8, residual_scale=0.1)
+    assert e.value.code == bsg.ERR_UNSUPPORTED
     lin.close()
