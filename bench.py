@@ -952,18 +952,17 @@ def run_layer(args) -> dict:
     }
 
 
-MMA_SYNC_BF16_TFLOPS = 594.0  # mma.sync m16n8k16 bf16 -> fp32, measured on GB300 at 2070 MHz (legacy tensor path)
 SFU_EX2_PER_SM_CLK = 16        # exponentials per SM per clock (special-function unit)
 
 
 def attention_roofline(batch: int, seq: int, heads: int, ms: float, sms: int, max_mhz: float, hbm_gbs: float,
                        bf16_tflops: float) -> dict:
     """The attention kernel against its floors: the tensor work (q k^T once,
-    P v twice for the two bf16 parts of P: 6 x batch x heads x seq^2 x 64
-    flops) at the measured dense bf16 rate, one exponential per score on the
-    special-function units, and the int8 QKV read once from HBM.  The
-    largest floor is the bound; the tensor floor at the rate the kernel's
-    mma.sync path itself can reach is reported beside it."""
+    P v twice for the two f16 parts of P: 6 x batch x heads x seq^2 x 64
+    flops) at the measured dense 16-bit rate (tcgen05 kind::f16 runs f16 at
+    the bf16 rate), one exponential per score on the special-function
+    units, and the int8 QKV read once from HBM.  The largest floor is the
+    bound."""
     macs = float(batch) * heads * seq * seq * 64
     clk = max_mhz * 1e6
     floors = {"tensor": 6 * macs / (bf16_tflops * 1e12),
@@ -971,18 +970,15 @@ def attention_roofline(batch: int, seq: int, heads: int, ms: float, sms: int, ma
               "hbm": float(batch) * seq * 3 * heads * 64 / (hbm_gbs * 1e9)}
     name = max(floors, key=floors.get)
     t = ms * 1e-3
-    mma_floor = 6 * macs / (MMA_SYNC_BF16_TFLOPS * 1e12)
     return {"kernel": "attention_kernel", "ms": round(ms, 6), "ops": 4 * macs,
             "achieved_tops": round(4 * macs / t / 1e12, 3),
             "floors_us": {k: round(v * 1e6, 3) for k, v in floors.items()},
             "bound": {"tensor": "tensor", "exp": "alu", "hbm": "hbm"}[name], "floor": name,
             "peak": bf16_tflops, "frac": round(floors[name] / t, 4),
-            "mma_sync_floor_us": round(mma_floor * 1e6, 3), "frac_of_mma_sync": round(mma_floor / t, 4),
             "basis": "graph of 200 launches, per launch; ops = 2 x (q k^T + P v) multiply-adds; floors: tensor = "
-                     "6 x MACs (P v twice: two bf16 parts) at the measured dense bf16 rate (MEASURED_PEAKS, burst), "
-                     "exp = one SFU exponential per score (16 per SM per clock at the max SM clock), hbm = QKV "
-                     "bytes at the measured copy rate; mma_sync = the tensor floor at the measured mma.sync m16n8k16 "
-                     "bf16 rate (594 TFLOP/s), the unit this kernel uses"}
+                     "6 x MACs (P v twice: two f16 parts) at the measured dense bf16 rate (MEASURED_PEAKS, burst; "
+                     "tcgen05.mma kind::f16), exp = one SFU exponential per score (16 per SM per clock at the max "
+                     "SM clock), hbm = QKV bytes at the measured copy rate"}
 
 
 def run_encoder(args) -> dict:

@@ -349,6 +349,16 @@ int bsgemm_attention(const int8_t* qkv, int batch, int seq, int heads, int head_
                      void* out, bsgemm_epilogue epi, void* stream);
 
 /*
+ * bsgemm_attention_status -- read (and with clear != 0, reset) the current
+ * device's attention status word: 0 when every wait of the attention
+ * kernel's launches completed; BSGEMM_STATUS_TIMEOUT when one gave up (a
+ * tensor-core MMA did not complete within the wait's limit; that launch's
+ * out is incomplete).  Synchronises the device.  Returns the status, or a
+ * negative BSGEMM_ERR_* code.
+ */
+int bsgemm_attention_status(int clear);
+
+/*
  * bsgemm_device_status -- read (and with clear != 0, reset) the handle's
  * device status word.  0 means every wait in the kernels completed; bit 0
  * (BSGEMM_STATUS_TIMEOUT) means a bounded wait on an asynchronous copy gave
@@ -372,10 +382,15 @@ int bsgemm_device_status(bsgemm_t h, int clear);
  *     its first grid barrier and the other CTAs give that barrier up after
  *     4096 polls; every CTA returns and bsgemm_block_prune returns
  *     BSGEMM_ERR_CUDA (keep is undefined).
+ *   BSGEMM_TEST_ATTN_SKIP_MMA: the attention kernel issues no tensor-core
+ *     MMA and gives each wait on one up after 64 polls (nothing is then in
+ *     flight when a CTA leaves); out is undefined and
+ *     bsgemm_attention_status reports BSGEMM_STATUS_TIMEOUT.
  * Not for production use.  Returns the previous bits.
  */
 #define BSGEMM_TEST_SKIP_TILE_COPY 1u
 #define BSGEMM_TEST_STALL_PRUNE_CTA 2u
+#define BSGEMM_TEST_ATTN_SKIP_MMA 4u
 uint32_t bsgemm_set_test_hooks(uint32_t bits);
 
 /*

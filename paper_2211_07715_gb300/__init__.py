@@ -92,6 +92,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_attention.restype = ctypes.c_int
     lib.bsgemm_device_status.argtypes = [vp, ctypes.c_int]
     lib.bsgemm_device_status.restype = ctypes.c_int
+    lib.bsgemm_attention_status.argtypes = [ctypes.c_int]
+    lib.bsgemm_attention_status.restype = ctypes.c_int
     lib.bsgemm_set_test_hooks.argtypes = [ctypes.c_uint32]
     lib.bsgemm_set_test_hooks.restype = ctypes.c_uint32
     lib.bsgemm_int8_peak.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
@@ -106,7 +108,7 @@ EXPORTED = ("bsgemm_create", "bsgemm_create_1x4", "bsgemm_create_2to4", "bsgemm_
             "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_layernorm",
             "bsgemm_attention", "bsgemm_destroy",
             "bsgemm_last_error", "bsgemm_last_status", "bsgemm_device_status", "bsgemm_max_k", "bsgemm_info",
-            "bsgemm_set_test_hooks", "bsgemm_int8_peak")
+            "bsgemm_set_test_hooks", "bsgemm_int8_peak", "bsgemm_attention_status")
 
 
 def _epi(kind: int, out_scale: float, flags: int = 0, residual: int = 0, residual_scale: float = 1.0) -> Epilogue:
@@ -339,6 +341,16 @@ def bsgemm_device_status(h: int, clear: bool = False) -> int:
 
 TEST_SKIP_TILE_COPY = 1  # BSGEMM_TEST_SKIP_TILE_COPY
 TEST_STALL_PRUNE_CTA = 2  # BSGEMM_TEST_STALL_PRUNE_CTA
+TEST_ATTN_SKIP_MMA = 4  # BSGEMM_TEST_ATTN_SKIP_MMA
+
+
+def bsgemm_attention_status(clear: bool = False) -> int:
+    """The current device's attention status word (STATUS_TIMEOUT when a
+    wait of the attention kernel gave up); synchronises the device."""
+    rc = _lib.bsgemm_attention_status(1 if clear else 0)
+    if rc < 0:
+        raise BsgemmError(rc, bsgemm_last_error())
+    return rc
 
 
 def bsgemm_set_test_hooks(bits: int) -> int:

@@ -28,7 +28,7 @@ def nvcc() -> str:
 
 
 def _inputs():
-    files = [os.path.join(CSRC, s) for s in SOURCES] + [os.path.join(CSRC, "bsgemm_device.cuh")]
+    files = [os.path.join(CSRC, s) for s in SOURCES] + [os.path.join(CSRC, h) for h in ("bsgemm_device.cuh", "bsgemm_tcgen05.cuh")]
     files += [os.path.join(CSRC, "bsgemm_internal.h"), os.path.join(INCLUDE, "bsgemm.h")]
     return files
 

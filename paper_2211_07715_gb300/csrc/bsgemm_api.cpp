@@ -934,6 +934,14 @@ int bsgemm_attention(const int8_t* qkv, int batch, int seq, int heads, int head_
     return BSGEMM_OK;
 }
 
+int bsgemm_attention_status(int clear) {
+    clear_error();
+    unsigned v = 0;
+    const cudaError_t e = bsg::attention_status(clear != 0, &v);
+    if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("reading the attention status", e));
+    return static_cast<int>(v);
+}
+
 int bsgemm_device_status(bsgemm_t h, int clear) {
     clear_error();
     if (!h) return fail(BSGEMM_ERR_INVALID, "NULL handle");

@@ -8,110 +8,112 @@
 //   out_t = (sum_j e_j v_j) * (qkv_scale / sum_j e_j)
 // No attention mask: every position of a sequence is a token.
 //
-// Both contractions run on the tensor cores (mma.sync m16n8k16, bf16
-// operands, fp32 accumulation):
-//   * q k^T is exact: int8 values are exact in bf16, the products (< 2^14)
+// Both contractions run on the fifth-generation tensor cores (tcgen05.mma
+// kind::f16, f16 operands, fp32 accumulators in tensor memory):
+//   * q k^T is exact: int8 values are exact in f16, the products (< 2^14)
 //     are exact, and every partial sum of 64 of them stays below 2^24, so
 //     the fp32 accumulator holds the int32 dot product;
-//   * P v takes P in two bf16 parts (p = hi + lo + r, |r| <= 2^-16 p) against
-//     the exact bf16 v, two MMAs per tile.
-// The softmax is taken online over blocks of 64 keys (running row maximum m
-// and sum l; when m grows, the context accumulator and l are scaled by the
-// same factor exp(m_old - m_new)), in fp32.
+//   * P v takes each weight in two f16 parts (e = hi + lo + r, |r| <= 2^-22
+//     e + 2^-25) against the exact f16 v, two MMAs per K step.
+// The softmax runs online over blocks of 128 keys in fp32: a thread keeps
+// its query's running maximum m of the exact dot products and its running
+// sum l; e_j = 2^((d_j - m) c log2(e)) with d_j - m exact, so the only
+// roundings inside the exponent are those of c log2(e) and of one product.
+// When m grows, the context and l are scaled by the same factor.
 //
-// One CTA = 64 queries of one (sequence, head), 4 warps of 16 queries.  The
-// head's keys and values for the whole sequence (seq <= BSGEMM_ATTN_MAX_SEQ,
-// padded to whole 64-key blocks with zeros) and the CTA's queries are
-// staged once into shared memory as bf16 rows of 64 (128 bytes, 16-byte
-// chunks XOR-swizzled by the row so that 8 consecutive rows of one chunk
-// lie in different banks); `ldmatrix` reads the MMA fragments: plain for
-// the queries and keys, transposed for the values.  The scores and
-// probabilities of a 16 x 64 block live in registers (the MMA output
-// layout of a score tile is the input layout of the P v MMA).
+// One CTA = 128 queries of one (sequence, head), 4 warps; thread i owns
+// query i = tensor-memory lane i.  Tensor memory (256 columns, so two CTAs
+// share an SM): S/P in columns 0-127 (the block's scores, then its weights
+// written back in place as f16 pairs: for keys 32c .. 32c + 31 the high
+// parts in columns 32c .. 32c + 15, the low parts in 32c + 16 .. 32c + 31),
+// the context O in 128-191, the CTA's queries (f16 pairs) in 192-223.  The
+// head's keys and values (seq <= BSGEMM_ATTN_MAX_SEQ, padded with zeros to
+// whole blocks) are staged once into shared memory as f16 rows of 64 with
+// the 128-byte swizzle: K is the K-major B operand of q k^T, V the MN-major
+// B operand of P v.  Per block one thread issues the 4 MMAs of S = Q K_b^T
+// (N = 128, K = 64) and, after the threads have written P, the 16 of O +=
+// P_hi V_b + P_lo V_b (N = 64, K = 128); completions arrive on two
+// mbarriers, every wait bounded.
+#include <cfloat>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
 
-#include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include "bsgemm.h"
+#include "bsgemm_device.cuh"
 #include "bsgemm_internal.h"
+#include "bsgemm_tcgen05.cuh"
 
 namespace bsg {
 namespace {
 
-constexpr int kAttnThreads = 128;  // 4 warps x 16 queries
-constexpr int kAttnQ = 64;         // queries per CTA
-constexpr int kKeyBlock = 64;      // keys per online-softmax block
+constexpr int kAttnThreads = 128;     // 4 warps, one query (TMEM lane) each
+constexpr int kAttnQ = 128;           // queries per CTA
+constexpr int kKeyBlock = 128;        // keys per online-softmax block
+constexpr uint32_t kBlockBytes = 16384;  // 128 rows x 64 f16
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kColS = 0, kColO = 128, kColQ = 192;
+constexpr uint32_t kIdescS = f16_idesc(128, 128, false);  // S = Q K_b^T
+constexpr uint32_t kIdescPV = f16_idesc(128, 64, true);   // O += P V_b
+
+// Bit 0 set when a wait of the attention kernel gave up (per device).
+__device__ unsigned g_attn_status;
 
 __device__ __forceinline__ int4 ld_nc16(const int8_t* p) {
     return __ldg(reinterpret_cast<const int4*>(p));
 }
 
-// Byte offset of 16-byte chunk c (bf16 elements 8c .. 8c+7) of row r in a
-// swizzled tile of 64-element bf16 rows.
-__device__ __forceinline__ uint32_t tile_off(int r, int c) {
-    return (static_cast<uint32_t>(r) << 7) | (static_cast<uint32_t>(c ^ (r & 7)) << 4);
+// Two int8 values (bytes sel of the biased word u = w ^ 0x80808080) as an
+// f16 pair, exactly: 0x64uu is the f16 1024 + uu, minus 1152 = the value.
+__device__ __forceinline__ uint32_t s8x2_f16x2(uint32_t u, uint32_t sel) {
+    const uint32_t b = __byte_perm(u, 0x64646464u, sel);
+    __half2 h;
+    memcpy(&h, &b, sizeof(h));
+    h = __hsub2(h, __half2(__ushort_as_half(0x6480u), __ushort_as_half(0x6480u)));  // 1152
+    uint32_t r;
+    memcpy(&r, &h, sizeof(r));
+    return r;
 }
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ uint32_t bf16x2(float lo, float hi) {
-    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    uint32_t u;
-    memcpy(&u, &v, sizeof(u));
-    return u;
-}
-
-// The bf16 pair of bf16x2(lo, hi) back in fp32.
-__device__ __forceinline__ float bf16_lo(uint32_t u) { return __uint_as_float(u << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
-
-// Byte k of w (w holds int8 values XOR 0x80, i.e. v + 128 as unsigned
-// bytes) as the float v: 0x4B0000uu is 2^23 + uu exactly.
-template <int k>
-__device__ __forceinline__ float widen_s8(uint32_t w) {
-    return __fsub_rn(__int_as_float(static_cast<int>(__byte_perm(w, 0x4B000000u, 0x7440u + k))), 8388736.0f);
-}
-
-// 16 int8 values (elements 16 ch .. 16 ch + 15 of row r) -> bf16 chunks
-// 2 ch and 2 ch + 1 of that row.
-__device__ __forceinline__ void store_row16(unsigned char* tile, int r, int ch, int4 v) {
+// 16 int8 values -> 8 f16 pairs, in order.
+__device__ __forceinline__ void widen16(int4 v, uint32_t (&o)[8]) {
     const uint32_t w[4] = {static_cast<uint32_t>(v.x) ^ 0x80808080u, static_cast<uint32_t>(v.y) ^ 0x80808080u,
                            static_cast<uint32_t>(v.z) ^ 0x80808080u, static_cast<uint32_t>(v.w) ^ 0x80808080u};
-    uint32_t o[8];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-        o[2 * q] = bf16x2(widen_s8<0>(w[q]), widen_s8<1>(w[q]));
-        o[2 * q + 1] = bf16x2(widen_s8<2>(w[q]), widen_s8<3>(w[q]));
+        o[2 * q] = s8x2_f16x2(w[q], 0x4140u);
+        o[2 * q + 1] = s8x2_f16x2(w[q], 0x4342u);
     }
-    *reinterpret_cast<int4*>(tile + tile_off(r, 2 * ch)) = make_int4(o[0], o[1], o[2], o[3]);
-    *reinterpret_cast<int4*>(tile + tile_off(r, 2 * ch + 1)) = make_int4(o[4], o[5], o[6], o[7]);
 }
 
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
-}
-
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
-}
-
-// d += A B for one m16n8k16 tile: A 16 x 16 (4 registers of bf16 pairs), B
-// 16 x 8 (2 registers), d 16 x 8 fp32 (rows g and g + 8, columns 2 t4 and
-// 2 t4 + 1 of lane 4 g + t4).
-__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
-                 "{%8, %9}, {%0, %1, %2, %3};\n"
-                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+// Rows 0 .. rows-1 (a multiple of 128) of one third of the head (src = its
+// row 0, rows ld bytes apart) into a swizzled f16 tile; rows >= seq are
+// zeros.  Row j, 16-byte chunk c (f16 8c .. 8c + 7) at j * 128 + (c ^ (j %
+// 8)) * 16.
+__device__ __forceinline__ void stage_rows(unsigned char* tile, const int8_t* src, int seq, int rows, int ld,
+                                           int tid) {
+    for (int u0 = 0; u0 < 4 * rows; u0 += 4 * kAttnThreads) {
+        int4 v[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int u = u0 + k * kAttnThreads + tid, j = u >> 2, ch = u & 3;
+            v[k] = j < seq ? ld_nc16(src + static_cast<long long>(j) * ld + 16 * ch) : make_int4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int u = u0 + k * kAttnThreads + tid, j = u >> 2, ch = u & 3;
+            uint32_t o[8];
+            widen16(v[k], o);
+            unsigned char* row = tile + static_cast<uint32_t>(j) * 128u;
+            *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) =
+                make_uint4(o[0], o[1], o[2], o[3]);
+            *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
+                make_uint4(o[4], o[5], o[6], o[7]);
+        }
+    }
 }
 
 __device__ __forceinline__ uint32_t pack2_s8(float v0, float v1, float inv) {
@@ -121,163 +123,221 @@ __device__ __forceinline__ uint32_t pack2_s8(float v0, float v1, float inv) {
     return d;  // q0 in byte 0, q1 in byte 1
 }
 
-__global__ void __launch_bounds__(kAttnThreads, 2)
-attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c, float vscale, int kind,
-                 float inv_out_scale, void* __restrict__ out) {
-    extern __shared__ __align__(128) unsigned char smem[];
-    const int nkb = (seq + kKeyBlock - 1) / kKeyBlock;
-    const int seq_pad = nkb * kKeyBlock;
-    unsigned char* Ks = smem;                    // [seq_pad][64] bf16
-    unsigned char* Vs = smem + 128 * seq_pad;    // [seq_pad][64] bf16
-    unsigned char* Qs = smem + 256 * seq_pad;    // [64][64] bf16
+// The f16 pair (a, b) -> u32 (a in the low half), and back.
+__device__ __forceinline__ uint32_t f16x2_bits(float a, float b) {
+    const __half2 h = __floats2half2_rn(a, b);
+    uint32_t r;
+    memcpy(&r, &h, sizeof(r));
+    return r;
+}
+__device__ __forceinline__ float2 f16x2_float2(uint32_t u) {
+    __half2 h;
+    memcpy(&h, &u, sizeof(h));
+    return __half22float2(h);
+}
 
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+// c2 = c log2(e).  skip_mma (a test hook) issues no MMA, so that every wait
+// gives up after wait_limit polls with nothing in flight.
+__global__ void __launch_bounds__(kAttnThreads, 2)
+attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c2, float vscale, int kind,
+                 float inv_out_scale, void* __restrict__ out, unsigned wait_limit, int skip_mma) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* sm =
+        reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const int nkb = (seq + kKeyBlock - 1) / kKeyBlock;
+    unsigned char* Ks = sm;                                  // [nkb * 128][64] f16, swizzled
+    unsigned char* Vs = sm + nkb * kBlockBytes;              // [nkb * 128][64] f16, swizzled
+    unsigned char* misc = sm + 2 * nkb * kBlockBytes;
+    const uint32_t bar_s = smem_addr(misc);                  // S_b complete
+    const uint32_t bar_o = bar_s + 8;                        // P_b V_b complete
+    const int tid = threadIdx.x, warp = tid >> 5;
     const int q0 = blockIdx.x * kAttnQ;
     const int h = blockIdx.y;
     const long long row0 = static_cast<long long>(blockIdx.z) * seq;  // first token row of the sequence
     const int8_t* head = qkv + row0 * ld + h * 64;
 
-    // 1. Queries, keys and values of the head -> bf16 tiles (rows past the
-    //    sequence are zeros).
-    const int4 zero = make_int4(0, 0, 0, 0);
-    for (int u = tid; u < 4 * kAttnQ; u += kAttnThreads) {
-        const int i = u >> 2, ch = u & 3;
-        const int4 v = q0 + i < seq ? ld_nc16(head + static_cast<long long>(q0 + i) * ld + 16 * ch) : zero;
-        store_row16(Qs, i, ch, v);
-    }
-    for (int u = tid; u < 4 * seq_pad; u += kAttnThreads) {
-        const int j = u >> 2, ch = u & 3;
-        int4 kv = zero, vv = zero;
-        if (j < seq) {
-            const int8_t* row = head + static_cast<long long>(j) * ld + 16 * ch;
-            kv = ld_nc16(row + d);
-            vv = ld_nc16(row + 2 * d);
-        }
-        store_row16(Ks, j, ch, kv);
-        store_row16(Vs, j, ch, vv);
-    }
+    if (tid == 0) mbar_init_n(bar_s, 2);
+    __syncwarp();
+    if (warp == 0) tmem_alloc(bar_s + 16, kTmemCols);
+    stage_rows(Ks, head + d, seq, nkb * kKeyBlock, ld, tid);
+    fence_proxy_async();
+    tc_fence_before();
     __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = *reinterpret_cast<volatile uint32_t*>(misc + 16);
+    const uint32_t lane = tm + (static_cast<uint32_t>(32 * warp) << 16);  // this warp's quarter of the lanes
 
-    // 2. The warp's 16 queries as A fragments (4 chunks of 16 channels).
-    uint32_t qa[4][4];
+    // The thread's query as f16 pairs into its lane.
     {
-        const int r = 16 * warp + (lane & 7) + 8 * ((lane >> 3) & 1);
+        const int q = q0 + tid;
+        uint32_t v[32];
 #pragma unroll
-        for (int kc = 0; kc < 4; ++kc)
-            ldsm_x4(smem_u32(Qs + tile_off(r, 2 * kc + (lane >> 4))), qa[kc][0], qa[kc][1], qa[kc][2], qa[kc][3]);
+        for (int k = 0; k < 4; ++k) {
+            const int4 x = q < seq ? ld_nc16(head + static_cast<long long>(q) * ld + 16 * k) : make_int4(0, 0, 0, 0);
+            uint32_t o[8];
+            widen16(x, o);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[8 * k + i] = o[i];
+        }
+        tmem_st32(lane + kColQ, v);
+        tmem_wait_st();
     }
-    const int t4 = lane & 3;
-    float o[8][4];
-#pragma unroll
-    for (int n = 0; n < 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.0f;
-    float m0 = -INFINITY, m1 = -INFINITY;  // running maxima of rows g and g + 8
-    float l0 = 0.0f, l1 = 0.0f;            // this lane's part of the running sums
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
 
-    for (int kb = 0; kb < nkb; ++kb) {
-        const int key0 = kb * kKeyBlock;
-        // scores of keys key0 + 8 nt .. + 7
-        float s[8][4];
+    const uint32_t ks = smem_addr(Ks), vs = smem_addr(Vs);
+    auto issue_s = [&](int b) {
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.0f;
+        for (int t = 0; t < 4; ++t)
+            mma_f16_ts(tm + kColS, tm + kColQ + 8 * t, sw128_desc(ks + b * kBlockBytes + 32 * t, 16, 1024), kIdescS,
+                       t > 0);
+        tc_commit(bar_s);
+    };
+    if (tid == 0 && !skip_mma) issue_s(0);
+    // The values land while the first scores are computed; they are visible
+    // to the MMAs after the block's barrier below.
+    stage_rows(Vs, head + 2 * d, seq, nkb * kKeyBlock, ld, tid);
+    fence_proxy_async();
+
+    float m = -INFINITY;  // running maximum of the exact dot products
+    float l = 0.0f;       // running sum of the weights
+    bool ok = true;
+    for (int b = 0; b < nkb; ++b) {
+        ok &= mbar_wait(bar_s, b & 1, wait_limit);
+        __syncwarp();
+        tc_fence_after();
+        float s[kKeyBlock];
+        {
+            uint32_t r[4][32];
 #pragma unroll
-            for (int kcp = 0; kcp < 2; ++kcp) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4(smem_u32(Ks + tile_off(key0 + 8 * nt + (lane & 7), 4 * kcp + (lane >> 3))), b0, b1, b2, b3);
-                mma_bf16(s[nt], qa[2 * kcp], b0, b1);
-                mma_bf16(s[nt], qa[2 * kcp + 1], b2, b3);
+            for (int k = 0; k < 4; ++k) tmem_ld32(lane + kColS + 32 * k, r[k]);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) tmem_wait_ld(r[k]);
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s[32 * k + i] = __uint_as_float(r[k][i]);
+        }
+        const int valid = seq - b * kKeyBlock;  // keys of the block inside the sequence, >= 1
+        if (valid < kKeyBlock) {
+#pragma unroll
+            for (int j = 0; j < kKeyBlock; ++j)
+                if (j >= valid) s[j] = -INFINITY;
+        }
+        float bm = s[0];
+#pragma unroll
+        for (int j = 1; j < kKeyBlock; ++j) bm = fmaxf(bm, s[j]);
+        const float mn = fmaxf(m, bm);  // finite: the block has a key
+        // A larger maximum scales the context and the sum by the same
+        // factor (1 for the lanes whose maximum did not move); tensor-memory
+        // loads and stores are warp-wide, so the whole warp takes the branch.
+        if (b > 0 && __any_sync(0xffffffffu, mn > m)) {
+            const float alpha = exp2f(__fmul_rn(__fsub_rn(m, mn), c2));
+            l = __fmul_rn(l, alpha);
+            uint32_t o[2][32];
+            tmem_ld32(lane + kColO, o[0]);
+            tmem_ld32(lane + kColO + 32, o[1]);
+            tmem_wait_ld(o[0]);
+            tmem_wait_ld(o[1]);
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+#pragma unroll
+                for (int i = 0; i < 32; ++i) o[k][i] = __float_as_uint(__fmul_rn(__uint_as_float(o[k][i]), alpha));
+            tmem_st32(lane + kColO, o[0]);
+            tmem_st32(lane + kColO + 32, o[1]);
+        }
+        m = mn;
+        // Weights of keys 32 cc .. 32 cc + 31: high f16 parts into columns
+        // 32 cc .. + 15, low parts into 32 cc + 16 .. + 31 (over the scores).
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+            uint32_t p[32];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const float e0 = exp2f(__fmul_rn(__fsub_rn(s[32 * cc + 2 * e], m), c2));
+                const float e1 = exp2f(__fmul_rn(__fsub_rn(s[32 * cc + 2 * e + 1], m), c2));
+                l = __fadd_rn(__fadd_rn(l, e0), e1);
+                const uint32_t hi = f16x2_bits(e0, e1);
+                const float2 hf = f16x2_float2(hi);
+                p[e] = hi;
+                p[16 + e] = f16x2_bits(__fsub_rn(e0, hf.x), __fsub_rn(e1, hf.y));
+            }
+            tmem_st32(lane + kColS + 32 * cc, p);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !skip_mma) {
+            tc_fence_after();
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {  // keys 16 t .. 16 t + 15 of the block
+                const uint64_t bd = sw128_desc(vs + b * kBlockBytes + 2048 * t, 1024, 1024);
+                const uint32_t a = tm + kColS + 32 * (t >> 1) + 8 * (t & 1);
+                mma_f16_ts(tm + kColO, a, bd, kIdescPV, (b > 0 || t > 0) ? 1u : 0u);
+                mma_f16_ts(tm + kColO, a + 16, bd, kIdescPV, 1u);
+            }
+            tc_commit(bar_o);
+            if (b + 1 < nkb) {  // the next scores overwrite P_b: wait until it is consumed
+                ok &= mbar_wait(bar_o, b & 1, wait_limit);
+                tc_fence_after();
+                issue_s(b + 1);
             }
         }
-        float bm0 = -INFINITY, bm1 = -INFINITY;
+    }
+
+    // Context row: O / l * qkv_scale.
+    ok &= mbar_wait(bar_o, (nkb - 1) & 1, wait_limit);
+    __syncwarp();
+    tc_fence_after();
+    uint32_t o[2][32];
+    tmem_ld32(lane + kColO, o[0]);
+    tmem_ld32(lane + kColO + 32, o[1]);
+    tmem_wait_ld(o[0]);
+    tmem_wait_ld(o[1]);
+    const int r = q0 + tid;
+    if (r < seq) {
+        const float f = __fdiv_rn(vscale, l);
+        const long long base = (row0 + r) * d + h * 64;
+        if (kind == 3) {
+            uint4* dst = reinterpret_cast<uint4*>(static_cast<int8_t*>(out) + base);
 #pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
+            for (int k = 0; k < 4; ++k) {
+                uint32_t w[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int key = key0 + 8 * nt + 2 * t4 + (e & 1);
-                s[nt][e] = key < seq ? __fmul_rn(s[nt][e], c) : -INFINITY;
-            }
-            bm0 = fmaxf(bm0, fmaxf(s[nt][0], s[nt][1]));
-            bm1 = fmaxf(bm1, fmaxf(s[nt][2], s[nt][3]));
-        }
-        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 1));
-        bm0 = fmaxf(bm0, __shfl_xor_sync(0xffffffffu, bm0, 2));
-        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 1));
-        bm1 = fmaxf(bm1, __shfl_xor_sync(0xffffffffu, bm1, 2));
-        const float mn0 = fmaxf(m0, bm0), mn1 = fmaxf(m1, bm1);  // finite: key0 < seq
-        const float a0 = expf(__fsub_rn(m0, mn0)), a1 = expf(__fsub_rn(m1, mn1));  // 0 in the first block
-        m0 = mn0;
-        m1 = mn1;
-        l0 = __fmul_rn(l0, a0);
-        l1 = __fmul_rn(l1, a1);
-#pragma unroll
-        for (int n = 0; n < 8; ++n) {
-            o[n][0] = __fmul_rn(o[n][0], a0), o[n][1] = __fmul_rn(o[n][1], a0);
-            o[n][2] = __fmul_rn(o[n][2], a1), o[n][3] = __fmul_rn(o[n][3], a1);
-        }
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            s[nt][0] = expf(__fsub_rn(s[nt][0], mn0)), s[nt][1] = expf(__fsub_rn(s[nt][1], mn0));
-            s[nt][2] = expf(__fsub_rn(s[nt][2], mn1)), s[nt][3] = expf(__fsub_rn(s[nt][3], mn1));
-            l0 = __fadd_rn(l0, __fadd_rn(s[nt][0], s[nt][1]));
-            l1 = __fadd_rn(l1, __fadd_rn(s[nt][2], s[nt][3]));
-        }
-        // context += P v, 32 keys (two k-chunks of 16) per transposed ldmatrix
-#pragma unroll
-        for (int kkp = 0; kkp < 2; ++kkp) {
-            uint32_t hi[2][4], lo[2][4];
-#pragma unroll
-            for (int x = 0; x < 2; ++x) {
-                const int nt = 2 * (2 * kkp + x);
-                const float* p[4] = {&s[nt][0], &s[nt][2], &s[nt + 1][0], &s[nt + 1][2]};
-#pragma unroll
-                for (int r = 0; r < 4; ++r) {
-                    hi[x][r] = bf16x2(p[r][0], p[r][1]);
-                    lo[x][r] = bf16x2(__fsub_rn(p[r][0], bf16_lo(hi[x][r])), __fsub_rn(p[r][1], bf16_hi(hi[x][r])));
+                for (int i = 0; i < 4; ++i) {
+                    const int j = 16 * k + 4 * i;
+                    const float y0 = __fmul_rn(__uint_as_float(o[j >> 5][j & 31]), f);
+                    const float y1 = __fmul_rn(__uint_as_float(o[(j + 1) >> 5][(j + 1) & 31]), f);
+                    const float y2 = __fmul_rn(__uint_as_float(o[(j + 2) >> 5][(j + 2) & 31]), f);
+                    const float y3 = __fmul_rn(__uint_as_float(o[(j + 3) >> 5][(j + 3) & 31]), f);
+                    w[i] = pack2_s8(y0, y1, inv_out_scale) | (pack2_s8(y2, y3, inv_out_scale) << 16);
                 }
+                dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
             }
+        } else {
+            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + base);
 #pragma unroll
-            for (int n = 0; n < 8; ++n) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4_t(smem_u32(Vs + tile_off(key0 + 32 * kkp + 8 * (lane >> 3) + (lane & 7), n)), b0, b1, b2, b3);
-                mma_bf16(o[n], hi[0], b0, b1);
-                mma_bf16(o[n], lo[0], b0, b1);
-                mma_bf16(o[n], hi[1], b2, b3);
-                mma_bf16(o[n], lo[1], b2, b3);
-            }
-        }
-    }
-
-    // 3. Row sums over the quad, scale, store rows g and g + 8.
-    l0 = __fadd_rn(l0, __shfl_xor_sync(0xffffffffu, l0, 1));
-    l0 = __fadd_rn(l0, __shfl_xor_sync(0xffffffffu, l0, 2));
-    l1 = __fadd_rn(l1, __shfl_xor_sync(0xffffffffu, l1, 1));
-    l1 = __fadd_rn(l1, __shfl_xor_sync(0xffffffffu, l1, 2));
-    const float f0 = __fdiv_rn(vscale, l0), f1 = __fdiv_rn(vscale, l1);
-    const int ra = q0 + 16 * warp + (lane >> 2);
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-        const int r = ra + 8 * half;
-        if (r >= seq) continue;
-        const float f = half ? f1 : f0;
-        const long long base = (row0 + r) * d + h * 64 + 2 * t4;
-#pragma unroll
-        for (int n = 0; n < 8; ++n) {
-            const float y0 = __fmul_rn(o[n][2 * half], f), y1 = __fmul_rn(o[n][2 * half + 1], f);
-            if (kind == 3) {
-                *reinterpret_cast<uint16_t*>(static_cast<int8_t*>(out) + base + 8 * n) =
-                    static_cast<uint16_t>(pack2_s8(y0, y1, inv_out_scale));
-            } else {
-                *reinterpret_cast<float2*>(static_cast<float*>(out) + base + 8 * n) = make_float2(y0, y1);
+            for (int k = 0; k < 16; ++k) {
+                const int j = 4 * k;
+                dst[k] = make_float4(__fmul_rn(__uint_as_float(o[j >> 5][j & 31]), f),
+                                     __fmul_rn(__uint_as_float(o[(j + 1) >> 5][(j + 1) & 31]), f),
+                                     __fmul_rn(__uint_as_float(o[(j + 2) >> 5][(j + 2) & 31]), f),
+                                     __fmul_rn(__uint_as_float(o[(j + 3) >> 5][(j + 3) & 31]), f));
             }
         }
     }
+    if (!ok) atomicOr(&g_attn_status, static_cast<unsigned>(kStatusTimeout));
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tm, kTmemCols);
 }
 
 }  // namespace
 
 size_t attention_smem_bytes(int seq) {
-    const size_t seq_pad = (static_cast<size_t>(seq) + kKeyBlock - 1) / kKeyBlock * kKeyBlock;
-    return 256 * seq_pad + 128 * kAttnQ;  // keys and values, queries: bf16 rows of 64
+    const size_t nkb = (static_cast<size_t>(seq) + kKeyBlock - 1) / kKeyBlock;
+    return 2 * nkb * kBlockBytes + 1024 + 64;  // K and V tiles, 1024-byte alignment, barriers + TMEM address
 }
 
 cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, int ld, float score_scale,
@@ -298,11 +358,22 @@ cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, i
             ready[dev] = true;
         }
     }
+    const float c2 = static_cast<float>(static_cast<double>(score_scale) * 1.4426950408889634);  // c log2(e)
+    const bool skip = (test_hooks() & BSGEMM_TEST_ATTN_SKIP_MMA) != 0;
     const dim3 grid(static_cast<unsigned>((seq + kAttnQ - 1) / kAttnQ), static_cast<unsigned>(heads),
                     static_cast<unsigned>(batch));
-    attention_kernel<<<grid, kAttnThreads, attention_smem_bytes(seq), s>>>(qkv, seq, heads * 64, ld, score_scale,
-                                                                         qkv_scale, kind, inv_out_scale, out);
+    attention_kernel<<<grid, kAttnThreads, attention_smem_bytes(seq), s>>>(
+        qkv, seq, heads * 64, ld, c2, qkv_scale, kind, inv_out_scale, out, skip ? 64u : kWaitLimit, skip ? 1 : 0);
     return cudaGetLastError();
+}
+
+cudaError_t attention_status(bool clear, unsigned* v) {
+    cudaError_t e = cudaMemcpyFromSymbol(v, g_attn_status, sizeof(unsigned));
+    if (e == cudaSuccess && clear && *v != 0) {
+        const unsigned zero = 0;
+        e = cudaMemcpyToSymbol(g_attn_status, &zero, sizeof(unsigned));
+    }
+    return e;
 }
 
 }  // namespace bsg

@@ -117,6 +117,9 @@ cudaError_t launch_layernorm(const float* z, int M, int N, const float* gamma, c
 size_t attention_smem_bytes(int seq);
 cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, int ld, float score_scale,
                              float qkv_scale, int kind, float inv_out_scale, void* out, cudaStream_t s);
+// The current device's attention status word (bit 0: a wait gave up),
+// reset to 0 when clear is set and it was not.
+cudaError_t attention_status(bool clear, unsigned* v);
 // x [M][K] -> swizzled token tiles in xb (the layout the kernel stages by TMA).
 cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, cudaStream_t s);
 // Average-magnitude block pruning of a dense fp32 W [N][K] (DEVICE) into

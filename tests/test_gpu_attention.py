@@ -1,20 +1,28 @@
 """Multi-head self-attention on device (bsgemm_attention) against the fp64
 oracle (oracle.attention_f64).
 
-Tolerance, derived from the kernel's arithmetic.  The scores are exact
-int32 dot products (bf16 tensor-core products of int8 values, partial sums
-below 2^24) times c = fl(qkv_scale^2 / 8), so each s_j carries a relative
-error of at most 2^-23; s_j - max s adds 2^-24 of |s_j - max s| and expf at
-most 2 ulp, so each weight e_j is within 2^-21 (S + 1) of its exact value
-(S = the largest |s_j|).  P enters the P v product as two bf16 parts, which
-drops at most 2^-16 of each weight.  The sums over the seq keys (of e_j in
-fp32 adds; of e_j v_j in the tensor cores' fp32 accumulation, counted with
-truncating adds) add at most seq 2^-24 and seq 2^-23 relative to their sums
-of magnitudes; the online softmax rescales the context and the sum by the
-same factors (one rounding each per block of 64 keys), and the final scale
-and product add 2 ulp.  In units of vmax = max |v| * qkv_scale that is at
-most
-    (3 seq 2^-24 + 2^-16 + 2^-21 (S + 1) + (2 ceil(seq / 64) + 4) 2^-24) vmax
+Tolerance, derived from the kernel's arithmetic (fifth-generation tensor
+cores, f16 operands, fp32 accumulators).  The scores are exact int32 dot
+products (int8 values are exact in f16, products below 2^14, partial sums
+of 64 below 2^24).  A weight is e_j = exp2f(fl((d_j - m) c2)) with d_j - m
+an exact difference of dot products and c2 = c log2(e) within 2^-23 of its
+exact value (c rounded once to fp32, the product once), so the exponent
+t_j is within 2^-22.4 |t_j| of the exact one; 2^t |t| ln 2 <= 1/e bounds
+the resulting error of a weight by 2^-23.8 absolute (the largest weight
+being 1), and exp2f adds 2 ulp (2^-22) relative.  The online softmax over
+blocks of 128 keys rescales the context and the sum by the same factor
+alpha (its exponent error is already counted, since the exponents add; its
+2 ulp and the two products add (2^-22 + 2^-24) per rescale, R =
+ceil(seq / 128) - 1 of them).  P enters the P v product as two f16 parts
+(hi + lo), which drops at most 2^-22 e + 2^-25 of each weight; the
+products with the exact f16 v are exact.  The sums of e_j (fp32, one add a
+key) and of e_j v_j (the tensor cores' fp32 accumulation, two products a
+key, counted as truncating adds) add at most seq_pad 2^-24 and 2 seq_pad
+2^-23 relative to their sums of magnitudes (seq_pad = 128 (R + 1)); the
+final scale and product add 2^-23.  A weight's error enters the numerator
+and the sum, so it counts twice.  In units of vmax = max |v| * qkv_scale
+that is at most
+    ((6 + 2 R) 2^-22 + 2 R 2^-24 + seq 2^-22.4 + 5 seq_pad 2^-24 + 2^-23) vmax
 per element.  A dropped or repeated key (weight ~ 1 / seq), a wrong scale
 or head offset moves an element by orders of magnitude more.  int8 outputs
 must equal rne(exact * inv) saturated, except within that bound (times inv)
@@ -51,16 +59,11 @@ def draw_qkv(rng, batch, seq, heads, pad=0, std=35.0):
 
 def bound(qkv, scale, batch, seq, heads):
     d = heads * HD
-    x = qkv[:, :3 * d].astype(np.int64)
-    smax = 0.0
-    for b in range(batch):
-        rows = slice(b * seq, (b + 1) * seq)
-        for h in range(heads):
-            qh = x[rows, h * HD:(h + 1) * HD]
-            kh = x[rows, d + h * HD:d + (h + 1) * HD]
-            smax = max(smax, float(np.abs(qh @ kh.T).max()) * scale * scale / 8.0)
-    vmax = float(np.abs(x[:, 2 * d:3 * d]).max()) * scale
-    return (3 * seq * 2.0 ** -24 + 2.0 ** -16 + 2.0 ** -21 * (smax + 1) + (2 * -(-seq // 64) + 4) * 2.0 ** -24) * vmax
+    vmax = float(np.abs(qkv[:, 2 * d:3 * d].astype(np.int64)).max()) * scale
+    r = -(-seq // 128) - 1
+    seq_pad = 128 * (r + 1)
+    return ((6 + 2 * r) * 2.0 ** -22 + 2 * r * 2.0 ** -24 + seq * 2.0 ** -22.4 + 5 * seq_pad * 2.0 ** -24
+            + 2.0 ** -23) * vmax
 
 
 def run_device(bsg, qkv, batch, seq, heads, scale, kind=None, out_scale=1.0, guard_rows=0, stream=None):
@@ -81,7 +84,8 @@ def run_device(bsg, qkv, batch, seq, heads, scale, kind=None, out_scale=1.0, gua
 
 @pytest.mark.parametrize("batch,seq,heads,pad,scale", [
     (1, 1, 1, 0, 0.05), (2, 5, 2, 16, 0.05), (1, 64, 12, 0, 0.05), (3, 65, 4, 0, 0.08),
-    (2, 130, 3, 48, 0.02), (1, 512, 2, 0, 0.05), (2, 384, 12, 0, 0.12)])
+    (2, 130, 3, 48, 0.02), (1, 512, 2, 0, 0.05), (2, 384, 12, 0, 0.12), (1, 128, 2, 0, 0.05),
+    (1, 129, 2, 0, 0.05), (2, 257, 1, 16, 0.05), (1, 383, 2, 0, 0.1), (1, 511, 1, 0, 0.05)])
 def test_attention_f32_parity(bsg, batch, seq, heads, pad, scale):
     rng = np.random.default_rng(7000 + 7 * seq + heads)
     qkv = draw_qkv(rng, batch, seq, heads, pad)
@@ -150,3 +154,21 @@ def test_attention_checks_on_device(bsg):
     out = bsg.attention(qkv, 2, 8, 1, 0.05)                    # all zero: the context is 0
     torch.cuda.synchronize()
     assert out.abs().max().item() == 0.0
+
+
+@pytest.mark.parametrize("order", ["rising", "falling"])
+def test_attention_running_maximum(bsg, order):
+    """Scores that rise from key to key make every block of 128 keys raise
+    the running maximum (the context and the sum are rescaled at each
+    block); falling scores never do.  Both against the oracle."""
+    seq, heads, scale = 500, 2, 0.02
+    d = heads * HD
+    rng = np.random.default_rng(7300)
+    ramp = np.rint(np.linspace(-127, 127, seq)).astype(np.int64)
+    if order == "falling":
+        ramp = ramp[::-1]
+    k = np.repeat(ramp[:, None], d, axis=1)
+    qkv = np.concatenate([np.full((seq, d), 60), k, rng.integers(-127, 128, size=(seq, d))], axis=1).astype(np.int8)
+    got = run_device(bsg, qkv, 1, seq, heads, scale)
+    want = oracle.attention_f64(qkv, scale, 1, seq, heads=heads, head_dim=HD)
+    assert np.abs(got.astype(np.float64) - want).max() <= bound(qkv, scale, 1, seq, heads)

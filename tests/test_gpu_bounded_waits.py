@@ -5,7 +5,8 @@ The test hooks (bsgemm_set_test_hooks) make the waits run out on purpose:
 the layer kernel issues no tile copy (so no copy is in flight when its CTAs
 leave) and polls its copy barriers 64 times; the pruning kernel's CTA 0
 leaves before the first grid barrier, which the other CTAs give up after
-4096 polls.  Each call must return, report the failure, and leave the
+4096 polls; the attention kernel issues no tensor-core MMA and polls the
+mbarriers its MMAs would complete 64 times.  Each call must return, report the failure, and leave the
 context usable: a normal run right after matches the oracle.
 """
 import os
@@ -97,3 +98,23 @@ def test_prune_grid_barrier_gives_up_and_the_call_fails(bsg, hooks):
     keep = bsg.block_prune(wd, 0.9)
     torch.cuda.synchronize()
     assert np.array_equal(keep.cpu().numpy().astype(bool), oracle.block_prune(w, 0.9))
+
+
+def test_attention_mma_wait_gives_up_and_reports_timeout(bsg, hooks):
+    from test_gpu_attention import HD, bound, draw_qkv
+    batch, seq, heads, scale = 2, 300, 3, 0.05
+    qkv = draw_qkv(np.random.default_rng(6403), batch, seq, heads)
+    qd = torch.from_numpy(qkv).cuda()
+    out = torch.zeros((batch * seq, heads * HD), dtype=torch.float32, device="cuda")
+    assert bsg.bsgemm_attention_status(clear=True) in (0, bsg.STATUS_TIMEOUT)
+    hooks(bsg.TEST_ATTN_SKIP_MMA)
+    bsg.attention(qd, batch, seq, heads, scale, out=out)  # returns: the waits are bounded
+    torch.cuda.synchronize()
+    hooks(0)
+    assert bsg.bsgemm_attention_status(clear=True) == bsg.STATUS_TIMEOUT
+    assert bsg.bsgemm_attention_status() == 0
+    bsg.attention(qd, batch, seq, heads, scale, out=out)
+    torch.cuda.synchronize()
+    want = oracle.attention_f64(qkv, scale, batch, seq, heads=heads, head_dim=HD, threads=2)
+    assert np.abs(out.cpu().numpy().astype(np.float64) - want).max() <= bound(qkv, scale, batch, seq, heads)
+    assert bsg.bsgemm_attention_status() == 0
