@@ -11,7 +11,7 @@ def test_attention_floors_follow_their_definitions():
     product.  Tensor floor = 6 x that many flops at the given bf16 rate,
     exp floor = one exponential per score at 16 per SM per clock, HBM floor
     = the int8 QKV rows once; the largest one is the bound."""
-    r = bench.attention_roofline(8, 384, 12, 0.0316, 152, 2070.0, 6783.5, 1903.9)
+    r = bench.attention_roofline(8, 384, 12, 0.0155, 152, 2070.0, 6783.5, 1903.9)
     macs = 8 * 12 * 384 * 384 * 64
     assert macs == 905_969_664
     assert r["ops"] == 4 * macs
@@ -19,10 +19,10 @@ def test_attention_floors_follow_their_definitions():
     assert abs(r["floors_us"]["exp"] - 8 * 12 * 384 * 384 / (152 * 16 * 2070e6) * 1e6) < 1e-3
     assert abs(r["floors_us"]["hbm"] - 8 * 384 * 2304 / 6783.5e9 * 1e6) < 1e-3
     assert r["bound"] == "tensor" and r["floor"] == "tensor"
-    assert abs(r["frac"] - r["floors_us"]["tensor"] / 31.6) < 1e-3
-    assert abs(r["mma_sync_floor_us"] - 6 * macs / 594e12 * 1e6) < 1e-3
+    assert abs(r["frac"] - r["floors_us"]["tensor"] / 15.5) < 1e-3
+    assert "mma_sync_floor_us" not in r  # the kernel runs on tcgen05, whose rate is the measured one
     # a slow exponential unit makes exp the bound
-    r = bench.attention_roofline(8, 384, 12, 0.0316, 1, 2070.0, 6783.5, 1903.9)
+    r = bench.attention_roofline(8, 384, 12, 0.0155, 1, 2070.0, 6783.5, 1903.9)
     assert r["bound"] == "alu" and r["floor"] == "exp"
 
 
