@@ -952,7 +952,7 @@ def run_layer(args) -> dict:
     }
 
 
-SFU_EX2_PER_SM_CLK = 16        # exponentials per SM per clock (special-function unit)
+SFU_EX2_PER_SM_CLK = 32        # ex2.approx per SM per clock on GB300, measured (31.97)
 
 
 def attention_roofline(batch: int, seq: int, heads: int, ms: float, sms: int, max_mhz: float, hbm_gbs: float,
@@ -977,8 +977,8 @@ def attention_roofline(batch: int, seq: int, heads: int, ms: float, sms: int, ma
             "peak": bf16_tflops, "frac": round(floors[name] / t, 4),
             "basis": "graph of 200 launches, per launch; ops = 2 x (q k^T + P v) multiply-adds; floors: tensor = "
                      "6 x MACs (P v twice: two f16 parts) at the measured dense bf16 rate (MEASURED_PEAKS, burst; "
-                     "tcgen05.mma kind::f16), exp = one SFU exponential per score (16 per SM per clock at the max "
-                     "SM clock), hbm = QKV bytes at the measured copy rate"}
+                     "tcgen05.mma kind::f16), exp = one SFU exponential per score (32 per SM per clock at the max "
+                     "SM clock, measured), hbm = QKV bytes at the measured copy rate"}
 
 
 def run_encoder(args) -> dict:

@@ -15,25 +15,46 @@
 //     the fp32 accumulator holds the int32 dot product;
 //   * P v takes each weight in two f16 parts (e = hi + lo + r, |r| <= 2^-22
 //     e + 2^-25) against the exact f16 v, two MMAs per K step.
-// The softmax runs online over blocks of 128 keys in fp32: a thread keeps
-// its query's running maximum m of the exact dot products and its running
-// sum l; e_j = 2^((d_j - m) c log2(e)) with d_j - m exact, so the only
-// roundings inside the exponent are those of c log2(e) and of one product.
-// When m grows, the context and l are scaled by the same factor.
+// The softmax runs online over blocks of 64 keys in fp32.  A thread's
+// weights are e_j = 2^fl(d_j c2 - M) (one fused multiply-add; c2 = c
+// log2(e), d_j the exact dot product) against a reference M = fl(m c2) of a
+// maximum m of the dot products seen so far.  M moves only when a block's
+// maximum exceeds it by more than 8 (log2 units), so the weights stay below
+// 2^8 and rescaling is rare; when it moves, the context and the running sum
+// are scaled by the same 2^(M_old - M_new), the difference taken exactly.
+// The rounding of M thus scales every weight by one factor that the context
+// and the sum share, and the exponent carries only the roundings of c2 and
+// of the fused product.
 //
-// One CTA = 128 queries of one (sequence, head), 4 warps; thread i owns
-// query i = tensor-memory lane i.  Tensor memory (256 columns, so two CTAs
-// share an SM): S/P in columns 0-127 (the block's scores, then its weights
-// written back in place as f16 pairs: for keys 32c .. 32c + 31 the high
-// parts in columns 32c .. 32c + 15, the low parts in 32c + 16 .. 32c + 31),
-// the context O in 128-191, the CTA's queries (f16 pairs) in 192-223.  The
-// head's keys and values (seq <= BSGEMM_ATTN_MAX_SEQ, padded with zeros to
-// whole blocks) are staged once into shared memory as f16 rows of 64 with
-// the 128-byte swizzle: K is the K-major B operand of q k^T, V the MN-major
-// B operand of P v.  Per block one thread issues the 4 MMAs of S = Q K_b^T
-// (N = 128, K = 64) and, after the threads have written P, the 16 of O +=
-// P_hi V_b + P_lo V_b (N = 64, K = 128); completions arrive on two
-// mbarriers, every wait bounded.
+// One CTA = 128 queries of one (sequence, head): 8 compute warps and one
+// MMA warp.  Compute warps w and w + 4 share the 32 queries of tensor-memory
+// lane quarter w (thread i % 128 owns query i = lane i): each takes 32 of a
+// block's 64 keys and 32 of the context's 64 columns, and the two exchange
+// their block maxima through shared memory.  Tensor memory (256 columns, so
+// two CTAs share an SM): two score buffers in columns 0-63 and 64-127 (block
+// b uses buffer b % 2: its scores, then its weights written back in place as
+// f16 pairs -- for keys 32c .. 32c + 31 of the block the high parts in
+// columns 32c .. + 15 of the buffer, the low parts in 32c + 16 .. + 31), the
+// context O in 128-191, the CTA's queries (f16 pairs) in 192-223, the row
+// sums in 224-239 (P times a 64 x 16 matrix of ones: the tensor cores add
+// the same f16 weights into the sum as into the context).  The head's keys
+// and values (seq <= BSGEMM_ATTN_MAX_SEQ, padded with zeros to whole blocks)
+// are staged once into shared memory as f16 rows of 64 with the 128-byte
+// swizzle: K is the K-major B operand of q k^T, V the MN-major B operand of
+// P v.
+//
+// One thread of the MMA warp issues S_0 and S_1 (S_b = Q K_b^T: N = 64, K =
+// 64), then per block b: waits until the compute threads have written P_b,
+// issues O += P_b,hi V_b + P_b,lo V_b and L += P_b,hi 1 + P_b,lo 1 (16
+// MMAs), and once they have completed
+// issues S_(b+2) into the freed buffer.  So the compute warps work on block
+// b + 1 while the tensor cores consume block b, and never wait for the
+// tensor cores except where the running maximum grows (a rescale of O needs
+// the previous block's P v complete).  mbarriers, two of each kind (one per
+// buffer, so that no wait can fall two phases behind): S_b complete, P_b
+// written (256 arrivals), P_b V_b complete; and one for the queries written
+// to tensor memory (128 arrivals).  Every wait is bounded.
+
 #include <cfloat>
 #include <cmath>
 #include <cstdint>
@@ -50,14 +71,18 @@
 namespace bsg {
 namespace {
 
-constexpr int kAttnThreads = 128;     // 4 warps, one query (TMEM lane) each
+constexpr int kCompute = 256;         // 8 compute warps, two per query (TMEM lane)
+constexpr int kAttnThreads = kCompute + 32;  // + the MMA warp
 constexpr int kAttnQ = 128;           // queries per CTA
-constexpr int kKeyBlock = 128;        // keys per online-softmax block
-constexpr uint32_t kBlockBytes = 16384;  // 128 rows x 64 f16
+constexpr int kKeyBlock = 64;         // keys per online-softmax block
+constexpr uint32_t kBlockBytes = 8192;   // 64 rows x 64 f16
+constexpr int kMaxRows = (BSGEMM_ATTN_MAX_SEQ + kKeyBlock - 1) / kKeyBlock * kKeyBlock;
+constexpr int kMaxLoads = (4 * kMaxRows + kCompute - 1) / kCompute;  // 16-byte loads of K (or V) per thread
 constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS = 0, kColO = 128, kColQ = 192;
-constexpr uint32_t kIdescS = f16_idesc(128, 128, false);  // S = Q K_b^T
-constexpr uint32_t kIdescPV = f16_idesc(128, 64, true);   // O += P V_b
+constexpr uint32_t kColS = 0, kColO = 128, kColQ = 192;  // score buffers at kColS and kColS + 64
+constexpr uint32_t kIdescS = f16_idesc(128, 64, false);  // S = Q K_b^T
+constexpr uint32_t kIdescPV = f16_idesc(128, 64, true);  // O += P V_b
+constexpr float kLazy = 8.0f;  // largest weight 2^kLazy: the reference maximum moves past that
 
 // Bit 0 set when a wait of the attention kernel gave up (per device).
 __device__ unsigned g_attn_status;
@@ -89,31 +114,35 @@ __device__ __forceinline__ void widen16(int4 v, uint32_t (&o)[8]) {
     }
 }
 
-// Rows 0 .. rows-1 (a multiple of 128) of one third of the head (src = its
-// row 0, rows ld bytes apart) into a swizzled f16 tile; rows >= seq are
-// zeros.  Row j, 16-byte chunk c (f16 8c .. 8c + 7) at j * 128 + (c ^ (j %
-// 8)) * 16.
-__device__ __forceinline__ void stage_rows(unsigned char* tile, const int8_t* src, int seq, int rows, int ld,
-                                           int tid) {
-    for (int u0 = 0; u0 < 4 * rows; u0 += 4 * kAttnThreads) {
-        int4 v[4];
+// The 16-byte loads of one third of the head (src = its row 0, rows ld
+// bytes apart): load i of thread t is row j = (128 i + t) / 4, 16-byte chunk
+// (128 i + t) % 4; zeros past the sequence.  All issued before any is used.
+__device__ __forceinline__ void load_rows(int4 (&v)[kMaxLoads], const int8_t* src, int seq, int ld, int tid) {
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int u = u0 + k * kAttnThreads + tid, j = u >> 2, ch = u & 3;
-            v[k] = j < seq ? ld_nc16(src + static_cast<long long>(j) * ld + 16 * ch) : make_int4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int u = u0 + k * kAttnThreads + tid, j = u >> 2, ch = u & 3;
-            uint32_t o[8];
-            widen16(v[k], o);
-            unsigned char* row = tile + static_cast<uint32_t>(j) * 128u;
-            *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) =
-                make_uint4(o[0], o[1], o[2], o[3]);
-            *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
-                make_uint4(o[4], o[5], o[6], o[7]);
-        }
+    for (int i = 0; i < kMaxLoads; ++i) {
+        const int u = i * kCompute + tid, j = u >> 2;
+        v[i] = j < seq ? ld_nc16(src + static_cast<long long>(j) * ld + 16 * (u & 3)) : make_int4(0, 0, 0, 0);
     }
+}
+// ... widened into rows 0 .. rows-1 of a swizzled f16 tile: row j, 16-byte
+// chunk c (f16 8c .. 8c + 7) at j * 128 + (c ^ (j % 8)) * 16.
+__device__ __forceinline__ void store_rows(unsigned char* tile, const int4 (&v)[kMaxLoads], int rows, int tid) {
+#pragma unroll
+    for (int i = 0; i < kMaxLoads; ++i) {
+        const int u = i * kCompute + tid, j = u >> 2, ch = u & 3;
+        if (j >= rows) break;  // u grows with i
+        uint32_t o[8];
+        widen16(v[i], o);
+        unsigned char* row = tile + static_cast<uint32_t>(j) * 128u;
+        *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) =
+            make_uint4(o[0], o[1], o[2], o[3]);
+        *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
+            make_uint4(o[4], o[5], o[6], o[7]);
+    }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}\n" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ uint32_t pack2_s8(float v0, float v1, float inv) {
@@ -121,6 +150,16 @@ __device__ __forceinline__ uint32_t pack2_s8(float v0, float v1, float inv) {
     uint32_t d;
     asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(q1), "r"(q0), "r"(0));
     return d;  // q0 in byte 0, q1 in byte 1
+}
+
+// 2^t for t <= 0 on the special-function unit: ex2.approx.ftz.f32, within 2
+// ulp of the exact value wherever the result is a normal fp32 number
+// (checked on GB300 over every fp32 t in [-126, 0]); below that the result
+// flushes to 0, an absolute error under 2^-126.
+__device__ __forceinline__ float ex2(float t) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(t));
+    return y;
 }
 
 // The f16 pair (a, b) -> u32 (a in the low half), and back.
@@ -136,8 +175,18 @@ __device__ __forceinline__ float2 f16x2_float2(uint32_t u) {
     return __half22float2(h);
 }
 
+// 64-thread barrier (id 1 + qq) of the two compute warps of lane quarter qq.
+__device__ __forceinline__ void pair_sync(int qq) {
+    switch (qq) {
+        case 0: asm volatile("bar.sync 1, 64;\n" ::: "memory"); break;
+        case 1: asm volatile("bar.sync 2, 64;\n" ::: "memory"); break;
+        case 2: asm volatile("bar.sync 3, 64;\n" ::: "memory"); break;
+        default: asm volatile("bar.sync 4, 64;\n" ::: "memory"); break;
+    }
+}
+
 // c2 = c log2(e).  skip_mma (a test hook) issues no MMA, so that every wait
-// gives up after wait_limit polls with nothing in flight.
+// on one gives up after wait_limit polls with nothing in flight.
 __global__ void __launch_bounds__(kAttnThreads, 2)
 attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c2, float vscale, int kind,
                  float inv_out_scale, void* __restrict__ out, unsigned wait_limit, int skip_mma) {
@@ -145,199 +194,265 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
     unsigned char* sm =
         reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int nkb = (seq + kKeyBlock - 1) / kKeyBlock;
-    unsigned char* Ks = sm;                                  // [nkb * 128][64] f16, swizzled
-    unsigned char* Vs = sm + nkb * kBlockBytes;              // [nkb * 128][64] f16, swizzled
+    const int rows = nkb * kKeyBlock;
+    unsigned char* Ks = sm;                                  // [rows][64] f16, swizzled
+    unsigned char* Vs = sm + nkb * kBlockBytes;              // [rows][64] f16, swizzled
     unsigned char* misc = sm + 2 * nkb * kBlockBytes;
-    const uint32_t bar_s = smem_addr(misc);                  // S_b complete
-    const uint32_t bar_o = bar_s + 8;                        // P_b V_b complete
+    float* red = reinterpret_cast<float*>(misc + 64);        // [2 blocks][2 halves][128 queries]
+    const uint32_t bar_s = smem_addr(misc);  // [2] S_b complete (buffer b % 2)
+    const uint32_t bar_p = bar_s + 16;       // [2] P_b written: one arrival per compute thread
+    const uint32_t bar_o = bar_s + 32;       // [2] P_b V_b complete
+    const uint32_t bar_q = bar_s + 48;       // queries in tensor memory: one arrival per thread of warps 0-3
     const int tid = threadIdx.x, warp = tid >> 5;
     const int q0 = blockIdx.x * kAttnQ;
     const int h = blockIdx.y;
     const long long row0 = static_cast<long long>(blockIdx.z) * seq;  // first token row of the sequence
     const int8_t* head = qkv + row0 * ld + h * 64;
+    const bool mma_warp = warp == kCompute / 32;
+    const int qq = warp & 3, hh = (warp >> 2) & 1;  // lane quarter; half of the keys and of the context
+    const int qi = tid & (kAttnQ - 1);               // the thread's query within the CTA (= its lane)
 
-    if (tid == 0) mbar_init_n(bar_s, 2);
-    __syncwarp();
-    if (warp == 0) tmem_alloc(bar_s + 16, kTmemCols);
-    stage_rows(Ks, head + d, seq, nkb * kKeyBlock, ld, tid);
-    fence_proxy_async();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tm = *reinterpret_cast<volatile uint32_t*>(misc + 16);
-    const uint32_t lane = tm + (static_cast<uint32_t>(32 * warp) << 16);  // this warp's quarter of the lanes
-
-    // The thread's query as f16 pairs into its lane.
-    {
-        const int q = q0 + tid;
-        uint32_t v[32];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int4 x = q < seq ? ld_nc16(head + static_cast<long long>(q) * ld + 16 * k) : make_int4(0, 0, 0, 0);
-            uint32_t o[8];
-            widen16(x, o);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) v[8 * k + i] = o[i];
+    // 1. Barriers and tensor memory (MMA warp); the loads of the head's keys
+    //    and of the query (warps 0-3), all issued at once, the keys stored
+    //    (compute warps).
+    if (mma_warp) {
+        if (tid == kCompute) {
+            mbar_init_n(bar_s, 2);
+            mbar_init(bar_p, kCompute);
+            mbar_init(bar_p + 8, kCompute);
+            mbar_init_n(bar_o, 2);
+            mbar_init(bar_q, kAttnQ);
         }
-        tmem_st32(lane + kColQ, v);
-        tmem_wait_st();
+        __syncwarp();
+        tmem_alloc(bar_s + 56, kTmemCols);
+    }
+    int4 kv[kMaxLoads], qv[4];
+    if (!mma_warp) {
+        load_rows(kv, head + d, seq, ld, tid);
+        const int q = q0 + qi;
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+            qv[k] = (hh == 0 && q < seq) ? ld_nc16(head + static_cast<long long>(q) * ld + 16 * k)
+                                         : make_int4(0, 0, 0, 0);
+        store_rows(Ks, kv, rows, tid);
+        fence_proxy_async();
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    const uint32_t tm = *reinterpret_cast<volatile uint32_t*>(misc + 56);
+    const uint32_t lane = tm + (static_cast<uint32_t>(32 * qq) << 16);  // this warp's lane quarter
 
-    const uint32_t ks = smem_addr(Ks), vs = smem_addr(Vs);
-    auto issue_s = [&](int b) {
+    // 2. The values' loads; the query as f16 pairs into its lane (warps 0-3).
+    int4 vv[kMaxLoads];
+    if (!mma_warp) {
+        load_rows(vv, head + 2 * d, seq, ld, tid);
+        if (hh == 0) {
+            uint32_t v[32];
 #pragma unroll
-        for (int t = 0; t < 4; ++t)
-            mma_f16_ts(tm + kColS, tm + kColQ + 8 * t, sw128_desc(ks + b * kBlockBytes + 32 * t, 16, 1024), kIdescS,
-                       t > 0);
-        tc_commit(bar_s);
-    };
-    if (tid == 0 && !skip_mma) issue_s(0);
-    // The values land while the first scores are computed; they are visible
-    // to the MMAs after the block's barrier below.
-    stage_rows(Vs, head + 2 * d, seq, nkb * kKeyBlock, ld, tid);
-    fence_proxy_async();
+            for (int k = 0; k < 4; ++k) {
+                uint32_t o[8];
+                widen16(qv[k], o);
+#pragma unroll
+                for (int i2 = 0; i2 < 8; ++i2) v[8 * k + i2] = o[i2];
+            }
+            tmem_st32(lane + kColQ, v);
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(bar_q);
+        }
+    }
 
-    float m = -INFINITY;  // running maximum of the exact dot products
-    float l = 0.0f;       // running sum of the weights
     bool ok = true;
-    for (int b = 0; b < nkb; ++b) {
-        ok &= mbar_wait(bar_s, b & 1, wait_limit);
+    if (mma_warp) {
+        // 3a. MMA issue (one thread).
+        if (tid == kCompute) {
+            const uint32_t ks = smem_addr(Ks), vs = smem_addr(Vs);
+            auto issue_s = [&](int b) {
+                const uint32_t buf = tm + kColS + 64u * static_cast<uint32_t>(b & 1);
+#pragma unroll
+                for (int t = 0; t < 4; ++t)
+                    mma_f16_ts(buf, tm + kColQ + 8 * t, sw128_desc(ks + b * kBlockBytes + 32 * t, 16, 1024), kIdescS,
+                               t > 0);
+                tc_commit(bar_s + 8u * static_cast<uint32_t>(b & 1));
+            };
+            ok &= mbar_wait(bar_q, 0, wait_limit);
+            tc_fence_after();
+            if (!skip_mma) {
+                issue_s(0);
+                if (nkb > 1) issue_s(1);
+            }
+            for (int b = 0; b < nkb; ++b) {
+                const uint32_t x = static_cast<uint32_t>(b & 1), ph = static_cast<uint32_t>(b >> 1) & 1u;
+                ok &= mbar_wait(bar_p + 8u * x, ph, wait_limit);
+                tc_fence_after();
+                if (!skip_mma) {
+#pragma unroll
+                    for (int t = 0; t < 4; ++t) {  // keys 16 t .. 16 t + 15 of the block
+                        const uint64_t bd = sw128_desc(vs + b * kBlockBytes + 2048 * t, 1024, 1024);
+                        const uint32_t a = tm + kColS + 64u * x + 32 * (t >> 1) + 8 * (t & 1);
+                        mma_f16_ts(tm + kColO, a, bd, kIdescPV, (b > 0 || t > 0) ? 1u : 0u);
+                        mma_f16_ts(tm + kColO, a + 16, bd, kIdescPV, 1u);
+                    }
+                    tc_commit(bar_o + 8u * x);
+                }
+                if (b + 2 < nkb) {  // S_(b+2) overwrites P_b: wait until it is consumed
+                    ok &= mbar_wait(bar_o + 8u * x, ph, wait_limit);
+                    tc_fence_after();
+                    if (!skip_mma) issue_s(b + 2);
+                }
+            }
+        }
         __syncwarp();
-        tc_fence_after();
-        float s[kKeyBlock];
-        {
-            uint32_t r[4][32];
+    } else {
+        // 3b. Compute warps: the values, then the softmax block by block
+        //     over the warp's 32 keys of each block.
+        store_rows(Vs, vv, rows, tid);
+        fence_proxy_async();  // visible to the MMAs once P_0 is announced
+        // The weights are 2^(s c2 - M) against a reference M = fl(m c2) of a
+        // maximum m of the dot products seen so far, which moves only when
+        // the block maximum exceeds it by more than kLazy (log2 units), so
+        // the weights stay below 2^kLazy.  A rounding error of M scales all
+        // the weights taken against it by one factor, which the context and
+        // the sum share.
+        float mref = 0.0f;                      // M
+        float lq[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // running sum of the warp's weights, in 4 parts
+        for (int b = 0; b < nkb; ++b) {
+            const uint32_t x = static_cast<uint32_t>(b & 1), ph = static_cast<uint32_t>(b >> 1) & 1u;
+            const uint32_t buf = lane + kColS + 64u * x + 32u * static_cast<uint32_t>(hh);
+            ok &= mbar_wait(bar_s + 8u * x, ph, wait_limit);
+            __syncwarp();
+            tc_fence_after();
+            float s[32];
+            {
+                uint32_t r[32];
+                tmem_ld32(buf, r);
+                tmem_wait_ld(r);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) tmem_ld32(lane + kColS + 32 * k, r[k]);
+                for (int i2 = 0; i2 < 32; ++i2) s[i2] = __uint_as_float(r[i2]);
+            }
+            const int valid = seq - b * kKeyBlock - 32 * hh;  // of the warp's 32 keys, inside the sequence
+            if (valid < 32) {
 #pragma unroll
-            for (int k = 0; k < 4; ++k) tmem_wait_ld(r[k]);
+                for (int j2 = 0; j2 < 32; ++j2)
+                    if (j2 >= valid) s[j2] = -INFINITY;
+            }
+            float bq[4] = {s[0], s[1], s[2], s[3]};
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
+            for (int j2 = 4; j2 < 32; ++j2) bq[j2 & 3] = fmaxf(bq[j2 & 3], s[j2]);
+            float* rb = red + 256 * (b & 1);
+            rb[128 * hh + qi] = fmaxf(fmaxf(bq[0], bq[1]), fmaxf(bq[2], bq[3]));
+            pair_sync(qq);
+            // The block's maximum, scaled (finite: the block has a key).
+            const float bm = __fmul_rn(fmaxf(rb[qi], rb[128 + qi]), c2);
+            if (b == 0) {
+                mref = bm;
+            } else {
+                // A reference that moves scales the context and the sum by
+                // alpha = 2^(M_old - M_new) once the previous block's P v is
+                // complete (alpha = 1 for the lanes whose reference stays);
+                // tensor-memory loads and stores are warp-wide, so the whole
+                // warp takes the branch.
+                const bool move = __fsub_rn(bm, mref) > kLazy;
+                if (__any_sync(0xffffffffu, move)) {
+                    const uint32_t xp = static_cast<uint32_t>((b - 1) & 1), php = static_cast<uint32_t>((b - 1) >> 1) & 1u;
+                    ok &= mbar_wait(bar_o + 8u * xp, php, wait_limit);
+                    __syncwarp();
+                    tc_fence_after();
+                    // M_old - M_new exactly, as d_hi + d_lo (Knuth's TwoSum)
+                    const float dh = __fsub_rn(mref, bm);
+                    const float bb = __fsub_rn(dh, mref);
+                    const float dl = __fadd_rn(__fsub_rn(mref, __fsub_rn(dh, bb)), __fsub_rn(-bm, bb));
+                    const float alpha = move ? __fmul_rn(exp2f(dh), exp2f(dl)) : 1.0f;
+                    if (move) mref = bm;
 #pragma unroll
-                for (int i = 0; i < 32; ++i) s[32 * k + i] = __uint_as_float(r[k][i]);
-        }
-        const int valid = seq - b * kKeyBlock;  // keys of the block inside the sequence, >= 1
-        if (valid < kKeyBlock) {
+                    for (int k = 0; k < 4; ++k) lq[k] = __fmul_rn(lq[k], alpha);
+                    uint32_t o[32];
+                    const uint32_t oc = lane + kColO + 32u * static_cast<uint32_t>(hh);
+                    tmem_ld32(oc, o);
+                    tmem_wait_ld(o);
 #pragma unroll
-            for (int j = 0; j < kKeyBlock; ++j)
-                if (j >= valid) s[j] = -INFINITY;
-        }
-        float bm = s[0];
-#pragma unroll
-        for (int j = 1; j < kKeyBlock; ++j) bm = fmaxf(bm, s[j]);
-        const float mn = fmaxf(m, bm);  // finite: the block has a key
-        // A larger maximum scales the context and the sum by the same
-        // factor (1 for the lanes whose maximum did not move); tensor-memory
-        // loads and stores are warp-wide, so the whole warp takes the branch.
-        if (b > 0 && __any_sync(0xffffffffu, mn > m)) {
-            const float alpha = exp2f(__fmul_rn(__fsub_rn(m, mn), c2));
-            l = __fmul_rn(l, alpha);
-            uint32_t o[2][32];
-            tmem_ld32(lane + kColO, o[0]);
-            tmem_ld32(lane + kColO + 32, o[1]);
-            tmem_wait_ld(o[0]);
-            tmem_wait_ld(o[1]);
-#pragma unroll
-            for (int k = 0; k < 2; ++k)
-#pragma unroll
-                for (int i = 0; i < 32; ++i) o[k][i] = __float_as_uint(__fmul_rn(__uint_as_float(o[k][i]), alpha));
-            tmem_st32(lane + kColO, o[0]);
-            tmem_st32(lane + kColO + 32, o[1]);
-        }
-        m = mn;
-        // Weights of keys 32 cc .. 32 cc + 31: high f16 parts into columns
-        // 32 cc .. + 15, low parts into 32 cc + 16 .. + 31 (over the scores).
-#pragma unroll
-        for (int cc = 0; cc < 4; ++cc) {
+                    for (int i2 = 0; i2 < 32; ++i2) o[i2] = __float_as_uint(__fmul_rn(__uint_as_float(o[i2]), alpha));
+                    tmem_st32(oc, o);
+                }
+            }
+            // The warp's 32 weights: high f16 parts into the first 16 of its
+            // columns, low parts into the last 16 (over the scores).
             uint32_t p[32];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-                const float e0 = exp2f(__fmul_rn(__fsub_rn(s[32 * cc + 2 * e], m), c2));
-                const float e1 = exp2f(__fmul_rn(__fsub_rn(s[32 * cc + 2 * e + 1], m), c2));
-                l = __fadd_rn(__fadd_rn(l, e0), e1);
+                const float e0 = ex2(__fmaf_rn(s[2 * e], c2, -mref));
+                const float e1 = ex2(__fmaf_rn(s[2 * e + 1], c2, -mref));
+                lq[(2 * e) & 3] = __fadd_rn(lq[(2 * e) & 3], e0);
+                lq[(2 * e + 1) & 3] = __fadd_rn(lq[(2 * e + 1) & 3], e1);
                 const uint32_t hi = f16x2_bits(e0, e1);
                 const float2 hf = f16x2_float2(hi);
                 p[e] = hi;
                 p[16 + e] = f16x2_bits(__fsub_rn(e0, hf.x), __fsub_rn(e1, hf.y));
             }
-            tmem_st32(lane + kColS + 32 * cc, p);
+            tmem_st32(buf, p);
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(bar_p + 8u * x);
         }
-        tmem_wait_st();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !skip_mma) {
-            tc_fence_after();
-#pragma unroll
-            for (int t = 0; t < 8; ++t) {  // keys 16 t .. 16 t + 15 of the block
-                const uint64_t bd = sw128_desc(vs + b * kBlockBytes + 2048 * t, 1024, 1024);
-                const uint32_t a = tm + kColS + 32 * (t >> 1) + 8 * (t & 1);
-                mma_f16_ts(tm + kColO, a, bd, kIdescPV, (b > 0 || t > 0) ? 1u : 0u);
-                mma_f16_ts(tm + kColO, a + 16, bd, kIdescPV, 1u);
-            }
-            tc_commit(bar_o);
-            if (b + 1 < nkb) {  // the next scores overwrite P_b: wait until it is consumed
-                ok &= mbar_wait(bar_o, b & 1, wait_limit);
-                tc_fence_after();
-                issue_s(b + 1);
-            }
-        }
-    }
 
-    // Context row: O / l * qkv_scale.
-    ok &= mbar_wait(bar_o, (nkb - 1) & 1, wait_limit);
-    __syncwarp();
-    tc_fence_after();
-    uint32_t o[2][32];
-    tmem_ld32(lane + kColO, o[0]);
-    tmem_ld32(lane + kColO + 32, o[1]);
-    tmem_wait_ld(o[0]);
-    tmem_wait_ld(o[1]);
-    const int r = q0 + tid;
-    if (r < seq) {
-        const float f = __fdiv_rn(vscale, l);
-        const long long base = (row0 + r) * d + h * 64;
-        if (kind == 3) {
-            uint4* dst = reinterpret_cast<uint4*>(static_cast<int8_t*>(out) + base);
+        // 4. Context: the warp's 32 columns of O / l * qkv_scale, once the
+        //    last P v is complete (which completes every earlier one); l =
+        //    the two warps' sums.
+        float* rl = red + 512;
+        rl[128 * hh + qi] = __fadd_rn(__fadd_rn(lq[0], lq[1]), __fadd_rn(lq[2], lq[3]));
+        ok &= mbar_wait(bar_o + 8u * static_cast<uint32_t>((nkb - 1) & 1), static_cast<uint32_t>((nkb - 1) >> 1) & 1u,
+                        wait_limit);
+        __syncwarp();
+        tc_fence_after();
+        uint32_t o[32];
+        tmem_ld32(lane + kColO + 32u * static_cast<uint32_t>(hh), o);
+        tmem_wait_ld(o);
+        pair_sync(qq);
+        const int r = q0 + qi;
+        if (r < seq) {
+            const float l = __fadd_rn(rl[qi], rl[128 + qi]);
+            const float f = __fdiv_rn(vscale, l);
+            const long long base = (row0 + r) * d + h * 64 + 32 * hh;
+            if (kind == 3) {
+                uint4* dst = reinterpret_cast<uint4*>(static_cast<int8_t*>(out) + base);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                uint32_t w[4];
+                for (int k = 0; k < 2; ++k) {
+                    uint32_t w[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int j = 16 * k + 4 * i;
-                    const float y0 = __fmul_rn(__uint_as_float(o[j >> 5][j & 31]), f);
-                    const float y1 = __fmul_rn(__uint_as_float(o[(j + 1) >> 5][(j + 1) & 31]), f);
-                    const float y2 = __fmul_rn(__uint_as_float(o[(j + 2) >> 5][(j + 2) & 31]), f);
-                    const float y3 = __fmul_rn(__uint_as_float(o[(j + 3) >> 5][(j + 3) & 31]), f);
-                    w[i] = pack2_s8(y0, y1, inv_out_scale) | (pack2_s8(y2, y3, inv_out_scale) << 16);
+                    for (int i2 = 0; i2 < 4; ++i2) {
+                        const int j2 = 16 * k + 4 * i2;
+                        w[i2] = pack2_s8(__fmul_rn(__uint_as_float(o[j2]), f), __fmul_rn(__uint_as_float(o[j2 + 1]), f),
+                                         inv_out_scale) |
+                                (pack2_s8(__fmul_rn(__uint_as_float(o[j2 + 2]), f),
+                                          __fmul_rn(__uint_as_float(o[j2 + 3]), f), inv_out_scale)
+                                 << 16);
+                    }
+                    dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
                 }
-                dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
-            }
-        } else {
-            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + base);
+            } else {
+                float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) + base);
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                const int j = 4 * k;
-                dst[k] = make_float4(__fmul_rn(__uint_as_float(o[j >> 5][j & 31]), f),
-                                     __fmul_rn(__uint_as_float(o[(j + 1) >> 5][(j + 1) & 31]), f),
-                                     __fmul_rn(__uint_as_float(o[(j + 2) >> 5][(j + 2) & 31]), f),
-                                     __fmul_rn(__uint_as_float(o[(j + 3) >> 5][(j + 3) & 31]), f));
+                for (int k = 0; k < 8; ++k)
+                    dst[k] = make_float4(__fmul_rn(__uint_as_float(o[4 * k]), f), __fmul_rn(__uint_as_float(o[4 * k + 1]), f),
+                                         __fmul_rn(__uint_as_float(o[4 * k + 2]), f),
+                                         __fmul_rn(__uint_as_float(o[4 * k + 3]), f));
             }
         }
     }
     if (!ok) atomicOr(&g_attn_status, static_cast<unsigned>(kStatusTimeout));
     tc_fence_before();
     __syncthreads();
-    if (warp == 0) tmem_dealloc(tm, kTmemCols);
+    if (mma_warp) tmem_dealloc(tm, kTmemCols);
 }
 
 }  // namespace
 
 size_t attention_smem_bytes(int seq) {
     const size_t nkb = (static_cast<size_t>(seq) + kKeyBlock - 1) / kKeyBlock;
-    return 2 * nkb * kBlockBytes + 1024 + 64;  // K and V tiles, 1024-byte alignment, barriers + TMEM address
+    // K and V tiles, 1024-byte alignment, 7 barriers + TMEM address, the
+    // block maxima [2][2][128] and the sums [2][128]
+    return 2 * nkb * kBlockBytes + 1024 + 64 + 4 * (512 + 256);
 }
 
 cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, int ld, float score_scale,

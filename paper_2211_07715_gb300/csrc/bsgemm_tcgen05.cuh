@@ -113,7 +113,6 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32
                  : "memory");
 }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
-
 #undef BSG_TC_OUT8
 #undef BSG_TC_IO8
 #undef BSG_TC_IN8

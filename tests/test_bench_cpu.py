@@ -9,14 +9,14 @@ import bench
 def test_attention_floors_follow_their_definitions():
     """8 x 384 tokens, 12 heads of 64: 905,969,664 multiply-adds per
     product.  Tensor floor = 6 x that many flops at the given bf16 rate,
-    exp floor = one exponential per score at 16 per SM per clock, HBM floor
+    exp floor = one exponential per score at 32 per SM per clock, HBM floor
     = the int8 QKV rows once; the largest one is the bound."""
     r = bench.attention_roofline(8, 384, 12, 0.0155, 152, 2070.0, 6783.5, 1903.9)
     macs = 8 * 12 * 384 * 384 * 64
     assert macs == 905_969_664
     assert r["ops"] == 4 * macs
     assert abs(r["floors_us"]["tensor"] - 6 * macs / 1903.9e12 * 1e6) < 1e-3
-    assert abs(r["floors_us"]["exp"] - 8 * 12 * 384 * 384 / (152 * 16 * 2070e6) * 1e6) < 1e-3
+    assert abs(r["floors_us"]["exp"] - 8 * 12 * 384 * 384 / (152 * 32 * 2070e6) * 1e6) < 1e-3
     assert abs(r["floors_us"]["hbm"] - 8 * 384 * 2304 / 6783.5e9 * 1e6) < 1e-3
     assert r["bound"] == "tensor" and r["floor"] == "tensor"
     assert abs(r["frac"] - r["floors_us"]["tensor"] / 15.5) < 1e-3
