@@ -1081,7 +1081,7 @@ def run_encoder(args) -> dict:
     def attn_only(i, s):
         b = bufs[i % nsets]
         bsg.bsgemm_attention(b["qkv"].data_ptr(), batch, seq, heads, 64, 2304, scales["qkv"], b["ctx"].data_ptr(),
-                             bsg.OUT_I8, scales["ctx"], s.cuda_stream)
+                             bsg.OUT_I8, scales["ctx"], s.cuda_stream, bsg.ACT_READY)
 
     attn_ms = graph_ms(attn_only, reps)
     ops = [2.0 * m * w.nnzb * 4 for w in weights]

@@ -337,7 +337,11 @@ int bsgemm_layernorm(const float* z, int M, int N, const float* gamma, const flo
  *          qkv_scale^2 / sqrt(head_dim) a normal fp32 number below 2^100.
  *   out    DEVICE [batch * seq][d], float (epi.kind BSGEMM_OUT_F32) or
  *          int8 (BSGEMM_OUT_I8, epi.out_scale as for bsgemm_run);
- *          16-byte aligned; must not overlap qkv.  Other epi fields unused.
+ *          16-byte aligned; must not overlap qkv.  epi.flags may be
+ *          BSGEMM_ACT_READY (qkv was complete before the stream's
+ *          preceding kernel began: the kernel then reads it while that
+ *          kernel still runs; out is written after it either way).  Other
+ *          epi fields unused.
  * head_dim must be 64 and seq <= BSGEMM_ATTN_MAX_SEQ (else
  * BSGEMM_ERR_UNSUPPORTED); 1 <= heads <= 65535, 0 <= batch <= 65535, seq >=
  * 1 unless batch = 0 (a no-op).  One kernel on `stream`, asynchronous.

@@ -293,11 +293,12 @@ ATTN_HEAD_DIM = 64
 
 
 def bsgemm_attention(qkv_ptr: int, batch: int, seq: int, heads: int, head_dim: int, ld: int, qkv_scale: float,
-                     out_ptr: int, kind: int, out_scale: float = 1.0, stream: int = 0) -> None:
+                     out_ptr: int, kind: int, out_scale: float = 1.0, stream: int = 0, flags: int = 0) -> None:
     """Enqueue multi-head self-attention on the int8 QKV rows (raw device
-    pointers; rows of ld bytes holding q | k | v)."""
+    pointers; rows of ld bytes holding q | k | v).  flags: 0 or ACT_READY
+    (qkv was complete before the stream's previous kernel began)."""
     rc = _lib.bsgemm_attention(qkv_ptr, int(batch), int(seq), int(heads), int(head_dim), int(ld), float(qkv_scale),
-                               out_ptr, _epi(kind, out_scale), stream)
+                               out_ptr, _epi(kind, out_scale, flags), stream)
     if rc != 0:
         raise BsgemmError(rc, bsgemm_last_error())
 

@@ -909,6 +909,8 @@ int bsgemm_attention(const int8_t* qkv, int batch, int seq, int heads, int head_
         return fail(BSGEMM_ERR_UNSUPPORTED, "seq exceeds BSGEMM_ATTN_MAX_SEQ = " + std::to_string(BSGEMM_ATTN_MAX_SEQ));
     if (epi.kind != BSGEMM_OUT_F32 && epi.kind != BSGEMM_OUT_I8)
         return fail(BSGEMM_ERR_INVALID, "attention writes BSGEMM_OUT_F32 or BSGEMM_OUT_I8");
+    if (epi.flags & ~static_cast<uint32_t>(BSGEMM_ACT_READY))
+        return fail(BSGEMM_ERR_INVALID, "unknown bits in epi.flags");
     const long long d = static_cast<long long>(heads) * head_dim;
     if (ld < 3 * d || ld % 16 != 0) return fail(BSGEMM_ERR_INVALID, "ld must be >= 3 * heads * head_dim and a multiple of 16");
     if (static_cast<long long>(batch) * seq > INT32_MAX) return fail(BSGEMM_ERR_INVALID, "batch * seq exceeds 2^31 - 1");
@@ -929,7 +931,8 @@ int bsgemm_attention(const int8_t* qkv, int batch, int seq, int heads, int head_
     if ((reinterpret_cast<uintptr_t>(qkv) & 15u) || (reinterpret_cast<uintptr_t>(out) & 15u))
         return fail(BSGEMM_ERR_INVALID, "qkv and out must be 16-byte aligned");
     const cudaError_t e = bsg::launch_attention(qkv, batch, seq, heads, ld, static_cast<float>(c), qkv_scale, epi.kind,
-                                                inv, out, static_cast<cudaStream_t>(stream));
+                                                inv, out, (epi.flags & BSGEMM_ACT_READY) != 0,
+                                                static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("attention launch", e));
     return BSGEMM_OK;
 }

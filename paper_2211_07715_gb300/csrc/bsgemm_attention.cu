@@ -77,7 +77,7 @@ constexpr int kAttnQ = 128;           // queries per CTA
 constexpr int kKeyBlock = 64;         // keys per online-softmax block
 constexpr uint32_t kBlockBytes = 8192;   // 64 rows x 64 f16
 constexpr int kMaxRows = (BSGEMM_ATTN_MAX_SEQ + kKeyBlock - 1) / kKeyBlock * kKeyBlock;
-constexpr int kMaxLoads = (4 * kMaxRows + kCompute - 1) / kCompute;  // 16-byte loads of K (or V) per thread
+constexpr int kMaxHalfUnits = (2 * kMaxRows + kCompute - 1) / kCompute;  // 16-byte units of V's second half a thread
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kColS = 0, kColO = 128, kColQ = 192;  // score buffers at kColS and kColS + 64
 constexpr uint32_t kIdescS = f16_idesc(128, 64, false);  // S = Q K_b^T
@@ -114,35 +114,34 @@ __device__ __forceinline__ void widen16(int4 v, uint32_t (&o)[8]) {
     }
 }
 
-// The 16-byte loads of one third of the head (src = its row 0, rows ld
-// bytes apart): load i of thread t is row j = (128 i + t) / 4, 16-byte chunk
-// (128 i + t) % 4; zeros past the sequence.  All issued before any is used.
-__device__ __forceinline__ void load_rows(int4 (&v)[kMaxLoads], const int8_t* src, int seq, int ld, int tid) {
-#pragma unroll
-    for (int i = 0; i < kMaxLoads; ++i) {
-        const int u = i * kCompute + tid, j = u >> 2;
-        v[i] = j < seq ? ld_nc16(src + static_cast<long long>(j) * ld + 16 * (u & 3)) : make_int4(0, 0, 0, 0);
-    }
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}\n" ::"r"(bar) : "memory");
 }
-// ... widened into rows 0 .. rows-1 of a swizzled f16 tile: row j, 16-byte
-// chunk c (f16 8c .. 8c + 7) at j * 128 + (c ^ (j % 8)) * 16.
-__device__ __forceinline__ void store_rows(unsigned char* tile, const int4 (&v)[kMaxLoads], int rows, int tid) {
-#pragma unroll
-    for (int i = 0; i < kMaxLoads; ++i) {
-        const int u = i * kCompute + tid, j = u >> 2, ch = u & 3;
-        if (j >= rows) break;  // u grows with i
+
+// 16 bytes global -> shared without registers (zeros when src_bytes is 0).
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;\n" ::: "memory");
+}
+// Barrier of the 8 compute warps (the MMA warp does not take part).
+__device__ __forceinline__ void compute_sync() { asm volatile("bar.sync 5, 256;\n" ::: "memory"); }
+
+// Rows [j0, j1) of int8 rows (64 bytes each, row-major from `src`) widened
+// into the swizzled f16 tile `tile` (row j, 16-byte chunk c at j * 128 + (c
+// ^ (j % 8)) * 16); thread t takes 16-byte units t, t + 256, ...
+__device__ __forceinline__ void widen_rows(unsigned char* tile, const unsigned char* src, int j0, int j1, int tid) {
+    for (int u = 4 * j0 + tid; u < 4 * j1; u += kCompute) {
+        const int j = u >> 2, ch = u & 3;
         uint32_t o[8];
-        widen16(v[i], o);
+        widen16(*reinterpret_cast<const int4*>(src + 16 * u), o);
         unsigned char* row = tile + static_cast<uint32_t>(j) * 128u;
         *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) =
             make_uint4(o[0], o[1], o[2], o[3]);
         *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
             make_uint4(o[4], o[5], o[6], o[7]);
     }
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}\n" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ uint32_t pack2_s8(float v0, float v1, float inv) {
@@ -189,7 +188,7 @@ __device__ __forceinline__ void pair_sync(int qq) {
 // on one gives up after wait_limit polls with nothing in flight.
 __global__ void __launch_bounds__(kAttnThreads, 2)
 attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c2, float vscale, int kind,
-                 float inv_out_scale, void* __restrict__ out, unsigned wait_limit, int skip_mma) {
+                 float inv_out_scale, void* __restrict__ out, unsigned wait_limit, int skip_mma, int act_ready) {
     extern __shared__ unsigned char smem_raw[];
     unsigned char* sm =
         reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -212,9 +211,16 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
     const int qq = warp & 3, hh = (warp >> 2) & 1;  // lane quarter; half of the keys and of the context
     const int qi = tid & (kAttnQ - 1);               // the thread's query within the CTA (= its lane)
 
-    // 1. Barriers and tensor memory (MMA warp); the loads of the head's keys
-    //    and of the query (warps 0-3), all issued at once, the keys stored
-    //    (compute warps).
+    // The kernel is launched with programmatic dependent launch: it lets the
+    // next kernel launch at once, and reads qkv only after the preceding
+    // kernel has completed -- unless act_ready says qkv was complete before
+    // that kernel began; global writes always come after it.
+    griddep_launch_dependents();
+
+    // 1. Barriers and tensor memory (MMA warp); the head's keys and values
+    //    copied as int8 into the value tile's space (keys in its first half,
+    //    values in its second) and the query loaded (warps 0-3), all issued
+    //    at once; the keys widened into their f16 tile (compute warps).
     if (mma_warp) {
         if (tid == kCompute) {
             mbar_init_n(bar_s, 2);
@@ -226,15 +232,25 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
         __syncwarp();
         tmem_alloc(bar_s + 56, kTmemCols);
     }
-    int4 kv[kMaxLoads], qv[4];
+    int4 qv[4];
     if (!mma_warp) {
-        load_rows(kv, head + d, seq, ld, tid);
+        if (!act_ready) griddep_wait();
         const int q = q0 + qi;
 #pragma unroll
         for (int k = 0; k < 4; ++k)
             qv[k] = (hh == 0 && q < seq) ? ld_nc16(head + static_cast<long long>(q) * ld + 16 * k)
                                          : make_int4(0, 0, 0, 0);
-        store_rows(Ks, kv, rows, tid);
+        // unit u of part p (0 = keys, 1 = values): row u / 4, 16-byte chunk u % 4,
+        // to Vs + p * rows * 64 + 16 u (zeros past the sequence)
+        const uint32_t vs8 = smem_addr(Vs);
+        for (int u = tid; u < 8 * rows; u += kCompute) {
+            const int p = u >= 4 * rows, r = u - 4 * rows * p, j = r >> 2;
+            const int8_t* src = head + (p + 1) * d + static_cast<long long>(j < seq ? j : 0) * ld + 16 * (r & 3);
+            cp_async16(vs8 + static_cast<uint32_t>(p * rows * 64 + 16 * r), src, j < seq ? 16u : 0u);
+        }
+        cp_async_wait_all();
+        compute_sync();  // every thread's copies have landed
+        widen_rows(Ks, Vs, 0, rows, tid);
         fence_proxy_async();
     }
     tc_fence_before();
@@ -243,10 +259,8 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
     const uint32_t tm = *reinterpret_cast<volatile uint32_t*>(misc + 56);
     const uint32_t lane = tm + (static_cast<uint32_t>(32 * qq) << 16);  // this warp's lane quarter
 
-    // 2. The values' loads; the query as f16 pairs into its lane (warps 0-3).
-    int4 vv[kMaxLoads];
+    // 2. The query as f16 pairs into its lane (warps 0-3).
     if (!mma_warp) {
-        load_rows(vv, head + 2 * d, seq, ld, tid);
         if (hh == 0) {
             uint32_t v[32];
 #pragma unroll
@@ -305,9 +319,36 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
         }
         __syncwarp();
     } else {
-        // 3b. Compute warps: the values, then the softmax block by block
-        //     over the warp's 32 keys of each block.
-        store_rows(Vs, vv, rows, tid);
+        // 3b. Compute warps: the values widened in place, then the softmax
+        //     block by block over the warp's 32 keys of each block.  The
+        //     int8 values sit at Vs + rows * 64: rows below rows / 2 widen
+        //     into the keys' int8 space (free now), the others over their
+        //     own int8 bytes, so those are read into registers first.
+        {
+            const unsigned char* v8 = Vs + rows * 64;
+            const int half = rows / 2;
+            widen_rows(Vs, v8, 0, half, tid);
+            int4 hv[kMaxHalfUnits];
+#pragma unroll
+            for (int i = 0; i < kMaxHalfUnits; ++i) {
+                const int u = 4 * half + i * kCompute + tid;
+                hv[i] = u < 4 * rows ? *reinterpret_cast<const int4*>(v8 + 16 * u) : make_int4(0, 0, 0, 0);
+            }
+            compute_sync();  // every read of the second half's int8 bytes is done
+#pragma unroll
+            for (int i = 0; i < kMaxHalfUnits; ++i) {
+                const int u = 4 * half + i * kCompute + tid;
+                if (u >= 4 * rows) break;
+                const int j = u >> 2, ch = u & 3;
+                uint32_t o[8];
+                widen16(hv[i], o);
+                unsigned char* row = Vs + static_cast<uint32_t>(j) * 128u;
+                *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) =
+                    make_uint4(o[0], o[1], o[2], o[3]);
+                *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
+                    make_uint4(o[4], o[5], o[6], o[7]);
+            }
+        }
         fence_proxy_async();  // visible to the MMAs once P_0 is announced
         // The weights are 2^(s c2 - M) against a reference M = fl(m c2) of a
         // maximum m of the dot products seen so far, which moves only when
@@ -410,6 +451,7 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
         tmem_wait_ld(o);
         pair_sync(qq);
         const int r = q0 + qi;
+        griddep_wait();  // the output is written after the preceding kernel
         if (r < seq) {
             const float l = __fadd_rn(rl[qi], rl[128 + qi]);
             const float f = __fdiv_rn(vscale, l);
@@ -440,7 +482,10 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
             }
         }
     }
-    if (!ok) atomicOr(&g_attn_status, static_cast<unsigned>(kStatusTimeout));
+    if (!ok) {
+        griddep_wait();
+        atomicOr(&g_attn_status, static_cast<unsigned>(kStatusTimeout));
+    }
     tc_fence_before();
     __syncthreads();
     if (mma_warp) tmem_dealloc(tm, kTmemCols);
@@ -456,7 +501,7 @@ size_t attention_smem_bytes(int seq) {
 }
 
 cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, int ld, float score_scale,
-                             float qkv_scale, int kind, float inv_out_scale, void* out, cudaStream_t s) {
+                             float qkv_scale, int kind, float inv_out_scale, void* out, bool act_ready, cudaStream_t s) {
     constexpr int kMaxDevices = 64;
     static std::mutex mu;
     static bool ready[kMaxDevices] = {};
@@ -477,9 +522,19 @@ cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, i
     const bool skip = (test_hooks() & BSGEMM_TEST_ATTN_SKIP_MMA) != 0;
     const dim3 grid(static_cast<unsigned>((seq + kAttnQ - 1) / kAttnQ), static_cast<unsigned>(heads),
                     static_cast<unsigned>(batch));
-    attention_kernel<<<grid, kAttnThreads, attention_smem_bytes(seq), s>>>(
-        qkv, seq, heads * 64, ld, c2, qkv_scale, kind, inv_out_scale, out, skip ? 64u : kWaitLimit, skip ? 1 : 0);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kAttnThreads);
+    cfg.dynamicSmemBytes = attention_smem_bytes(seq);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, attention_kernel, qkv, seq, heads * 64, ld, c2, qkv_scale, kind, inv_out_scale, out,
+                           skip ? 64u : kWaitLimit, skip ? 1 : 0, act_ready ? 1 : 0);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 cudaError_t attention_status(bool clear, unsigned* v) {

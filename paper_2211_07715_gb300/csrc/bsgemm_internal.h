@@ -116,7 +116,7 @@ cudaError_t launch_layernorm(const float* z, int M, int N, const float* gamma, c
 // 64] (kind 1: fp32, 3: int8); score_scale = qkv_scale^2 / 8.
 size_t attention_smem_bytes(int seq);
 cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, int ld, float score_scale,
-                             float qkv_scale, int kind, float inv_out_scale, void* out, cudaStream_t s);
+                             float qkv_scale, int kind, float inv_out_scale, void* out, bool act_ready, cudaStream_t s);
 // The current device's attention status word (bit 0: a wait gave up),
 // reset to 0 when clear is set and it was not.
 cudaError_t attention_status(bool clear, unsigned* v);
