@@ -30,30 +30,30 @@
 // MMA warp.  Compute warps w and w + 4 share the 32 queries of tensor-memory
 // lane quarter w (thread i % 128 owns query i = lane i): each takes 32 of a
 // block's 64 keys and 32 of the context's 64 columns, and the two exchange
-// their block maxima through shared memory.  Tensor memory (256 columns, so
-// two CTAs share an SM): two score buffers in columns 0-63 and 64-127 (block
-// b uses buffer b % 2: its scores, then its weights written back in place as
-// f16 pairs -- for keys 32c .. 32c + 31 of the block the high parts in
-// columns 32c .. + 15 of the buffer, the low parts in 32c + 16 .. + 31), the
-// context O in 128-191, the CTA's queries (f16 pairs) in 192-223, the row
-// sums in 224-239 (P times a 64 x 16 matrix of ones: the tensor cores add
-// the same f16 weights into the sum as into the context).  The head's keys
+// their block maxima through shared memory and keep their running sums of
+// the weights in registers.  Tensor memory (256 columns, so two CTAs share
+// an SM): two score buffers in columns 0-63 and 64-127 (block b uses
+// buffer b % 2: its scores, then its weights written back in place as f16
+// pairs -- for keys 32c .. 32c + 31 of the block the high parts in columns
+// 32c .. + 15 of the buffer, the low parts in 32c + 16 .. + 31), the context
+// O in 128-191, the CTA's queries (f16 pairs) in 192-223.  The head's keys
 // and values (seq <= BSGEMM_ATTN_MAX_SEQ, padded with zeros to whole blocks)
-// are staged once into shared memory as f16 rows of 64 with the 128-byte
-// swizzle: K is the K-major B operand of q k^T, V the MN-major B operand of
-// P v.
+// are copied into shared memory as int8 (cp.async, no registers) and widened
+// there into f16 rows of 64 with the 128-byte swizzle: K is the K-major B
+// operand of q k^T, V the MN-major B operand of P v.
 //
 // One thread of the MMA warp issues S_0 and S_1 (S_b = Q K_b^T: N = 64, K =
 // 64), then per block b: waits until the compute threads have written P_b,
-// issues O += P_b,hi V_b + P_b,lo V_b and L += P_b,hi 1 + P_b,lo 1 (16
-// MMAs), and once they have completed
-// issues S_(b+2) into the freed buffer.  So the compute warps work on block
-// b + 1 while the tensor cores consume block b, and never wait for the
-// tensor cores except where the running maximum grows (a rescale of O needs
-// the previous block's P v complete).  mbarriers, two of each kind (one per
-// buffer, so that no wait can fall two phases behind): S_b complete, P_b
-// written (256 arrivals), P_b V_b complete; and one for the queries written
-// to tensor memory (128 arrivals).  Every wait is bounded.
+// issues O += P_b,hi V_b + P_b,lo V_b (8 MMAs) and right behind them
+// S_(b+2) into the same buffer: the MMAs one thread issues run in issue
+// order, so S_(b+2) writes the buffer only after P_b V_b has read it.  The
+// compute warps thus work on block b + 1 while the tensor cores consume
+// block b, and wait for the tensor cores only where the running maximum
+// grows (a rescale of O needs the previous block's P v complete).
+// mbarriers, two of each kind (one per buffer, so that no wait can fall two
+// phases behind): S_b complete, P_b written (256 arrivals), P_b V_b
+// complete; and one for the queries written to tensor memory (128
+// arrivals).  Every wait is bounded.
 
 #include <cfloat>
 #include <cmath>
@@ -310,11 +310,9 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
                     }
                     tc_commit(bar_o + 8u * x);
                 }
-                if (b + 2 < nkb) {  // S_(b+2) overwrites P_b: wait until it is consumed
-                    ok &= mbar_wait(bar_o + 8u * x, ph, wait_limit);
-                    tc_fence_after();
-                    if (!skip_mma) issue_s(b + 2);
-                }
+                // S_(b+2) overwrites P_b.  MMAs issued by one thread run in
+                // issue order, so it follows P_b V_b without a wait here.
+                if (b + 2 < nkb && !skip_mma) issue_s(b + 2);
             }
         }
         __syncwarp();
