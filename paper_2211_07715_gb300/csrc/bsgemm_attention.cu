@@ -122,25 +122,38 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
 }
-__device__ __forceinline__ void cp_async_wait_all() {
-    asm volatile("cp.async.commit_group;\n cp.async.wait_group 0;\n" ::: "memory");
-}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+// Wait until at most N of this thread's committed groups are in flight.
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
 // Barrier of the 8 compute warps (the MMA warp does not take part).
 __device__ __forceinline__ void compute_sync() { asm volatile("bar.sync 5, 256;\n" ::: "memory"); }
 
 // Rows [j0, j1) of int8 rows (64 bytes each, row-major from `src`) widened
 // into the swizzled f16 tile `tile` (row j, 16-byte chunk c at j * 128 + (c
-// ^ (j % 8)) * 16); thread t takes 16-byte units t, t + 256, ...
+// ^ (j % 8)) * 16); thread t takes 16-byte units t, t + 256, ... (at most
+// NU of them: all loads first, then the widening and stores).
+__device__ __forceinline__ void store_unit(unsigned char* tile, int u, int4 v) {
+    const int j = u >> 2, ch = u & 3;
+    uint32_t o[8];
+    widen16(v, o);
+    unsigned char* row = tile + static_cast<uint32_t>(j) * 128u;
+    *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+    *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
+        make_uint4(o[4], o[5], o[6], o[7]);
+}
+template <int NU>
 __device__ __forceinline__ void widen_rows(unsigned char* tile, const unsigned char* src, int j0, int j1, int tid) {
-    for (int u = 4 * j0 + tid; u < 4 * j1; u += kCompute) {
-        const int j = u >> 2, ch = u & 3;
-        uint32_t o[8];
-        widen16(*reinterpret_cast<const int4*>(src + 16 * u), o);
-        unsigned char* row = tile + static_cast<uint32_t>(j) * 128u;
-        *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) =
-            make_uint4(o[0], o[1], o[2], o[3]);
-        *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
-            make_uint4(o[4], o[5], o[6], o[7]);
+    int4 v[NU];
+#pragma unroll
+    for (int i = 0; i < NU; ++i) {
+        const int u = 4 * j0 + tid + i * kCompute;
+        v[i] = u < 4 * j1 ? *reinterpret_cast<const int4*>(src + 16 * u) : make_int4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int i = 0; i < NU; ++i) {
+        const int u = 4 * j0 + tid + i * kCompute;
+        if (u < 4 * j1) store_unit(tile, u, v[i]);
     }
 }
 
@@ -241,16 +254,21 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
             qv[k] = (hh == 0 && q < seq) ? ld_nc16(head + static_cast<long long>(q) * ld + 16 * k)
                                          : make_int4(0, 0, 0, 0);
         // unit u of part p (0 = keys, 1 = values): row u / 4, 16-byte chunk u % 4,
-        // to Vs + p * rows * 64 + 16 u (zeros past the sequence)
+        // to Vs + p * rows * 64 + 16 u (zeros past the sequence); one
+        // commit group per part, so the keys widen while the values land
         const uint32_t vs8 = smem_addr(Vs);
-        for (int u = tid; u < 8 * rows; u += kCompute) {
-            const int p = u >= 4 * rows, r = u - 4 * rows * p, j = r >> 2;
-            const int8_t* src = head + (p + 1) * d + static_cast<long long>(j < seq ? j : 0) * ld + 16 * (r & 3);
-            cp_async16(vs8 + static_cast<uint32_t>(p * rows * 64 + 16 * r), src, j < seq ? 16u : 0u);
+#pragma unroll
+        for (int p = 0; p < 2; ++p) {
+            for (int u = tid; u < 4 * rows; u += kCompute) {
+                const int j = u >> 2;
+                const int8_t* src = head + (p + 1) * d + static_cast<long long>(j < seq ? j : 0) * ld + 16 * (u & 3);
+                cp_async16(vs8 + static_cast<uint32_t>(p * rows * 64 + 16 * u), src, j < seq ? 16u : 0u);
+            }
+            cp_async_commit();
         }
-        cp_async_wait_all();
-        compute_sync();  // every thread's copies have landed
-        widen_rows(Ks, Vs, 0, rows, tid);
+        cp_async_wait<1>();
+        compute_sync();  // every thread's copies of the keys have landed
+        widen_rows<4 * kMaxRows / kCompute>(Ks, Vs, 0, rows, tid);
         fence_proxy_async();
     }
     tc_fence_before();
@@ -323,28 +341,22 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
         //     into the keys' int8 space (free now), the others over their
         //     own int8 bytes, so those are read into registers first.
         {
+            cp_async_wait<0>();
+            compute_sync();  // every thread's copies of the values have landed
             const unsigned char* v8 = Vs + rows * 64;
             const int half = rows / 2;
-            widen_rows(Vs, v8, 0, half, tid);
-            int4 hv[kMaxHalfUnits];
+            int4 hv[kMaxHalfUnits];  // the second half's int8 bytes, loaded with the first half's
 #pragma unroll
             for (int i = 0; i < kMaxHalfUnits; ++i) {
                 const int u = 4 * half + i * kCompute + tid;
                 hv[i] = u < 4 * rows ? *reinterpret_cast<const int4*>(v8 + 16 * u) : make_int4(0, 0, 0, 0);
             }
+            widen_rows<kMaxHalfUnits>(Vs, v8, 0, half, tid);
             compute_sync();  // every read of the second half's int8 bytes is done
 #pragma unroll
             for (int i = 0; i < kMaxHalfUnits; ++i) {
                 const int u = 4 * half + i * kCompute + tid;
-                if (u >= 4 * rows) break;
-                const int j = u >> 2, ch = u & 3;
-                uint32_t o[8];
-                widen16(hv[i], o);
-                unsigned char* row = Vs + static_cast<uint32_t>(j) * 128u;
-                *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch) ^ (j & 7)) << 4)) =
-                    make_uint4(o[0], o[1], o[2], o[3]);
-                *reinterpret_cast<uint4*>(row + ((static_cast<uint32_t>(2 * ch + 1) ^ (j & 7)) << 4)) =
-                    make_uint4(o[4], o[5], o[6], o[7]);
+                if (u < 4 * rows) store_unit(Vs, u, hv[i]);
             }
         }
         fence_proxy_async();  // visible to the MMAs once P_0 is announced
