@@ -174,6 +174,36 @@ __device__ __forceinline__ float ex2(float t) {
     return y;
 }
 
+// Two fp32 lanes at once (sm_100+ packed instructions, each lane rounded
+// as the scalar instruction rounds): a * b + c, a + b, a - b; and the
+// largest of three values.
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+    float2 r;
+    asm("{\n .reg .b64 ra, rb, rc, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mov.b64 rc, {%6, %7};\n"
+        " fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}\n"
+        : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return r;
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+        " add.rn.f32x2 rd, ra, rb;\n mov.b64 {%0, %1}, rd;\n}\n"
+        : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n"
+        " sub.rn.f32x2 rd, ra, rb;\n mov.b64 {%0, %1}, rd;\n}\n"
+        : "=f"(r.x), "=f"(r.y) : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
 // The f16 pair (a, b) -> u32 (a in the low half), and back.
 __device__ __forceinline__ uint32_t f16x2_bits(float a, float b) {
     const __half2 h = __floats2half2_rn(a, b);
@@ -390,9 +420,11 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
             }
             float bq[4] = {s[0], s[1], s[2], s[3]};
 #pragma unroll
-            for (int j2 = 4; j2 < 32; ++j2) bq[j2 & 3] = fmaxf(bq[j2 & 3], s[j2]);
+            for (int j2 = 4; j2 < 32; j2 += 8)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) bq[k] = max3(bq[k], s[j2 + k], s[j2 + 4 + k]);
             float* rb = red + 256 * (b & 1);
-            rb[128 * hh + qi] = fmaxf(fmaxf(bq[0], bq[1]), fmaxf(bq[2], bq[3]));
+            rb[128 * hh + qi] = fmaxf(max3(bq[0], bq[1], bq[2]), bq[3]);
             pair_sync(qq);
             // The block's maximum, scaled (finite: the block has a key).
             const float bm = __fmul_rn(fmaxf(rb[qi], rb[128 + qi]), c2);
@@ -429,18 +461,28 @@ attention_kernel(const int8_t* __restrict__ qkv, int seq, int d, int ld, float c
             }
             // The warp's 32 weights: high f16 parts into the first 16 of its
             // columns, low parts into the last 16 (over the scores).
+            // (pairs of lanes: the packed fp32 instructions round each lane
+            // as the scalar ones do, so the values are those of one lane at a
+            // time; the sums go to lq[0], lq[1] for even e, lq[2], lq[3] for
+            // odd e, as before)
             uint32_t p[32];
+            float2 l01 = make_float2(lq[0], lq[1]), l23 = make_float2(lq[2], lq[3]);
+            const float2 c22 = make_float2(c2, c2), nm2 = make_float2(-mref, -mref);
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-                const float e0 = ex2(__fmaf_rn(s[2 * e], c2, -mref));
-                const float e1 = ex2(__fmaf_rn(s[2 * e + 1], c2, -mref));
-                lq[(2 * e) & 3] = __fadd_rn(lq[(2 * e) & 3], e0);
-                lq[(2 * e + 1) & 3] = __fadd_rn(lq[(2 * e + 1) & 3], e1);
-                const uint32_t hi = f16x2_bits(e0, e1);
-                const float2 hf = f16x2_float2(hi);
+                const float2 t = fma2(make_float2(s[2 * e], s[2 * e + 1]), c22, nm2);
+                const float2 ee = make_float2(ex2(t.x), ex2(t.y));
+                if (e & 1) l23 = add2(l23, ee);
+                else l01 = add2(l01, ee);
+                const uint32_t hi = f16x2_bits(ee.x, ee.y);
+                const float2 lo = sub2(ee, f16x2_float2(hi));
                 p[e] = hi;
-                p[16 + e] = f16x2_bits(__fsub_rn(e0, hf.x), __fsub_rn(e1, hf.y));
+                p[16 + e] = f16x2_bits(lo.x, lo.y);
             }
+            lq[0] = l01.x;
+            lq[1] = l01.y;
+            lq[2] = l23.x;
+            lq[3] = l23.y;
             tmem_st32(buf, p);
             tmem_wait_st();
             tc_fence_before();
