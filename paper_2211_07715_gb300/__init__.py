@@ -304,11 +304,13 @@ def bsgemm_attention(qkv_ptr: int, batch: int, seq: int, heads: int, head_dim: i
 
 
 def attention(qkv, batch: int, seq: int, heads: int, qkv_scale: float, kind: int = OUT_F32, out_scale: float = 1.0,
-              out=None, stream=None):
+              out=None, stream=None, flags: int = 0):
     """Multi-head self-attention (head width 64) on the CUDA int8 tensor qkv
     [batch * seq][>= 3 * heads * 64] (the QKV linear's output, q | k | v;
     its row stride may be padded to a multiple of 16).  Returns the context
-    [batch * seq][heads * 64], float32 or int8 by kind (or fills `out`)."""
+    [batch * seq][heads * 64], float32 or int8 by kind (or fills `out`).
+    flags: 0 or ACT_READY (qkv was complete before the stream's previous
+    kernel began)."""
     import torch
     if qkv.dtype != torch.int8 or not qkv.is_cuda or qkv.dim() != 2 or qkv.stride(1) != 1:
         raise ValueError("qkv must be a CUDA int8 [M][row] tensor with unit column stride")
@@ -325,7 +327,7 @@ def attention(qkv, batch: int, seq: int, heads: int, qkv_scale: float, kind: int
         raise ValueError(f"out must be a contiguous {dtype} [{m}][{d}] tensor")
     s = torch.cuda.current_stream() if stream is None else stream
     bsgemm_attention(qkv.data_ptr(), batch, seq, heads, ATTN_HEAD_DIM, qkv.stride(0), qkv_scale, out.data_ptr(), kind,
-                     out_scale, s.cuda_stream)
+                     out_scale, s.cuda_stream, flags)
     return out
 
 

@@ -955,7 +955,10 @@ cudaError_t launch(const DeviceWeights& w, const LaunchArgs& a_in, const Schedul
 // then the variance from the centred squares; out = fmaf((z - mean) *
 // rstd, gamma, beta), fp32 or requantised to int8 (kind 3: fp32 multiply
 // by 1 / out_scale, round half even, saturate).  With N % 4 == 0 and
-// 16-byte aligned arrays the row moves as float4 (and 4-byte int8 words).
+// 16-byte aligned arrays the row moves as float4 (and 4-byte int8 words),
+// and for N <= 1024 it is read once into registers for all three passes.
+// Launched with programmatic dependent launch: z is read after the
+// previous kernel completes.
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -971,17 +974,61 @@ __device__ __forceinline__ void ln_store(int kind, void* out, long long idx, flo
     }
 }
 
+constexpr int kLnVec = 8;  // float4s a lane keeps in registers: rows of N <= 1024 take one read
+
 __global__ void __launch_bounds__(256)
 layernorm_kernel(const float* __restrict__ z, int M, int N, const float* __restrict__ gamma,
                  const float* __restrict__ beta, float eps, int kind, float inv_out_scale, void* __restrict__ out) {
+    griddep_launch_dependents();
     const int lane = threadIdx.x & 31;
     const long long m = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
     if (m >= M) return;
+    griddep_wait();  // z is the previous kernel's output
     const float* row = z + m * N;
-    const float c = __ldg(row);
     const bool vec = (N & 3) == 0 && (reinterpret_cast<uintptr_t>(z) & 15) == 0 &&
                      (reinterpret_cast<uintptr_t>(gamma) & 15) == 0 && (reinterpret_cast<uintptr_t>(beta) & 15) == 0 &&
                      (reinterpret_cast<uintptr_t>(out) & 15) == 0;
+    if (vec && N <= 128 * kLnVec) {
+        // the row in registers (lane l: float4s l, l + 32, ...), read once;
+        // the same operations in the same order as the loops below
+        float4 v[kLnVec];
+#pragma unroll
+        for (int i = 0; i < kLnVec; ++i) {
+            const int n = 4 * lane + 128 * i;
+            v[i] = n < N ? __ldg(reinterpret_cast<const float4*>(row + n)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        const float c = __shfl_sync(0xffffffffu, v[0].x, 0);
+        float s1 = 0.0f;
+#pragma unroll
+        for (int i = 0; i < kLnVec; ++i)
+            if (4 * lane + 128 * i < N) s1 += ((v[i].x - c) + (v[i].y - c)) + ((v[i].z - c) + (v[i].w - c));
+        const float mean = c + warp_sum(s1) / N;
+        float s2 = 0.0f;
+#pragma unroll
+        for (int i = 0; i < kLnVec; ++i) {
+            if (4 * lane + 128 * i < N) {
+                const float a = v[i].x - mean, b = v[i].y - mean, d = v[i].z - mean, e = v[i].w - mean;
+                s2 += (a * a + b * b) + (d * d + e * e);
+            }
+        }
+        const float rstd = rsqrtf(warp_sum(s2) / N + eps);
+        const long long base = m * N;
+#pragma unroll
+        for (int i = 0; i < kLnVec; ++i) {
+            const int n = 4 * lane + 128 * i;
+            if (n >= N) continue;
+            const float4 g = __ldg(reinterpret_cast<const float4*>(gamma + n));
+            const float4 b = __ldg(reinterpret_cast<const float4*>(beta + n));
+            const float y0 = __fmaf_rn((v[i].x - mean) * rstd, g.x, b.x), y1 = __fmaf_rn((v[i].y - mean) * rstd, g.y, b.y);
+            const float y2 = __fmaf_rn((v[i].z - mean) * rstd, g.z, b.z), y3 = __fmaf_rn((v[i].w - mean) * rstd, g.w, b.w);
+            if (kind == 3)
+                *reinterpret_cast<uint32_t*>(static_cast<int8_t*>(out) + base + n) = requant4_s8(y0, y1, y2, y3, inv_out_scale);
+            else
+                *reinterpret_cast<float4*>(static_cast<float*>(out) + base + n) = make_float4(y0, y1, y2, y3);
+        }
+        return;
+    }
+    const float c = __ldg(row);
     float s1 = 0.0f;
     if (vec) {
         for (int n = 4 * lane; n < N; n += 128) {
@@ -1032,8 +1079,17 @@ cudaError_t launch_layernorm(const float* z, int M, int N, const float* gamma, c
                              float inv_out_scale, void* out, cudaStream_t s) {
     const int rows_per_block = 8;
     const unsigned grid = static_cast<unsigned>((static_cast<long long>(M) + rows_per_block - 1) / rows_per_block);
-    layernorm_kernel<<<grid, 32 * rows_per_block, 0, s>>>(z, M, N, gamma, beta, eps, kind, inv_out_scale, out);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(32 * rows_per_block);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // its set-up overlaps the previous kernel's end
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, layernorm_kernel, z, M, N, gamma, beta, eps, kind, inv_out_scale, out);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 size_t tiled_bytes(int K, long long M) {

@@ -111,10 +111,11 @@ def test_block_prune_rejects_bad_arguments(bsg):
 def test_attention_rejects_bad_arguments(bsg):
     """Shape, stride, scale, kind and pointer checks come before any CUDA
     call; batch = 0 is a no-op."""
-    def code(batch=2, seq=8, heads=12, head_dim=64, ld=2304, scale=0.05, qkv=16, out=16, kind=None, out_scale=1.0):
+    def code(batch=2, seq=8, heads=12, head_dim=64, ld=2304, scale=0.05, qkv=16, out=16, kind=None, out_scale=1.0,
+             flags=0):
         with pytest.raises(bsg.BsgemmError) as e:
             bsg.bsgemm_attention(qkv, batch, seq, heads, head_dim, ld, scale, out,
-                                 bsg.OUT_F32 if kind is None else kind, out_scale)
+                                 bsg.OUT_F32 if kind is None else kind, out_scale, 0, flags)
         return e.value.code
     assert code(head_dim=32) == bsg.ERR_UNSUPPORTED
     assert code(seq=bsg.ATTN_MAX_SEQ + 1) == bsg.ERR_UNSUPPORTED
@@ -132,6 +133,7 @@ def test_attention_rejects_bad_arguments(bsg):
     assert code(kind=bsg.OUT_I32) == bsg.ERR_INVALID
     assert code(kind=bsg.OUT_F32_GELU) == bsg.ERR_INVALID
     assert code(kind=bsg.OUT_I8, out_scale=0.0) == bsg.ERR_INVALID
+    assert code(flags=2) == bsg.ERR_INVALID                 # only BSGEMM_ACT_READY is defined
     assert code(qkv=0) == bsg.ERR_INVALID
     assert code(out=0) == bsg.ERR_INVALID
     assert code(qkv=24) == bsg.ERR_INVALID                  # not 16-byte aligned

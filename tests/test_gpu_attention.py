@@ -194,3 +194,26 @@ def test_attention_every_block_boundary(bsg):
         want = oracle.attention_f64(qkv, 0.05, 1, seq, heads=1, head_dim=HD)
         assert np.abs(got.astype(np.float64) - want).max() <= bound(qkv, 0.05, 1, seq, 1), seq
     assert bsg.bsgemm_attention_status() == 0
+
+
+def test_attention_act_ready_back_to_back(bsg):
+    """Independent batches launched back to back on one stream with
+    ACT_READY, as the bench times the kernel: each launch may read its qkv
+    while the previous launch still runs (programmatic dependent launch) and
+    writes its output only after it; every output matches the oracle."""
+    import torch
+    batch, seq, heads, scale = 2, 384, 12, 0.05
+    rng = np.random.default_rng(7500)
+    qkvs = [draw_qkv(rng, batch, seq, heads) for _ in range(4)]
+    dev = [torch.from_numpy(q).cuda() for q in qkvs]
+    outs = [torch.full((batch * seq, heads * HD), 1234.5, dtype=torch.float32, device="cuda") for _ in qkvs]
+    s = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    for rep in range(3):
+        for q, o in zip(dev, outs):
+            bsg.attention(q, batch, seq, heads, scale, bsg.OUT_F32, out=o, stream=s, flags=bsg.ACT_READY)
+    torch.cuda.synchronize()
+    for q, o in zip(qkvs, outs):
+        want = oracle.attention_f64(q, scale, batch, seq, heads=heads, head_dim=HD, threads=8)
+        assert np.abs(o.cpu().numpy().astype(np.float64) - want).max() <= bound(q, scale, batch, seq, heads)
+    assert bsg.bsgemm_attention_status() == 0
