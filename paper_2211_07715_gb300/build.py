@@ -1,6 +1,6 @@
 """Compile libbsgemm.so in-tree with nvcc for sm_103a (GB300).
 
-Five translation units (layer kernels, pruning kernel, attention kernel, int8 peak probes, host ABI) compile in parallel, then link
+Six translation units (layer kernels, pruning kernel, attention kernel, sparse tensor-core kernel, int8 peak probes, host ABI) compile in parallel, then link
 into one shared library with the CUDA runtime linked statically, so the
 library needs nothing but the NVIDIA driver at run time.
 """
@@ -16,7 +16,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libbsgemm.so")
-SOURCES = ["bsgemm_kernel.cu", "bsgemm_prune.cu", "bsgemm_attention.cu", "bsgemm_peaks.cu", "bsgemm_api.cpp"]
+SOURCES = ["bsgemm_kernel.cu", "bsgemm_prune.cu", "bsgemm_attention.cu", "bsgemm_sparse24.cu", "bsgemm_peaks.cu",
+           "bsgemm_api.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -28,6 +28,11 @@ struct bsgemm_ctx {
     size_t arena_bytes = 0;
     std::vector<int32_t> cost;  // schedule prefix cost of the row groups [ngroups + 1]
     bsg::DeviceWeights w{};
+    // 2:4 weights with N and K multiples of 128: the sparse tensor cores'
+    // operands (launch_sparse24), in their own allocation; NULL otherwise
+    void* tc_arena = nullptr;
+    const unsigned char* tc_aimg = nullptr;
+    const uint32_t* tc_meta = nullptr;
     std::mutex sched_mu;        // guards the cached schedule of the last token count
     long long sched_m = -1;
     int sched_grid = 0;
@@ -56,6 +61,19 @@ std::string cuda_msg(const char* what, cudaError_t e) {
 }
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// IEEE binary16 bits of an int8 value (exact: |v| <= 128 needs at most 8
+// significant bits).
+uint16_t f16_of_int(int8_t v8) {
+    int v = v8;
+    if (v == 0) return 0;
+    const uint16_t sign = v < 0 ? 0x8000u : 0u;
+    unsigned a = static_cast<unsigned>(v < 0 ? -v : v);
+    int ex = 0;
+    while ((a >> ex) > 1) ++ex;                      // a = 1.f x 2^ex
+    const unsigned mant = (a << (10 - ex)) & 0x3FFu;  // 10 fraction bits
+    return static_cast<uint16_t>(sign | ((ex + 15) << 10) | mant);
+}
 
 const int kZeroStatus = 0;
 
@@ -631,7 +649,69 @@ bsgemm_t bsgemm_create_2to4(int N, int K, const int8_t* values, const uint8_t* i
         indices[r + 1] = static_cast<int32_t>(cols.size());
     }
     indices.insert(indices.end(), cols.begin(), cols.end());
-    return bsgemm_create(N, K, BSGEMM_BLOCK, indices.data(), vals.empty() ? nullptr : vals.data(), scales, bias);
+    bsgemm_t h = bsgemm_create(N, K, BSGEMM_BLOCK, indices.data(), vals.empty() ? nullptr : vals.data(), scales, bias);
+    if (!h || N % 128 != 0 || K % 128 != 0 || K > 4096) return h;
+
+    // The sparse tensor cores' operands.  Per (channel tile ct, stage s of
+    // 128 columns): the stored values of rows 128 ct .. + 127 and columns
+    // 128 s .. + 127 as the shared-memory image the MMA reads (row m: 64 f16,
+    // element e = 2 (group - 32 s) + t in 16-byte chunk e / 8, placed at chunk
+    // (e / 8) ^ (m % 8) of the row's 128 bytes); and the metadata of its 4
+    // MMAs (MMA i: columns 128 s + 32 i .. + 31, 8 groups): row m's word has
+    // nibble g = first position | second position << 2 of group 8 i + g, and
+    // within every 16 rows the tensor memory lanes hold (lane r < 8: row r's
+    // groups 0-3 | row r + 8's groups 0-3; lane 8 + r: row r's groups 4-7 |
+    // row r + 8's groups 4-7) -- the layout tcgen05.mma.sp reads.
+    const int ntile = N / 128, nst = K / 128;
+    std::vector<uint16_t> aimg(static_cast<size_t>(ntile) * nst * (bsg::kTc24AImage / 2), 0);
+    std::vector<uint32_t> meta(static_cast<size_t>(ntile) * nst * 128 * 4, 0);
+    for (int ct = 0; ct < ntile; ++ct) {
+        for (int st = 0; st < nst; ++st) {
+            uint16_t* img = &aimg[(static_cast<size_t>(ct) * nst + st) * (bsg::kTc24AImage / 2)];
+            uint32_t word[4][128];
+            for (int m = 0; m < 128; ++m) {
+                const int n = 128 * ct + m;
+                for (int e = 0; e < 64; ++e) {
+                    const size_t p = static_cast<size_t>(n) * half + 64 * st + e;
+                    const int c = e / 8;
+                    img[(128 * m + 16 * (c ^ (m % 8))) / 2 + e % 8] = f16_of_int(values[p]);
+                }
+                for (int i = 0; i < 4; ++i) {
+                    uint32_t w = 0;
+                    for (int g = 0; g < 8; ++g) {
+                        const size_t p = static_cast<size_t>(n) * half + 64 * st + 16 * i + 2 * g;
+                        w |= static_cast<uint32_t>(idx[p] | (idx[p + 1] << 2)) << (4 * g);
+                    }
+                    word[i][m] = w;
+                }
+            }
+            uint32_t* mt = &meta[(static_cast<size_t>(ct) * nst + st) * 128 * 4];
+            for (int i = 0; i < 4; ++i) {
+                for (int b16 = 0; b16 < 128; b16 += 16) {
+                    for (int r = 0; r < 8; ++r) {
+                        const uint32_t lo = word[i][b16 + r], hi = word[i][b16 + 8 + r];
+                        mt[4 * (b16 + r) + i] = (lo & 0xFFFFu) | (hi << 16);
+                        mt[4 * (b16 + 8 + r) + i] = (lo >> 16) | (hi & 0xFFFF0000u);
+                    }
+                }
+            }
+        }
+    }
+    const size_t abytes = aimg.size() * sizeof(uint16_t), mbytes = meta.size() * sizeof(uint32_t);
+    void* arena = nullptr;
+    cudaError_t e = cudaMalloc(&arena, abytes + mbytes);
+    if (e == cudaSuccess) e = cudaMemcpy(arena, aimg.data(), abytes, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(static_cast<char*>(arena) + abytes, meta.data(), mbytes, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        if (arena) cudaFree(arena);
+        bsgemm_destroy(h);
+        fail(BSGEMM_ERR_CUDA, cuda_msg("sparse tensor-core operands", e));
+        return nullptr;
+    }
+    h->tc_arena = arena;
+    h->tc_aimg = static_cast<const unsigned char*>(arena);
+    h->tc_meta = reinterpret_cast<const uint32_t*>(static_cast<const char*>(arena) + abytes);
+    return h;
 }
 
 // mode: 0 = gather from act (no scratch), 1 = relayout act into workspace
@@ -706,6 +786,14 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
     a.skip_copy = (g_test_hooks.load() & BSGEMM_TEST_SKIP_TILE_COPY) != 0;
     a.wait_limit = a.skip_copy ? 64u : 0u;
+    // 2:4 weights on the sparse tensor cores: row-major act, any kind but the residual
+    if (h->tc_aimg && (mode == 0 || mode == 1) && epi.kind != BSGEMM_OUT_F32_RESID &&
+        (reinterpret_cast<uintptr_t>(act) & 15u) == 0) {
+        e = bsg::launch_sparse24(act, M, h->w.N, h->w.K, h->tc_aimg, h->tc_meta, h->w.scale, h->w.bias, out, epi.kind,
+                                 inv, (epi.flags & BSGEMM_ACT_READY) != 0, h->w.status, s);
+        if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("sparse tensor-core kernel launch", e));
+        return BSGEMM_OK;
+    }
     const long long ntiles = (static_cast<long long>(M) + bsg::kTile - 1) / bsg::kTile;
     const long long upt = h->w.ngroups;  // units per token tile
     long long cap = static_cast<long long>(h->num_sms) * h->ctas_per_sm;
@@ -958,6 +1046,7 @@ int bsgemm_device_status(bsgemm_t h, int clear) {
 void bsgemm_destroy(bsgemm_t h) {
     if (!h) return;
     if (h->arena) cudaFree(h->arena);
+    if (h->tc_arena) cudaFree(h->tc_arena);
     delete h;
 }
 

@@ -1,0 +1,298 @@
+// Weights with 2:4 structured sparsity along K on the sparse tensor cores.
+//
+// A 2:4 weight (two values in every group of 4 consecutive input columns of
+// a row; Sec. 1 cites the pattern as the one sparse tensor cores take) is a
+// dense contraction of its stored half, so here it runs on the
+// fifth-generation tensor cores' sparse MMA (`tcgen05.mma.sp ... kind::f16`):
+// out^T = W x^T with the weight as the sparse A operand (M = 128 output
+// channels a tile, its stored values as f16 plus 2-bit positions) and the
+// token tile as the dense B operand (N = 128 tokens).  int8 values are exact
+// in f16 and their products (|v x| <= 127 * 128) exact in fp32; every
+// partial sum of at most 1024 products stays below 2^24, so each chunk of
+// 2048 input columns (1024 stored values a row) accumulates exactly in its
+// own fp32 accumulator in tensor memory, and the chunks are added in int32
+// by the epilogue: the int32 result of the definition, bit for bit.
+//
+// Per CTA (128 channels x 128 tokens, all of K in stages of 128 columns):
+//   * the create step lays out every (channel tile, stage) of the weight as
+//     the 16 KB shared-memory image of its stored values (128 rows of 64 f16,
+//     the 128-byte swizzle) and the stage's 4 x 128 metadata words (one
+//     tensor-memory column per MMA); one thread of the MMA warp brings the
+//     image in with a bulk copy;
+//   * the 4 converter warps (thread t = token row t and tensor-memory lane t)
+//     copy the stage's int8 activations with cp.async, widen them to f16 into
+//     the B image (two 128-row x 64-column sub-tiles, 128-byte swizzle), and
+//     store the stage's metadata into tensor memory;
+//   * one thread of the MMA warp issues the stage's 4 MMAs (K = 32 each)
+//     into the chunk's accumulator (tensor-memory columns 0-127 and
+//     128-255) and commits them to the stage's "empty" barrier; two stages
+//     are in flight; each MMA's metadata column sits on a 32-column boundary
+//     (columns 256 + 32 j);
+//   * the epilogue (the converter warps again; lane m = channel m of the
+//     tile): the chunks' accumulators read from tensor memory 32 tokens at a
+//     time, converted to int32 exactly, added, and the fused epilogue
+//     (dequantise + bias, GELU, requantise) stored as out[token][channel].
+// Every wait is bounded; a wait that gives up sets the handle's status word.
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "bsgemm.h"
+#include "bsgemm_device.cuh"
+#include "bsgemm_internal.h"
+#include "bsgemm_tcgen05.cuh"
+
+namespace bsg {
+namespace {
+
+constexpr int kTcThreads = 160;            // 4 converter / epilogue warps + 1 MMA warp
+constexpr uint32_t kAImg = kTc24AImage;    // bytes of a stage's weight image
+constexpr uint32_t kXImg = 128 * 128;      // a stage's int8 token tile (128 tokens x 128 columns)
+constexpr uint32_t kBImg = 2 * 128 * 128;  // its f16 form: two 128 x 64 sub-tiles
+constexpr uint32_t kStageBytes = kAImg + kXImg + kBImg;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColMeta = 256;         // metadata of MMA i of stage buffer b at column 256 + 32 (4 b + i)
+
+// Instruction descriptor of the sparse MMA: f16 A and B, fp32 accumulator,
+// both K-major, N = 128, M = 128, sparsity flag (bit 2).
+constexpr uint32_t kIdescSp = f16_idesc(128, 128, false) | (1u << 2);
+
+__device__ __forceinline__ void mma_sp(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t meta, uint32_t acc) {
+    asm volatile("{\n .reg .pred p;\n setp.ne.u32 p, %5, 0;\n"
+                 " tcgen05.mma.sp.cta_group::1.kind::f16 [%0], %1, %2, [%3], %4, p;\n}\n"
+                 ::"r"(d), "l"(adesc), "l"(bdesc), "r"(meta), "r"(kIdescSp), "r"(acc) : "memory");
+}
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+__device__ __forceinline__ void arrive(uint32_t bar) {
+    asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}\n" ::"r"(bar) : "memory");
+}
+// Two int8 values (bytes sel of u = w ^ 0x80808080) as an exact f16 pair:
+// 0x64uu is the f16 1024 + uu, minus 1152 = the value.
+__device__ __forceinline__ uint32_t s8x2_f16x2(uint32_t u, uint32_t sel) {
+    const uint32_t b = __byte_perm(u, 0x64646464u, sel);
+    uint32_t r;
+    asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(b), "r"(0x64806480u));
+    return r;
+}
+
+template <int KIND>
+__global__ void __launch_bounds__(kTcThreads, 1)
+sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigned char* __restrict__ aimg,
+                const uint32_t* __restrict__ meta, const float* __restrict__ scale, const float* __restrict__ bias,
+                void* __restrict__ out, float inv_out_scale, int act_ready, unsigned wait_limit, int* status) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* sm =
+        reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    __shared__ __align__(8) unsigned long long s_bar[7];  // a_full[2], b_full[2], empty[2], done
+    __shared__ uint32_t s_tmem;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const bool mma_warp = warp == 4;
+    const int ct = blockIdx.x;                    // channel tile
+    const long long t0 = static_cast<long long>(blockIdx.y) * 128;  // first token
+    const int nst = K / 128;                      // stages
+    const uint32_t bar = smem_addr(&s_bar[0]);
+    const uint32_t a_full = bar, b_full = bar + 16, empty = bar + 32, done = bar + 48;
+    auto stage_base = [&](int b) { return sm + static_cast<uint32_t>(b) * kStageBytes; };
+
+    griddep_launch_dependents();
+    if (tid == kTcThreads - 32) {
+        mbar_init(a_full, 1);
+        mbar_init(a_full + 8, 1);
+        mbar_init(b_full, 128);
+        mbar_init(b_full + 8, 128);
+        mbar_init(empty, 1);
+        mbar_init(empty + 8, 1);
+        mbar_init(done, 1);
+    }
+    if (mma_warp) tmem_alloc(smem_addr(&s_tmem), kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = s_tmem;
+    bool ok = true;
+
+    if (mma_warp) {
+        if (tid == kTcThreads - 32) {
+            // the weight images of stages 0 and 1, then stage s + 1's once stage
+            // s - 1's MMAs (issued before stage s's) have read its buffer
+            auto load_a = [&](int s) {
+                const uint32_t b = static_cast<uint32_t>(s & 1);
+                mbar_arrive_expect_tx(a_full + 8u * b, kAImg);
+                bulk_g2s(smem_addr(stage_base(s & 1)), aimg + (static_cast<size_t>(ct) * nst + s) * kAImg, kAImg,
+                         a_full + 8u * b);
+            };
+            load_a(0);
+            if (nst > 1) load_a(1);
+            for (int s = 0; s < nst; ++s) {
+                const uint32_t b = static_cast<uint32_t>(s & 1), ph = static_cast<uint32_t>(s >> 1) & 1u;
+                ok &= mbar_wait(a_full + 8u * b, ph, wait_limit);
+                ok &= mbar_wait(b_full + 8u * b, ph, wait_limit);
+                tc_fence_after();
+                const uint32_t as = smem_addr(stage_base(s & 1)), bs = as + kAImg + kXImg;
+                const uint32_t d = tm + 128u * static_cast<uint32_t>(s / 16);  // the chunk's accumulator (two at most)
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    mma_sp(d, sw128_desc(as + 32u * i, 16, 1024), sw128_desc(bs + 16384u * (i >> 1) + 64u * (i & 1), 16, 1024),
+                           tm + kColMeta + 32u * (4u * b + static_cast<uint32_t>(i)), (s % 16 != 0 || i > 0) ? 1u : 0u);
+                tc_commit(empty + 8u * b);
+                if (s >= 1 && s + 1 < nst) {
+                    ok &= mbar_wait(empty + 8u * (b ^ 1u), static_cast<uint32_t>((s - 1) >> 1) & 1u, wait_limit);
+                    tc_fence_after();
+                    load_a(s + 1);
+                }
+            }
+            tc_commit(done);
+        }
+        __syncwarp();
+    } else {
+        // converter warps: thread tid = token row tid of the tile
+        if (!act_ready) griddep_wait();
+        const long long tok = t0 + tid;
+        const int8_t* xrow = x + (tok < M ? tok : 0) * static_cast<long long>(K);
+        const uint32_t src_bytes = tok < M ? 16u : 0u;
+        // the stage's 128 columns of this thread's token: 8 copies of 16 bytes,
+        // chunk c of row tid at tid * 128 + (c ^ (tid % 8)) * 16 (conflict-free
+        // reads by 8 consecutive threads)
+        auto copy_x = [&](int s) {
+            const uint32_t xs = smem_addr(stage_base(s & 1) + kAImg) + 128u * static_cast<uint32_t>(tid);
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                cp_async16(xs + ((static_cast<uint32_t>(c) ^ (tid & 7)) << 4), xrow + 128 * s + 16 * c, src_bytes);
+            cp_async_commit();
+        };
+        copy_x(0);
+        for (int s = 0; s < nst; ++s) {
+            const uint32_t b = static_cast<uint32_t>(s & 1);
+            if (s + 1 < nst) {
+                copy_x(s + 1);
+                cp_async_wait<1>();
+            } else {
+                cp_async_wait<0>();
+            }
+            if (s >= 2) {  // stage s - 2's MMAs have read this buffer's B image and metadata
+                ok &= mbar_wait(empty + 8u * b, static_cast<uint32_t>((s - 2) >> 1) & 1u, wait_limit);
+                tc_fence_after();
+            }
+            unsigned char* st = stage_base(s & 1);
+            const unsigned char* xs = st + kAImg + 128u * static_cast<uint32_t>(tid);
+            unsigned char* bs = st + kAImg + kXImg;
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const int4 v = *reinterpret_cast<const int4*>(xs + ((static_cast<uint32_t>(c) ^ (tid & 7)) << 4));
+                const uint32_t w[4] = {static_cast<uint32_t>(v.x) ^ 0x80808080u, static_cast<uint32_t>(v.y) ^ 0x80808080u,
+                                       static_cast<uint32_t>(v.z) ^ 0x80808080u, static_cast<uint32_t>(v.w) ^ 0x80808080u};
+                uint32_t o[8];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    o[2 * q] = s8x2_f16x2(w[q], 0x4140u);
+                    o[2 * q + 1] = s8x2_f16x2(w[q], 0x4342u);
+                }
+                // columns 16c .. 16c + 15 = f16 chunks 2c, 2c + 1 of the row: sub-tile
+                // (2c) / 8, chunk (2c) % 8 of its 128-byte row, swizzled
+                unsigned char* row = bs + 16384u * static_cast<uint32_t>(c >> 2) + 128u * static_cast<uint32_t>(tid);
+                const uint32_t c0 = static_cast<uint32_t>((2 * c) & 7), c1 = c0 + 1;
+                *reinterpret_cast<uint4*>(row + ((c0 ^ (tid & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+                *reinterpret_cast<uint4*>(row + ((c1 ^ (tid & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
+            }
+            fence_proxy_async();  // the B image, for the tensor cores
+            // the stage's metadata: word tid of each of its 4 MMAs into this lane,
+            // one column each (32-column aligned)
+            const uint4 mv = __ldg(reinterpret_cast<const uint4*>(meta + ((static_cast<size_t>(ct) * nst + s) * 128 + tid) * 4));
+            const uint32_t mw[4] = {mv.x, mv.y, mv.z, mv.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};\n"
+                             ::"r"(tm + (static_cast<uint32_t>(32 * warp) << 16) + kColMeta + 32u * (4u * b + i)), "r"(mw[i])
+                             : "memory");
+            tmem_wait_st();
+            tc_fence_before();
+            arrive(b_full + 8u * b);
+        }
+
+        // epilogue: lane tid = channel ch of the tile
+        ok &= mbar_wait(done, 0, wait_limit);
+        __syncwarp();
+        tc_fence_after();
+        const int ch = ct * 128 + tid;
+        const float sc = scale[ch], bi = bias[ch];
+        const int nchunks = (nst + 15) / 16;
+        griddep_wait();  // outputs after the preceding kernel
+        for (int n0 = 0; n0 < 128; n0 += 32) {
+            int acc[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) acc[j] = 0;
+            for (int c = 0; c < nchunks; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tm + (static_cast<uint32_t>(32 * warp) << 16) + 128u * static_cast<uint32_t>(c) +
+                              static_cast<uint32_t>(n0), v);
+                tmem_wait_ld(v);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) acc[j] += __float2int_rn(__uint_as_float(v[j]));  // an exact integer
+            }
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                const long long t = t0 + n0 + j;
+                if (t >= M) break;
+                const size_t o = static_cast<size_t>(t) * N + ch;
+                if (KIND == 0) {
+                    static_cast<int32_t*>(out)[o] = acc[j];
+                } else if (KIND == 1 || KIND == 2) {
+                    static_cast<float*>(out)[o] = epilogue_value<KIND>(acc[j], sc, bi);
+                } else {
+                    const int qv = __float2int_rn(__fmul_rn(epilogue_value<KIND>(acc[j], sc, bi), inv_out_scale));
+                    static_cast<int8_t*>(out)[o] = static_cast<int8_t>(qv > 127 ? 127 : (qv < -128 ? -128 : qv));
+                }
+            }
+        }
+    }
+    if (!ok) {
+        griddep_wait();
+        atomicOr(status, kStatusTimeout);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (mma_warp) tmem_dealloc(tm, kTmemCols);
+}
+
+}  // namespace
+
+cudaError_t launch_sparse24(const int8_t* x, int M, int N, int K, const unsigned char* aimg, const uint32_t* meta,
+                            const float* scale, const float* bias, void* out, int kind, float inv_out_scale,
+                            bool act_ready, int* status, cudaStream_t s) {
+    const void* fn = nullptr;
+    switch (kind) {
+    case 0: fn = reinterpret_cast<const void*>(&sparse24_kernel<0>); break;
+    case 1: fn = reinterpret_cast<const void*>(&sparse24_kernel<1>); break;
+    case 2: fn = reinterpret_cast<const void*>(&sparse24_kernel<2>); break;
+    case 3: fn = reinterpret_cast<const void*>(&sparse24_kernel<3>); break;
+    case 4: fn = reinterpret_cast<const void*>(&sparse24_kernel<4>); break;
+    default: return cudaErrorNotSupported;
+    }
+    const int smem = static_cast<int>(2 * kStageBytes + 1024);
+    cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(N / 128), static_cast<unsigned>((M + 127) / 128));
+    cfg.blockDim = dim3(kTcThreads);
+    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const unsigned wl = kWaitLimit;
+    const int ar = act_ready ? 1 : 0;
+    void* args[] = {const_cast<int8_t**>(&x), &M, &N, &K, const_cast<unsigned char**>(&aimg), const_cast<uint32_t**>(&meta),
+                    const_cast<float**>(&scale), const_cast<float**>(&bias), &out, &inv_out_scale,
+                    const_cast<int*>(&ar), const_cast<unsigned*>(&wl), &status};
+    e = cudaLaunchKernelExC(&cfg, fn, args);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
+}  // namespace bsg

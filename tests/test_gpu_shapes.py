@@ -5,8 +5,10 @@ oracle's linear on the oracle's own decompression of the same arrays
     natively by the kernel's 1 x 4 form (bsgemm_create_1x4): every kind but
     the residual, both staging paths, ragged K (relayout path), K = 4,
     N not a multiple of 4, rows without blocks, one token;
-  * 2:4-sparse weights (bsgemm_create_2to4: the 4 x 1 blocks that hold
-    them)."""
+  * 2:4-sparse weights (bsgemm_create_2to4): N and K multiples of 128 on
+    the sparse tensor cores (tcgen05.mma.sp, exact fp32 chunks of 2048
+    columns added in int32), other shapes as the 4 x 1 blocks that hold
+    them."""
 import numpy as np
 import pytest
 
@@ -74,6 +76,39 @@ def test_2to4_through_the_layer(bsg, n_out, k_in, m):
     for kind in KINDS:
         want = oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
         check(gpu_run(lin, x, kind, 0.05), want, kind, f"2:4 kind {kind}")
+    lin.close()
+
+
+@pytest.mark.parametrize("n_out,k_in,m", [(128, 128, 1), (256, 2048, 130), (768, 3072, 300), (128, 2176, 64),
+                                          (384, 1024, 257)])
+def test_2to4_on_the_sparse_tensor_cores(bsg, n_out, k_in, m):
+    """Every kind, ragged token tiles, one and two exact accumulator chunks
+    (a chunk holds 2048 columns), a chunk boundary at the last stage."""
+    rng = synth.rng_for(8200 + n_out + k_in + m)
+    wt = synth.draw_weight_2to4(rng, n_out, k_in)
+    w = oracle.sparse2to4_to_dense(wt.values, wt.idx)
+    lin = bsg.SparseInt8Linear.from_2to4(wt.values, wt.idx, wt.scales, wt.bias)
+    x = synth.draw_x(rng, m, k_in, "u127")
+    for kind in KINDS:
+        want = oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
+        check(gpu_run(lin, x, kind, 0.05), want, kind, f"2:4 tensor cores kind {kind}")
+    lin.close()
+
+
+def test_2to4_tensor_cores_at_the_fp32_limit(bsg):
+    """Every stored value -128 and every activation -128: each product is
+    2^14 and a chunk's 1024 of them sum to exactly 2^24, the largest partial
+    sum the exact fp32 accumulation has to hold; then mixed extremes."""
+    n_out, k_in, m = 128, 3072, 70
+    rng = synth.rng_for(8300)
+    wt = synth.draw_weight_2to4(rng, n_out, k_in)
+    values = np.full_like(wt.values, -128)
+    w = oracle.sparse2to4_to_dense(values, wt.idx)
+    lin = bsg.SparseInt8Linear.from_2to4(values, wt.idx, wt.scales, wt.bias)
+    for x in (np.full((m, k_in), -128, dtype=np.int8),
+              rng.choice(np.array([-128, 127], dtype=np.int8), size=(m, k_in))):
+        want = oracle.linear(x, w, wt.scales, wt.bias, synth.I32, threads=8)
+        check(gpu_run(lin, x, synth.I32, 1.0), want, synth.I32, "2:4 extremes")
     lin.close()
 
 
