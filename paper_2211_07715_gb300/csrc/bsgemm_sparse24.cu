@@ -19,18 +19,19 @@
 //     the 128-byte swizzle) and the stage's 4 x 128 metadata words (one
 //     tensor-memory column per MMA); one thread of the MMA warp brings the
 //     image in with a bulk copy;
-//   * the 4 converter warps (thread t = token row t and tensor-memory lane t)
+//   * the 8 converter warps (two threads a token row, one per 64 columns)
 //     copy the stage's int8 activations with cp.async, widen them to f16 into
 //     the B image (two 128-row x 64-column sub-tiles, 128-byte swizzle), and
-//     store the stage's metadata into tensor memory;
+//     store the stage's metadata into tensor memory (warps 0-3: lane r =
+//     weight row r);
 //   * one thread of the MMA warp issues the stage's 4 MMAs (K = 32 each)
 //     into the chunk's accumulator (tensor-memory columns 0-127 and
 //     128-255) and commits them to the stage's "empty" barrier; two stages
 //     are in flight; each MMA's metadata column sits on a 32-column boundary
 //     (columns 256 + 32 j);
 //   * the epilogue (the converter warps again; lane m = channel m of the
-//     tile): the chunks' accumulators read from tensor memory 32 tokens at a
-//     time, converted to int32 exactly, added, and the fused epilogue
+//     tile, warps w and w + 4 the two halves of the tokens): the chunks'
+//     accumulators read from tensor memory 32 tokens at a time, converted to int32 exactly, added, and the fused epilogue
 //     (dequantise + bias, GELU, requantise) stored as out[token][channel].
 // Every wait is bounded; a wait that gives up sets the handle's status word.
 
@@ -45,7 +46,7 @@
 namespace bsg {
 namespace {
 
-constexpr int kTcThreads = 160;            // 4 converter / epilogue warps + 1 MMA warp
+constexpr int kTcThreads = 288;            // 8 converter / epilogue warps + 1 MMA warp
 constexpr uint32_t kAImg = kTc24AImage;    // bytes of a stage's weight image
 constexpr uint32_t kXImg = 128 * 128;      // a stage's int8 token tile (128 tokens x 128 columns)
 constexpr uint32_t kBImg = 2 * 128 * 128;  // its f16 form: two 128 x 64 sub-tiles
@@ -91,7 +92,7 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
     __shared__ __align__(8) unsigned long long s_bar[7];  // a_full[2], b_full[2], empty[2], done
     __shared__ uint32_t s_tmem;
     const int tid = threadIdx.x, warp = tid >> 5;
-    const bool mma_warp = warp == 4;
+    const bool mma_warp = warp == 8;
     const int ct = blockIdx.x;                    // channel tile
     const long long t0 = static_cast<long long>(blockIdx.y) * 128;  // first token
     const int nst = K / 128;                      // stages
@@ -103,8 +104,8 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
     if (tid == kTcThreads - 32) {
         mbar_init(a_full, 1);
         mbar_init(a_full + 8, 1);
-        mbar_init(b_full, 128);
-        mbar_init(b_full + 8, 128);
+        mbar_init(b_full, 256);
+        mbar_init(b_full + 8, 256);
         mbar_init(empty, 1);
         mbar_init(empty + 8, 1);
         mbar_init(done, 1);
@@ -150,19 +151,21 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
         }
         __syncwarp();
     } else {
-        // converter warps: thread tid = token row tid of the tile
+        // converter warps: thread tid takes token row r = tid % 128 of the tile
+        // and its columns 64 h .. 64 h + 63 of each stage, h = tid / 128 (f16
+        // sub-tile h of the B image)
+        const int r = tid & 127, h = tid >> 7;
         if (!act_ready) griddep_wait();
-        const long long tok = t0 + tid;
-        const int8_t* xrow = x + (tok < M ? tok : 0) * static_cast<long long>(K);
+        const long long tok = t0 + r;
+        const int8_t* xrow = x + (tok < M ? tok : 0) * static_cast<long long>(K) + 64 * h;
         const uint32_t src_bytes = tok < M ? 16u : 0u;
-        // the stage's 128 columns of this thread's token: 8 copies of 16 bytes,
-        // chunk c of row tid at tid * 128 + (c ^ (tid % 8)) * 16 (conflict-free
-        // reads by 8 consecutive threads)
+        // 4 copies of 16 bytes: chunk c (= 4 h + cc) of row r at r * 128 + (c ^
+        // (r % 8)) * 16 (conflict-free reads by 8 consecutive threads)
         auto copy_x = [&](int s) {
-            const uint32_t xs = smem_addr(stage_base(s & 1) + kAImg) + 128u * static_cast<uint32_t>(tid);
+            const uint32_t xs = smem_addr(stage_base(s & 1) + kAImg) + 128u * static_cast<uint32_t>(r);
 #pragma unroll
-            for (int c = 0; c < 8; ++c)
-                cp_async16(xs + ((static_cast<uint32_t>(c) ^ (tid & 7)) << 4), xrow + 128 * s + 16 * c, src_bytes);
+            for (int cc = 0; cc < 4; ++cc)
+                cp_async16(xs + ((static_cast<uint32_t>(4 * h + cc) ^ (r & 7)) << 4), xrow + 128 * s + 16 * cc, src_bytes);
             cp_async_commit();
         };
         copy_x(0);
@@ -179,11 +182,12 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
                 tc_fence_after();
             }
             unsigned char* st = stage_base(s & 1);
-            const unsigned char* xs = st + kAImg + 128u * static_cast<uint32_t>(tid);
-            unsigned char* bs = st + kAImg + kXImg;
+            const unsigned char* xs = st + kAImg + 128u * static_cast<uint32_t>(r);
+            unsigned char* row = st + kAImg + kXImg + 16384u * static_cast<uint32_t>(h) + 128u * static_cast<uint32_t>(r);
 #pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                const int4 v = *reinterpret_cast<const int4*>(xs + ((static_cast<uint32_t>(c) ^ (tid & 7)) << 4));
+            for (int cc = 0; cc < 4; ++cc) {
+                const int c = 4 * h + cc;
+                const int4 v = *reinterpret_cast<const int4*>(xs + ((static_cast<uint32_t>(c) ^ (r & 7)) << 4));
                 const uint32_t w[4] = {static_cast<uint32_t>(v.x) ^ 0x80808080u, static_cast<uint32_t>(v.y) ^ 0x80808080u,
                                        static_cast<uint32_t>(v.z) ^ 0x80808080u, static_cast<uint32_t>(v.w) ^ 0x80808080u};
                 uint32_t o[8];
@@ -192,43 +196,45 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
                     o[2 * q] = s8x2_f16x2(w[q], 0x4140u);
                     o[2 * q + 1] = s8x2_f16x2(w[q], 0x4342u);
                 }
-                // columns 16c .. 16c + 15 = f16 chunks 2c, 2c + 1 of the row: sub-tile
-                // (2c) / 8, chunk (2c) % 8 of its 128-byte row, swizzled
-                unsigned char* row = bs + 16384u * static_cast<uint32_t>(c >> 2) + 128u * static_cast<uint32_t>(tid);
-                const uint32_t c0 = static_cast<uint32_t>((2 * c) & 7), c1 = c0 + 1;
-                *reinterpret_cast<uint4*>(row + ((c0 ^ (tid & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
-                *reinterpret_cast<uint4*>(row + ((c1 ^ (tid & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
+                // columns 16 c .. + 15 = f16 chunks 2 cc, 2 cc + 1 of the row of sub-tile h, swizzled
+                const uint32_t c0 = static_cast<uint32_t>(2 * cc), c1 = c0 + 1;
+                *reinterpret_cast<uint4*>(row + ((c0 ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+                *reinterpret_cast<uint4*>(row + ((c1 ^ (r & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
             }
             fence_proxy_async();  // the B image, for the tensor cores
-            // the stage's metadata: word tid of each of its 4 MMAs into this lane,
-            // one column each (32-column aligned)
-            const uint4 mv = __ldg(reinterpret_cast<const uint4*>(meta + ((static_cast<size_t>(ct) * nst + s) * 128 + tid) * 4));
-            const uint32_t mw[4] = {mv.x, mv.y, mv.z, mv.w};
+            if (h == 0) {
+                // the stage's metadata: word r of each of its 4 MMAs into lane r, one
+                // column each (32-column aligned)
+                const uint4 mv =
+                    __ldg(reinterpret_cast<const uint4*>(meta + ((static_cast<size_t>(ct) * nst + s) * 128 + r) * 4));
+                const uint32_t mw[4] = {mv.x, mv.y, mv.z, mv.w};
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
-                asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};\n"
-                             ::"r"(tm + (static_cast<uint32_t>(32 * warp) << 16) + kColMeta + 32u * (4u * b + i)), "r"(mw[i])
-                             : "memory");
-            tmem_wait_st();
+                for (int i = 0; i < 4; ++i)
+                    asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};\n"
+                                 ::"r"(tm + (static_cast<uint32_t>(32 * warp) << 16) + kColMeta + 32u * (4u * b + i)),
+                                   "r"(mw[i])
+                                 : "memory");
+                tmem_wait_st();
+            }
             tc_fence_before();
             arrive(b_full + 8u * b);
         }
 
-        // epilogue: lane tid = channel ch of the tile
+        // epilogue: lane r = channel ch of the tile, tokens 64 h .. 64 h + 63
         ok &= mbar_wait(done, 0, wait_limit);
         __syncwarp();
         tc_fence_after();
-        const int ch = ct * 128 + tid;
+        const int ch = ct * 128 + r;
         const float sc = scale[ch], bi = bias[ch];
         const int nchunks = (nst + 15) / 16;
         griddep_wait();  // outputs after the preceding kernel
-        for (int n0 = 0; n0 < 128; n0 += 32) {
+        for (int n0 = 64 * h; n0 < 64 * h + 64; n0 += 32) {
             int acc[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j) acc[j] = 0;
             for (int c = 0; c < nchunks; ++c) {
                 uint32_t v[32];
-                tmem_ld32(tm + (static_cast<uint32_t>(32 * warp) << 16) + 128u * static_cast<uint32_t>(c) +
+                tmem_ld32(tm + (static_cast<uint32_t>(32 * (warp & 3)) << 16) + 128u * static_cast<uint32_t>(c) +
                               static_cast<uint32_t>(n0), v);
                 tmem_wait_ld(v);
 #pragma unroll
