@@ -584,8 +584,11 @@ def run_shapes(args) -> dict:
     """Other block shapes on the FFN2 shape (768 <- 3072, M = 4096): a
     weight sparse in 1 x 4 blocks at 90%, run natively by the kernel's 1 x 4
     form and, for comparison, as the 4 x 1 blocks that hold it; and a 2:4
-    weight (run as its 4 x 1 blocks).  value = effective TOPS of the useful
-    multiply-adds (2 ops each) of the native 1 x 4 path."""
+    weight, run on the sparse tensor cores (tcgen05.mma.sp, its roofline
+    the measured dense bf16/f16 rate: the sparse MMA does the stored half
+    at the dense rate) and, for comparison, as the 4 x 1 blocks that hold
+    it.  value = effective TOPS of the useful multiply-adds (2 ops each) of
+    the native 1 x 4 path."""
     import torch
     import paper_2211_07715_gb300 as bsg
 
@@ -616,7 +619,24 @@ def run_shapes(args) -> dict:
     lin.close()
     w24 = synth.draw_weight_2to4(rng, n_out, k_in)
     useful24 = 2.0 * m * n_out * k_in / 2
+    tensor_peak = 1903.9
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            tensor_peak = float(json.load(f).get("bf16_tflops", tensor_peak))
+    except (OSError, ValueError):
+        pass
     lin = bsg.SparseInt8Linear.from_2to4(w24.values, w24.idx, w24.scales, w24.bias)
+    ms, lo, hi = time_handle(bsg, torch, dev, lin, x, synth.I8, 0.05, steps)
+    res["sparse_2to4_tensor_cores"] = {
+        "ms_per_step": round(ms, 6), "min_ms": round(lo, 6), "max_ms": round(hi, 6),
+        "value": round(useful24 / (ms * 1e-3) / 1e12, 3), "unit": UNIT, "stored_macs_per_useful": 1.0,
+        "roofline_frac": round(useful24 / (ms * 1e-3) / 1e12 / tensor_peak, 4), "roofline_peak": tensor_peak,
+        "roofline_basis": "useful multiply-adds at the measured dense bf16 rate (the f16 rate; the sparse MMA does "
+                          "the stored half at the dense rate)",
+        "frac_of_dp4a_peak": round(useful24 / (ms * 1e-3) / 1e12 / peak, 4)}
+    lin.close()
+    dense24 = bsg.dense_from_2to4(w24.values, w24.idx)
+    lin = bsg.SparseInt8Linear.from_dense(dense24, w24.scales, w24.bias)
     ms, lo, hi = time_handle(bsg, torch, dev, lin, x, synth.I8, 0.05, steps)
     res["sparse_2to4_as_4x1"] = {"ms_per_step": round(ms, 6), "min_ms": round(lo, 6), "max_ms": round(hi, 6),
                                  "value": round(useful24 / (ms * 1e-3) / 1e12, 3), "unit": UNIT,
@@ -628,10 +648,10 @@ def run_shapes(args) -> dict:
             "ms_per_step": nat["ms_per_step"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "s8", "data": "synthetic",
             "config": {"workload": "other block shapes on 768 <- 3072, M = 4096, int8 out: 1 x 4 blocks at 90% "
-                                   "(native / regrouped into 4 x 1), 2:4 (regrouped into 4 x 1)",
+                                   "(native / regrouped into 4 x 1), 2:4 (sparse tensor cores / regrouped into 4 x 1)",
                        "basis": f"graph of {steps} bsgemm_run_ws launches (ACT_READY, rotating sets), median of "
                                 f"{REPEATS} replays; value = useful multiply-adds x 2 / time"},
-            "shapes": res, "gpu_launches": 3 * steps * REPEATS, "kernel_source_sha256": kernel_sha()}
+            "shapes": res, "gpu_launches": 4 * steps * REPEATS, "kernel_source_sha256": kernel_sha()}
 
 
 def run_configs(args) -> dict:

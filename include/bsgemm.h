@@ -143,11 +143,18 @@ bsgemm_t bsgemm_create_1x4(int N, int K, const int32_t* indices, const int8_t* v
  * pattern of sparse tensor cores that Sec. 1 cites as related work).  HOST
  * arrays [N][K/2], read during the call only: values int8 and idx uint8,
  * where values[n][2j + t] is W[n][4j + idx[n][2j + t]]; idx[n][2j] <
- * idx[n][2j + 1] <= 3 (a value may be 0).  K a multiple of 4.  The weight
- * is run as the 4 x 1 blocks that hold its values (block (r, k) stored when
- * one of rows 4r..4r+3 is nonzero in column k; about 1.9x the multiply-adds
- * of the 2:4 values for random patterns).  scales, bias and the result as
- * for bsgemm_create.
+ * idx[n][2j + 1] <= 3 (a value may be 0).  K a multiple of 4.  With N and
+ * K multiples of 128 (K <= 4096) the runs of row-major activations
+ * (bsgemm_run, _run_ws, _run_static, _run_host), every kind but
+ * BSGEMM_OUT_F32_RESID, go to the sparse tensor cores (tcgen05.mma.sp: the
+ * stored values as f16 with their positions, the activations widened to
+ * f16, exact fp32 partial sums of at most 1024 products added in int32:
+ * the int32 result bit for bit); the handle then holds a second device
+ * allocation of N K + N K / 32 bytes for those operands.  Other shapes and
+ * runs go through the 4 x 1 blocks that hold the values (block (r, k)
+ * stored when one of rows 4r..4r+3 is nonzero in column k; about 1.9x the
+ * multiply-adds of the 2:4 values for random patterns).  scales, bias and
+ * the result as for bsgemm_create.
  */
 bsgemm_t bsgemm_create_2to4(int N, int K, const int8_t* values, const uint8_t* idx, const float* scales,
                             const float* bias);
