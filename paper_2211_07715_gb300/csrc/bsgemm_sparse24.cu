@@ -18,9 +18,10 @@
 //     the 16 KB shared-memory image of its stored values (128 rows of 64 f16,
 //     the 128-byte swizzle) and the stage's 4 x 128 metadata words (one
 //     tensor-memory column per MMA); one thread of the MMA warp brings the
-//     image in with a bulk copy;
+//     images in by bulk copies, three stages ahead (a ring of four);
 //   * the 8 converter warps (two threads a token row, one per 64 columns)
-//     copy the stage's int8 activations with cp.async, widen them to f16 into
+//     copy the stage's int8 activations with cp.async two stages ahead (a
+//     ring of three int8 tiles), widen them to f16 into
 //     the B image (two 128-row x 64-column sub-tiles, 128-byte swizzle), and
 //     store the stage's metadata into tensor memory (warps 0-3: lane r =
 //     weight row r);
@@ -50,7 +51,10 @@ constexpr int kTcThreads = 288;            // 8 converter / epilogue warps + 1 M
 constexpr uint32_t kAImg = kTc24AImage;    // bytes of a stage's weight image
 constexpr uint32_t kXImg = 128 * 128;      // a stage's int8 token tile (128 tokens x 128 columns)
 constexpr uint32_t kBImg = 2 * 128 * 128;  // its f16 form: two 128 x 64 sub-tiles
-constexpr uint32_t kStageBytes = kAImg + kXImg + kBImg;
+constexpr int kARing = 4;                  // weight images in flight (loaded three stages ahead)
+constexpr int kXRing = 3;                  // int8 token tiles in flight (copied two stages ahead)
+// shared memory: the weight-image ring, the two f16 token images, the int8 ring
+constexpr uint32_t kBOff = kARing * kAImg, kXOff = kBOff + 2 * kBImg, kSmemBytes = kXOff + kXRing * kXImg;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColMeta = 256;         // metadata of MMA i of stage buffer b at column 256 + 32 (4 b + i)
 
@@ -89,7 +93,7 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
     extern __shared__ unsigned char smem_raw[];
     unsigned char* sm =
         reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    __shared__ __align__(8) unsigned long long s_bar[7];  // a_full[2], b_full[2], empty[2], done
+    __shared__ __align__(8) unsigned long long s_bar[9];  // a_full[4], b_full[2], empty[2], done
     __shared__ uint32_t s_tmem;
     const int tid = threadIdx.x, warp = tid >> 5;
     const bool mma_warp = warp == 8;
@@ -97,13 +101,14 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
     const long long t0 = static_cast<long long>(blockIdx.y) * 128;  // first token
     const int nst = K / 128;                      // stages
     const uint32_t bar = smem_addr(&s_bar[0]);
-    const uint32_t a_full = bar, b_full = bar + 16, empty = bar + 32, done = bar + 48;
-    auto stage_base = [&](int b) { return sm + static_cast<uint32_t>(b) * kStageBytes; };
+    const uint32_t a_full = bar, b_full = bar + 32, empty = bar + 48, done = bar + 64;
+    auto a_base = [&](int s) { return sm + static_cast<uint32_t>(s % kARing) * kAImg; };
+    auto b_base = [&](int s) { return sm + kBOff + static_cast<uint32_t>(s & 1) * kBImg; };
+    auto x_base = [&](int s) { return sm + kXOff + static_cast<uint32_t>(s % kXRing) * kXImg; };
 
     griddep_launch_dependents();
     if (tid == kTcThreads - 32) {
-        mbar_init(a_full, 1);
-        mbar_init(a_full + 8, 1);
+        for (int i = 0; i < kARing; ++i) mbar_init(a_full + 8u * i, 1);
         mbar_init(b_full, 256);
         mbar_init(b_full + 8, 256);
         mbar_init(empty, 1);
@@ -119,32 +124,32 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
 
     if (mma_warp) {
         if (tid == kTcThreads - 32) {
-            // the weight images of stages 0 and 1, then stage s + 1's once stage
-            // s - 1's MMAs (issued before stage s's) have read its buffer
+            // the weight images of stages 0-3, then stage s + 3's once stage
+            // s - 1's MMAs (issued before stage s's) have read its ring slot
             auto load_a = [&](int s) {
-                const uint32_t b = static_cast<uint32_t>(s & 1);
-                mbar_arrive_expect_tx(a_full + 8u * b, kAImg);
-                bulk_g2s(smem_addr(stage_base(s & 1)), aimg + (static_cast<size_t>(ct) * nst + s) * kAImg, kAImg,
-                         a_full + 8u * b);
+                const uint32_t slot = static_cast<uint32_t>(s % kARing);
+                mbar_arrive_expect_tx(a_full + 8u * slot, kAImg);
+                bulk_g2s(smem_addr(a_base(s)), aimg + (static_cast<size_t>(ct) * nst + s) * kAImg, kAImg,
+                         a_full + 8u * slot);
             };
-            load_a(0);
-            if (nst > 1) load_a(1);
+            for (int s = 0; s < kARing && s < nst; ++s) load_a(s);
             for (int s = 0; s < nst; ++s) {
                 const uint32_t b = static_cast<uint32_t>(s & 1), ph = static_cast<uint32_t>(s >> 1) & 1u;
-                ok &= mbar_wait(a_full + 8u * b, ph, wait_limit);
+                ok &= mbar_wait(a_full + 8u * static_cast<uint32_t>(s % kARing), static_cast<uint32_t>(s / kARing) & 1u,
+                                wait_limit);
                 ok &= mbar_wait(b_full + 8u * b, ph, wait_limit);
                 tc_fence_after();
-                const uint32_t as = smem_addr(stage_base(s & 1)), bs = as + kAImg + kXImg;
+                const uint32_t as = smem_addr(a_base(s)), bs = smem_addr(b_base(s));
                 const uint32_t d = tm + 128u * static_cast<uint32_t>(s / 16);  // the chunk's accumulator (two at most)
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
                     mma_sp(d, sw128_desc(as + 32u * i, 16, 1024), sw128_desc(bs + 16384u * (i >> 1) + 64u * (i & 1), 16, 1024),
                            tm + kColMeta + 32u * (4u * b + static_cast<uint32_t>(i)), (s % 16 != 0 || i > 0) ? 1u : 0u);
                 tc_commit(empty + 8u * b);
-                if (s >= 1 && s + 1 < nst) {
+                if (s >= 1 && s + kARing - 1 < nst) {
                     ok &= mbar_wait(empty + 8u * (b ^ 1u), static_cast<uint32_t>((s - 1) >> 1) & 1u, wait_limit);
                     tc_fence_after();
-                    load_a(s + 1);
+                    load_a(s + kARing - 1);
                 }
             }
             tc_commit(done);
@@ -162,17 +167,28 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
         // 4 copies of 16 bytes: chunk c (= 4 h + cc) of row r at r * 128 + (c ^
         // (r % 8)) * 16 (conflict-free reads by 8 consecutive threads)
         auto copy_x = [&](int s) {
-            const uint32_t xs = smem_addr(stage_base(s & 1) + kAImg) + 128u * static_cast<uint32_t>(r);
+            const uint32_t xs = smem_addr(x_base(s)) + 128u * static_cast<uint32_t>(r);
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc)
                 cp_async16(xs + ((static_cast<uint32_t>(4 * h + cc) ^ (r & 7)) << 4), xrow + 128 * s + 16 * cc, src_bytes);
             cp_async_commit();
         };
         copy_x(0);
+        if (nst > 1) copy_x(1);
+        // the metadata words of this lane (warps 0-3: lane r = weight row r), a stage ahead
+        auto load_meta = [&](int s) {
+            return h == 0 ? __ldg(reinterpret_cast<const uint4*>(meta + ((static_cast<size_t>(ct) * nst + s) * 128 + r) * 4))
+                          : make_uint4(0u, 0u, 0u, 0u);
+        };
+        uint4 mv = load_meta(0);
         for (int s = 0; s < nst; ++s) {
             const uint32_t b = static_cast<uint32_t>(s & 1);
-            if (s + 1 < nst) {
-                copy_x(s + 1);
+            // stage s's copies landed (groups are committed in stage order; the
+            // ring slot of stage s + 2 was last read by this thread for stage s - 1)
+            if (s + 2 < nst) {
+                copy_x(s + 2);
+                cp_async_wait<2>();
+            } else if (s + 1 < nst) {
                 cp_async_wait<1>();
             } else {
                 cp_async_wait<0>();
@@ -181,9 +197,8 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
                 ok &= mbar_wait(empty + 8u * b, static_cast<uint32_t>((s - 2) >> 1) & 1u, wait_limit);
                 tc_fence_after();
             }
-            unsigned char* st = stage_base(s & 1);
-            const unsigned char* xs = st + kAImg + 128u * static_cast<uint32_t>(r);
-            unsigned char* row = st + kAImg + kXImg + 16384u * static_cast<uint32_t>(h) + 128u * static_cast<uint32_t>(r);
+            const unsigned char* xs = x_base(s) + 128u * static_cast<uint32_t>(r);
+            unsigned char* row = b_base(s) + 16384u * static_cast<uint32_t>(h) + 128u * static_cast<uint32_t>(r);
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc) {
                 const int c = 4 * h + cc;
@@ -205,8 +220,6 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
             if (h == 0) {
                 // the stage's metadata: word r of each of its 4 MMAs into lane r, one
                 // column each (32-column aligned)
-                const uint4 mv =
-                    __ldg(reinterpret_cast<const uint4*>(meta + ((static_cast<size_t>(ct) * nst + s) * 128 + r) * 4));
                 const uint32_t mw[4] = {mv.x, mv.y, mv.z, mv.w};
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
@@ -218,6 +231,7 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
             }
             tc_fence_before();
             arrive(b_full + 8u * b);
+            if (s + 1 < nst) mv = load_meta(s + 1);
         }
 
         // epilogue: lane r = channel ch of the tile, tokens 64 h .. 64 h + 63
@@ -279,7 +293,7 @@ cudaError_t launch_sparse24(const int8_t* x, int M, int N, int K, const unsigned
     case 4: fn = reinterpret_cast<const void*>(&sparse24_kernel<4>); break;
     default: return cudaErrorNotSupported;
     }
-    const int smem = static_cast<int>(2 * kStageBytes + 1024);
+    const int smem = static_cast<int>(kSmemBytes + 1024);
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
