@@ -109,7 +109,8 @@ typedef struct bsgemm_ctx* bsgemm_t; /* opaque handle */
  * The call allocates device memory on the CURRENT CUDA device, copies the
  * repacked weights there and synchronises.  Returns NULL on failure.
  *
- * Other block shapes: bsgemm_create_1x4 and bsgemm_create_2to4 below.
+ * Other block shapes: bsgemm_create_1x4 and bsgemm_create_2to4 below; the
+ * same weight run dense on the tensor cores: bsgemm_create_tc.
  */
 #define BSGEMM_MAX_N (4 * 65535) /* block-row indices are 16-bit inside the kernel */
 bsgemm_t bsgemm_create(int N, int K, int block, const int32_t* indices, const int8_t* values,
@@ -143,8 +144,8 @@ bsgemm_t bsgemm_create_1x4(int N, int K, const int32_t* indices, const int8_t* v
  * pattern of sparse tensor cores that Sec. 1 cites as related work).  HOST
  * arrays [N][K/2], read during the call only: values int8 and idx uint8,
  * where values[n][2j + t] is W[n][4j + idx[n][2j + t]]; idx[n][2j] <
- * idx[n][2j + 1] <= 3 (a value may be 0).  K a multiple of 4.  With N and
- * K multiples of 128 (K <= 4096) the runs of row-major activations
+ * idx[n][2j + 1] <= 3 (a value may be 0).  K a multiple of 4, at most
+ * bsgemm_max_k().  With N and K multiples of 128 the runs of row-major activations
  * (bsgemm_run, _run_ws, _run_static, _run_host), every kind but
  * BSGEMM_OUT_F32_RESID, go to the sparse tensor cores (tcgen05.mma.sp: the
  * stored values as f16 with their positions, the activations widened to
@@ -158,6 +159,25 @@ bsgemm_t bsgemm_create_1x4(int N, int K, const int32_t* indices, const int8_t* v
  */
 bsgemm_t bsgemm_create_2to4(int N, int K, const int8_t* values, const uint8_t* idx, const float* scales,
                             const float* bias);
+
+/*
+ * bsgemm_create_tc -- the block-compressed weight of bsgemm_create (same
+ * arguments, same validation, same result), also laid out to run DENSE
+ * over K on the tensor cores: the contraction of Algorithm 1 with every
+ * column multiplied, zeros included (tcgen05.mma kind::f16 on the int8
+ * values as f16, the activations widened to f16, exact fp32 partial sums
+ * of at most 1024 products added in int32: the int32 result bit for bit).
+ * With N and K multiples of 128 (K <= bsgemm_max_k() as for every
+ * handle) the runs of row-major activations (bsgemm_run, _run_ws,
+ * _run_static, _run_host), every kind but BSGEMM_OUT_F32_RESID, take that
+ * path, and the handle holds a second
+ * device allocation of 2 N K bytes (the f16 image); other shapes and runs
+ * take the block-sparse kernel.  This is the tensor-core alternative to
+ * the block-sparse int8 kernel, for comparison: its time does not fall
+ * with sparsity.
+ */
+bsgemm_t bsgemm_create_tc(int N, int K, int block, const int32_t* indices, const int8_t* values,
+                          const float* scales, const float* bias);
 
 /*
  * bsgemm_run -- out = epilogue(X * W^T) on `stream`.
@@ -445,8 +465,8 @@ int bsgemm_max_k(void);
  * the inner loop; the last quad of a block-row is padded with zero-weight
  * entries), [4] token-tile height of the kernel, [5] CTAs of a launch once
  * M is large enough to fill the GPU (SMs x resident CTAs per SM), [6] device
- * bytes held by the handle.  Returns the number of entries available (7),
- * or BSGEMM_ERR_INVALID.
+ * bytes held by the handle (the tensor-core operands' allocation included).
+ * Returns the number of entries available (7), or BSGEMM_ERR_INVALID.
  */
 int bsgemm_info(bsgemm_t h, int64_t* out, int n);
 

@@ -55,6 +55,8 @@ def _load() -> ctypes.CDLL:
     lib.bsgemm_create_1x4.restype = vp
     lib.bsgemm_create_2to4.argtypes = [ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]
     lib.bsgemm_create_2to4.restype = vp
+    lib.bsgemm_create_tc.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, vp, vp, vp, vp]
+    lib.bsgemm_create_tc.restype = vp
     lib.bsgemm_run.argtypes = [vp, vp, ctypes.c_int, vp, Epilogue, vp]
     lib.bsgemm_run.restype = ctypes.c_int
     lib.bsgemm_destroy.argtypes = [vp]
@@ -103,7 +105,7 @@ def _load() -> ctypes.CDLL:
 
 _lib = _load()
 
-EXPORTED = ("bsgemm_create", "bsgemm_create_1x4", "bsgemm_create_2to4", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
+EXPORTED = ("bsgemm_create", "bsgemm_create_1x4", "bsgemm_create_2to4", "bsgemm_create_tc", "bsgemm_run", "bsgemm_run_ws", "bsgemm_run_static", "bsgemm_workspace_bytes",
             "bsgemm_tile_activations", "bsgemm_run_tiled", "bsgemm_run_kmajor",
             "bsgemm_host_workspace_bytes", "bsgemm_run_host", "bsgemm_block_prune", "bsgemm_layernorm",
             "bsgemm_attention", "bsgemm_destroy",
@@ -141,6 +143,20 @@ def bsgemm_create(n_out: int, k_in: int, block: int, indices, values, scales, bi
     bias = None if bias is None else _host_array(bias, np.float32)
     h = _lib.bsgemm_create(int(n_out), int(k_in), int(block), indices.ctypes.data, values.ctypes.data,
                            scales.ctypes.data, None if bias is None else bias.ctypes.data)
+    if not h:
+        raise BsgemmError(bsgemm_last_status(), bsgemm_last_error())
+    return h
+
+
+def bsgemm_create_tc(n_out: int, k_in: int, block: int, indices, values, scales, bias=None) -> int:
+    """As bsgemm_create, and with N and K multiples of 128 (K <= 4096) the
+    row-major runs go dense over K to the tensor cores (see include/bsgemm.h)."""
+    indices = _host_array(indices, np.int32)
+    values = _host_array(values, np.int8)
+    scales = _host_array(scales, np.float32)
+    bias = None if bias is None else _host_array(bias, np.float32)
+    h = _lib.bsgemm_create_tc(int(n_out), int(k_in), int(block), indices.ctypes.data, values.ctypes.data,
+                              scales.ctypes.data, None if bias is None else bias.ctypes.data)
     if not h:
         raise BsgemmError(bsgemm_last_status(), bsgemm_last_error())
     return h
@@ -465,19 +481,22 @@ def dense_from_2to4(values, idx) -> np.ndarray:
 class SparseInt8Linear:
     """One block-sparse int8 linear layer resident on the current CUDA device."""
 
-    def __init__(self, n_out: int, k_in: int, indptr, colidx, values, scales, bias=None):
+    def __init__(self, n_out: int, k_in: int, indptr, colidx, values, scales, bias=None, tensor_cores: bool = False):
+        """tensor_cores: create through bsgemm_create_tc (the weight also run
+        dense over K on the tensor cores when N and K are multiples of 128)."""
         indices = np.concatenate([_host_array(indptr, np.int32), _host_array(colidx, np.int32)])
         self.n_out, self.k_in = int(n_out), int(k_in)
-        self._h = bsgemm_create(n_out, k_in, BLOCK, indices, values, scales, bias)
+        create = bsgemm_create_tc if tensor_cores else bsgemm_create
+        self._h = create(n_out, k_in, BLOCK, indices, values, scales, bias)
         self.info = bsgemm_info(self._h)
 
     @classmethod
-    def from_dense(cls, w, scales, bias=None, keep=None) -> "SparseInt8Linear":
+    def from_dense(cls, w, scales, bias=None, keep=None, tensor_cores: bool = False) -> "SparseInt8Linear":
         """From a dense int8 weight [N][K]; `keep` [N/4][K] (e.g. from
         block_prune) selects the stored blocks."""
         w = _host_array(w, np.int8)
         indptr, colidx, values = dense_to_blocks(w, keep)
-        return cls(w.shape[0], w.shape[1], indptr, colidx, values, scales, bias)
+        return cls(w.shape[0], w.shape[1], indptr, colidx, values, scales, bias, tensor_cores=tensor_cores)
 
     @classmethod
     def _of_handle(cls, h: int, n_out: int, k_in: int) -> "SparseInt8Linear":
@@ -499,8 +518,9 @@ class SparseInt8Linear:
     @classmethod
     def from_2to4(cls, values, idx, scales, bias=None) -> "SparseInt8Linear":
         """A 2:4-sparse weight (values, idx [N][K/2]) through
-        bsgemm_create_2to4: run as the 4 x 1 blocks that hold its values
-        (~94% of all blocks for random 2:4 patterns)."""
+        bsgemm_create_2to4: on the sparse tensor cores when N and K are
+        multiples of 128 (K <= 4096), else as the 4 x 1 blocks that hold its
+        values (~94% of all blocks for random 2:4 patterns)."""
         values = np.asarray(values)
         n_out, k_in = values.shape[0], 2 * values.shape[1]
         return cls._of_handle(bsgemm_create_2to4(n_out, k_in, values, idx, scales, bias), n_out, k_in)

@@ -28,11 +28,14 @@ struct bsgemm_ctx {
     size_t arena_bytes = 0;
     std::vector<int32_t> cost;  // schedule prefix cost of the row groups [ngroups + 1]
     bsg::DeviceWeights w{};
-    // 2:4 weights with N and K multiples of 128: the sparse tensor cores'
-    // operands (launch_sparse24), in their own allocation; NULL otherwise
+    // Handles of bsgemm_create_2to4 / bsgemm_create_tc with N and K
+    // multiples of 128: the tensor cores' operands (launch_tc_linear), in
+    // their own allocation; NULL otherwise.  tc_dense: the dense MMA's image.
     void* tc_arena = nullptr;
     const unsigned char* tc_aimg = nullptr;
     const uint32_t* tc_meta = nullptr;
+    bool tc_dense = false;
+    size_t tc_bytes = 0;
     std::mutex sched_mu;        // guards the cached schedule of the last token count
     long long sched_m = -1;
     int sched_grid = 0;
@@ -359,6 +362,30 @@ bsgemm_t upload(const Repacked& rp, const float* scales, const float* bias) {
 }  // namespace
 
 unsigned bsg::test_hooks() { return g_test_hooks.load(); }
+
+// Upload the tensor cores' operands of handle h into their own allocation;
+// on failure destroys h and returns NULL.
+static bsgemm_t attach_tc(bsgemm_t h, const std::vector<uint16_t>& aimg, const std::vector<uint32_t>& meta,
+                          bool dense) {
+    const size_t abytes = aimg.size() * sizeof(uint16_t), mbytes = meta.size() * sizeof(uint32_t);
+    void* arena = nullptr;
+    cudaError_t e = cudaMalloc(&arena, abytes + mbytes);
+    if (e == cudaSuccess) e = cudaMemcpy(arena, aimg.data(), abytes, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && mbytes)
+        e = cudaMemcpy(static_cast<char*>(arena) + abytes, meta.data(), mbytes, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        if (arena) cudaFree(arena);
+        bsgemm_destroy(h);
+        fail(BSGEMM_ERR_CUDA, cuda_msg("tensor-core operands", e));
+        return nullptr;
+    }
+    h->tc_arena = arena;
+    h->tc_aimg = static_cast<const unsigned char*>(arena);
+    h->tc_meta = mbytes ? reinterpret_cast<const uint32_t*>(static_cast<const char*>(arena) + abytes) : nullptr;
+    h->tc_dense = dense;
+    h->tc_bytes = abytes + mbytes;
+    return h;
+}
 
 extern "C" {
 
@@ -697,21 +724,35 @@ bsgemm_t bsgemm_create_2to4(int N, int K, const int8_t* values, const uint8_t* i
             }
         }
     }
-    const size_t abytes = aimg.size() * sizeof(uint16_t), mbytes = meta.size() * sizeof(uint32_t);
-    void* arena = nullptr;
-    cudaError_t e = cudaMalloc(&arena, abytes + mbytes);
-    if (e == cudaSuccess) e = cudaMemcpy(arena, aimg.data(), abytes, cudaMemcpyHostToDevice);
-    if (e == cudaSuccess) e = cudaMemcpy(static_cast<char*>(arena) + abytes, meta.data(), mbytes, cudaMemcpyHostToDevice);
-    if (e != cudaSuccess) {
-        if (arena) cudaFree(arena);
-        bsgemm_destroy(h);
-        fail(BSGEMM_ERR_CUDA, cuda_msg("sparse tensor-core operands", e));
-        return nullptr;
+    return attach_tc(h, aimg, meta, false);
+}
+
+// Any block-compressed weight, also run dense over K on the tensor cores
+// (launch_tc_linear, dense form) when N and K are multiples of 128: per
+// (channel tile ct, stage s of 128 columns) the weight's 128 x 128 values
+// as f16, row m = channel 128 ct + m, in two sub-tiles of 64 columns, the
+// 16-byte chunk c of a sub-tile row placed at chunk c ^ (m % 8) of its 128
+// bytes; zero where no block is stored.
+bsgemm_t bsgemm_create_tc(int N, int K, int block, const int32_t* indices, const int8_t* values, const float* scales,
+                          const float* bias) {
+    bsgemm_t h = bsgemm_create(N, K, block, indices, values, scales, bias);
+    if (!h || N % 128 != 0 || K % 128 != 0 || K > 4096) return h;
+    const int nbr = N / 4, nst = K / 128;
+    constexpr size_t kImg = bsg::kTcDenseAImage / 2;  // f16 values per (tile, stage)
+    std::vector<uint16_t> aimg(static_cast<size_t>(N / 128) * nst * kImg, 0);
+    const int32_t* indptr = indices;
+    const int32_t* colidx = indices + nbr + 1;
+    for (int r = 0; r < nbr; ++r) {
+        for (int j = indptr[r]; j < indptr[r + 1]; ++j) {
+            const int k = colidx[j], st = k / 128, kk = k % 128, c = (kk % 64) / 8;
+            for (int i = 0; i < 4; ++i) {
+                const int n = 4 * r + i, m = n % 128;
+                aimg[(static_cast<size_t>(n / 128) * nst + st) * kImg + (kk / 64) * (kImg / 2) + 64 * m +
+                     8 * (c ^ (m % 8)) + kk % 8] = f16_of_int(values[4 * static_cast<size_t>(j) + i]);
+            }
+        }
     }
-    h->tc_arena = arena;
-    h->tc_aimg = static_cast<const unsigned char*>(arena);
-    h->tc_meta = reinterpret_cast<const uint32_t*>(static_cast<const char*>(arena) + abytes);
-    return h;
+    return attach_tc(h, aimg, std::vector<uint32_t>(), true);
 }
 
 // mode: 0 = gather from act (no scratch), 1 = relayout act into workspace
@@ -786,12 +827,13 @@ static int run_common(bsgemm_t h, const int8_t* act, int M, void* out, bsgemm_ep
     a.x_vec16 = (reinterpret_cast<uintptr_t>(act) % 16 == 0) && (h->w.K % 16 == 0);
     a.skip_copy = (g_test_hooks.load() & BSGEMM_TEST_SKIP_TILE_COPY) != 0;
     a.wait_limit = a.skip_copy ? 64u : 0u;
-    // 2:4 weights on the sparse tensor cores: row-major act, any kind but the residual
+    // weights on the tensor cores (2:4 sparse, or dense over K): row-major
+    // act, any kind but the residual
     if (h->tc_aimg && (mode == 0 || mode == 1) && epi.kind != BSGEMM_OUT_F32_RESID &&
         (reinterpret_cast<uintptr_t>(act) & 15u) == 0) {
-        e = bsg::launch_sparse24(act, M, h->w.N, h->w.K, h->tc_aimg, h->tc_meta, h->w.scale, h->w.bias, out, epi.kind,
-                                 inv, (epi.flags & BSGEMM_ACT_READY) != 0, h->w.status, s);
-        if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("sparse tensor-core kernel launch", e));
+        e = bsg::launch_tc_linear(act, M, h->w.N, h->w.K, h->tc_aimg, h->tc_meta, h->tc_dense, h->w.scale, h->w.bias,
+                                  out, epi.kind, inv, (epi.flags & BSGEMM_ACT_READY) != 0, h->w.status, s);
+        if (e != cudaSuccess) return fail(BSGEMM_ERR_CUDA, cuda_msg("tensor-core kernel launch", e));
         return BSGEMM_OK;
     }
     const long long ntiles = (static_cast<long long>(M) + bsg::kTile - 1) / bsg::kTile;
@@ -1054,7 +1096,7 @@ int bsgemm_info(bsgemm_t h, int64_t* out, int n) {
     clear_error();
     if (!h || (!out && n > 0)) return fail(BSGEMM_ERR_INVALID, "NULL handle or output");
     const int64_t v[7] = {h->w.N, h->w.K, h->nnzb, 4 * static_cast<int64_t>(h->w.S), bsg::kTile,
-                          static_cast<int64_t>(h->num_sms) * h->ctas_per_sm, static_cast<int64_t>(h->arena_bytes)};
+                          static_cast<int64_t>(h->num_sms) * h->ctas_per_sm, static_cast<int64_t>(h->arena_bytes + h->tc_bytes)};
     for (int i = 0; i < n && i < 7; ++i) out[i] = v[i];
     return 7;
 }

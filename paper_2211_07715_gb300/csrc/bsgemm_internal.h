@@ -120,15 +120,19 @@ cudaError_t launch_attention(const int8_t* qkv, int batch, int seq, int heads, i
 // The current device's attention status word (bit 0: a wait gave up),
 // reset to 0 when clear is set and it was not.
 cudaError_t attention_status(bool clear, unsigned* v);
-// 2:4-sparse weights on the sparse tensor cores (bsgemm_sparse24.cu), for N
-// and K multiples of 128, K <= 4096: aimg = per (128-channel tile, 128-column
-// stage) the kTc24AImage-byte shared-memory image of the stored values
-// (128 rows x 64 f16, 128-byte swizzle); meta = per (tile, stage, lane) the 4
-// sparse-MMA metadata words.  kind 0-4 (no residual).
+// Weights on the tensor cores (bsgemm_sparse24.cu), for N and K multiples
+// of 128, K <= 4096, M >= 1.  2:4-sparse (dense = false): aimg = per
+// (128-channel tile, 128-column stage) the kTc24AImage-byte shared-memory
+// image of the stored values (128 rows x 64 f16, 128-byte swizzle); meta =
+// per (tile, stage, lane) the 4 sparse-MMA metadata words.  Dense over K
+// (dense = true, meta unused): aimg = per (tile, stage) the kTcDenseAImage-
+// byte image of all 128 columns (two 128-row x 64-f16 sub-tiles, 128-byte
+// swizzle).  kind 0-4 (no residual).
 constexpr uint32_t kTc24AImage = 16384;
-cudaError_t launch_sparse24(const int8_t* x, int M, int N, int K, const unsigned char* aimg, const uint32_t* meta,
-                            const float* scale, const float* bias, void* out, int kind, float inv_out_scale,
-                            bool act_ready, int* status, cudaStream_t s);
+constexpr uint32_t kTcDenseAImage = 32768;
+cudaError_t launch_tc_linear(const int8_t* x, int M, int N, int K, const unsigned char* aimg, const uint32_t* meta,
+                             bool dense, const float* scale, const float* bias, void* out, int kind,
+                             float inv_out_scale, bool act_ready, int* status, cudaStream_t s);
 // x [M][K] -> swizzled token tiles in xb (the layout the kernel stages by TMA).
 cudaError_t launch_pretile(const int8_t* x, int M, int K, int8_t* xb, int sms, cudaStream_t s);
 // Average-magnitude block pruning of a dense fp32 W [N][K] (DEVICE) into

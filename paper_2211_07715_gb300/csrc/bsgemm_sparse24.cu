@@ -35,6 +35,16 @@
 //     accumulators read from tensor memory 32 tokens at a time, converted to int32 exactly, added, and the fused epilogue
 //     (dequantise + bias, GELU, requantise) stored as out[token][channel].
 // Every wait is bounded; a wait that gives up sets the handle's status word.
+//
+// The same kernel with DENSE set runs any int8 weight, stored in full, on
+// the dense MMA (`tcgen05.mma ... kind::f16`, K = 16): every block-sparse
+// weight taken as dense over K, the tensor-core form of Algorithm 1's
+// contraction that skips no zero block.  A stage's weight image is then
+// 32 KB (128 rows x 128 f16 as two 64-column sub-tiles, the B image's
+// layout; a ring of three, loaded two stages ahead), its 8 MMAs read no
+// metadata, and a chunk of exactly-accumulated columns is 1024 (8 stages:
+// at most 1024 products below 2^14 in magnitude each), four chunks for K =
+// 4096 filling the 512 tensor-memory columns.
 
 #include <cstdint>
 #include <cuda_runtime.h>
@@ -48,19 +58,27 @@ namespace bsg {
 namespace {
 
 constexpr int kTcThreads = 288;            // 8 converter / epilogue warps + 1 MMA warp
-constexpr uint32_t kAImg = kTc24AImage;    // bytes of a stage's weight image
 constexpr uint32_t kXImg = 128 * 128;      // a stage's int8 token tile (128 tokens x 128 columns)
 constexpr uint32_t kBImg = 2 * 128 * 128;  // its f16 form: two 128 x 64 sub-tiles
-constexpr int kARing = 4;                  // weight images in flight (loaded three stages ahead)
 constexpr int kXRing = 3;                  // int8 token tiles in flight (copied two stages ahead)
+// bytes of a stage's weight image; weight images in flight (the sparse
+// form loads three stages ahead, the dense form two); stages of one exact
+// fp32 accumulator chunk
+__host__ __device__ constexpr uint32_t a_img_bytes(bool dense) { return dense ? kBImg : kTc24AImage; }
+__host__ __device__ constexpr int a_ring(bool dense) { return dense ? 3 : 4; }
+__host__ __device__ constexpr int chunk_stages(bool dense) { return dense ? 8 : 16; }
 // shared memory: the weight-image ring, the two f16 token images, the int8 ring
-constexpr uint32_t kBOff = kARing * kAImg, kXOff = kBOff + 2 * kBImg, kSmemBytes = kXOff + kXRing * kXImg;
+__host__ __device__ constexpr uint32_t b_off(bool dense) { return a_ring(dense) * a_img_bytes(dense); }
+__host__ __device__ constexpr uint32_t x_off(bool dense) { return b_off(dense) + 2 * kBImg; }
+__host__ __device__ constexpr uint32_t smem_bytes(bool dense) { return x_off(dense) + kXRing * kXImg; }
+static_assert(smem_bytes(true) + 1024 <= 227 * 1024 && smem_bytes(false) + 1024 <= 227 * 1024, "shared memory");
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColMeta = 256;         // metadata of MMA i of stage buffer b at column 256 + 32 (4 b + i)
 
-// Instruction descriptor of the sparse MMA: f16 A and B, fp32 accumulator,
-// both K-major, N = 128, M = 128, sparsity flag (bit 2).
-constexpr uint32_t kIdescSp = f16_idesc(128, 128, false) | (1u << 2);
+// Instruction descriptors: f16 A and B, fp32 accumulator, both K-major,
+// N = 128, M = 128; the sparse MMA's with the sparsity flag (bit 2).
+constexpr uint32_t kIdesc = f16_idesc(128, 128, false);
+constexpr uint32_t kIdescSp = kIdesc | (1u << 2);
 
 __device__ __forceinline__ void mma_sp(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t meta, uint32_t acc) {
     asm volatile("{\n .reg .pred p;\n setp.ne.u32 p, %5, 0;\n"
@@ -85,11 +103,13 @@ __device__ __forceinline__ uint32_t s8x2_f16x2(uint32_t u, uint32_t sel) {
     return r;
 }
 
-template <int KIND>
+template <int KIND, bool DENSE>
 __global__ void __launch_bounds__(kTcThreads, 1)
 sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigned char* __restrict__ aimg,
                 const uint32_t* __restrict__ meta, const float* __restrict__ scale, const float* __restrict__ bias,
                 void* __restrict__ out, float inv_out_scale, int act_ready, unsigned wait_limit, int* status) {
+    constexpr uint32_t kAImg = a_img_bytes(DENSE);
+    constexpr int kARing = a_ring(DENSE), kChunk = chunk_stages(DENSE);
     extern __shared__ unsigned char smem_raw[];
     unsigned char* sm =
         reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -103,8 +123,8 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
     const uint32_t bar = smem_addr(&s_bar[0]);
     const uint32_t a_full = bar, b_full = bar + 32, empty = bar + 48, done = bar + 64;
     auto a_base = [&](int s) { return sm + static_cast<uint32_t>(s % kARing) * kAImg; };
-    auto b_base = [&](int s) { return sm + kBOff + static_cast<uint32_t>(s & 1) * kBImg; };
-    auto x_base = [&](int s) { return sm + kXOff + static_cast<uint32_t>(s % kXRing) * kXImg; };
+    auto b_base = [&](int s) { return sm + b_off(DENSE) + static_cast<uint32_t>(s & 1) * kBImg; };
+    auto x_base = [&](int s) { return sm + x_off(DENSE) + static_cast<uint32_t>(s % kXRing) * kXImg; };
 
     griddep_launch_dependents();
     if (tid == kTcThreads - 32) {
@@ -124,13 +144,16 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
 
     if (mma_warp) {
         if (tid == kTcThreads - 32) {
-            // the weight images of stages 0-3, then stage s + 3's once stage
-            // s - 1's MMAs (issued before stage s's) have read its ring slot
+            // the weight images of the first kARing stages, then stage s +
+            // kARing - 1's once stage s - 1's MMAs (issued before stage s's)
+            // have read its ring slot
             auto load_a = [&](int s) {
                 const uint32_t slot = static_cast<uint32_t>(s % kARing);
                 mbar_arrive_expect_tx(a_full + 8u * slot, kAImg);
-                bulk_g2s(smem_addr(a_base(s)), aimg + (static_cast<size_t>(ct) * nst + s) * kAImg, kAImg,
-                         a_full + 8u * slot);
+#pragma unroll
+                for (uint32_t o = 0; o < kAImg; o += 16384u)  // copies of 16 KB
+                    bulk_g2s(smem_addr(a_base(s)) + o, aimg + (static_cast<size_t>(ct) * nst + s) * kAImg + o, 16384u,
+                             a_full + 8u * slot);
             };
             for (int s = 0; s < kARing && s < nst; ++s) load_a(s);
             for (int s = 0; s < nst; ++s) {
@@ -140,11 +163,22 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
                 ok &= mbar_wait(b_full + 8u * b, ph, wait_limit);
                 tc_fence_after();
                 const uint32_t as = smem_addr(a_base(s)), bs = smem_addr(b_base(s));
-                const uint32_t d = tm + 128u * static_cast<uint32_t>(s / 16);  // the chunk's accumulator (two at most)
+                const uint32_t d = tm + 128u * static_cast<uint32_t>(s / kChunk);  // the chunk's accumulator
+                if (DENSE) {
+                    // MMA i: columns 16 i .. 16 i + 15 of the stage, in sub-tile i / 4 of both images
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    mma_sp(d, sw128_desc(as + 32u * i, 16, 1024), sw128_desc(bs + 16384u * (i >> 1) + 64u * (i & 1), 16, 1024),
-                           tm + kColMeta + 32u * (4u * b + static_cast<uint32_t>(i)), (s % 16 != 0 || i > 0) ? 1u : 0u);
+                    for (int i = 0; i < 8; ++i) {
+                        const uint32_t off = 16384u * static_cast<uint32_t>(i >> 2) + 32u * static_cast<uint32_t>(i & 3);
+                        mma_f16_ss(d, sw128_desc(as + off, 16, 1024), sw128_desc(bs + off, 16, 1024), kIdesc,
+                                   (s % kChunk != 0 || i > 0) ? 1u : 0u);
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        mma_sp(d, sw128_desc(as + 32u * i, 16, 1024),
+                               sw128_desc(bs + 16384u * (i >> 1) + 64u * (i & 1), 16, 1024),
+                               tm + kColMeta + 32u * (4u * b + static_cast<uint32_t>(i)), (s % kChunk != 0 || i > 0) ? 1u : 0u);
+                }
                 tc_commit(empty + 8u * b);
                 if (s >= 1 && s + kARing - 1 < nst) {
                     ok &= mbar_wait(empty + 8u * (b ^ 1u), static_cast<uint32_t>((s - 1) >> 1) & 1u, wait_limit);
@@ -177,7 +211,7 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
         if (nst > 1) copy_x(1);
         // the metadata words of this lane (warps 0-3: lane r = weight row r), a stage ahead
         auto load_meta = [&](int s) {
-            return h == 0 ? __ldg(reinterpret_cast<const uint4*>(meta + ((static_cast<size_t>(ct) * nst + s) * 128 + r) * 4))
+            return !DENSE && h == 0 ? __ldg(reinterpret_cast<const uint4*>(meta + ((static_cast<size_t>(ct) * nst + s) * 128 + r) * 4))
                           : make_uint4(0u, 0u, 0u, 0u);
         };
         uint4 mv = load_meta(0);
@@ -217,7 +251,7 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
                 *reinterpret_cast<uint4*>(row + ((c1 ^ (r & 7)) << 4)) = make_uint4(o[4], o[5], o[6], o[7]);
             }
             fence_proxy_async();  // the B image, for the tensor cores
-            if (h == 0) {
+            if (!DENSE && h == 0) {
                 // the stage's metadata: word r of each of its 4 MMAs into lane r, one
                 // column each (32-column aligned)
                 const uint32_t mw[4] = {mv.x, mv.y, mv.z, mv.w};
@@ -240,7 +274,7 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
         tc_fence_after();
         const int ch = ct * 128 + r;
         const float sc = scale[ch], bi = bias[ch];
-        const int nchunks = (nst + 15) / 16;
+        const int nchunks = (nst + kChunk - 1) / kChunk;
         griddep_wait();  // outputs after the preceding kernel
         for (int n0 = 64 * h; n0 < 64 * h + 64; n0 += 32) {
             int acc[32];
@@ -281,19 +315,25 @@ sparse24_kernel(const int8_t* __restrict__ x, int M, int N, int K, const unsigne
 
 }  // namespace
 
-cudaError_t launch_sparse24(const int8_t* x, int M, int N, int K, const unsigned char* aimg, const uint32_t* meta,
-                            const float* scale, const float* bias, void* out, int kind, float inv_out_scale,
-                            bool act_ready, int* status, cudaStream_t s) {
+cudaError_t launch_tc_linear(const int8_t* x, int M, int N, int K, const unsigned char* aimg, const uint32_t* meta,
+                             bool dense, const float* scale, const float* bias, void* out, int kind,
+                             float inv_out_scale, bool act_ready, int* status, cudaStream_t s) {
     const void* fn = nullptr;
-    switch (kind) {
-    case 0: fn = reinterpret_cast<const void*>(&sparse24_kernel<0>); break;
-    case 1: fn = reinterpret_cast<const void*>(&sparse24_kernel<1>); break;
-    case 2: fn = reinterpret_cast<const void*>(&sparse24_kernel<2>); break;
-    case 3: fn = reinterpret_cast<const void*>(&sparse24_kernel<3>); break;
-    case 4: fn = reinterpret_cast<const void*>(&sparse24_kernel<4>); break;
+    switch (kind + (dense ? 8 : 0)) {
+    case 0: fn = reinterpret_cast<const void*>(&sparse24_kernel<0, false>); break;
+    case 1: fn = reinterpret_cast<const void*>(&sparse24_kernel<1, false>); break;
+    case 2: fn = reinterpret_cast<const void*>(&sparse24_kernel<2, false>); break;
+    case 3: fn = reinterpret_cast<const void*>(&sparse24_kernel<3, false>); break;
+    case 4: fn = reinterpret_cast<const void*>(&sparse24_kernel<4, false>); break;
+    case 8: fn = reinterpret_cast<const void*>(&sparse24_kernel<0, true>); break;
+    case 9: fn = reinterpret_cast<const void*>(&sparse24_kernel<1, true>); break;
+    case 10: fn = reinterpret_cast<const void*>(&sparse24_kernel<2, true>); break;
+    case 11: fn = reinterpret_cast<const void*>(&sparse24_kernel<3, true>); break;
+    case 12: fn = reinterpret_cast<const void*>(&sparse24_kernel<4, true>); break;
     default: return cudaErrorNotSupported;
     }
-    const int smem = static_cast<int>(kSmemBytes + 1024);
+    if (K % 128 != 0 || K > 4096 || N % 128 != 0 || (!dense && meta == nullptr)) return cudaErrorInvalidValue;
+    const int smem = static_cast<int>(smem_bytes(dense) + 1024);
     cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};

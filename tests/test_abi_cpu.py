@@ -50,13 +50,19 @@ def test_max_k(bsg):
     assert 3072 <= k < 131072  # covers the DistilBERT FFN2 (K = 3072)
 
 
-def _create(bsg, *args):
-    with pytest.raises(bsg.BsgemmError) as e:
-        bsg.bsgemm_create(*args)
-    return e.value.code
+@pytest.fixture(params=["bsgemm_create", "bsgemm_create_tc"])
+def create_fn(request):
+    return request.param
 
 
-def test_create_rejects_bad_arrays(bsg):
+def test_create_rejects_bad_arrays(bsg, create_fn):
+    """bsgemm_create and bsgemm_create_tc (the same weight, also laid out
+    for the tensor cores) validate the same way, before any device call."""
+    def _create(bsg, *args):
+        with pytest.raises(bsg.BsgemmError) as e:
+            getattr(bsg, create_fn)(*args)
+        return e.value.code
+
     ones = [1.0] * 8
     assert _create(bsg, 6, 8, 4, [0, 1, 1, 8], [[1] * 4], [1.0] * 6) == bsg.ERR_INVALID  # N = 6 (2 block-rows): column = K
     assert _create(bsg, 8, 8, 2, [0, 0, 0], [], ones) == bsg.ERR_UNSUPPORTED         # block != 4

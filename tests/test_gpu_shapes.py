@@ -8,7 +8,10 @@ oracle's linear on the oracle's own decompression of the same arrays
   * 2:4-sparse weights (bsgemm_create_2to4): N and K multiples of 128 on
     the sparse tensor cores (tcgen05.mma.sp, exact fp32 chunks of 2048
     columns added in int32), other shapes as the 4 x 1 blocks that hold
-    them."""
+    them;
+  * 4 x 1 block weights run dense over K on the tensor cores
+    (bsgemm_create_tc: tcgen05.mma kind::f16, exact fp32 chunks of 1024
+    columns added in int32)."""
 import numpy as np
 import pytest
 
@@ -109,6 +112,52 @@ def test_2to4_tensor_cores_at_the_fp32_limit(bsg):
               rng.choice(np.array([-128, 127], dtype=np.int8), size=(m, k_in))):
         want = oracle.linear(x, w, wt.scales, wt.bias, synth.I32, threads=8)
         check(gpu_run(lin, x, synth.I32, 1.0), want, synth.I32, "2:4 extremes")
+    lin.close()
+
+
+@pytest.mark.parametrize("n_out,k_in,m,sparsity", [(128, 128, 1, 0.0), (256, 2048, 130, 0.9), (768, 3072, 300, 0.9),
+                                                    (384, 1152, 257, 0.5), (256, 2944, 64, 0.8), (128, 256, 70, 1.0)])
+def test_dense_over_k_on_the_tensor_cores(bsg, n_out, k_in, m, sparsity):
+    """bsgemm_create_tc: every kind, ragged token tiles, one to three exact
+    accumulator chunks (a chunk holds 1024 columns; K = 1152 ends with a
+    chunk of one stage, K = 2944 with one of seven), a weight without
+    stored blocks; then an act
+    pointer off the 16-byte boundary, which the block-sparse kernel takes."""
+    rng = synth.rng_for(8400 + n_out + k_in + m)
+    wt = synth.draw_weight(rng, n_out, k_in, sparsity)
+    w = oracle.bsr_to_dense(n_out, k_in, wt.indptr, wt.colidx, wt.values)
+    lin = bsg.SparseInt8Linear(n_out, k_in, wt.indptr, wt.colidx, wt.values, wt.scales, wt.bias, tensor_cores=True)
+    assert lin.info["nnzb"] == wt.nnzb
+    assert lin.info["device_bytes"] >= 2 * n_out * k_in  # the f16 image of the dense form
+    x = synth.draw_x(rng, m, k_in, "u127")
+    for kind in KINDS:
+        want = oracle.linear(x, w, wt.scales, wt.bias, kind, out_scale=0.05, threads=8)
+        check(gpu_run(lin, x, kind, 0.05), want, kind, f"dense tensor cores kind {kind}")
+    buf = torch.empty(m * k_in + 4, dtype=torch.int8, device="cuda")
+    xd = buf[4:].view(m, k_in)
+    xd.copy_(torch.from_numpy(x))
+    out = torch.empty((m, n_out), dtype=torch.int32, device="cuda")
+    lin.run(xd, out, synth.I32, 1.0)
+    torch.cuda.synchronize()
+    check(out.cpu().numpy(), oracle.linear(x, w, wt.scales, wt.bias, synth.I32, threads=8), synth.I32, "offset act")
+    lin.close()
+
+
+def test_dense_tensor_cores_at_the_fp32_limit(bsg):
+    """Every weight -128 and every activation -128: each product is 2^14 and
+    a chunk's 1024 of them sum to exactly 2^24, the largest partial sum the
+    exact fp32 accumulation has to hold (three chunks); then mixed
+    extremes."""
+    n_out, k_in, m = 128, 3072, 70
+    rng = synth.rng_for(8500)
+    wt = synth.draw_weight(rng, n_out, k_in, 0.0)
+    values = np.full_like(wt.values, -128)
+    w = oracle.bsr_to_dense(n_out, k_in, wt.indptr, wt.colidx, values)
+    lin = bsg.SparseInt8Linear(n_out, k_in, wt.indptr, wt.colidx, values, wt.scales, wt.bias, tensor_cores=True)
+    for x in (np.full((m, k_in), -128, dtype=np.int8),
+              rng.choice(np.array([-128, 127], dtype=np.int8), size=(m, k_in))):
+        want = oracle.linear(x, w, wt.scales, wt.bias, synth.I32, threads=8)
+        check(gpu_run(lin, x, synth.I32, 1.0), want, synth.I32, "dense extremes")
     lin.close()
 
 
