@@ -820,8 +820,16 @@ def run_reference(args, rank: int) -> dict | None:
 LAYER_SCALES = os.path.join(ROOT, "tests", "golden", "layer_scales.json")
 
 
+# form of the layer linears in the layer / encoder / stack / production
+# workloads: "sparse" (the block-sparse kernel) or "tensor-cores" (the same
+# weights dense over K on the tensor cores, bsgemm_create_tc); --linear-form
+LINEAR_FORM = "sparse"
+
+
 def _layer_linears(bsg, weights):
-    return [bsg.SparseInt8Linear(w.n_out, w.k_in, w.indptr, w.colidx, w.values, w.scales, w.bias) for w in weights]
+    tc = LINEAR_FORM == "tensor-cores"
+    return [bsg.SparseInt8Linear(w.n_out, w.k_in, w.indptr, w.colidx, w.values, w.scales, w.bias, tensor_cores=tc)
+            for w in weights]
 
 
 def _peak_tops(props, max_mhz) -> float:
@@ -1516,7 +1524,12 @@ def main():
     p.add_argument("--no-configs", action="store_true", help="skip the other configurations' sub-objects")
     p.add_argument("--soak-seconds", type=float, default=1.0, help="untimed load before the timed region")
     p.add_argument("--e2e-steps", type=int, default=200, help="steps of the end-to-end (host buffers) timing")
+    p.add_argument("--linear-form", choices=("sparse", "tensor-cores"), default="sparse",
+                   help="layer, encoder, stack, production: the block-sparse kernel, or the same weights dense "
+                        "over K on the tensor cores (bsgemm_create_tc)")
     args = p.parse_args()
+    global LINEAR_FORM
+    LINEAR_FORM = args.linear_form
     if args.warmup < 3:
         p.error("--warmup must be >= 3")
 
@@ -1550,6 +1563,8 @@ def main():
         if world > 1:
             import torch.distributed as dist
             dist.destroy_process_group()
+    if res is not None and args.workload in ("layer", "encoder", "stack", "production"):
+        res["config"]["linear_form"] = LINEAR_FORM
     if res is not None:
         print(json.dumps(res), flush=True)
 
